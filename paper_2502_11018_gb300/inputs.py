@@ -1,0 +1,301 @@
+"""Seeded synthetic inputs for the verify pass (shared by tests, bench, smoke).
+
+This module only *synthesises* inputs: draft trees, draft tokens, planted
+hidden states, random weights and caches, uniforms.  It holds none of the
+verify pass's arithmetic (no attention, projection, selection or acceptance)
+and imports neither the CUDA library nor the oracle.
+
+Workload shapes follow GRIFFIN's evaluation: batch 1 (Section 5), a dynamic
+draft tree of 60 tokens and depth 6 built EAGLE-2 style from top-k
+expansions (Appendix C), T in {0, 1} (Section 5), LLaMA-2/LLaMA-3/Mixtral
+shaped target models (Section 5).  The MT-Bench / HumanEval / GSM8K prompts
+the paper decodes are not used: seeded random weights, caches and trees of
+the same shapes stand in for them.
+"""
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+import torch
+
+# --------------------------------------------------------------------------
+# Workload configurations.  Layer counts are the public model shapes.
+# --------------------------------------------------------------------------
+
+CONFIGS = {
+    # One attention layer + LM head, fp32, MHA 8 x 64, vocab 4096, prefix 256,
+    # 16-node tree of depth 4 with branching <= 4.
+    "tiny_f32": dict(dtype="f32", B=1, L=1, H=512, Hq=8, Hkv=8, d=64, V=4096,
+                     P=(256,), N=16, D=4, branch=4, rope_base=10000.0,
+                     std_w=0.02, std_kv=0.02, temperature=0.0),
+    # LLaMA-2-7B shaped: MHA 32 x 128, vocab 32000, prefix 2048, 60 nodes depth 6.
+    "llama2_7b": dict(dtype="bf16", B=1, L=32, H=4096, Hq=32, Hkv=32, d=128, V=32000,
+                      P=(2048,), N=60, D=6, branch=10, rope_base=10000.0,
+                      std_w=0.02, std_kv=1.0, temperature=0.0),
+    # LLaMA-3-8B shaped: GQA 32q / 8kv x 128, vocab 128256, prefix 4096, depth 8.
+    "llama3_8b": dict(dtype="bf16", B=1, L=32, H=4096, Hq=32, Hkv=8, d=128, V=128256,
+                      P=(4096,), N=60, D=8, branch=10, rope_base=500000.0,
+                      std_w=0.02, std_kv=1.0, temperature=0.0),
+    # LLaMA-2-13B shaped, batch 4 with ragged prefixes.
+    "llama2_13b_b4": dict(dtype="bf16", B=4, L=40, H=5120, Hq=40, Hkv=40, d=128, V=32000,
+                          P=(1024, 3072, 6144, 8192), N=60, D=6, branch=10,
+                          rope_base=10000.0, std_w=0.02, std_kv=1.0, temperature=0.0),
+    # Mixtral-8x7B attention shape, long context, temperature-1 acceptance.
+    "mixtral_attn": dict(dtype="bf16", B=1, L=32, H=4096, Hq=32, Hkv=8, d=128, V=32000,
+                         P=(16384,), N=60, D=8, branch=10, rope_base=1000000.0,
+                         std_w=0.02, std_kv=1.0, temperature=1.0),
+}
+
+
+def config(name, **overrides):
+    cfg = dict(CONFIGS[name])
+    cfg.update(overrides)
+    cfg["name"] = name
+    cfg["P"] = tuple(cfg["P"])
+    if len(cfg["P"]) != cfg["B"]:
+        cfg["P"] = tuple(cfg["P"][i % len(cfg["P"])] for i in range(cfg["B"]))
+    cfg.setdefault("S_max", max(cfg["P"]) + 64 + 64)
+    return cfg
+
+
+# --------------------------------------------------------------------------
+# Draft trees.
+# --------------------------------------------------------------------------
+
+def make_tree(rng, N, D, branch, V):
+    """EAGLE-2 style dynamic draft tree with ``N`` nodes (root included).
+
+    Every expanded node proposes ``branch`` candidate children with distinct
+    tokens and seeded log-probabilities; a candidate's score is its parent's
+    score plus its own log-probability.  The best-scoring chain of first
+    candidates is kept down to depth ``D`` (so the tree reaches depth ``D``);
+    the remaining ``N - 1 - D`` slots take the best-scoring candidates whose
+    parent is already kept.  Nodes are then renumbered breadth first (by
+    depth, then by parent, then by candidate rank), so ``parents[i] < i`` and
+    the first child of a node is its best candidate.
+
+    Returns ``parents`` (int32[N], ``parents[0] = -1``) and ``tokens``
+    (int32[N]; ``tokens[0]`` is the root, i.e. the last committed token).
+    """
+    assert N >= D + 1, "tree must hold a chain of depth D"
+    # Candidate table: id -> (parent id, depth, score, rank, token)
+    cand = [(-1, 0, 0.0, 0, int(rng.integers(V)))]
+    children = {}
+
+    def expand(u):
+        if u in children:
+            return children[u]
+        par, dep, score, _, _ = cand[u]
+        g = np.sort(rng.normal(0.0, 2.0, size=branch))[::-1]
+        logp = g - (g.max() + math.log(np.exp(g - g.max()).sum() + 1.0))  # strictly < 0
+        toks = rng.choice(V, size=branch, replace=False)
+        ids = []
+        for r in range(branch):
+            cand.append((u, dep + 1, score + float(logp[r]), r, int(toks[r])))
+            ids.append(len(cand) - 1)
+        children[u] = ids
+        return ids
+
+    kept = [0]
+    keptset = {0}
+    u = 0
+    for _ in range(D):
+        c = expand(u)[0]
+        kept.append(c)
+        keptset.add(c)
+        u = c
+    # Expand every node of depth < D that is kept, repeatedly, best first.
+    while len(kept) < N:
+        for k in list(kept):
+            if cand[k][1] < D:
+                expand(k)
+        best = None
+        for cid in range(1, len(cand)):
+            if cid in keptset or cand[cid][0] not in keptset:
+                continue
+            if best is None or cand[cid][2] > cand[best][2]:
+                best = cid
+        if best is None:
+            raise ValueError(f"branch {branch} and depth {D} cannot hold {N} nodes")
+        kept.append(best)
+        keptset.add(best)
+    # Breadth-first renumbering.
+    order = sorted(kept, key=lambda cid: (cand[cid][1], _bfs_key(cand, cid)))
+    new_id = {cid: i for i, cid in enumerate(order)}
+    parents = np.full(N, -1, dtype=np.int32)
+    tokens = np.zeros(N, dtype=np.int32)
+    for cid in order:
+        i = new_id[cid]
+        par = cand[cid][0]
+        parents[i] = -1 if par == -1 else new_id[par]
+        tokens[i] = cand[cid][4]
+    return parents, tokens
+
+
+def _bfs_key(cand, cid):
+    key = []
+    while cid != -1:
+        key.append(cand[cid][3])
+        cid = cand[cid][0]
+    return tuple(reversed(key))
+
+
+def children_of(parents):
+    ch = [[] for _ in range(len(parents))]
+    for i in range(1, len(parents)):
+        ch[int(parents[i])].append(i)
+    return ch
+
+
+def plant_choices(rng, parents, tokens, V, p_match=0.5):
+    """Planted target choice per node for greedy verification.
+
+    For a node with children, with probability ``p_match`` the planted choice
+    is the token of its first child (so that child matches), otherwise a
+    token none of its children carries; leaves get a random token.
+    """
+    ch = children_of(parents)
+    out = np.zeros(len(parents), dtype=np.int32)
+    for u in range(len(parents)):
+        kids = {int(tokens[c]) for c in ch[u]}
+        if ch[u] and rng.random() < p_match:
+            out[u] = tokens[ch[u][0]]
+        else:
+            while True:
+                t = int(rng.integers(V))
+                if t not in kids:
+                    break
+            out[u] = t
+    return out
+
+
+# --------------------------------------------------------------------------
+# Tensors.
+# --------------------------------------------------------------------------
+
+def torch_dtype(cfg):
+    return torch.bfloat16 if cfg["dtype"] == "bf16" else torch.float32
+
+
+def randn(gen, shape, std, dtype, device):
+    x = torch.randn(shape, generator=gen, dtype=torch.float32, device=device)
+    if std != 1.0:
+        x.mul_(std)
+    return x.to(dtype)
+
+
+def planted_hidden(gen, W, targets, alpha=1.0, eps_rel=0.05, weights=None):
+    """Rows ``h[r] = sum_k a_k W[t_rk] / |W[t_rk]| + eps * n_r``.
+
+    With ``targets`` of shape ``[rows]`` this is ``alpha * W[t] / |W[t]| +
+    eps * n`` (``eps = eps_rel * alpha / sqrt(H)``): the planted token's score
+    is about ``alpha * |W[t]|`` while every other score is a small random
+    projection, so the planted token is the row's maximum by a wide margin.
+    With ``targets`` of shape ``[rows][k]`` and per-column ``weights`` the row
+    is a weighted mix (used to shape temperature-1 target distributions:
+    the score of ``t_rk`` is then about ``weights[k]``).
+    """
+    Wf = W.float()
+    t = torch.as_tensor(targets, device=W.device, dtype=torch.long)
+    H = W.shape[1]
+    if t.dim() == 1:
+        rowsW = Wf[t]
+        h = alpha * rowsW / rowsW.norm(dim=1, keepdim=True)
+        eps = eps_rel * alpha / math.sqrt(H)
+    else:
+        wts = torch.as_tensor(weights, device=W.device, dtype=torch.float32)
+        h = torch.zeros(t.shape[0], H, device=W.device)
+        for k in range(t.shape[1]):
+            rowsW = Wf[t[:, k]]
+            h += wts[k] * rowsW / (rowsW.norm(dim=1, keepdim=True) ** 2)
+        eps = eps_rel / math.sqrt(H)
+    n = torch.randn(h.shape, generator=gen, device=W.device, dtype=torch.float32)
+    return (h + eps * n).to(W.dtype)
+
+
+@dataclass
+class StepInputs:
+    """All inputs of one verify step (device or host tensors)."""
+    cfg: dict
+    parents: torch.Tensor            # int32 [B][N]
+    tokens: torch.Tensor             # int32 [B][N]
+    prefix_len: torch.Tensor         # int32 [B]
+    planted: torch.Tensor            # int32 [B][N]  planted greedy choice (T = 0)
+    q: torch.Tensor                  # [L][B][N][Hq][d]
+    k_new: torch.Tensor              # [L][B][N][Hkv][d]
+    v_new: torch.Tensor              # [L][B][N][Hkv][d]
+    cacheK: torch.Tensor             # [L][B][Hkv][S_max][d]
+    cacheV: torch.Tensor             # [L][B][Hkv][S_max][d]
+    h: torch.Tensor                  # [B*N][H]
+    W: torch.Tensor                  # [V][H]
+    draft_logits: torch.Tensor = None  # fp32 [B][N][V]   (T > 0)
+    u_acc: torch.Tensor = None         # fp32 [B][N]      (T > 0)
+    u_res: torch.Tensor = None         # fp32 [B][N]      (T > 0)
+    extra: dict = field(default_factory=dict)
+
+
+def make_step_inputs(cfg, seed, device="cpu", layers=None):
+    """Build one seeded verify step for ``cfg`` on ``device``.
+
+    ``layers`` overrides the layer count (tests use fewer layers than the
+    bench; each layer's tensors are drawn independently).
+    """
+    L = cfg["L"] if layers is None else layers
+    B, N, D, V, H = cfg["B"], cfg["N"], cfg["D"], cfg["V"], cfg["H"]
+    Hq, Hkv, d, S_max = cfg["Hq"], cfg["Hkv"], cfg["d"], cfg["S_max"]
+    dt = torch_dtype(cfg)
+    rng = np.random.default_rng(seed)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed))
+
+    parents = np.zeros((B, N), dtype=np.int32)
+    tokens = np.zeros((B, N), dtype=np.int32)
+    planted = np.zeros((B, N), dtype=np.int32)
+    for b in range(B):
+        parents[b], tokens[b] = make_tree(rng, N, D, cfg["branch"], V)
+        planted[b] = plant_choices(rng, parents[b], tokens[b], V)
+
+    W = randn(gen, (V, H), cfg["std_w"], dt, device)
+    std = cfg["std_kv"]
+    q = randn(gen, (L, B, N, Hq, d), std, dt, device)
+    k_new = randn(gen, (L, B, N, Hkv, d), std, dt, device)
+    v_new = randn(gen, (L, B, N, Hkv, d), std, dt, device)
+    cacheK = randn(gen, (L, B, Hkv, S_max, d), std, dt, device)
+    cacheV = randn(gen, (L, B, Hkv, S_max, d), std, dt, device)
+
+    draft_logits = u_acc = u_res = None
+    T = cfg.get("temperature", 0.0)
+    if T > 0.0:
+        # Temperature-1 workload: each node's target distribution is shaped by
+        # three planted tokens (scores about 10, 9, 8 over a near-flat tail);
+        # the draft logits carry the same planted scores plus N(0, 1) noise on
+        # every token; each node's children are then drawn i.i.d. from the
+        # draft distribution of the parent, as speculative sampling assumes.
+        hot = np.stack([rng.choice(V, size=3, replace=False) for _ in range(B * N)])
+        h = planted_hidden(gen, W, hot, weights=[10.0, 9.0, 8.0])
+        dl = torch.randn((B, N, V), generator=gen, device=device, dtype=torch.float32)
+        hot_t = torch.as_tensor(hot, device=device, dtype=torch.long).view(B, N, 3)
+        dl.scatter_add_(2, hot_t, torch.tensor([10.0, 9.0, 8.0], device=device).expand(B, N, 3).contiguous())
+        draft_logits = dl
+        for b in range(B):
+            ch = children_of(parents[b])
+            for u in range(N):
+                if not ch[u]:
+                    continue
+                qd = torch.softmax(dl[b, u].double() / T, dim=0)
+                draws = torch.multinomial(qd.float(), len(ch[u]), replacement=True, generator=gen)
+                for c, x in zip(ch[u], draws.tolist()):
+                    tokens[b, c] = x
+        u_acc = torch.rand((B, N), generator=gen, device=device, dtype=torch.float32)
+        u_res = torch.rand((B, N), generator=gen, device=device, dtype=torch.float32)
+    else:
+        h = planted_hidden(gen, W, planted.reshape(-1))
+
+    def i32(a):
+        return torch.as_tensor(a, dtype=torch.int32).to(device)
+
+    return StepInputs(cfg=dict(cfg, L=L), parents=i32(parents), tokens=i32(tokens),
+                      prefix_len=i32(np.array(cfg["P"], dtype=np.int32)), planted=i32(planted),
+                      q=q, k_new=k_new, v_new=v_new, cacheK=cacheK, cacheV=cacheV,
+                      h=h, W=W, draft_logits=draft_logits, u_acc=u_acc, u_res=u_res)
