@@ -1,0 +1,331 @@
+"""Benchmark of one draft-tree verify step (GRIFFIN, arXiv 2502.11018).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+
+A step is one pass of the whole verify path over one seeded synthetic batch:
+tree build, tree attention for every layer, LM head + argmax (or logits for
+T = 1), acceptance and KV compaction, all through the C ABI of libgv.so,
+replayed as one CUDA graph.  The default workload is the LLaMA-3-8B shaped
+step (32 layers, GQA 32/8 x 128, prefix 4096, vocab 128256, 60-node tree of
+depth 8).  Its working set (1.6 GB of weights and caches) is far above the
+129 MB L2, so no L2 flush is needed between steps.
+
+Prints one JSON line (rank 0).  Under torchrun with N > 1 every rank runs an
+independent replica of the step on its own GPU (the verify path of one
+decoding stream does not shard: replicas only), and `value` is the total over
+ranks divided by the slowest rank's time.
+"""
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from paper_2502_11018_gb300 import build as gv_build  # noqa: E402
+from paper_2502_11018_gb300 import gv, inputs  # noqa: E402
+
+METRIC = "verify steps/s and accepted tok/s (LLaMA-3-8B shape, 60-node tree); % HBM roofline"
+UNIT = "verify_steps/s"
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "source": "fallback"}
+
+
+def step_bytes(cfg, accept_len):
+    """Algorithmic HBM bytes of one step: what the method must move once."""
+    es = 2 if cfg["dtype"] == "bf16" else 4
+    L, B, N, H, V = cfg["L"], cfg["B"], cfg["N"], cfg["H"], cfg["V"]
+    Hq, Hkv, d = cfg["Hq"], cfg["Hkv"], cfg["d"]
+    attn = 0
+    for P in cfg["P"]:
+        attn += 2 * P * Hkv * d * es                       # prefix K and V, read once
+    attn += B * N * (Hq + 2 * Hkv) * d * es               # tree q, k, v read
+    attn += B * N * Hq * d * es + 2 * B * N * Hkv * d * es  # output + tree K/V scratch written
+    attn *= L
+    lm = V * H * es + B * N * H * es                      # W once, hidden states
+    if cfg.get("temperature", 0.0) > 0:
+        lm += B * N * V * 4                               # fp32 logits written
+        lm += 2 * B * N * V * 4                           # target + draft logits read by accept
+    else:
+        lm += B * N * 8
+    compact = 2 * 2 * int(sum(accept_len)) * Hkv * d * es * L   # K,V rows read + written
+    return {"attention": attn, "lmhead": lm, "compact": compact,
+            "total": attn + lm + compact + B * N * 64}
+
+
+def lmhead_bytes(cfg):
+    es = 2 if cfg["dtype"] == "bf16" else 4
+    B, N, H, V = cfg["B"], cfg["N"], cfg["H"], cfg["V"]
+    b = V * H * es + B * N * H * es
+    if cfg.get("temperature", 0.0) > 0:
+        b += B * N * V * 4
+    return b
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = max(mx, float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def event_time_ms(fn, iters, stream):
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(iters):
+        fn()
+    end.record(stream)
+    end.synchronize()
+    return start.elapsed_time(end) / iters
+
+
+def cpu_baseline(cfg, seed, rank0):
+    """The float64 oracle timed on the host cores on a bounded sample."""
+    import numpy as np
+    import oracle
+    cfg1 = dict(cfg)
+    frac_v = 16 if cfg["V"] >= 64000 else 4
+    Vs = cfg["V"] // frac_v
+    inp = inputs.make_step_inputs(dict(cfg, V=Vs), seed, device="cpu", layers=1)
+    t0 = time.perf_counter()
+    oracle.verify_step(inp, layers=1, skip_compact=False)
+    t_sample = time.perf_counter() - t0
+    # Split the sample time into its attention and LM-head parts to extrapolate.
+    t1 = time.perf_counter()
+    oracle.lmhead_logits(oracle.step.as_f64(inp.h), oracle.step.as_f64(inp.W))
+    t_lm = time.perf_counter() - t1
+    t_rest = max(t_sample - t_lm, 0.0)
+    est = cfg["L"] * t_rest + frac_v * t_lm
+    cores = os.cpu_count()
+    return {"value": 1.0 / est, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": (f"1 of {cfg['L']} layers (tree build, attention, accept, compaction) and "
+                       f"{Vs} of {cfg['V']} vocabulary rows of the LM head, float64 numpy; "
+                       f"full-step time extrapolated linearly ({est:.2f} s/step; sample took "
+                       f"{t_sample:.2f} s)"),
+            "seconds_per_step": est}
+
+
+def run_reference(args):
+    """The reference arm: the float64 oracle on the host cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    cfg = inputs.config(args.config)
+    res = None
+    for _ in range(args.warmup):
+        cpu_baseline(cfg, 1000, True)
+    vals = []
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        res = cpu_baseline(cfg, 1000 + i, True)
+        vals.append(res["seconds_per_step"])
+    wall = time.perf_counter() - t0
+    v = 1.0 / statistics.mean(vals)
+    line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1000.0 * statistics.mean(vals),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": cfg["name"], "batch": cfg["B"], "layers": cfg["L"],
+                       "prefix": list(cfg["P"]), "tree_nodes": cfg["N"], "vocab": cfg["V"]},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": res["cores"], "kind": "oracle",
+                             "sample": res["sample"]},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "wall_s": wall}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="llama3_8b", choices=sorted(inputs.CONFIGS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--seed", type=int, default=1000)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
+
+    if args.impl == "reference":
+        run_reference(args)
+        return
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if rank == 0:
+        gv_build.build()
+    if dist is not None:
+        dist.barrier()
+    gv.lib()
+
+    from paper_2502_11018_gb300.step import VerifyStep
+    cfg = inputs.config(args.config)
+    inp = inputs.make_step_inputs(cfg, args.seed + rank, device=dev)
+    step = VerifyStep(inp)
+    step.capture()
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        step.replay()
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ms = event_time_ms(step.replay, args.steps, stream)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    clk = clocks.stop()
+    accept_len = step.accept_len.cpu().tolist()
+    t_max = ms
+    if dist is not None:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        t_max = float(t.item())
+
+    # Dominant kernel (LM head) timed alone on its own launch stream.
+    lm_ms = event_time_ms(step.lmhead, 20, stream)
+    peaks = load_peaks()
+    lm_gbs = lmhead_bytes(cfg) / (lm_ms * 1e-3) / 1e9
+    sb = step_bytes(cfg, accept_len)
+    step_gbs = sb["total"] / (t_max * 1e-3) / 1e9
+
+    # End to end through the public API with host buffers: pinned host inputs
+    # copied in, step, result read back, every step.
+    e2e = e2e_measure(step, inp, args.e2e_steps, stream)
+
+    launches_per_step = 1 + 3 * cfg["L"] + 2 + 1 + 1
+    line = {
+        "metric": METRIC, "value": world * 1000.0 / t_max, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg["dtype"],
+        "data": "synthetic (seeded random weights, caches and draft trees)",
+        "config": {"workload": cfg["name"], "batch": cfg["B"], "layers": cfg["L"],
+                   "hidden": cfg["H"], "heads_q": cfg["Hq"], "heads_kv": cfg["Hkv"],
+                   "head_dim": cfg["d"], "vocab": cfg["V"], "prefix": list(cfg["P"]),
+                   "tree_nodes": cfg["N"], "tree_depth": cfg["D"],
+                   "temperature": cfg.get("temperature", 0.0),
+                   "l2": "working set above L2 (no flush needed)", "parallelism": f"replicas{world}"},
+        "accepted_tok_per_s": world * sum(accept_len) * 1000.0 / t_max,
+        "accept_len": accept_len,
+        "hbm_roofline": {"step_bytes": sb["total"], "achieved_gbs": step_gbs,
+                         "peak_gbs": peaks["hbm_gbs"], "frac": step_gbs / peaks["hbm_gbs"],
+                         "peak_source": peaks["source"]},
+        "roofline": {"kernel": "lmhead_select", "bound": "hbm", "achieved": lm_gbs,
+                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": lm_gbs / peaks["hbm_gbs"],
+                     "traffic": None, "ms_per_launch": lm_ms},
+        "gpu_launches": launches_per_step * args.steps,
+        "e2e": e2e,
+        "clocks": clk,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = {k: v for k, v in cpu_baseline(cfg, args.seed, True).items()
+                                if k != "seconds_per_step"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def e2e_measure(step, inp, steps, stream):
+    """Same metric through VerifyStep with host buffers: the step's inputs
+    (tree, tokens, per-layer q/k/v, hidden states, uniforms) are copied from
+    pinned host memory, the step runs, and the accepted tokens are read back."""
+    names = ["parents", "tokens", "prefix_len", "q", "k_new", "v_new", "h"]
+    if inp.draft_logits is not None:
+        names += ["draft_logits", "u_acc", "u_res"]
+    host = {n: getattr(inp, n).cpu().pin_memory() for n in names}
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    outs = [step.accept_len, step.out_tokens, step.path]
+    d2h = sum(t.numel() * t.element_size() for t in outs)
+    pinned_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
+
+    def one():
+        for n in names:
+            getattr(inp, n).copy_(host[n], non_blocking=True)
+        step.replay()
+        for dst, src in zip(pinned_out, outs):
+            dst.copy_(src, non_blocking=True)
+
+    one()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one()
+        torch.cuda.current_stream().synchronize()
+    dt = (time.perf_counter() - t0) / steps
+    return {"value": 1.0 / dt, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": dt * 1000.0}
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,231 @@
+/*
+ * gv.h -- C ABI of the GB300 draft-tree verification library (libgv.so).
+ *
+ * One verify step of GRIFFIN-style speculative decoding (arXiv 2502.11018):
+ * the draft model proposes a tree of tokens, the target model verifies all of
+ * them in a single forward pass and accepts a subset (Section 3, the
+ * draft-and-verify cycle; Appendix C, the dynamic draft tree of 60 tokens).
+ * The calls below are that pass's data-parallel steps, in order:
+ *
+ *   gv_tree_build        positions and ancestor bitmasks from a parent array
+ *   gv_verify_attention  tree-masked attention of one layer (call per layer)
+ *   gv_lmhead_select     LM-head projection fused with argmax / top-k / logits
+ *   gv_accept            longest accepted root chain (T = 0) or recursive
+ *                        rejection sampling (T > 0)
+ *   gv_kv_compact        commit the accepted chain's K/V into the cache
+ *
+ * Conventions shared by every call:
+ *  - Every pointer argument is DEVICE memory owned by the caller, unless the
+ *    argument says otherwise.  The library never allocates on these paths:
+ *    scratch memory is queried with the matching *_workspace call and passed
+ *    in.  The library keeps no state between calls (the only persistent state
+ *    of a decoding loop is the caller's cache and prefix lengths).
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Calls only enqueue work; they are asynchronous with respect to
+ *    the host and can be captured into a CUDA graph.
+ *  - Return value: a gv_status.  Argument errors the host can see (null
+ *    pointers, bad sizes, misalignment, unsupported shapes) return
+ *    synchronously before anything is enqueued.  A CUDA launch error returns
+ *    GV_ERR_CUDA (text from gv_last_error()).  Data-dependent errors (an
+ *    invalid parent array, cache overflow) cannot be seen by the host without
+ *    a synchronisation; they are written to the per-sequence status array
+ *    `seq_status[B]` on the device, and every later call that takes
+ *    `seq_status` leaves a sequence whose status is non-zero untouched.
+ *  - Index layouts are row-major with the last index contiguous.  Node 0 of
+ *    every tree is the root (the last committed token, whose K/V is not yet
+ *    in the cache); nodes are in topological order, parents[i] < i.
+ *  - Limits: 1 <= N <= 64 nodes per tree; head dim d in {64, 128}; Hq a
+ *    multiple of Hkv.
+ */
+#ifndef GV_H
+#define GV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    GV_OK = 0,
+    GV_ERR_ARG = -1,          /* bad pointer, size, alignment or mode          */
+    GV_ERR_INVALID_TREE = -2, /* parent array breaks the topological rule, or
+                                 a node is deeper than the caller's D         */
+    GV_ERR_CAPACITY = -3,     /* prefix_len + accept_len would exceed S_max    */
+    GV_ERR_UNSUPPORTED = -4,  /* shape outside the supported limits, or no
+                                 sm_103 device                                */
+    GV_ERR_CUDA = -5,         /* a CUDA runtime call failed                    */
+    GV_ERR_TIMEOUT = -6       /* a bounded device-side wait gave up            */
+} gv_status;
+
+typedef enum { GV_BF16 = 0, GV_F32 = 1 } gv_dtype;
+
+typedef enum {
+    GV_SELECT_ARGMAX = 0,     /* ids[rows], vals[rows] = max logit             */
+    GV_SELECT_TOPK = 1,       /* ids[rows][k], vals[rows][k], k <= 16          */
+    GV_SELECT_LOGITS = 2      /* logits[rows][V] fp32, row_max[rows], row_lse[rows] */
+} gv_select_mode;
+
+/* Shape of one attention layer of the verify pass. */
+typedef struct {
+    int B;            /* sequences                                            */
+    int N;            /* tree nodes per sequence, root included (<= 64)       */
+    int Hq;           /* query heads                                          */
+    int Hkv;          /* key/value heads (Hq % Hkv == 0; GQA when Hq > Hkv)   */
+    int d;            /* head dimension (64 or 128)                           */
+    int S_max;        /* cache rows per (sequence, KV head)                   */
+    float rope_base;  /* RoPE frequency base                                  */
+    gv_dtype dt;      /* GV_BF16 (tensor-core path) or GV_F32                 */
+} gv_attn_shape;
+
+/*
+ * gv_tree_build -- depths, RoPE positions and ancestor bitmasks of B trees.
+ * Section 4.1: a rejected draft token takes every later token of its draft
+ * sequence with it, so the ancestor-or-self set of a node is what decides both
+ * its attention mask and its acceptance; Appendix C: dynamic tree, <= 64 nodes.
+ *
+ *   parents    int32 [B][N]  parent index per node; parents[b][0] == -1 and
+ *                            0 <= parents[b][i] < i for i >= 1
+ *   prefix_len int32 [B]     cached tokens per sequence (P_b)
+ *   depth      int32 [B][N]  out: edges from the root
+ *   pos        int32 [B][N]  out: P_b + depth (RoPE position)
+ *   anc        uint64[B][N]  out: bit j set iff node j is on the root-to-i chain
+ *   seq_status int32 [B]     out: GV_OK, or GV_ERR_INVALID_TREE for a parent
+ *                            array that breaks the rule above; such a tree gets
+ *                            depth 0, pos P_b and anc[i] = 1 << i.
+ * Returns GV_ERR_INVALID_TREE synchronously when N < 1 or N > 64.
+ */
+int gv_tree_build(const int32_t* parents, const int32_t* prefix_len, int B, int N,
+                  int32_t* depth, int32_t* pos, uint64_t* anc, int32_t* seq_status,
+                  void* stream);
+
+/*
+ * gv_verify_attention -- one attention layer of the verify forward pass.
+ * Section 3: the target model verifies all draft tokens in one forward pass.
+ * Draft node i of sequence b, query head h, attends to the cached prefix rows
+ * 0..P_b-1 of KV head g = h / (Hq/Hkv) and to the tree nodes j with bit j of
+ * anc[b][i] set, which equals causal attention over [prefix ; root chain of i].
+ * RoPE (rotate-half, frequencies rope_base^(-2j/d), angles formed in double)
+ * is applied to q and k_new at pos[b][i]; softmax scale is 1/sqrt(d).
+ *
+ *   q          [B][N][Hq][d]      tree queries, unrotated           (dt)
+ *   k_new      [B][N][Hkv][d]     tree keys, unrotated              (dt)
+ *   v_new      [B][N][Hkv][d]     tree values                       (dt)
+ *   cacheK/V   [B][Hkv][S_max][d] cache of this layer; rows < P_b are
+ *                                 read (keys stored already rotated)  (dt)
+ *   prefix_len int32 [B]          P_b <= S_max
+ *   pos, anc   from gv_tree_build
+ *   treeK/V    [B][Hkv][N][d]     out: rotated tree keys / the values, the
+ *                                 scratch gv_kv_compact reads        (dt)
+ *   out        [B][N][Hq][d]      out: attention output              (dt)
+ *   workspace  >= gv_verify_attention_workspace(s) bytes, 256-byte aligned;
+ *              contents need no initialisation and are clobbered.
+ * All tensors 16-byte aligned.  Two calls that share a workspace must be
+ * ordered on the device (same stream or an event between them).
+ */
+size_t gv_verify_attention_workspace(const gv_attn_shape* s);
+int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new,
+                        const void* v_new, const void* cacheK, const void* cacheV,
+                        const int32_t* prefix_len, const int32_t* pos, const uint64_t* anc,
+                        void* treeK, void* treeV, void* out,
+                        void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * gv_lmhead_select -- LM head fused with the per-node selection.
+ * Section 3 / Eq. 1: the LM head maps a final hidden feature to a token;
+ * Section 4.1 ranks candidates by their top-k; Section 5 decodes at T in {0,1}.
+ * logits[r][v] = sum_k h[r][k] * W[v][k], accumulated in fp32.
+ *
+ *   h        [rows][H]   final hidden states of the tree nodes     (dt)
+ *   W        [V][H]      LM-head weight, row-major                 (dt)
+ *   mode GV_SELECT_ARGMAX: ids int32[rows] = argmax (lowest id on ties),
+ *                          vals fp32[rows] = its logit; no logits are written
+ *                          to memory.
+ *   mode GV_SELECT_TOPK:   ids int32[rows][k], vals fp32[rows][k], by
+ *                          decreasing logit, lower id first on ties; 1<=k<=16.
+ *   mode GV_SELECT_LOGITS: logits fp32[rows][V], row_max fp32[rows],
+ *                          row_lse fp32[rows] = max + log(sum exp(l - max)).
+ *   Unused outputs may be NULL.
+ *   workspace >= gv_lmhead_workspace(rows, H, V, dt, mode, k) bytes.
+ * H must be a multiple of 64 (bf16) or 4 (fp32); rows >= 1.
+ */
+size_t gv_lmhead_workspace(int rows, int H, int V, int dt, int mode, int k);
+int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int dt, int mode,
+                     int k, int32_t* ids, float* vals, float* logits, float* row_max,
+                     float* row_lse, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * gv_accept -- accept the longest verified root chain of each tree.
+ * Section 3: the target accepts a subset of the drafts; Section 4.1: a
+ * rejected token discards its whole subtree; Section 5: lossless at T = 0 and
+ * T = 1.
+ *
+ * temperature == 0 (greedy): node j > 0 matches when
+ *   tokens[b][j] == choice[b*N + parent(j)]; the accepted node is the deepest
+ *   node whose whole root chain matches (smallest index among equals).
+ * temperature > 0: multi-draft recursive rejection sampling.  From the root:
+ *   p = softmax(target_logits[b][u] / T), q = softmax(draft_logits[b][u] / T);
+ *   children c of u in increasing index are accepted when
+ *   u_acc[b][c] <= p(x_c) / q(x_c) (always when q(x_c) == 0), otherwise
+ *   p <- max(p - q, 0) / sum(max(p - q, 0)) (kept if that sum is 0); when no
+ *   child is accepted the bonus token is the smallest v with
+ *   sum_{w<=v} p(w) > u_res[b][u] * sum(p).
+ *
+ *   tokens        int32 [B][N]      draft token per node (tokens[b][0] = root)
+ *   anc, depth    from gv_tree_build
+ *   choice        int32 [B*N]       target argmax per node (T == 0; else NULL)
+ *   target_logits fp32  [B][N][V]   (T > 0; else NULL)
+ *   draft_logits  fp32  [B][N][V]   (T > 0; else NULL)
+ *   u_acc, u_res  fp32  [B][N]      uniforms in [0, 1) (T > 0; else NULL)
+ *   path          int32 [B][D+1]    out: accepted chain, root first, -1 padded
+ *   accept_len    int32 [B]         out: entries of path (1 .. D+1)
+ *   out_tokens    int32 [B][D+1]    out: accepted drafts then the bonus token
+ *   seq_status    int32 [B]         in/out: non-zero sequences are skipped
+ *                                   (accept_len 0, rows of -1); a tree with a
+ *                                   node deeper than D gets GV_ERR_INVALID_TREE.
+ *   workspace >= gv_accept_workspace(B, V, temperature) bytes (0 for T == 0).
+ */
+size_t gv_accept_workspace(int B, int V, float temperature);
+int gv_accept(int B, int N, int D, int V, float temperature, const int32_t* tokens,
+              const uint64_t* anc, const int32_t* depth, const int32_t* choice,
+              const float* target_logits, const float* draft_logits, const float* u_acc,
+              const float* u_res, int32_t* path, int32_t* accept_len, int32_t* out_tokens,
+              int32_t* seq_status, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * gv_kv_compact -- append the accepted chain's K/V to every layer's cache.
+ * Section 4.1: only the accepted chain survives verification.  For every
+ * layer l, sequence b, KV head h and t < accept_len[b]:
+ *   cache[l][b][h][P_b + t][:] = tree[l][b][h][path[b][t]][:]
+ * and new_len[b] = P_b + accept_len[b].  Nothing else is written.
+ *
+ *   treeK/V    [L][B][Hkv][N][d]      tree scratch of every layer   (dt)
+ *   cacheK/V   [L][B][Hkv][S_max][d]  caches, updated in place       (dt)
+ *   path       int32 [B][D+1], accept_len int32 [B] from gv_accept
+ *   prefix_len int32 [B]
+ *   new_len    int32 [B]   out
+ *   seq_status int32 [B]   in/out: non-zero sequences are left untouched
+ *                          (new_len = P_b); P_b + accept_len > S_max sets
+ *                          GV_ERR_CAPACITY and writes nothing for that sequence.
+ * Rows must be 16-byte multiples (d * sizeof(dt) % 16 == 0).
+ */
+int gv_kv_compact(int L, int B, int N, int D, int Hkv, int d, int S_max, int dt,
+                  const void* treeK, const void* treeV, void* cacheK, void* cacheV,
+                  const int32_t* path, const int32_t* accept_len, const int32_t* prefix_len,
+                  int32_t* new_len, int32_t* seq_status, void* stream);
+
+/* Static name of a status code. */
+const char* gv_status_string(int status);
+
+/* Detail of the last error returned on the calling host thread ("" if none). */
+const char* gv_last_error(void);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int gv_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GV_H */

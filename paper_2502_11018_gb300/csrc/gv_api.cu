@@ -1,0 +1,337 @@
+// extern "C" entry points of libgv.so: argument validation, workspace
+// carving, and dispatch to the kernels.  The declarations and the contract of
+// every call are in include/gv.h.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <cmath>
+
+#include "gv_internal.cuh"
+#include "attention.cuh"
+
+namespace gv {
+
+// ------------------------------------------------------------- bookkeeping --
+static thread_local char g_err[512];
+
+void set_error(const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+}
+
+void clear_error() { g_err[0] = '\0'; }
+
+int check_launch(const char* what) {
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) {
+        set_error("%s: %s", what, cudaGetErrorString(e));
+        return GV_ERR_CUDA;
+    }
+    return GV_OK;
+}
+
+int sm_count() {
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (cache[dev] == 0) {
+        int n = 0;
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        cache[dev] = n > 0 ? n : 148;
+    }
+    return cache[dev];
+}
+
+int device_cc() {
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    if (cache[dev] == 0) {
+        int ma = 0, mi = 0;
+        cudaDeviceGetAttribute(&ma, cudaDevAttrComputeCapabilityMajor, dev);
+        cudaDeviceGetAttribute(&mi, cudaDevAttrComputeCapabilityMinor, dev);
+        cache[dev] = ma * 10 + mi;
+    }
+    return cache[dev];
+}
+
+static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Kernel launchers defined in the other translation units.
+int launch_tree_build(const int32_t*, const int32_t*, int, int, int32_t*, int32_t*, uint64_t*,
+                      int32_t*, cudaStream_t);
+int launch_kv_compact(int, int, int, int, int, int, int, int, const void*, const void*, void*,
+                      void*, const int32_t*, const int32_t*, const int32_t*, int32_t*, int32_t*,
+                      cudaStream_t);
+int launch_accept(int, int, int, int, float, const int32_t*, const uint64_t*, const int32_t*,
+                  const int32_t*, const float*, const float*, const float*, const float*,
+                  int32_t*, int32_t*, int32_t*, int32_t*, void*, cudaStream_t);
+int launch_lmhead_cc(const void*, const void*, int, int, int, int, int, int, float*,
+                     SelectPartials, int32_t*, float*, float*, float*, cudaStream_t);
+
+// ---------------------------------------------------------- attention plan --
+constexpr int KPS = 256;   // prefix keys per split
+
+struct AttnPlan {
+    size_t q_rot, part_o, part_ml, counters, total;
+    int nsplit, q_rows_pad;
+};
+
+static bool attn_shape_ok(const gv_attn_shape* s) {
+    return s && s->B >= 1 && s->N >= 1 && s->N <= 64 && s->Hkv >= 1 && s->Hq >= s->Hkv &&
+           s->Hq % s->Hkv == 0 && (s->d == 64 || s->d == 128) && s->S_max >= 1 &&
+           (s->dt == GV_BF16 || s->dt == GV_F32) && s->rope_base > 0.0f &&
+           std::isfinite(s->rope_base);
+}
+
+static AttnPlan attn_plan(const gv_attn_shape* s) {
+    AttnPlan p{};
+    const int R = (s->Hq / s->Hkv) * s->N;
+    p.q_rows_pad = (R + 127) / 128 * 128;
+    p.nsplit = (s->S_max + KPS - 1) / KPS + 1;
+    const size_t bh = (size_t)s->B * s->Hkv;
+    size_t off = 0;
+    p.q_rot = off;
+    off += align256(bh * p.q_rows_pad * s->d * sizeof(float));
+    p.part_o = off;
+    off += align256(bh * p.nsplit * R * s->d * sizeof(float));
+    p.part_ml = off;
+    off += align256(bh * p.nsplit * R * 2 * sizeof(float));
+    p.counters = off;
+    off += align256(bh * sizeof(unsigned));
+    p.total = off;
+    return p;
+}
+
+// ------------------------------------------------------------ lmhead plan --
+constexpr int CC_TV = 64;
+
+struct LmPlan {
+    size_t val, id, m, s, total;
+    int slots, K;
+};
+
+static LmPlan lm_plan(int rows, int V, int mode, int k) {
+    LmPlan p{};
+    p.slots = (V + CC_TV - 1) / CC_TV;
+    p.K = mode == GV_SELECT_TOPK ? k : 1;
+    const size_t n = (size_t)p.slots * rows;
+    size_t off = 0;
+    p.val = off;
+    off += align256(n * p.K * sizeof(float));
+    p.id = off;
+    off += align256(n * p.K * sizeof(int));
+    p.m = off;
+    off += align256(n * sizeof(float));
+    p.s = off;
+    off += align256(n * sizeof(float));
+    p.total = off;
+    return p;
+}
+
+}  // namespace gv
+
+using namespace gv;
+
+extern "C" {
+
+int gv_version(void) { return 100; }
+
+const char* gv_last_error(void) { return g_err; }
+
+const char* gv_status_string(int status) {
+    switch (status) {
+        case GV_OK: return "GV_OK";
+        case GV_ERR_ARG: return "GV_ERR_ARG";
+        case GV_ERR_INVALID_TREE: return "GV_ERR_INVALID_TREE";
+        case GV_ERR_CAPACITY: return "GV_ERR_CAPACITY";
+        case GV_ERR_UNSUPPORTED: return "GV_ERR_UNSUPPORTED";
+        case GV_ERR_CUDA: return "GV_ERR_CUDA";
+        case GV_ERR_TIMEOUT: return "GV_ERR_TIMEOUT";
+        default: return "GV_ERR_UNKNOWN";
+    }
+}
+
+int gv_tree_build(const int32_t* parents, const int32_t* prefix_len, int B, int N, int32_t* depth,
+                  int32_t* pos, uint64_t* anc, int32_t* seq_status, void* stream) {
+    clear_error();
+    if (N < 1 || N > 64) {
+        set_error("gv_tree_build: N=%d outside 1..64", N);
+        return GV_ERR_INVALID_TREE;
+    }
+    GV_CHECK_ARG(B >= 1, "gv_tree_build: B=%d", B);
+    GV_CHECK_ARG(parents && prefix_len && depth && pos && anc && seq_status,
+                 "gv_tree_build: null pointer");
+    GV_CHECK_ARG(((uintptr_t)anc & 7u) == 0, "gv_tree_build: anc not 8-byte aligned");
+    return launch_tree_build(parents, prefix_len, B, N, depth, pos, anc, seq_status,
+                             as_stream(stream));
+}
+
+size_t gv_verify_attention_workspace(const gv_attn_shape* s) {
+    if (!attn_shape_ok(s)) return 0;
+    return attn_plan(s).total;
+}
+
+int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new,
+                        const void* v_new, const void* cacheK, const void* cacheV,
+                        const int32_t* prefix_len, const int32_t* pos, const uint64_t* anc,
+                        void* treeK, void* treeV, void* out, void* workspace, size_t ws_bytes,
+                        void* stream) {
+    clear_error();
+    if (s && (s->N < 1 || s->N > 64)) {
+        set_error("gv_verify_attention: N=%d outside 1..64", s->N);
+        return GV_ERR_UNSUPPORTED;
+    }
+    if (s && !(s->d == 64 || s->d == 128)) {
+        set_error("gv_verify_attention: head dim %d not in {64, 128}", s->d);
+        return GV_ERR_UNSUPPORTED;
+    }
+    GV_CHECK_ARG(attn_shape_ok(s), "gv_verify_attention: invalid shape");
+    const void* ptrs[] = {q, k_new, v_new, cacheK, cacheV, treeK, treeV, out};
+    for (const void* p : ptrs)
+        GV_CHECK_ARG(p && aligned16(p), "gv_verify_attention: tensor null or not 16-byte aligned");
+    GV_CHECK_ARG(prefix_len && pos && anc, "gv_verify_attention: null index pointer");
+    const AttnPlan plan = attn_plan(s);
+    GV_CHECK_ARG(workspace && ((uintptr_t)workspace & 255u) == 0,
+                 "gv_verify_attention: workspace null or not 256-byte aligned");
+    GV_CHECK_ARG(ws_bytes >= plan.total, "gv_verify_attention: workspace %zu < %zu bytes",
+                 ws_bytes, plan.total);
+    char* ws = static_cast<char*>(workspace);
+    AttnArgs a{};
+    a.B = s->B;
+    a.N = s->N;
+    a.Hq = s->Hq;
+    a.Hkv = s->Hkv;
+    a.d = s->d;
+    a.S_max = s->S_max;
+    a.G = s->Hq / s->Hkv;
+    a.R = a.G * s->N;
+    a.q_rows_pad = plan.q_rows_pad;
+    a.rope_base = s->rope_base;
+    a.scale = 1.0f / sqrtf((float)s->d);
+    a.q = q;
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.cacheK = cacheK;
+    a.cacheV = cacheV;
+    a.prefix_len = prefix_len;
+    a.pos = pos;
+    a.anc = reinterpret_cast<const unsigned long long*>(anc);
+    a.treeK = treeK;
+    a.treeV = treeV;
+    a.out = out;
+    a.q_rot = ws + plan.q_rot;
+    a.part_o = reinterpret_cast<float*>(ws + plan.part_o);
+    a.part_ml = reinterpret_cast<float*>(ws + plan.part_ml);
+    a.counters = reinterpret_cast<unsigned*>(ws + plan.counters);
+    a.nsplit = plan.nsplit;
+    a.kps = KPS;
+    cudaStream_t st = as_stream(stream);
+    int rc;
+    if (s->dt == GV_F32) {
+        if ((rc = launch_rope_tree<float, float>(a, st)) != GV_OK) return rc;
+        if ((rc = launch_attn_cc<float>(a, st)) != GV_OK) return rc;
+        return launch_attn_combine<float>(a, st);
+    }
+    if ((rc = launch_rope_tree<__nv_bfloat16, float>(a, st)) != GV_OK) return rc;
+    if ((rc = launch_attn_cc<__nv_bfloat16>(a, st)) != GV_OK) return rc;
+    return launch_attn_combine<__nv_bfloat16>(a, st);
+}
+
+size_t gv_lmhead_workspace(int rows, int H, int V, int dt, int mode, int k) {
+    if (rows < 1 || H < 1 || V < 1 || mode < 0 || mode > 2) return 0;
+    if (mode == GV_SELECT_TOPK && (k < 1 || k > 16)) return 0;
+    (void)dt;
+    return lm_plan(rows, V, mode, k).total;
+}
+
+int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int dt, int mode, int k,
+                     int32_t* ids, float* vals, float* logits, float* row_max, float* row_lse,
+                     void* workspace, size_t ws_bytes, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(rows >= 1 && H >= 1 && V >= 1, "gv_lmhead_select: rows=%d H=%d V=%d", rows, H, V);
+    GV_CHECK_ARG(dt == GV_BF16 || dt == GV_F32, "gv_lmhead_select: dtype %d", dt);
+    GV_CHECK_ARG(mode >= 0 && mode <= 2, "gv_lmhead_select: mode %d", mode);
+    GV_CHECK_ARG(mode != GV_SELECT_TOPK || (k >= 1 && k <= 16), "gv_lmhead_select: k=%d", k);
+    GV_CHECK_ARG(h && W && aligned16(h) && aligned16(W), "gv_lmhead_select: h/W null or unaligned");
+    if (mode == GV_SELECT_LOGITS)
+        GV_CHECK_ARG(logits, "gv_lmhead_select: logits output is null");
+    else
+        GV_CHECK_ARG(ids, "gv_lmhead_select: ids output is null");
+    const LmPlan plan = lm_plan(rows, V, mode, k);
+    GV_CHECK_ARG(workspace && ((uintptr_t)workspace & 255u) == 0,
+                 "gv_lmhead_select: workspace null or not 256-byte aligned");
+    GV_CHECK_ARG(ws_bytes >= plan.total, "gv_lmhead_select: workspace %zu < %zu bytes", ws_bytes,
+                 plan.total);
+    char* ws = static_cast<char*>(workspace);
+    SelectPartials part;
+    part.val = reinterpret_cast<float*>(ws + plan.val);
+    part.id = reinterpret_cast<int*>(ws + plan.id);
+    part.m = reinterpret_cast<float*>(ws + plan.m);
+    part.s = reinterpret_cast<float*>(ws + plan.s);
+    part.slots = plan.slots;
+    part.rows = rows;
+    part.K = plan.K;
+    return launch_lmhead_cc(h, W, rows, H, V, dt, mode, plan.K, logits, part, ids, vals, row_max,
+                            row_lse, as_stream(stream));
+}
+
+size_t gv_accept_workspace(int B, int V, float temperature) {
+    if (B < 1) return 0;
+    if (temperature == 0.0f) return 0;
+    return align256((size_t)B * 2 * (size_t)V * sizeof(float));
+}
+
+int gv_accept(int B, int N, int D, int V, float temperature, const int32_t* tokens,
+              const uint64_t* anc, const int32_t* depth, const int32_t* choice,
+              const float* target_logits, const float* draft_logits, const float* u_acc,
+              const float* u_res, int32_t* path, int32_t* accept_len, int32_t* out_tokens,
+              int32_t* seq_status, void* workspace, size_t ws_bytes, void* stream) {
+    clear_error();
+    if (N < 1 || N > 64) {
+        set_error("gv_accept: N=%d outside 1..64", N);
+        return GV_ERR_INVALID_TREE;
+    }
+    GV_CHECK_ARG(B >= 1 && D >= 0, "gv_accept: B=%d D=%d", B, D);
+    GV_CHECK_ARG(std::isfinite(temperature) && temperature >= 0.0f, "gv_accept: temperature %g",
+                 (double)temperature);
+    GV_CHECK_ARG(tokens && anc && depth && path && accept_len && out_tokens && seq_status,
+                 "gv_accept: null pointer");
+    if (temperature == 0.0f) {
+        GV_CHECK_ARG(choice, "gv_accept: greedy acceptance needs choice");
+    } else {
+        GV_CHECK_ARG(V >= 1, "gv_accept: V=%d", V);
+        GV_CHECK_ARG(target_logits && draft_logits && u_acc && u_res,
+                     "gv_accept: sampling needs logits and uniforms");
+        GV_CHECK_ARG(workspace && ws_bytes >= gv_accept_workspace(B, V, temperature),
+                     "gv_accept: workspace too small");
+    }
+    return launch_accept(B, N, D, V, temperature, tokens, anc, depth, choice, target_logits,
+                         draft_logits, u_acc, u_res, path, accept_len, out_tokens, seq_status,
+                         workspace, as_stream(stream));
+}
+
+int gv_kv_compact(int L, int B, int N, int D, int Hkv, int d, int S_max, int dt, const void* treeK,
+                  const void* treeV, void* cacheK, void* cacheV, const int32_t* path,
+                  const int32_t* accept_len, const int32_t* prefix_len, int32_t* new_len,
+                  int32_t* seq_status, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(L >= 1 && B >= 1 && N >= 1 && N <= 64 && D >= 0 && Hkv >= 1 && d >= 1 &&
+                     S_max >= 1,
+                 "gv_kv_compact: bad sizes");
+    GV_CHECK_ARG(dt == GV_BF16 || dt == GV_F32, "gv_kv_compact: dtype %d", dt);
+    const int esize = dt == GV_BF16 ? 2 : 4;
+    GV_CHECK_ARG((d * esize) % 16 == 0, "gv_kv_compact: row of %d bytes is not a 16-byte multiple",
+                 d * esize);
+    const void* ptrs[] = {treeK, treeV, cacheK, cacheV};
+    for (const void* p : ptrs)
+        GV_CHECK_ARG(p && aligned16(p), "gv_kv_compact: tensor null or not 16-byte aligned");
+    GV_CHECK_ARG(path && accept_len && prefix_len && new_len && seq_status,
+                 "gv_kv_compact: null index pointer");
+    return launch_kv_compact(L, B, N, D, Hkv, d, S_max, esize, treeK, treeV, cacheK, cacheV, path,
+                             accept_len, prefix_len, new_len, seq_status, as_stream(stream));
+}
+
+}  // extern "C"

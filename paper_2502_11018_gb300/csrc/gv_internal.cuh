@@ -1,0 +1,79 @@
+// Internal helpers of libgv.so (not part of the C ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "gv.h"
+
+namespace gv {
+
+// ---- host-side error bookkeeping -------------------------------------------
+void set_error(const char* fmt, ...);
+void clear_error();
+
+#define GV_CHECK_ARG(cond, ...)                                     \
+    do {                                                            \
+        if (!(cond)) {                                              \
+            ::gv::set_error(__VA_ARGS__);                           \
+            return GV_ERR_ARG;                                      \
+        }                                                           \
+    } while (0)
+
+// Launch-error check after a kernel launch.
+int check_launch(const char* what);
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+inline cudaStream_t as_stream(void* s) { return reinterpret_cast<cudaStream_t>(s); }
+
+// Number of SMs of the current device (cached per device).
+int sm_count();
+// Compute capability major*10+minor of the current device.
+int device_cc();
+
+// ---- device helpers ---------------------------------------------------------
+constexpr unsigned FULL = 0xffffffffu;
+
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <typename T> __device__ __forceinline__ T from_f32(float x);
+template <> __device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) {
+    return __float2bfloat16_rn(x);
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(FULL, v, o));
+    return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
+    return v;
+}
+
+// (value, id) ordering used by every selection: larger value first, then
+// smaller id.  NaN never wins.
+__device__ __forceinline__ bool better(float va, int ia, float vb, int ib) {
+    return (va > vb) || (va == vb && ia < ib) || (vb != vb && va == va);
+}
+
+// Per-(slot, row) partial results of the LM-head selection, merged by
+// lmhead_merge_kernel.  Layout in the workspace (slots = producing tiles):
+//   float val[slots][rows][K]; int id[slots][rows][K];  (top-K, K = k or 1)
+//   float m[slots][rows]; float s[slots][rows];          (logits mode: max, sum exp)
+struct SelectPartials {
+    float* val;
+    int* id;
+    float* m;
+    float* s;
+    int slots;
+    int rows;
+    int K;
+};
+
+}  // namespace gv

@@ -1,0 +1,196 @@
+"""ctypes binding of libgv.so: the C-ABI calls of include/gv.h under the same
+names, taking torch CUDA tensors.
+
+This layer only marshals arguments (device pointers, sizes, the current
+stream); every step of the verify pass runs in the library's CUDA kernels.
+There is no fallback: if libgv.so is missing, or a tensor is not on a CUDA
+device, the calls raise.
+"""
+
+import ctypes
+import os
+
+import torch
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libgv.so")
+
+GV_OK = 0
+GV_ERR_ARG = -1
+GV_ERR_INVALID_TREE = -2
+GV_ERR_CAPACITY = -3
+GV_ERR_UNSUPPORTED = -4
+GV_ERR_CUDA = -5
+GV_ERR_TIMEOUT = -6
+
+GV_BF16 = 0
+GV_F32 = 1
+
+GV_SELECT_ARGMAX = 0
+GV_SELECT_TOPK = 1
+GV_SELECT_LOGITS = 2
+
+# Every symbol include/gv.h declares.
+EXPORTS = ("gv_tree_build", "gv_verify_attention_workspace", "gv_verify_attention",
+           "gv_lmhead_workspace", "gv_lmhead_select", "gv_accept_workspace", "gv_accept",
+           "gv_kv_compact", "gv_status_string", "gv_last_error", "gv_version")
+
+
+class GvError(RuntimeError):
+    def __init__(self, call, status, detail):
+        super().__init__(f"{call} -> {status_string(status)} ({status}): {detail}")
+        self.status = status
+
+
+class gv_attn_shape(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("N", ctypes.c_int), ("Hq", ctypes.c_int),
+                ("Hkv", ctypes.c_int), ("d", ctypes.c_int), ("S_max", ctypes.c_int),
+                ("rope_base", ctypes.c_float), ("dt", ctypes.c_int)]
+
+
+_lib = None
+_vp = ctypes.c_void_p
+_i = ctypes.c_int
+_f = ctypes.c_float
+_sz = ctypes.c_size_t
+
+
+def lib():
+    """Load libgv.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                           "`python -m paper_2502_11018_gb300.build` (nvcc, sm_103a)")
+    L = ctypes.CDLL(LIB_PATH)
+    sig = {
+        "gv_tree_build": ([_vp, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
+        "gv_verify_attention_workspace": ([ctypes.POINTER(gv_attn_shape)], _sz),
+        "gv_verify_attention": ([ctypes.POINTER(gv_attn_shape)] + [_vp] * 12 + [_sz, _vp], _i),
+        "gv_lmhead_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
+        "gv_lmhead_select": ([_vp, _vp, _i, _i, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp,
+                              _sz, _vp], _i),
+        "gv_accept_workspace": ([_i, _i, _f], _sz),
+        "gv_accept": ([_i, _i, _i, _i, _f] + [_vp] * 12 + [_vp, _sz, _vp], _i),
+        "gv_kv_compact": ([_i] * 8 + [_vp] * 9 + [_vp], _i),
+        "gv_status_string": ([_i], ctypes.c_char_p),
+        "gv_last_error": ([], ctypes.c_char_p),
+        "gv_version": ([], _i),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(L, name)
+        fn.argtypes = args
+        fn.restype = res
+    _lib = L
+    return L
+
+
+def status_string(status):
+    return lib().gv_status_string(int(status)).decode()
+
+
+def last_error():
+    return lib().gv_last_error().decode()
+
+
+def _check(call, rc):
+    if rc != GV_OK:
+        raise GvError(call, rc, last_error())
+    return rc
+
+
+def _ptr(t, name):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name}: expected a torch tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name}: tensor must live on a CUDA device (no CPU path)")
+    if not t.is_contiguous():
+        raise ValueError(f"{name}: tensor must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def dtype_code(t):
+    if t.dtype == torch.bfloat16:
+        return GV_BF16
+    if t.dtype == torch.float32:
+        return GV_F32
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+# ------------------------------------------------------------------- calls --
+
+def gv_tree_build(parents, prefix_len, depth, pos, anc, seq_status, stream=None):
+    B, N = parents.shape
+    return _check("gv_tree_build", lib().gv_tree_build(
+        _ptr(parents, "parents"), _ptr(prefix_len, "prefix_len"), B, N, _ptr(depth, "depth"),
+        _ptr(pos, "pos"), _ptr(anc, "anc"), _ptr(seq_status, "seq_status"), _stream(stream)))
+
+
+def attn_shape(B, N, Hq, Hkv, d, S_max, rope_base, dt):
+    return gv_attn_shape(B, N, Hq, Hkv, d, S_max, float(rope_base), int(dt))
+
+
+def gv_verify_attention_workspace(shape):
+    return int(lib().gv_verify_attention_workspace(ctypes.byref(shape)))
+
+
+def gv_verify_attention(shape, q, k_new, v_new, cacheK, cacheV, prefix_len, pos, anc, treeK,
+                        treeV, out, workspace, stream=None):
+    return _check("gv_verify_attention", lib().gv_verify_attention(
+        ctypes.byref(shape), _ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"),
+        _ptr(cacheK, "cacheK"), _ptr(cacheV, "cacheV"), _ptr(prefix_len, "prefix_len"),
+        _ptr(pos, "pos"), _ptr(anc, "anc"), _ptr(treeK, "treeK"), _ptr(treeV, "treeV"),
+        _ptr(out, "out"), _ptr(workspace, "workspace"), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
+
+
+def gv_lmhead_workspace(rows, H, V, dt, mode, k=1):
+    return int(lib().gv_lmhead_workspace(rows, H, V, dt, mode, k))
+
+
+def gv_lmhead_select(h, W, mode, k, ids, vals, logits, row_max, row_lse, workspace, stream=None):
+    rows, H = h.shape
+    V = W.shape[0]
+    return _check("gv_lmhead_select", lib().gv_lmhead_select(
+        _ptr(h, "h"), _ptr(W, "W"), rows, H, V, dtype_code(h), mode, k, _ptr(ids, "ids"),
+        _ptr(vals, "vals"), _ptr(logits, "logits"), _ptr(row_max, "row_max"),
+        _ptr(row_lse, "row_lse"), _ptr(workspace, "workspace"),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def gv_accept_workspace(B, V, temperature):
+    return int(lib().gv_accept_workspace(B, V, float(temperature)))
+
+
+def gv_accept(D, temperature, tokens, anc, depth, choice, target_logits, draft_logits, u_acc,
+              u_res, path, accept_len, out_tokens, seq_status, workspace=None, V=0, stream=None):
+    B, N = tokens.shape
+    if target_logits is not None:
+        V = target_logits.shape[-1]
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    return _check("gv_accept", lib().gv_accept(
+        B, N, D, V, float(temperature), _ptr(tokens, "tokens"), _ptr(anc, "anc"),
+        _ptr(depth, "depth"), _ptr(choice, "choice"), _ptr(target_logits, "target_logits"),
+        _ptr(draft_logits, "draft_logits"), _ptr(u_acc, "u_acc"), _ptr(u_res, "u_res"),
+        _ptr(path, "path"), _ptr(accept_len, "accept_len"), _ptr(out_tokens, "out_tokens"),
+        _ptr(seq_status, "seq_status"), _ptr(workspace, "workspace"), ws_bytes, _stream(stream)))
+
+
+def gv_kv_compact(D, treeK, treeV, cacheK, cacheV, path, accept_len, prefix_len, new_len,
+                  seq_status, stream=None):
+    L, B, Hkv, N, d = treeK.shape
+    S_max = cacheK.shape[3]
+    return _check("gv_kv_compact", lib().gv_kv_compact(
+        L, B, N, D, Hkv, d, S_max, dtype_code(treeK), _ptr(treeK, "treeK"), _ptr(treeV, "treeV"),
+        _ptr(cacheK, "cacheK"), _ptr(cacheV, "cacheV"), _ptr(path, "path"),
+        _ptr(accept_len, "accept_len"), _ptr(prefix_len, "prefix_len"), _ptr(new_len, "new_len"),
+        _ptr(seq_status, "seq_status"), _stream(stream)))

@@ -1,0 +1,130 @@
+"""One whole verify step through the C ABI, with torch-allocated buffers.
+
+``VerifyStep`` owns the outputs and workspaces of one workload and issues the
+five calls of include/gv.h in order on one stream (GRIFFIN Section 3: draft,
+then one verify forward over every draft token, then accept):
+
+1. ``gv_tree_build``;
+2. ``gv_verify_attention`` for every layer (per-layer tree K/V scratch);
+3. ``gv_lmhead_select`` (argmax for T = 0, fp32 logits + LSE for T > 0);
+4. ``gv_accept``;
+5. ``gv_kv_compact`` into every layer's cache.
+
+No host synchronisation happens inside ``run``; it can be captured into a
+CUDA graph (``capture``/``replay``).
+"""
+
+import torch
+
+from . import gv
+from .inputs import StepInputs
+
+
+class VerifyStep:
+    def __init__(self, inp: StepInputs):
+        cfg = inp.cfg
+        self.inp = inp
+        self.cfg = cfg
+        dev = inp.q.device
+        if dev.type != "cuda":
+            raise ValueError("VerifyStep needs device tensors")
+        L, B, N, D, V, H = cfg["L"], cfg["B"], cfg["N"], cfg["D"], cfg["V"], cfg["H"]
+        Hq, Hkv, d, S_max = cfg["Hq"], cfg["Hkv"], cfg["d"], cfg["S_max"]
+        dt = inp.q.dtype
+        self.dt_code = gv.dtype_code(inp.q)
+        self.T = float(cfg.get("temperature", 0.0))
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.depth = torch.zeros(B, N, **i32)
+        self.pos = torch.zeros(B, N, **i32)
+        self.anc = torch.zeros(B, N, dtype=torch.int64, device=dev)
+        self.seq_status = torch.zeros(B, **i32)
+        self.treeK = torch.zeros(L, B, Hkv, N, d, dtype=dt, device=dev)
+        self.treeV = torch.zeros(L, B, Hkv, N, d, dtype=dt, device=dev)
+        self.attn_out = torch.zeros(L, B, N, Hq, d, dtype=dt, device=dev)
+        self.shape = gv.attn_shape(B, N, Hq, Hkv, d, S_max, cfg["rope_base"], self.dt_code)
+        ws = gv.gv_verify_attention_workspace(self.shape)
+        self.attn_ws = torch.empty(max(ws, 256), dtype=torch.uint8, device=dev)
+        rows = B * N
+        if self.T == 0.0:
+            self.lm_mode = gv.GV_SELECT_ARGMAX
+            self.ids = torch.zeros(rows, **i32)
+            self.vals = torch.zeros(rows, dtype=torch.float32, device=dev)
+            self.logits = self.row_max = self.row_lse = None
+        else:
+            self.lm_mode = gv.GV_SELECT_LOGITS
+            self.ids = self.vals = None
+            self.logits = torch.zeros(rows, V, dtype=torch.float32, device=dev)
+            self.row_max = torch.zeros(rows, dtype=torch.float32, device=dev)
+            self.row_lse = torch.zeros(rows, dtype=torch.float32, device=dev)
+        lw = gv.gv_lmhead_workspace(rows, H, V, self.dt_code, self.lm_mode, 1)
+        self.lm_ws = torch.empty(max(lw, 256), dtype=torch.uint8, device=dev)
+        self.path = torch.zeros(B, D + 1, **i32)
+        self.accept_len = torch.zeros(B, **i32)
+        self.out_tokens = torch.zeros(B, D + 1, **i32)
+        aw = gv.gv_accept_workspace(B, V, self.T)
+        self.acc_ws = torch.empty(max(aw, 256), dtype=torch.uint8, device=dev)
+        self.new_len = torch.zeros(B, **i32)
+        self.graph = None
+
+    # -------------------------------------------------------------- stages --
+    def tree(self, stream=None):
+        i = self.inp
+        gv.gv_tree_build(i.parents, i.prefix_len, self.depth, self.pos, self.anc, self.seq_status,
+                         stream)
+
+    def attention(self, layer, stream=None):
+        i = self.inp
+        gv.gv_verify_attention(self.shape, i.q[layer], i.k_new[layer], i.v_new[layer],
+                               i.cacheK[layer], i.cacheV[layer], i.prefix_len, self.pos, self.anc,
+                               self.treeK[layer], self.treeV[layer], self.attn_out[layer],
+                               self.attn_ws, stream)
+
+    def lmhead(self, stream=None):
+        i = self.inp
+        gv.gv_lmhead_select(i.h, i.W, self.lm_mode, 1, self.ids, self.vals, self.logits,
+                            self.row_max, self.row_lse, self.lm_ws, stream)
+
+    def accept(self, stream=None):
+        i = self.inp
+        B, N, V = self.cfg["B"], self.cfg["N"], self.cfg["V"]
+        if self.T == 0.0:
+            gv.gv_accept(self.cfg["D"], 0.0, i.tokens, self.anc, self.depth, self.ids, None, None,
+                         None, None, self.path, self.accept_len, self.out_tokens, self.seq_status,
+                         None, V, stream)
+        else:
+            gv.gv_accept(self.cfg["D"], self.T, i.tokens, self.anc, self.depth, None,
+                         self.logits.view(B, N, V), i.draft_logits, i.u_acc, i.u_res, self.path,
+                         self.accept_len, self.out_tokens, self.seq_status, self.acc_ws, V, stream)
+
+    def compact(self, stream=None):
+        i = self.inp
+        L = self.cfg["L"]
+        gv.gv_kv_compact(self.cfg["D"], self.treeK, self.treeV, i.cacheK[:L], i.cacheV[:L],
+                         self.path, self.accept_len, i.prefix_len, self.new_len, self.seq_status,
+                         stream)
+
+    def run(self, stream=None):
+        self.tree(stream)
+        for layer in range(self.cfg["L"]):
+            self.attention(layer, stream)
+        self.lmhead(stream)
+        self.accept(stream)
+        self.compact(stream)
+
+    # -------------------------------------------------------------- graphs --
+    def capture(self):
+        """Capture ``run`` into a CUDA graph (after one eager warm-up run)."""
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            self.run(s)
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.run(torch.cuda.current_stream())
+        self.graph = g
+        return g
+
+    def replay(self):
+        self.graph.replay()

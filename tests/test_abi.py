@@ -1,0 +1,67 @@
+"""The C-ABI library loads on a host without a GPU and exports every function
+include/gv.h declares; host-side argument checks answer without launching
+anything (no GPU is touched by these tests)."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2502_11018_gb300 import build, gv
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return gv.lib()
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "gv.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(gv_[a-z_]+)\s*\(", src)))
+
+
+def test_exports_match_header(lib):
+    names = declared_functions()
+    assert len(names) >= 11
+    for n in names:
+        assert hasattr(lib, n), n
+    assert sorted(gv.EXPORTS) == names
+
+
+def test_status_strings(lib):
+    assert gv.status_string(0) == "GV_OK"
+    assert gv.status_string(-2) == "GV_ERR_INVALID_TREE"
+    assert gv.status_string(-3) == "GV_ERR_CAPACITY"
+    assert gv.status_string(123) == "GV_ERR_UNKNOWN"
+    assert lib.gv_version() >= 100
+
+
+def test_host_side_validation(lib):
+    nul = None
+    # N outside 1..64 is rejected before any device work.
+    assert lib.gv_tree_build(nul, nul, 1, 65, nul, nul, nul, nul, nul) == gv.GV_ERR_INVALID_TREE
+    assert lib.gv_tree_build(nul, nul, 1, 0, nul, nul, nul, nul, nul) == gv.GV_ERR_INVALID_TREE
+    assert lib.gv_tree_build(nul, nul, 1, 4, nul, nul, nul, nul, nul) == gv.GV_ERR_ARG
+    assert "null" in gv.last_error()
+    shape = gv.attn_shape(1, 60, 32, 8, 96, 4224, 5e5, gv.GV_BF16)
+    assert lib.gv_verify_attention(ctypes.byref(shape), *([nul] * 12), 0, nul) == gv.GV_ERR_UNSUPPORTED
+    shape = gv.attn_shape(1, 60, 30, 8, 128, 4224, 5e5, gv.GV_BF16)
+    assert gv.gv_verify_attention_workspace(shape) == 0     # Hq not a multiple of Hkv
+    assert lib.gv_lmhead_select(nul, nul, 60, 4096, 1000, 0, 1, 17, *([nul] * 6), 0, nul) == gv.GV_ERR_ARG
+    assert lib.gv_accept(1, 60, 6, 0, -1.0, *([nul] * 12), nul, 0, nul) == gv.GV_ERR_ARG
+    assert lib.gv_kv_compact(1, 1, 60, 6, 8, 3, 100, 0, *([nul] * 9), nul) == gv.GV_ERR_ARG
+    assert "16-byte" in gv.last_error()
+
+
+def test_workspace_queries(lib):
+    shape = gv.attn_shape(1, 60, 32, 8, 128, 4224, 5e5, gv.GV_BF16)
+    assert gv.gv_verify_attention_workspace(shape) > 0
+    assert gv.gv_lmhead_workspace(60, 4096, 128256, gv.GV_BF16, gv.GV_SELECT_ARGMAX) > 0
+    assert gv.gv_lmhead_workspace(60, 4096, 128256, gv.GV_BF16, gv.GV_SELECT_TOPK, 0) == 0
+    assert gv.gv_accept_workspace(1, 32000, 0.0) == 0
+    assert gv.gv_accept_workspace(2, 32000, 1.0) >= 2 * 2 * 32000 * 4
