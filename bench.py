@@ -138,56 +138,124 @@ def event_time_ms(fn, iters, stream):
     return start.elapsed_time(end) / iters
 
 
-def cpu_baseline(cfg, seed, rank0):
-    """The float64 oracle timed on the host cores on a bounded sample."""
-    import numpy as np
+def oracle_step_sample(inp, cfg, ls, vs):
+    """Time the float64 oracle on a bounded sample of one step.
+
+    The sample is the whole step with attention on the first ``ls`` layers and
+    the LM head on the first ``vs`` vocabulary rows (acceptance then runs on
+    that slice).  Returns the full-step time extrapolated linearly in layers
+    and vocabulary rows, and the time the sample took.
+    """
     import oracle
-    cfg1 = dict(cfg)
-    frac_v = 16 if cfg["V"] >= 64000 else 4
-    Vs = cfg["V"] // frac_v
-    inp = inputs.make_step_inputs(dict(cfg, V=Vs), seed, device="cpu", layers=1)
+    from oracle.step import as_f64
+    T = cfg.get("temperature", 0.0)
+    P = as_f64(inp.prefix_len)
+    parents, tokens = as_f64(inp.parents), as_f64(inp.tokens)
     t0 = time.perf_counter()
-    oracle.verify_step(inp, layers=1, skip_compact=False)
-    t_sample = time.perf_counter() - t0
-    # Split the sample time into its attention and LM-head parts to extrapolate.
+    depth, pos, anc, st = oracle.tree_build(parents, P)
+    tk, tv = [], []
+    for layer in range(ls):
+        _, k_, v_ = oracle.tree_attention(as_f64(inp.q[layer]), as_f64(inp.k_new[layer]),
+                                          as_f64(inp.v_new[layer]), as_f64(inp.cacheK[layer]),
+                                          as_f64(inp.cacheV[layer]), P, pos, anc, cfg["rope_base"])
+        tk.append(k_)
+        tv.append(v_)
     t1 = time.perf_counter()
-    oracle.lmhead_logits(oracle.step.as_f64(inp.h), oracle.step.as_f64(inp.W))
-    t_lm = time.perf_counter() - t1
-    t_rest = max(t_sample - t_lm, 0.0)
-    est = cfg["L"] * t_rest + frac_v * t_lm
-    cores = os.cpu_count()
-    return {"value": 1.0 / est, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": (f"1 of {cfg['L']} layers (tree build, attention, accept, compaction) and "
-                       f"{Vs} of {cfg['V']} vocabulary rows of the LM head, float64 numpy; "
-                       f"full-step time extrapolated linearly ({est:.2f} s/step; sample took "
-                       f"{t_sample:.2f} s)"),
-            "seconds_per_step": est}
+    logits = oracle.lmhead_logits(as_f64(inp.h), as_f64(inp.W[:vs]))
+    t2 = time.perf_counter()
+    D = cfg["D"]
+    if T == 0.0:
+        choice, _ = oracle.select_argmax(logits)
+        path, alen, _, st = oracle.accept_greedy(parents, tokens, choice, D, st)
+    else:
+        B, N = parents.shape
+        path, alen, _, st, _ = oracle.accept_sampling(
+            parents, tokens % vs, logits.reshape(B, N, vs), as_f64(inp.draft_logits[..., :vs]),
+            as_f64(inp.u_acc), as_f64(inp.u_res), D, T, st)
+    import numpy as np
+    oracle.kv_compact(np.stack(tk), np.stack(tv), as_f64(inp.cacheK[:ls]), as_f64(inp.cacheV[:ls]),
+                      path, alen, P, st)
+    t3 = time.perf_counter()
+    est = (t1 - t0) * cfg["L"] / ls + (t2 - t1) * cfg["V"] / vs + (t3 - t2)
+    return est, t3 - t0
+
+
+def sample_desc(cfg, ls, vs, est, took):
+    return (f"float64 numpy oracle: whole step with attention on {ls} of {cfg['L']} layers and the "
+            f"LM head on {vs} of {cfg['V']} vocabulary rows; full-step time extrapolated linearly "
+            f"in layers and rows ({est:.2f} s/step; the sample took {took:.1f} s)")
+
+
+def host_inputs(cfg, seed, layers, dev_inp=None):
+    """Host copy of the first `layers` layers of the workload (from the device
+    inputs when given, else generated on the host)."""
+    if dev_inp is None:
+        return inputs.make_step_inputs(cfg, seed, device="cpu", layers=layers)
+    import dataclasses
+    kw = {}
+    for f in dataclasses.fields(dev_inp):
+        v = getattr(dev_inp, f.name)
+        if isinstance(v, torch.Tensor):
+            v = v[:layers] if f.name in ("q", "k_new", "v_new", "cacheK", "cacheV") else v
+            v = v.cpu()
+        kw[f.name] = v
+    return type(dev_inp)(**kw)
+
+
+def cpu_baseline(cfg, seed, dev_inp=None, budget_s=15.0):
+    """The oracle as it stands, timed on the host cores on a bounded sample
+    sized to roughly `budget_s` seconds."""
+    ls = min(cfg["L"], 4)
+    inp = host_inputs(cfg, seed, ls, dev_inp)
+    # Calibrate on one layer and an eighth of the vocabulary, then size the sample.
+    v8 = max(1, cfg["V"] // 8)
+    est1, took1 = oracle_step_sample(inp, cfg, 1, v8)
+    ls, vs = sample_size(cfg, est1, budget_s)
+    est, took = oracle_step_sample(inp, cfg, ls, vs)
+    return {"value": 1.0 / est, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": sample_desc(cfg, ls, vs, est, took), "seconds_per_step": est,
+            "layers": ls, "vocab_rows": vs}
+
+
+def sample_size(cfg, est_full, budget_s):
+    """Layers (<= 4) and vocabulary rows whose oracle time is about budget_s."""
+    frac = min(1.0, budget_s / max(est_full, 1e-6))
+    ls = max(1, min(4, int(round(cfg["L"] * frac))))
+    vs = max(256, min(cfg["V"], int(cfg["V"] * frac)))
+    return ls, vs
 
 
 def run_reference(args):
-    """The reference arm: the float64 oracle on the host cores."""
+    """The reference arm: the float64 oracle on the host cores, each step a
+    bounded sample of the workload sized so the whole run takes a few minutes."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     cfg = inputs.config(args.config)
-    res = None
+    inp = host_inputs(cfg, args.seed, min(cfg["L"], 4))
+    budget = max(0.5, min(20.0, 150.0 / max(1, args.steps + args.warmup)))
+    est1, _ = oracle_step_sample(inp, cfg, 1, max(1, cfg["V"] // 8))
+    ls, vs = sample_size(cfg, est1, budget)
     for _ in range(args.warmup):
-        cpu_baseline(cfg, 1000, True)
+        oracle_step_sample(inp, cfg, ls, vs)
     vals = []
     t0 = time.perf_counter()
-    for i in range(args.steps):
-        res = cpu_baseline(cfg, 1000 + i, True)
-        vals.append(res["seconds_per_step"])
+    took = 0.0
+    for _ in range(args.steps):
+        est, tk = oracle_step_sample(inp, cfg, ls, vs)
+        vals.append(est)
+        took += tk
     wall = time.perf_counter() - t0
     v = 1.0 / statistics.mean(vals)
+    desc = sample_desc(cfg, ls, vs, statistics.mean(vals), took / max(1, args.steps))
     line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1000.0 * statistics.mean(vals),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "impl": "reference",
+            "data": "synthetic (seeded random weights, caches and draft trees)", "impl": "reference",
             "config": {"workload": cfg["name"], "batch": cfg["B"], "layers": cfg["L"],
                        "prefix": list(cfg["P"]), "tree_nodes": cfg["N"], "vocab": cfg["V"]},
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": res["cores"], "kind": "oracle",
-                             "sample": res["sample"]},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": desc},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "wall_s": wall}
     print(json.dumps(line), flush=True)
@@ -203,6 +271,9 @@ def main():
     ap.add_argument("--seed", type=int, default=1000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention"],
+                    help="step: the benchmark; lmhead / attention: time that call alone "
+                         "(a small, self-contained launch sequence for profiler captures)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
 
@@ -227,6 +298,9 @@ def main():
 
     from paper_2502_11018_gb300.step import VerifyStep
     cfg = inputs.config(args.config)
+    if args.kernel != "step":
+        run_kernel_only(args, cfg, dev)
+        return
     inp = inputs.make_step_inputs(cfg, args.seed + rank, device=dev)
     step = VerifyStep(inp)
     step.capture()
@@ -288,12 +362,40 @@ def main():
         "clocks": clk,
     }
     if rank == 0 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = {k: v for k, v in cpu_baseline(cfg, args.seed, True).items()
-                                if k != "seconds_per_step"}
+        cb = cpu_baseline(cfg, args.seed, dev_inp=inp)
+        line["cpu_baseline"] = {k: cb[k] for k in ("value", "unit", "cores", "kind", "sample")}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
+
+
+def run_kernel_only(args, cfg, dev):
+    """Time one call of the verify path alone (one layer for attention), on a
+    workload whose inputs hold only that call's tensors."""
+    from paper_2502_11018_gb300.step import VerifyStep
+    layers = 1
+    inp = inputs.make_step_inputs(cfg, args.seed, device=dev, layers=layers)
+    step = VerifyStep(inp)
+    step.tree()
+    stream = torch.cuda.current_stream()
+    fn = step.lmhead if args.kernel == "lmhead" else (lambda: step.attention(0))
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    ms = event_time_ms(fn, args.steps, stream)
+    if args.kernel == "lmhead":
+        nbytes = lmhead_bytes(cfg)
+    else:
+        es = 2 if cfg["dtype"] == "bf16" else 4
+        B, N, Hq, Hkv, d = cfg["B"], cfg["N"], cfg["Hq"], cfg["Hkv"], cfg["d"]
+        nbytes = sum(2 * P * Hkv * d * es for P in cfg["P"])
+        nbytes += B * N * (2 * Hq + 4 * Hkv) * d * es
+    peaks = load_peaks()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    print(json.dumps({"kernel": args.kernel, "workload": cfg["name"], "ms_per_call": ms,
+                      "algorithmic_bytes": nbytes, "achieved_gbs": gbs,
+                      "frac_of_measured_hbm": gbs / peaks["hbm_gbs"]}), flush=True)
 
 
 def e2e_measure(step, inp, steps, stream):

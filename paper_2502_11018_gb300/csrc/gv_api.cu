@@ -68,8 +68,13 @@ int launch_kv_compact(int, int, int, int, int, int, int, int, const void*, const
 int launch_accept(int, int, int, int, float, const int32_t*, const uint64_t*, const int32_t*,
                   const int32_t*, const float*, const float*, const float*, const float*,
                   int32_t*, int32_t*, int32_t*, int32_t*, void*, cudaStream_t);
-int launch_lmhead_cc(const void*, const void*, int, int, int, int, int, int, float*,
-                     SelectPartials, int32_t*, float*, float*, float*, cudaStream_t);
+int launch_lmhead_cc(const float*, const float*, int, int, int, int, int, float*, SelectPartials,
+                     int32_t*, float*, float*, float*, cudaStream_t);
+int launch_lmhead_tc(const void*, const void*, int, int, int, int, int, float*, SelectPartials, int*,
+                     cudaStream_t);
+int launch_lmhead_merge(SelectPartials, int, int, int32_t*, float*, float*, float*, const int*,
+                        cudaStream_t);
+int lmhead_tc_grid(int slots_capacity);
 
 // ---------------------------------------------------------- attention plan --
 constexpr int KPS = 256;   // prefix keys per split
@@ -106,16 +111,17 @@ static AttnPlan attn_plan(const gv_attn_shape* s) {
 }
 
 // ------------------------------------------------------------ lmhead plan --
-constexpr int CC_TV = 64;
+constexpr int CC_TV = 64;        // vocabulary tile of the CUDA-core (fp32) kernel
+constexpr int TC_SLOTS = 256;    // partial slots of the tensor-core kernel (one per CTA)
 
 struct LmPlan {
-    size_t val, id, m, s, total;
+    size_t val, id, m, s, err, total;
     int slots, K;
 };
 
-static LmPlan lm_plan(int rows, int V, int mode, int k) {
+static LmPlan lm_plan(int rows, int V, int dt, int mode, int k) {
     LmPlan p{};
-    p.slots = (V + CC_TV - 1) / CC_TV;
+    p.slots = dt == GV_F32 ? (V + CC_TV - 1) / CC_TV : TC_SLOTS;
     p.K = mode == GV_SELECT_TOPK ? k : 1;
     const size_t n = (size_t)p.slots * rows;
     size_t off = 0;
@@ -127,6 +133,8 @@ static LmPlan lm_plan(int rows, int V, int mode, int k) {
     off += align256(n * sizeof(float));
     p.s = off;
     off += align256(n * sizeof(float));
+    p.err = off;
+    off += 256;
     p.total = off;
     return p;
 }
@@ -243,8 +251,8 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
 size_t gv_lmhead_workspace(int rows, int H, int V, int dt, int mode, int k) {
     if (rows < 1 || H < 1 || V < 1 || mode < 0 || mode > 2) return 0;
     if (mode == GV_SELECT_TOPK && (k < 1 || k > 16)) return 0;
-    (void)dt;
-    return lm_plan(rows, V, mode, k).total;
+    if (dt != GV_BF16 && dt != GV_F32) return 0;
+    return lm_plan(rows, V, dt, mode, k).total;
 }
 
 int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int dt, int mode, int k,
@@ -260,7 +268,11 @@ int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int d
         GV_CHECK_ARG(logits, "gv_lmhead_select: logits output is null");
     else
         GV_CHECK_ARG(ids, "gv_lmhead_select: ids output is null");
-    const LmPlan plan = lm_plan(rows, V, mode, k);
+    if (dt == GV_BF16)
+        GV_CHECK_ARG(H % 8 == 0, "gv_lmhead_select: bf16 rows need H %% 8 == 0 (16-byte rows), H=%d", H);
+    if (mode == GV_SELECT_LOGITS)
+        GV_CHECK_ARG(aligned16(logits), "gv_lmhead_select: logits not 16-byte aligned");
+    const LmPlan plan = lm_plan(rows, V, dt, mode, k);
     GV_CHECK_ARG(workspace && ((uintptr_t)workspace & 255u) == 0,
                  "gv_lmhead_select: workspace null or not 256-byte aligned");
     GV_CHECK_ARG(ws_bytes >= plan.total, "gv_lmhead_select: workspace %zu < %zu bytes", ws_bytes,
@@ -274,8 +286,16 @@ int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int d
     part.slots = plan.slots;
     part.rows = rows;
     part.K = plan.K;
-    return launch_lmhead_cc(h, W, rows, H, V, dt, mode, plan.K, logits, part, ids, vals, row_max,
-                            row_lse, as_stream(stream));
+    cudaStream_t st = as_stream(stream);
+    if (dt == GV_F32)
+        return launch_lmhead_cc(static_cast<const float*>(h), static_cast<const float*>(W), rows, H,
+                                V, mode, plan.K, logits, part, ids, vals, row_max, row_lse, st);
+    int* err = reinterpret_cast<int*>(ws + plan.err);
+    if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return check_launch("memset");
+    part.slots = lmhead_tc_grid(TC_SLOTS);
+    int rc = launch_lmhead_tc(h, W, rows, H, V, mode, plan.K, logits, part, err, st);
+    if (rc != GV_OK) return rc;
+    return launch_lmhead_merge(part, mode, plan.K, ids, vals, row_max, row_lse, err, st);
 }
 
 size_t gv_accept_workspace(int B, int V, float temperature) {

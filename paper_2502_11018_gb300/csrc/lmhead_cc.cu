@@ -131,13 +131,24 @@ lmhead_cc_kernel(const T* __restrict__ h, const T* __restrict__ W, int rows, int
 __global__ void __launch_bounds__(256)
 lmhead_merge_kernel(SelectPartials part, int mode, int K, int32_t* __restrict__ ids,
                     float* __restrict__ vals, float* __restrict__ row_max,
-                    float* __restrict__ row_lse) {
+                    float* __restrict__ row_lse, const int* __restrict__ err) {
     __shared__ float sv[8][16];
     __shared__ int si[8][16];
     __shared__ float red[33];
     const int r = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int rows = part.rows;
+    if (err != nullptr && *err != 0) {
+        // A bounded wait in the projection kernel gave up: no valid result.
+        if (mode == GV_SELECT_LOGITS) {
+            if (tid == 0 && row_max) row_max[r] = NAN;
+            if (tid == 0 && row_lse) row_lse[r] = NAN;
+        } else if (tid < K) {
+            ids[(size_t)r * K + tid] = -1;
+            if (vals) vals[(size_t)r * K + tid] = NAN;
+        }
+        return;
+    }
     if (mode == GV_SELECT_LOGITS) {
         float m = -INFINITY;
         for (int s = tid; s < part.slots; s += blockDim.x) m = fmaxf(m, part.m[(size_t)s * rows + r]);
@@ -222,22 +233,20 @@ lmhead_merge_kernel(SelectPartials part, int mode, int K, int32_t* __restrict__ 
     }
 }
 
-int launch_lmhead_cc(const void* h, const void* W, int rows, int H, int V, int dt, int mode,
-                     int K, float* logits, SelectPartials part, int32_t* ids, float* vals,
-                     float* row_max, float* row_lse, cudaStream_t st) {
-    dim3 grid((V + CC_TV - 1) / CC_TV, (rows + CC_TR - 1) / CC_TR);
-    if (dt == GV_F32)
-        lmhead_cc_kernel<float><<<grid, 256, 0, st>>>(static_cast<const float*>(h),
-                                                      static_cast<const float*>(W), rows, H, V,
-                                                      mode, K, logits, part);
-    else
-        lmhead_cc_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
-            static_cast<const __nv_bfloat16*>(h), static_cast<const __nv_bfloat16*>(W), rows, H, V,
-            mode, K, logits, part);
-    int rc = check_launch("lmhead_cc_kernel");
-    if (rc != GV_OK) return rc;
-    lmhead_merge_kernel<<<rows, 256, 0, st>>>(part, mode, K, ids, vals, row_max, row_lse);
+int launch_lmhead_merge(SelectPartials part, int mode, int K, int32_t* ids, float* vals,
+                        float* row_max, float* row_lse, const int* err, cudaStream_t st) {
+    lmhead_merge_kernel<<<part.rows, 256, 0, st>>>(part, mode, K, ids, vals, row_max, row_lse, err);
     return check_launch("lmhead_merge_kernel");
+}
+
+int launch_lmhead_cc(const float* h, const float* W, int rows, int H, int V, int mode, int K,
+                     float* logits, SelectPartials part, int32_t* ids, float* vals, float* row_max,
+                     float* row_lse, cudaStream_t st) {
+    dim3 grid((V + CC_TV - 1) / CC_TV, (rows + CC_TR - 1) / CC_TR);
+    lmhead_cc_kernel<float><<<grid, 256, 0, st>>>(h, W, rows, H, V, mode, K, logits, part);
+    const int rc = check_launch("lmhead_cc_kernel");
+    if (rc != GV_OK) return rc;
+    return launch_lmhead_merge(part, mode, K, ids, vals, row_max, row_lse, nullptr, st);
 }
 
 }  // namespace gv

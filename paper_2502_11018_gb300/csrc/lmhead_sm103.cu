@@ -1,0 +1,396 @@
+// gv_lmhead_select, bf16 tensor-core path for sm_103a.
+//
+// GRIFFIN Section 3 / Eq. 1: the LM head maps each draft node's final hidden
+// state to vocabulary scores; greedy verification (Section 5, T = 0) needs
+// only each node's argmax, so the scores are reduced on chip and never
+// written (the paper's closing remark on fusing kernels to cut memory
+// traffic).  The weight W[V][H] is read from HBM exactly once.
+//
+// One persistent CTA per SM walks vocabulary tiles of BN rows (round robin).
+// Per tile:  S[r][v] = sum_k h[r][k] W[v][k]  with the hidden rows on the MMA
+// M side (128 rows per M tile, rows beyond `rows` are zero-filled by TMA) and
+// BN vocabulary rows on the N side, both operands K-major with the 128-byte
+// swizzle, fp32 accumulators in tensor memory, double-buffered so the MMA of
+// tile i+1 overlaps the epilogue of tile i.
+//
+// Warp roles (192 threads):
+//   warp 0     one lane issues TMA loads of h and W k-blocks into a ring of
+//              shared-memory stages (W with an evict-first L2 hint, h with
+//              evict-last: h is re-read for every tile, W never);
+//   warp 1     allocates TMEM; one lane issues tcgen05.mma and commits each
+//              stage back to the producer and each finished tile to the
+//              epilogue;
+//   warps 2-5  one thread per M-tile row (TMEM lane): read the tile's scores
+//              32 columns at a time and fold them into a running per-row
+//              argmax / top-K / (max, sum exp) state; logits mode also stores
+//              the scores.
+// Each CTA finally writes its per-row partial result to the workspace, and
+// lmhead_merge_kernel combines the CTAs' partials.  Every wait is bounded.
+#include "gv_internal.cuh"
+#include "sm103.cuh"
+
+namespace gv {
+using namespace sm103;
+
+constexpr int LM_THREADS = 192;
+constexpr int LM_A_TILE_BYTES = 128 * 128;   // 128 rows x 64 bf16
+
+struct LmTcArgs {
+    int rows;          // rows of this launch (<= 256)
+    int row0;          // first global row of this launch (partials are indexed globally)
+    int V, BN, mt, n_tiles, kblocks, stages, stage_bytes;
+    uint32_t tmem_cols;
+    int mode, K;
+    float* logits;     // [rows_total][V] (mode LOGITS)
+    SelectPartials part;
+    int* err;
+};
+
+template <int KM>
+__global__ void __launch_bounds__(LM_THREADS, 1)
+lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_constant__ CUtensorMap tmap_w,
+                 LmTcArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~static_cast<uintptr_t>(1023));
+    uint8_t* stage_base = smem;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)a.stages * a.stage_bytes);
+    uint64_t* full = bars;
+    uint64_t* empty = bars + a.stages;
+    uint64_t* tfull = empty + a.stages;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < a.stages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int c = 0; c < 2; ++c) {
+            mbar_init(&tfull[c], 1);
+            mbar_init(&tempty[c], 4);
+        }
+        mbar_init(drain, 1);
+        *abort = 0;
+        fence_mbar_init();
+        prefetch_tmap(&tmap_h);
+        prefetch_tmap(&tmap_w);
+    }
+    if (warp == 1) tmem_alloc(tmem_holder, a.tmem_cols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+    const int acc_cols = a.mt * a.BN;
+
+    if (warp == 0) {
+        // ------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            const uint64_t pol_w = policy_evict_first();
+            const uint64_t pol_h = policy_evict_last();
+            const uint32_t tx = (uint32_t)(a.mt * LM_A_TILE_BYTES + a.BN * 128);
+            int s = 0;
+            uint32_t ph = 0;
+            int issued[8];   // parity of the last load issued into each stage, or -1
+            for (int q = 0; q < 8; ++q) issued[q] = -1;
+            for (int t = blockIdx.x; t < a.n_tiles; t += gridDim.x) {
+                for (int kb = 0; kb < a.kblocks; ++kb) {
+                    if (!mbar_wait(&empty[s], ph ^ 1u, abort)) goto producer_done;
+                    mbar_arrive_expect_tx(&full[s], tx);
+                    uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
+                    for (int m = 0; m < a.mt; ++m)
+                        tma_load_2d(st + m * LM_A_TILE_BYTES, &tmap_h, &full[s], kb * 64, m * 128, pol_h);
+                    tma_load_2d(st + a.mt * LM_A_TILE_BYTES, &tmap_w, &full[s], kb * 64, t * a.BN, pol_w);
+                    issued[s] = (int)ph;
+                    if (++s == a.stages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+            }
+        producer_done:
+            // On abort, let the copies this thread issued land before the CTA
+            // exits (each wait bounded on its own).
+            if (*abort) {
+                for (int q = 0; q < a.stages; ++q)
+                    if (issued[q] >= 0) mbar_wait_timeout_only(&full[q], (uint32_t)issued[q]);
+            }
+        }
+    } else if (warp == 1) {
+        // -------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(128, a.BN);
+            int s = 0;
+            uint32_t ph = 0;
+            int i = 0;
+            for (int t = blockIdx.x; t < a.n_tiles; t += gridDim.x, ++i) {
+                const int acc = i & 1;
+                if (!mbar_wait(&tempty[acc], ((uint32_t)(i >> 1) & 1u) ^ 1u, abort)) break;
+                tc_fence_after();
+                const uint32_t d_base = tmem + (uint32_t)(acc * acc_cols);
+                bool ok = true;
+                for (int kb = 0; kb < a.kblocks; ++kb) {
+                    if (!mbar_wait(&full[s], ph, abort)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
+                    const uint64_t bdesc = sdesc_kmajor_sw128(smem_u32(st + a.mt * LM_A_TILE_BYTES));
+                    for (int m = 0; m < a.mt; ++m) {
+                        const uint64_t adesc = sdesc_kmajor_sw128(smem_u32(st + m * LM_A_TILE_BYTES));
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk)
+                            mma_bf16(d_base + (uint32_t)(m * a.BN), adesc + 2u * kk, bdesc + 2u * kk,
+                                     idesc, (kb | kk) != 0);
+                    }
+                    mma_commit(&empty[s]);
+                    if (++s == a.stages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                mma_commit(&tfull[acc]);
+            }
+            // Every MMA this thread issued has completed once `drain` flips.
+            mma_commit(drain);
+            mbar_wait_timeout_only(drain, 0);
+        }
+    } else {
+        // ----------------------------------------------------------- epilogue
+        const int sub = warp & 3;                 // TMEM lane quarter this warp may access
+        const int row_in_tile = sub * 32 + lane;
+        float lv[2][KM];
+        int li[2][KM];
+        float rm[2], rs[2];
+#pragma unroll
+        for (int m = 0; m < 2; ++m) {
+            rm[m] = -INFINITY;
+            rs[m] = 0.f;
+#pragma unroll
+            for (int q = 0; q < KM; ++q) {
+                lv[m][q] = -INFINITY;
+                li[m][q] = INT32_MAX;
+            }
+        }
+        int i = 0;
+        for (int t = blockIdx.x; t < a.n_tiles; t += gridDim.x, ++i) {
+            const int acc = i & 1;
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(&tfull[acc], (uint32_t)(i >> 1) & 1u, abort);
+            ok = __shfl_sync(FULL, ok, 0);
+            if (!ok) break;
+            __syncwarp();
+            tc_fence_after();
+            const int v_tile = t * a.BN;
+#pragma unroll
+            for (int m = 0; m < 2; ++m) {
+                if (m >= a.mt) break;
+                const int r = a.row0 + m * 128 + row_in_tile;
+                const bool row_ok = m * 128 + row_in_tile < a.rows;
+                for (int c0 = 0; c0 < a.BN; c0 += 32) {
+                    uint32_t v[32];
+                    tmem_ld32(tmem + ((uint32_t)(sub * 32) << 16) +
+                                  (uint32_t)(acc * acc_cols + m * a.BN + c0), v);
+                    tmem_wait_ld();
+                    const int id0 = v_tile + c0;
+                    if (a.mode == GV_SELECT_LOGITS) {
+                        float cmax = -INFINITY;
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (id0 + j < a.V) cmax = fmaxf(cmax, __uint_as_float(v[j]));
+                        const float mnew = fmaxf(rm[m], cmax);
+                        float sum = 0.f;
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (id0 + j < a.V) sum += __expf(__uint_as_float(v[j]) - mnew);
+                        rs[m] = rs[m] * __expf(rm[m] - mnew) + sum;
+                        rm[m] = mnew;
+                        if (row_ok) {
+                            float* dst = a.logits + (size_t)r * a.V + id0;
+                            if (id0 + 32 <= a.V && (a.V & 3) == 0) {
+#pragma unroll
+                                for (int j = 0; j < 32; j += 4)
+                                    *reinterpret_cast<float4*>(dst + j) = make_float4(
+                                        __uint_as_float(v[j]), __uint_as_float(v[j + 1]),
+                                        __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
+                            } else {
+                                for (int j = 0; j < 32 && id0 + j < a.V; ++j) dst[j] = __uint_as_float(v[j]);
+                            }
+                        }
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) {
+                            float cv = __uint_as_float(v[j]);
+                            int ci = id0 + j;
+                            // ids only grow, so a strict '>' keeps the lower id on ties
+                            if (ci < a.V && cv > lv[m][KM - 1]) {
+#pragma unroll
+                                for (int q = 0; q < KM; ++q) {
+                                    if (cv > lv[m][q]) {
+                                        const float tv = lv[m][q];
+                                        const int ti = li[m][q];
+                                        lv[m][q] = cv;
+                                        li[m][q] = ci;
+                                        cv = tv;
+                                        ci = ti;
+                                    }
+                                }
+                            }
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+        }
+        // Per-CTA partial of every row this thread owns.
+        const int slot = blockIdx.x;
+#pragma unroll
+        for (int m = 0; m < 2; ++m) {
+            if (m >= a.mt) break;
+            if (m * 128 + row_in_tile >= a.rows) continue;
+            const int r = a.row0 + m * 128 + row_in_tile;
+            const size_t pr = (size_t)slot * a.part.rows + r;
+            if (a.mode == GV_SELECT_LOGITS) {
+                a.part.m[pr] = rm[m];
+                a.part.s[pr] = rm[m] == -INFINITY ? 0.f : rs[m];
+            } else {
+#pragma unroll
+                for (int q = 0; q < KM; ++q) {
+                    if (q < a.K) {
+                        a.part.val[pr * a.K + q] = lv[m][q];
+                        a.part.id[pr * a.K + q] = li[m][q];
+                    }
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, a.tmem_cols);
+    if (threadIdx.x == 0 && *abort) atomicExch(a.err, GV_ERR_TIMEOUT);
+}
+
+// ----------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn tensor_map_encoder() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [rows][cols] matrix, box [box_rows][64]
+// with the 128-byte swizzle.
+int make_map_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                uint64_t row_stride_bytes) {
+    EncodeTiledFn enc = tensor_map_encoder();
+    if (!enc) {
+        set_error("cuTensorMapEncodeTiled unavailable");
+        return GV_ERR_CUDA;
+    }
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {row_stride_bytes};
+    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        set_error("cuTensorMapEncodeTiled failed (%d)", (int)r);
+        return GV_ERR_CUDA;
+    }
+    return GV_OK;
+}
+
+// Vocabulary tile width: the multiple of 32 (<= 256 / mt) that minimises the
+// estimated time ceil(tiles / ctas) * (BN + per-tile overhead).
+int lmhead_pick_bn(int V, int mt, int ctas) {
+    int best = 64;
+    long best_cost = -1;
+    for (int bn = 64; bn * mt <= 256; bn += 32) {
+        const long tiles = (V + bn - 1) / bn;
+        const long waves = (tiles + ctas - 1) / ctas;
+        const long cost = waves * (bn + 16);
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best = bn;
+        }
+    }
+    return best;
+}
+
+// Number of CTAs (= partial slots) the tensor-core LM head launches with.
+int lmhead_tc_grid(int slots_capacity) {
+    const int c = sm_count();
+    return c < slots_capacity ? c : slots_capacity;
+}
+
+// Launches the kernel once per chunk of <= 256 rows; every launch uses the
+// same grid, and a CTA with no vocabulary tile writes neutral partials, so
+// the merge can read `grid` slots for every row.
+int launch_lmhead_tc(const void* h, const void* W, int rows, int H, int V, int mode, int K,
+                     float* logits, SelectPartials part, int* err, cudaStream_t st) {
+    const int grid = part.slots;
+    constexpr int SMEM_BUDGET = 220 * 1024;
+    for (int row0 = 0; row0 < rows; row0 += 256) {
+        const int r = rows - row0 < 256 ? rows - row0 : 256;
+        LmTcArgs a{};
+        a.rows = r;
+        a.row0 = row0;
+        a.V = V;
+        a.mt = (r + 127) / 128;
+        a.BN = lmhead_pick_bn(V, a.mt, grid);
+        a.n_tiles = (V + a.BN - 1) / a.BN;
+        a.kblocks = (H + 63) / 64;
+        a.stage_bytes = a.mt * LM_A_TILE_BYTES + a.BN * 128;
+        a.stages = (SMEM_BUDGET - 2048) / a.stage_bytes;
+        if (a.stages > 8) a.stages = 8;
+        const int cols = 2 * a.mt * a.BN;
+        a.tmem_cols = cols <= 32 ? 32 : cols <= 64 ? 64 : cols <= 128 ? 128 : cols <= 256 ? 256 : 512;
+        a.mode = mode;
+        a.K = K;
+        a.logits = logits;
+        a.part = part;
+        a.err = err;
+        CUtensorMap mh, mw;
+        const char* hb = static_cast<const char*>(h) + (size_t)row0 * H * 2;
+        int rc = make_map_2d(&mh, hb, (uint64_t)r, (uint64_t)H, 128, (uint64_t)H * 2);
+        if (rc != GV_OK) return rc;
+        rc = make_map_2d(&mw, W, (uint64_t)V, (uint64_t)H, (uint32_t)a.BN, (uint64_t)H * 2);
+        if (rc != GV_OK) return rc;
+        const size_t smem = 1024 + (size_t)a.stages * a.stage_bytes + 8 * (2 * a.stages + 5) + 16;
+        if (mode == GV_SELECT_TOPK) {
+            cudaFuncSetAttribute(lmhead_tc_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem);
+            lmhead_tc_kernel<16><<<grid, LM_THREADS, smem, st>>>(mh, mw, a);
+        } else {
+            cudaFuncSetAttribute(lmhead_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem);
+            lmhead_tc_kernel<1><<<grid, LM_THREADS, smem, st>>>(mh, mw, a);
+        }
+        rc = check_launch("lmhead_tc_kernel");
+        if (rc != GV_OK) return rc;
+    }
+    return GV_OK;
+}
+
+}  // namespace gv
