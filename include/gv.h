@@ -8,6 +8,7 @@
  * The calls below are that pass's data-parallel steps, in order:
  *
  *   gv_tree_build        positions and ancestor bitmasks from a parent array
+ *   gv_rope_table        RoPE cos/sin of every node (shared by all layers)
  *   gv_verify_attention  tree-masked attention of one layer (call per layer)
  *   gv_lmhead_select     LM-head projection fused with argmax / top-k / logits
  *   gv_accept            longest accepted root chain (T = 0) or recursive
@@ -75,7 +76,6 @@ typedef struct {
     int Hkv;          /* key/value heads (Hq % Hkv == 0; GQA when Hq > Hkv)   */
     int d;            /* head dimension (64 or 128)                           */
     int S_max;        /* cache rows per (sequence, KV head)                   */
-    float rope_base;  /* RoPE frequency base                                  */
     gv_dtype dt;      /* GV_BF16 (tensor-core path) or GV_F32                 */
 } gv_attn_shape;
 
@@ -101,13 +101,27 @@ int gv_tree_build(const int32_t* parents, const int32_t* prefix_len, int B, int 
                   void* stream);
 
 /*
+ * gv_rope_table -- RoPE cos/sin of every tree node, once per verify step.
+ * Every layer of the verify forward pass (Section 3) rotates the draft
+ * tokens' queries and keys at the same positions, so the angles are formed
+ * once: rope[b][i][j] = {cos(a), sin(a)} with a = pos[b][i] * rope_base^(-2j/d)
+ * computed in double and rounded to fp32, for j < d/2 (rotate-half RoPE).
+ *
+ *   pos   int32 [B][N]          from gv_tree_build
+ *   rope  fp32  [B][N][d/2][2]  out
+ * d must be even, 2 <= d <= 256.
+ */
+int gv_rope_table(const int32_t* pos, int B, int N, int d, float rope_base, float* rope,
+                  void* stream);
+
+/*
  * gv_verify_attention -- one attention layer of the verify forward pass.
  * Section 3: the target model verifies all draft tokens in one forward pass.
  * Draft node i of sequence b, query head h, attends to the cached prefix rows
  * 0..P_b-1 of KV head g = h / (Hq/Hkv) and to the tree nodes j with bit j of
  * anc[b][i] set, which equals causal attention over [prefix ; root chain of i].
- * RoPE (rotate-half, frequencies rope_base^(-2j/d), angles formed in double)
- * is applied to q and k_new at pos[b][i]; softmax scale is 1/sqrt(d).
+ * RoPE (rotate-half) is applied to q and k_new of node i with the cos/sin of
+ * rope[b][i] from gv_rope_table; softmax scale is 1/sqrt(d).
  *
  *   q          [B][N][Hq][d]      tree queries, unrotated           (dt)
  *   k_new      [B][N][Hkv][d]     tree keys, unrotated              (dt)
@@ -115,7 +129,8 @@ int gv_tree_build(const int32_t* parents, const int32_t* prefix_len, int B, int 
  *   cacheK/V   [B][Hkv][S_max][d] cache of this layer; rows < P_b are
  *                                 read (keys stored already rotated)  (dt)
  *   prefix_len int32 [B]          P_b <= S_max
- *   pos, anc   from gv_tree_build
+ *   rope       fp32 [B][N][d/2][2] from gv_rope_table
+ *   anc        uint64 [B][N]       from gv_tree_build
  *   treeK/V    [B][Hkv][N][d]     out: rotated tree keys / the values, the
  *                                 scratch gv_kv_compact reads        (dt)
  *   out        [B][N][Hq][d]      out: attention output              (dt)
@@ -127,7 +142,7 @@ int gv_tree_build(const int32_t* parents, const int32_t* prefix_len, int B, int 
 size_t gv_verify_attention_workspace(const gv_attn_shape* s);
 int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new,
                         const void* v_new, const void* cacheK, const void* cacheV,
-                        const int32_t* prefix_len, const int32_t* pos, const uint64_t* anc,
+                        const int32_t* prefix_len, const float* rope, const uint64_t* anc,
                         void* treeK, void* treeV, void* out,
                         void* workspace, size_t ws_bytes, void* stream);
 

@@ -11,7 +11,6 @@ struct AttnArgs {
     int G;            // Hq / Hkv
     int R;            // query rows per (sequence, KV head) = G * N
     int q_rows_pad;   // row stride of q_rot per (sequence, KV head)
-    float rope_base;
     float scale;      // 1 / sqrt(d)
     const void* q;
     const void* k_new;
@@ -19,22 +18,26 @@ struct AttnArgs {
     const void* cacheK;
     const void* cacheV;
     const int32_t* prefix_len;
-    const int32_t* pos;
+    const float* rope;   // [B][N][d/2][2] cos, sin per node (gv_rope_table)
     const unsigned long long* anc;
     void* treeK;
     void* treeV;
     void* out;
     // workspace pieces
     void* q_rot;      // [B*Hkv][q_rows_pad][d]  rotated queries (fp32 or bf16)
-    float* part_o;    // [B*Hkv][nsplit][R][d]
-    float* part_ml;   // [B*Hkv][nsplit][R][2]
-    int nsplit;       // prefix splits + 1 tree split
-    int kps;          // prefix keys per split
-    unsigned* counters;  // [B*Hkv] arrival tickets (tensor-core path)
+    float* part_o;    // [B*Hkv][nsplit][R][d]   per-split partial outputs
+    float* part_ml;   // [B*Hkv][nsplit][R][2] (m, l) on the CUDA-core path,
+                      // [B*Hkv][nsplit][R] log2-sum-exp on the tensor-core path
+    int nsplit;       // prefix splits + 1 tree split (CUDA-core path)
+    int kps;          // prefix keys per split (CUDA-core path)
+    int csize;        // CTAs per cluster, one cluster per (sequence, KV head) (tensor-core path)
 };
 
-template <typename T, typename TQ> int launch_rope_tree(const AttnArgs& a, cudaStream_t st);
-template <typename T> int launch_attn_combine(const AttnArgs& a, cudaStream_t st);
-template <typename T> int launch_attn_cc(const AttnArgs& a, cudaStream_t st);
+int launch_rope_table(const int32_t* pos, int B, int N, int d, float base, float* rope,
+                      cudaStream_t st);
+int launch_rope_tree_f32(const AttnArgs& a, cudaStream_t st);
+int launch_attn_combine_f32(const AttnArgs& a, cudaStream_t st);
+int launch_attn_cc_f32(const AttnArgs& a, cudaStream_t st);
+int launch_attn_tc(const AttnArgs& a, cudaStream_t st);
 
 }  // namespace gv

@@ -1,5 +1,7 @@
-// gv_verify_attention: RoPE prologue, split combine, and the CUDA-core
-// (fp32-operand) split-KV tree attention.
+// gv_rope_table, and the fp32 path of gv_verify_attention: RoPE prologue,
+// CUDA-core (FFMA) split-KV tree attention and split combine.  fp32 operands
+// stay on CUDA cores: tf32 tensor-core inputs would round them to 10-bit
+// mantissas, outside the 1e-4 relative tolerance fp32 results are held to.
 //
 // GRIFFIN Section 3: all draft tokens are verified in one target forward
 // pass; in each attention layer node i attends to the cached prefix and to
@@ -18,58 +20,78 @@
 
 namespace gv {
 
+// -------------------------------------------------------------- rope table --
+// One thread per (sequence, node, frequency j < d/2): the angle
+// pos * base^(-2j/d) is formed in double once per verify step and stored as
+// fp32 (cos, sin); every layer's RoPE reads this table.
+__global__ void __launch_bounds__(64)
+rope_table_kernel(const int32_t* __restrict__ pos, int B, int N, int d, double base,
+                  float2* __restrict__ rope) {
+    const int half = d >> 1;
+    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= B * N * half) return;
+    const int j = idx % half;
+    const int bi = idx / half;
+    const double theta = pow(base, -2.0 * (double)j / (double)d);
+    double sn, cs;
+    sincos((double)pos[bi] * theta, &sn, &cs);
+    rope[idx] = make_float2((float)cs, (float)sn);
+}
+
+int launch_rope_table(const int32_t* pos, int B, int N, int d, float base, float* rope,
+                      cudaStream_t st) {
+    const int total = B * N * (d / 2);
+    rope_table_kernel<<<(total + 63) / 64, 64, 0, st>>>(pos, B, N, d, (double)base,
+                                                        reinterpret_cast<float2*>(rope));
+    return check_launch("rope_table_kernel");
+}
+
 // ---------------------------------------------------------------- prologue --
-// One thread per (sequence, node, frequency j < d/2).  The angle
-// pos * base^(-2j/d) is formed in double and rounded to fp32 cos/sin once.
-template <typename T, typename TQ>
+// fp32 path: one thread per (sequence, node, frequency) rotates that
+// frequency's pair of every query head (into the q_rot workspace, grouped by
+// KV head) and of every key head (into the tree K scratch), and copies v.
 __global__ void __launch_bounds__(128)
-rope_tree_kernel(const T* __restrict__ q, const T* __restrict__ k_new, const T* __restrict__ v_new,
-                 const int32_t* __restrict__ pos, int B, int N, int Hq, int Hkv, int d,
-                 double rope_base, TQ* __restrict__ q_rot, T* __restrict__ treeK,
-                 T* __restrict__ treeV, int q_rows_pad) {
+rope_tree_f32_kernel(const float* __restrict__ q, const float* __restrict__ k_new,
+                     const float* __restrict__ v_new, const float2* __restrict__ rope, int B, int N,
+                     int Hq, int Hkv, int d, float* __restrict__ q_rot, float* __restrict__ treeK,
+                     float* __restrict__ treeV, int q_rows_pad) {
     const int half = d >> 1;
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= B * N * half) return;
     const int j = idx % half;
     const int i = (idx / half) % N;
     const int b = idx / (half * N);
-    const double theta = pow(rope_base, -2.0 * (double)j / (double)d);
-    double sn, cs;
-    sincos((double)pos[(size_t)b * N + i] * theta, &sn, &cs);
-    const float c = (float)cs, s = (float)sn;
+    const float2 r = rope[idx];
+    const float c = r.x, s = r.y;
     const int G = Hq / Hkv;
     for (int h = 0; h < Hq; ++h) {
         const size_t src = (((size_t)b * N + i) * Hq + h) * d;
-        const float x0 = to_f32(q[src + j]), x1 = to_f32(q[src + j + half]);
+        const float x0 = q[src + j], x1 = q[src + j + half];
         const int g = h / G, hl = h % G;
         const size_t dst = (((size_t)b * Hkv + g) * q_rows_pad + (size_t)hl * N + i) * d;
-        q_rot[dst + j] = from_f32<TQ>(x0 * c - x1 * s);
-        q_rot[dst + j + half] = from_f32<TQ>(x1 * c + x0 * s);
+        q_rot[dst + j] = x0 * c - x1 * s;
+        q_rot[dst + j + half] = x1 * c + x0 * s;
     }
     for (int g = 0; g < Hkv; ++g) {
         const size_t src = (((size_t)b * N + i) * Hkv + g) * d;
         const size_t dst = (((size_t)b * Hkv + g) * N + i) * d;
-        const float x0 = to_f32(k_new[src + j]), x1 = to_f32(k_new[src + j + half]);
-        treeK[dst + j] = from_f32<T>(x0 * c - x1 * s);
-        treeK[dst + j + half] = from_f32<T>(x1 * c + x0 * s);
+        const float x0 = k_new[src + j], x1 = k_new[src + j + half];
+        treeK[dst + j] = x0 * c - x1 * s;
+        treeK[dst + j + half] = x1 * c + x0 * s;
         treeV[dst + j] = v_new[src + j];
         treeV[dst + j + half] = v_new[src + j + half];
     }
 }
 
-template <typename T, typename TQ>
-int launch_rope_tree(const AttnArgs& a, cudaStream_t st) {
+int launch_rope_tree_f32(const AttnArgs& a, cudaStream_t st) {
     const int total = a.B * a.N * (a.d / 2);
-    rope_tree_kernel<T, TQ><<<(total + 127) / 128, 128, 0, st>>>(
-        static_cast<const T*>(a.q), static_cast<const T*>(a.k_new), static_cast<const T*>(a.v_new),
-        a.pos, a.B, a.N, a.Hq, a.Hkv, a.d, (double)a.rope_base, static_cast<TQ*>(a.q_rot),
-        static_cast<T*>(a.treeK), static_cast<T*>(a.treeV), a.q_rows_pad);
-    return check_launch("rope_tree_kernel");
+    rope_tree_f32_kernel<<<(total + 127) / 128, 128, 0, st>>>(
+        static_cast<const float*>(a.q), static_cast<const float*>(a.k_new),
+        static_cast<const float*>(a.v_new), reinterpret_cast<const float2*>(a.rope), a.B, a.N, a.Hq,
+        a.Hkv, a.d, static_cast<float*>(a.q_rot), static_cast<float*>(a.treeK),
+        static_cast<float*>(a.treeV), a.q_rows_pad);
+    return check_launch("rope_tree_f32_kernel");
 }
-
-template int launch_rope_tree<float, float>(const AttnArgs&, cudaStream_t);
-template int launch_rope_tree<__nv_bfloat16, float>(const AttnArgs&, cudaStream_t);
-template int launch_rope_tree<__nv_bfloat16, __nv_bfloat16>(const AttnArgs&, cudaStream_t);
 
 // ----------------------------------------------------------------- combine --
 // One warp per output row (b, node, head): out = sum_s e^{m_s - M} o_s / sum_s e^{m_s - M} l_s.
@@ -103,21 +125,18 @@ attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ 
     for (int j = 0; j < D / 32; ++j) o[lane + 32 * j] = from_f32<T>(acc[j] * inv);
 }
 
-template <typename T>
-int launch_attn_combine(const AttnArgs& a, cudaStream_t st) {
+int launch_attn_combine_f32(const AttnArgs& a, cudaStream_t st) {
     const int warps = a.B * a.N * a.Hq;
     const int blocks = (warps * 32 + 255) / 256;
+    float* out = static_cast<float*>(a.out);
     if (a.d == 128)
-        attn_combine_kernel<T, 128><<<blocks, 256, 0, st>>>(a.part_o, a.part_ml, a.B, a.N, a.Hq,
-                                                            a.Hkv, a.nsplit, a.R, static_cast<T*>(a.out));
+        attn_combine_kernel<float, 128><<<blocks, 256, 0, st>>>(a.part_o, a.part_ml, a.B, a.N, a.Hq,
+                                                                a.Hkv, a.nsplit, a.R, out);
     else
-        attn_combine_kernel<T, 64><<<blocks, 256, 0, st>>>(a.part_o, a.part_ml, a.B, a.N, a.Hq,
-                                                           a.Hkv, a.nsplit, a.R, static_cast<T*>(a.out));
+        attn_combine_kernel<float, 64><<<blocks, 256, 0, st>>>(a.part_o, a.part_ml, a.B, a.N, a.Hq,
+                                                               a.Hkv, a.nsplit, a.R, out);
     return check_launch("attn_combine_kernel");
 }
-
-template int launch_attn_combine<float>(const AttnArgs&, cudaStream_t);
-template int launch_attn_combine<__nv_bfloat16>(const AttnArgs&, cudaStream_t);
 
 // -------------------------------------------------------- CUDA-core splits --
 // Block = (sequence, KV head, 64-row chunk of the query rows) x split.
@@ -250,12 +269,8 @@ static int launch_cc(const AttnArgs& a, cudaStream_t st) {
     return check_launch("attn_cc_kernel");
 }
 
-template <typename T>
-int launch_attn_cc(const AttnArgs& a, cudaStream_t st) {
-    return a.d == 128 ? launch_cc<T, 128>(a, st) : launch_cc<T, 64>(a, st);
+int launch_attn_cc_f32(const AttnArgs& a, cudaStream_t st) {
+    return a.d == 128 ? launch_cc<float, 128>(a, st) : launch_cc<float, 64>(a, st);
 }
-
-template int launch_attn_cc<float>(const AttnArgs&, cudaStream_t);
-template int launch_attn_cc<__nv_bfloat16>(const AttnArgs&, cudaStream_t);
 
 }  // namespace gv

@@ -1,0 +1,717 @@
+// gv_verify_attention, bf16 tensor-core path for sm_103a.
+//
+// GRIFFIN Section 3: every draft token is verified in one target forward
+// pass; in each attention layer tree node i attends to the cached prefix and
+// to the nodes on its own root chain (Section 4.1: rejecting a token drops
+// its subtree, so the ancestor set is exactly what node i may see).
+//
+// One thread-block cluster of C CTAs per (sequence b, KV head g).  The keys
+// of (b, g) are cut into 64-key blocks: ceil(P_b / 64) prefix blocks and one
+// tree block (the N <= 64 tree keys, masked per query row by its ancestor
+// bitmask).  CTA `rank` of the cluster takes blocks rank, rank + C, ...; the
+// CTA that owns the tree block runs it first.  All G * N query rows of KV
+// head g share every K/V block; row r = i * G + hl holds node i and query
+// head g * G + hl, and 128 rows form one MMA M tile (MT = 1 or 2 tiles).
+//
+// Per block j of a CTA:
+//   S_j = Q K_j^T          tcgen05.mma, Q and K K-major 128B-swizzled in smem,
+//                          fp32 S in TMEM (two buffers: S_{j+1} overlaps the
+//                          softmax of block j)
+//   softmax                one thread per query row reads its S row from TMEM,
+//                          masks with a branch-free 64-bit validity mask
+//                          (prefix end, or the row's ancestor bitmask), keeps a
+//                          running max in the log2 domain and rescales O only
+//                          when the max grew by more than 2^8 (exact: O and l
+//                          always share one max), writes P = exp2(s - m) as
+//                          bf16 to one of two smem buffers
+//   O += P_j V_j           tcgen05.mma, P K-major, V MN-major (d contiguous)
+// Each CTA then leaves o = O / l and lse = m + log2(l) of its rows in its own
+// shared memory; after a cluster barrier every CTA reduces a 1/C share of the
+// rows across the cluster through distributed shared memory and writes the
+// final bf16 output.  No partial result goes through global memory.
+//
+// Warp roles: warp 0 issues the TMA loads (K/V blocks, raw Q tiles); warp 1
+// owns TMEM and issues the MMAs; warps 2.. (4 per M tile) rotate Q in place
+// (RoPE from the per-step table), build the tree K/V tile, and run the
+// softmax and the epilogue; all warps share the cluster reduction.
+//
+// Launch: cluster launch with programmatic dependent launch.  Before
+// griddepcontrol.wait a CTA only initialises barriers and TMEM and starts
+// streaming its K/V cache blocks (the cache is not written by the kernels it
+// overlaps); queries, RoPE table, ancestor masks and the output are touched
+// after it.  Every mbarrier wait is bounded; a CTA that gives up marks its
+// rows' lse NaN, which turns the affected outputs into NaN, and still
+// reaches both cluster barriers.
+#include "gv_internal.cuh"
+#include "attention.cuh"
+#include "sm103.cuh"
+
+namespace gv {
+using namespace sm103;
+
+constexpr int AT_BK = 64;                   // keys per block
+constexpr int AT_QHALF = 128 * 128;         // one M tile, 64 of the 128 d columns (bf16)
+constexpr int AT_QTILE = 2 * AT_QHALF;      // one M tile of Q
+constexpr int AT_PTILE = 128 * 128;         // one M tile of P: 128 rows x 64 keys bf16
+constexpr int AT_KV_HALF = AT_BK * 128;     // 64 keys x 64 d bf16 (one swizzle sub-tile)
+constexpr int AT_STAGE = 4 * AT_KV_HALF;    // K (2 halves) + V (2 halves)
+constexpr int AT_RED_STRIDE = 512 + 16;     // bytes per fp32 row of the reduction buffer
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+__device__ __forceinline__ void grid_dep_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dep_launch() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Shared::cluster address of the same smem location in CTA `rank`.
+__device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ float4 ld_cluster_v4(uint32_t addr) {
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ float fast_exp2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+// Byte offset of 16-byte chunk c of row r inside a 128B-swizzled tile whose
+// rows are 128 bytes apart (the layout TMA writes and tcgen05 reads).
+__device__ __forceinline__ uint32_t sw128(int r, int c) {
+    return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+__device__ __forceinline__ float2 unpack_bf16(uint32_t u) {
+    __nv_bfloat162 v = *reinterpret_cast<__nv_bfloat162*>(&u);
+    return __bfloat1622float2(v);
+}
+
+// Rotate 8 consecutive elements of the low half (lo) and the matching 8 of the
+// high half (hi) with 8 (cos, sin) pairs held as 4 float4; results as bf16.
+__device__ __forceinline__ void rope8(const uint4& lo, const uint4& hi, const float4* cs, uint4& olo,
+                                      uint4& ohi) {
+    const uint32_t* l = reinterpret_cast<const uint32_t*>(&lo);
+    const uint32_t* h = reinterpret_cast<const uint32_t*>(&hi);
+    uint32_t* ol = reinterpret_cast<uint32_t*>(&olo);
+    uint32_t* oh = reinterpret_cast<uint32_t*>(&ohi);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float2 a = unpack_bf16(l[e]);
+        const float2 b = unpack_bf16(h[e]);
+        const float4 c = cs[e];   // (cos, sin) of element 2e, then of 2e+1
+        ol[e] = pack_bf16(a.x * c.x - b.x * c.y, a.y * c.z - b.y * c.w);
+        oh[e] = pack_bf16(b.x * c.x + a.x * c.y, b.y * c.z + a.y * c.w);
+    }
+}
+
+template <int MT>
+__global__ void __launch_bounds__(64 + 128 * MT, 1)
+attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
+               const __grid_constant__ CUtensorMap map_q, AttnArgs a) {
+    constexpr int NSM = 128 * MT;            // softmax threads
+    constexpr int NTH = 64 + NSM;            // all threads
+    constexpr int ST = MT == 1 ? 4 : 3;      // K/V stages
+    const int C = a.csize;
+    const int rank = (int)cluster_rank();
+    const int bg = blockIdx.x / C;
+    const int b = bg / a.Hkv, g = bg % a.Hkv;
+    // prefix_len is a step input written before the previous kernel in the
+    // stream started, so it may be read before griddepcontrol.wait.
+    const int P = min(max(a.prefix_len[b], 0), a.S_max);
+    const int nb_pre = (P + AT_BK - 1) / AT_BK;
+    const int T = nb_pre + 1;                            // + the tree block
+    const int nblk = T > rank ? (T - 1 - rank) / C + 1 : 0;
+    const bool has_tree = nb_pre % C == rank;
+    const int nb_per_tile = 128 / a.G;                   // nodes per M tile
+    // Prefix block index of this CTA's j-th block (the tree block, if owned,
+    // is j = 0 and returns -1).
+    auto prefix_block = [&](int j) -> int {
+        if (has_tree) return j == 0 ? -1 : rank + C * (j - 1);
+        return rank + C * j;
+    };
+
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~static_cast<uintptr_t>(1023));
+    uint8_t* sQ = smem;                                  // MT x 32 KB
+    uint8_t* sP = sQ + MT * AT_QTILE;                    // 2 buffers x MT x 16 KB
+    uint8_t* sKV = sP + 2 * MT * AT_PTILE;               // ST x 32 KB
+    uint8_t* sRed = sP;                                  // reduction rows (after the last PV)
+    float* sLse = reinterpret_cast<float*>(sRed + MT * 128 * AT_RED_STRIDE);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + ST * AT_STAGE);
+    uint64_t* kv_full = bars;
+    uint64_t* kv_empty = kv_full + ST;
+    uint64_t* s_full = kv_empty + ST;
+    uint64_t* s_free = s_full + 2;
+    uint64_t* p_full = s_free + 2;
+    uint64_t* o_done = p_full + 2;
+    uint64_t* q_raw = o_done + 2;
+    uint64_t* q_full = q_raw + 1;
+    uint64_t* drain = q_full + 1;
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < ST; ++s) {
+            mbar_init(&kv_full[s], 1);
+            mbar_init(&kv_empty[s], 1);
+        }
+        for (int c = 0; c < 2; ++c) {
+            mbar_init(&s_full[c], 1);
+            mbar_init(&s_free[c], 4 * MT);
+            mbar_init(&p_full[c], 4 * MT);
+            mbar_init(&o_done[c], 1);
+        }
+        mbar_init(q_raw, 1);
+        mbar_init(q_full, 4 * MT);
+        mbar_init(drain, 1);
+        *abort = 0;
+        fence_mbar_init();
+        if (nblk > 0) {
+            prefetch_tmap(&map_q);
+            prefetch_tmap(&map_k);
+            prefetch_tmap(&map_v);
+        }
+    }
+    if (warp == 1) tmem_alloc(tmem_holder, 256 * MT);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+    grid_dep_launch();
+
+    // Row owned by a softmax thread (valid for warps >= 2).
+    const int t = threadIdx.x - 64;
+    const int m = (warp - 2) >> 2;                       // M tile of this warp
+    const int sub = warp & 3;                            // TMEM lane quarter
+    const int row = sub * 32 + lane;                     // row inside the M tile
+    const int node = m * nb_per_tile + row / a.G;        // tree node of this row
+    const bool row_ok = warp >= 2 && node < a.N;
+    const int grow = m * 128 + row;                      // = node * G + head in group
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+
+    if (nblk > 0) {
+        if (warp == 0) {
+            // ----------------------------------------------------- TMA producer
+            if (lane == 0) {
+                const uint64_t pol_kv = policy_evict_first();
+                const uint64_t pol_q = policy_evict_last();
+                int issued[ST];
+                for (int q = 0; q < ST; ++q) issued[q] = -1;
+                bool q_issued = false;
+                auto issue_q = [&]() {
+                    grid_dep_wait();
+                    mbar_arrive_expect_tx(q_raw, MT * AT_QTILE);
+                    for (int mm = 0; mm < MT; ++mm) {
+                        const int z = b * a.N + mm * nb_per_tile;
+                        tma_load_3d(sQ + mm * AT_QTILE, &map_q, q_raw, 0, g * a.G, z, pol_q);
+                        tma_load_3d(sQ + mm * AT_QTILE + AT_QHALF, &map_q, q_raw, 64, g * a.G, z, pol_q);
+                    }
+                    q_issued = true;
+                };
+                for (int j = 0; j < nblk; ++j) {
+                    const int s = j % ST;
+                    const uint32_t ph = (uint32_t)(j / ST) & 1u;
+                    if (j == ST) issue_q();          // the first ST blocks are in flight
+                    const int k = prefix_block(j);
+                    if (k < 0) continue;             // tree block: built by the softmax warps
+                    if (!mbar_wait(&kv_empty[s], ph ^ 1u, abort)) break;
+                    mbar_arrive_expect_tx(&kv_full[s], AT_STAGE);
+                    uint8_t* st = sKV + s * AT_STAGE;
+                    const int y = bg * a.S_max + k * AT_BK;
+                    tma_load_2d(st, &map_k, &kv_full[s], 0, y, pol_kv);
+                    tma_load_2d(st + AT_KV_HALF, &map_k, &kv_full[s], 64, y, pol_kv);
+                    tma_load_2d(st + 2 * AT_KV_HALF, &map_v, &kv_full[s], 0, y, pol_kv);
+                    tma_load_2d(st + 3 * AT_KV_HALF, &map_v, &kv_full[s], 64, y, pol_kv);
+                    issued[s] = (int)ph;
+                }
+                if (!q_issued && !*abort) issue_q();
+                if (*abort) {
+                    for (int q = 0; q < ST; ++q)
+                        if (issued[q] >= 0) mbar_wait_timeout_only(&kv_full[q], (uint32_t)issued[q]);
+                    if (q_issued) mbar_wait_timeout_only(q_raw, 0);
+                }
+            }
+        } else if (warp == 1) {
+            // ------------------------------------------------------- MMA issuer
+            if (lane == 0) {
+                const uint32_t idesc_s = idesc_bf16(128, AT_BK);
+                const uint32_t idesc_o = idesc_bf16(128, 128, /*b_mn_major=*/true);
+                bool mok = mbar_wait(q_full, 0, abort);
+                tc_fence_after();
+                auto issue_pv = [&](int jj) -> bool {
+                    const int pb = jj & 1;
+                    if (!mbar_wait(&p_full[pb], (uint32_t)(jj >> 1) & 1u, abort)) return false;
+                    tc_fence_after();
+                    const int sp = jj % ST;
+                    // V as the MN-major B operand: rows = keys (128 B apart, SBO =
+                    // 1 KB per 8 keys), the two 64-wide halves of d LBO = 8 KB apart.
+                    uint64_t vdesc = sdesc_kmajor_sw128(smem_u32(sKV + sp * AT_STAGE + 2 * AT_KV_HALF));
+                    vdesc = (vdesc & ~(0x3FFFull << 16)) | ((uint64_t)(AT_KV_HALF >> 4) << 16);
+#pragma unroll
+                    for (int mm = 0; mm < MT; ++mm) {
+                        const uint64_t pdesc =
+                            sdesc_kmajor_sw128(smem_u32(sP + (pb * MT + mm) * AT_PTILE));
+#pragma unroll
+                        for (int kk = 0; kk < AT_BK / 16; ++kk)
+                            mma_bf16(tmem + (uint32_t)(mm * 256 + 128), pdesc + 2u * kk,
+                                     vdesc + (uint64_t)(kk * 128), idesc_o, (jj | kk) != 0);
+                    }
+                    mma_commit(&kv_empty[sp]);
+                    mma_commit(&o_done[pb]);
+                    return true;
+                };
+                for (int j = 0; mok && j < nblk; ++j) {
+                    const int s = j % ST, buf = j & 1;
+                    if (!mbar_wait(&kv_full[s], (uint32_t)(j / ST) & 1u, abort) ||
+                        !mbar_wait(&s_free[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort)) {
+                        mok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t kbase = smem_u32(sKV + s * AT_STAGE);
+#pragma unroll
+                    for (int mm = 0; mm < MT; ++mm) {
+#pragma unroll
+                        for (int kb = 0; kb < 2; ++kb) {
+                            const uint64_t qdesc =
+                                sdesc_kmajor_sw128(smem_u32(sQ + mm * AT_QTILE + kb * AT_QHALF));
+                            const uint64_t kdesc = sdesc_kmajor_sw128(kbase + kb * AT_KV_HALF);
+#pragma unroll
+                            for (int kk = 0; kk < 4; ++kk)
+                                mma_bf16(tmem + (uint32_t)(mm * 256 + buf * AT_BK), qdesc + 2u * kk,
+                                         kdesc + 2u * kk, idesc_s, (kb | kk) != 0);
+                        }
+                    }
+                    mma_commit(&s_full[buf]);
+                    if (j >= 1 && !issue_pv(j - 1)) {
+                        mok = false;
+                        break;
+                    }
+                }
+                if (mok) issue_pv(nblk - 1);
+                mma_commit(drain);
+                mbar_wait_timeout_only(drain, 0);
+            }
+        } else {
+            // -------------------------- Q rotation, tree tile, softmax, epilogue
+            grid_dep_wait();
+            const float4* rope_b = reinterpret_cast<const float4*>(a.rope) + (size_t)b * a.N * 32;
+            if (has_tree) {
+                // Rotated tree keys and the values into stage 0 (and into the
+                // tree K/V scratch in global memory for gv_kv_compact).
+                uint8_t* st = sKV;
+                for (int e = t; e < AT_BK * 8; e += NSM) {
+                    const int j = e >> 3, c = e & 7;
+                    uint4 klo = make_uint4(0, 0, 0, 0), khi = klo, vlo = klo, vhi = klo;
+                    if (j < a.N) {
+                        const size_t src = (((size_t)b * a.N + j) * a.Hkv + g) * 16;
+                        const uint4* kr = reinterpret_cast<const uint4*>(a.k_new) + src;
+                        const uint4* vr = reinterpret_cast<const uint4*>(a.v_new) + src;
+                        const uint4 k0 = __ldg(kr + c), k1 = __ldg(kr + 8 + c);
+                        vlo = __ldg(vr + c);
+                        vhi = __ldg(vr + 8 + c);
+                        float4 cs[4];
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) cs[q] = __ldg(rope_b + (size_t)j * 32 + c * 4 + q);
+                        rope8(k0, k1, cs, klo, khi);
+                        uint4* tk = reinterpret_cast<uint4*>(a.treeK) + ((size_t)bg * a.N + j) * 16;
+                        uint4* tv = reinterpret_cast<uint4*>(a.treeV) + ((size_t)bg * a.N + j) * 16;
+                        tk[c] = klo;
+                        tk[8 + c] = khi;
+                        tv[c] = vlo;
+                        tv[8 + c] = vhi;
+                    }
+                    *reinterpret_cast<uint4*>(st + sw128(j, c)) = klo;
+                    *reinterpret_cast<uint4*>(st + AT_KV_HALF + sw128(j, c)) = khi;
+                    *reinterpret_cast<uint4*>(st + 2 * AT_KV_HALF + sw128(j, c)) = vlo;
+                    *reinterpret_cast<uint4*>(st + 3 * AT_KV_HALF + sw128(j, c)) = vhi;
+                }
+                fence_proxy_async_smem();
+                named_bar_sync(1, NSM);
+                if (t == 0) mbar_arrive(&kv_full[0]);
+            }
+            // RoPE of this thread's Q row, in place once the raw tile has landed.
+            {
+                float4 cs[32];
+                if (row_ok) {
+#pragma unroll
+                    for (int q = 0; q < 32; ++q) cs[q] = __ldg(rope_b + (size_t)node * 32 + q);
+                }
+                int w = 1;
+                if (lane == 0) w = mbar_wait(q_raw, 0, abort);
+                w = __shfl_sync(FULL, w, 0);
+                uint8_t* qt = sQ + m * AT_QTILE;
+                if (w) {
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        uint4* plo = reinterpret_cast<uint4*>(qt + sw128(row, c));
+                        uint4* phi = reinterpret_cast<uint4*>(qt + AT_QHALF + sw128(row, c));
+                        uint4 olo = make_uint4(0, 0, 0, 0), ohi = olo;
+                        if (row_ok) rope8(*plo, *phi, cs + 4 * c, olo, ohi);
+                        *plo = olo;
+                        *phi = ohi;
+                    }
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(q_full);
+            }
+            const unsigned long long anc_row =
+                (has_tree && row_ok) ? __ldg(a.anc + (size_t)b * a.N + node) : 0ull;
+            const float sl2 = a.scale * 1.4426950408889634f;     // scale * log2(e)
+            for (int j = 0; j < nblk; ++j) {
+                const int buf = j & 1, s = j % ST;
+                int w = 1;
+                if (lane == 0) w = mbar_wait(&s_full[buf], (uint32_t)(j >> 1) & 1u, abort);
+                if (!__shfl_sync(FULL, w, 0)) {
+                    ok = false;
+                    break;
+                }
+                __syncwarp();
+                tc_fence_after();
+                uint32_t sv[64];
+                const uint32_t scol =
+                    tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(m * 256 + buf * AT_BK);
+                tmem_ld32(scol, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+                tmem_ld32(scol + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+                tmem_wait_ld();
+#pragma unroll
+                for (int c = 0; c < 64; ++c) asm volatile("" : "+r"(sv[c]));  // uses stay after the wait
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&s_free[buf]);
+                // Branch-free validity mask of the block's 64 keys for this row.
+                const int k = prefix_block(j);
+                uint32_t vlo, vhi;
+                int nvalid = AT_BK;
+                if (k < 0) {
+                    vlo = (uint32_t)anc_row;
+                    vhi = (uint32_t)(anc_row >> 32);
+                } else {
+                    nvalid = min(AT_BK, P - k * AT_BK);
+                    vlo = nvalid >= 32 ? 0xFFFFFFFFu : ((1u << nvalid) - 1u);
+                    vhi = nvalid >= 64 ? 0xFFFFFFFFu : (nvalid > 32 ? ((1u << (nvalid - 32)) - 1u) : 0u);
+                }
+                float mx = -INFINITY;
+#pragma unroll
+                for (int c = 0; c < 64; ++c) {
+                    const uint32_t bit = c < 32 ? (vlo >> c) & 1u : (vhi >> (c - 32)) & 1u;
+                    const float x = bit ? __uint_as_float(sv[c]) * sl2 : -INFINITY;
+                    sv[c] = __float_as_uint(x);
+                    mx = fmaxf(mx, x);
+                }
+                const float m_new = fmaxf(m_used, mx);
+                const bool need = m_new > m_used + 8.0f;     // also true the first time
+                float alpha = 1.0f;
+                if (need) {
+                    alpha = fast_exp2(m_used - m_new);       // 0 when m_used = -inf
+                    m_used = m_new;
+                }
+                float ps[4] = {0.f, 0.f, 0.f, 0.f};
+                uint32_t pk[32];
+#pragma unroll
+                for (int c = 0; c < 32; ++c) {
+                    // masked keys give 0 (also for a padding row whose max is -inf)
+                    const float x0 = __uint_as_float(sv[2 * c]), x1 = __uint_as_float(sv[2 * c + 1]);
+                    const float p0 = x0 == -INFINITY ? 0.f : fast_exp2(x0 - m_used);
+                    const float p1 = x1 == -INFINITY ? 0.f : fast_exp2(x1 - m_used);
+                    ps[c & 3] += p0 + p1;
+                    pk[c] = pack_bf16(p0, p1);
+                }
+                l = l * alpha + ((ps[0] + ps[1]) + (ps[2] + ps[3]));
+                const int pb = j & 1;
+                if (j >= 2) {
+                    // P buffer pb was last read by PV_{j-2}.
+                    if (lane == 0) w = mbar_wait(&o_done[pb], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort);
+                    if (!__shfl_sync(FULL, w, 0)) {
+                        ok = false;
+                        break;
+                    }
+                }
+                if (j >= 1 && __any_sync(FULL, need)) {
+                    // Rescale O: PV_{j-1} must have landed first.
+                    if (lane == 0)
+                        w = mbar_wait(&o_done[(j - 1) & 1], (uint32_t)((j - 1) >> 1) & 1u, abort);
+                    if (!__shfl_sync(FULL, w, 0)) {
+                        ok = false;
+                        break;
+                    }
+                    __syncwarp();
+                    tc_fence_after();
+                    const uint32_t ocol = tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(m * 256 + 128);
+#pragma unroll
+                    for (int c0 = 0; c0 < 128; c0 += 32) {
+                        uint32_t ov[32];
+                        tmem_ld32(ocol + c0, ov);
+                        tmem_wait_ld();
+                        uint32_t lo[16], hi[16];
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            lo[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
+                            hi[e] = __float_as_uint(__uint_as_float(ov[16 + e]) * alpha);
+                        }
+                        tmem_st16(ocol + c0, lo);
+                        tmem_st16(ocol + c0 + 16, hi);
+                    }
+                    tmem_wait_st();
+                }
+                uint8_t* pt = sP + (pb * MT + m) * AT_PTILE;
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                    *reinterpret_cast<uint4*>(pt + sw128(row, c)) =
+                        make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+                if (k >= 0 && nvalid < AT_BK && m == 0) {
+                    // Zero the V rows past the prefix end (they may hold anything).
+                    int w2 = 1;
+                    if (lane == 0) w2 = mbar_wait(&kv_full[s], (uint32_t)(j / ST) & 1u, abort);
+                    if (__shfl_sync(FULL, w2, 0)) {
+                        uint8_t* vt = sKV + s * AT_STAGE + 2 * AT_KV_HALF;
+                        for (int e = row; e < (AT_BK - nvalid) * 16; e += 128) {
+                            const int key = nvalid + (e >> 4), c = e & 15;
+                            *reinterpret_cast<uint4*>(vt + (c >> 3) * AT_KV_HALF + sw128(key, c & 7)) =
+                                make_uint4(0, 0, 0, 0);
+                        }
+                    }
+                }
+                fence_proxy_async_smem();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&p_full[pb]);
+            }
+        }
+    }
+
+    // ---------------------------------------------- this CTA's partial rows
+    // Every MMA has completed once the final o_done phase (or the drain in the
+    // MMA thread) is observed; the P/K/V area is then reused for the rows.
+    if (warp >= 2) {
+        int w = ok && nblk > 0 ? 1 : 0;
+        if (w && lane == 0)
+            w = mbar_wait(&o_done[(nblk - 1) & 1], (uint32_t)((nblk - 1) >> 1) & 1u, abort);
+        w = __shfl_sync(FULL, w, 0);
+        uint8_t* dst = sRed + (size_t)grow * AT_RED_STRIDE;
+        if (w) {
+            __syncwarp();
+            tc_fence_after();
+            const uint32_t ocol = tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(m * 256 + 128);
+            const float inv = 1.0f / l;
+#pragma unroll
+            for (int c0 = 0; c0 < 128; c0 += 32) {
+                uint32_t ov[32];
+                tmem_ld32(ocol + c0, ov);
+                tmem_wait_ld();
+#pragma unroll
+                for (int e = 0; e < 32; e += 4)
+                    *reinterpret_cast<float4*>(dst + (c0 + e) * 4) =
+                        make_float4(__uint_as_float(ov[e]) * inv, __uint_as_float(ov[e + 1]) * inv,
+                                    __uint_as_float(ov[e + 2]) * inv, __uint_as_float(ov[e + 3]) * inv);
+            }
+        }
+        // lse: -inf for a CTA without blocks, NaN for one that gave up.
+        sLse[grow] = w ? m_used + log2f(l) : (nblk > 0 ? NAN : -INFINITY);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, 256 * MT);
+
+    // ------------------------------------------ cluster reduction of the rows
+    cluster_sync();
+    grid_dep_wait();   // the output may be written only after the previous grid
+    {
+        const int R = a.G * a.N;
+        const int Rc = (R + C - 1) / C;
+        const int r_lo = rank * Rc, r_hi = min(R, r_lo + Rc);
+        const uint32_t red_base = smem_u32(sRed);
+        const uint32_t lse_base = smem_u32(sLse);
+        for (int r = r_lo + warp; r < r_hi; r += NTH / 32) {
+            float lse = -INFINITY;
+            if (lane < C) lse = ld_cluster_f32(map_rank(lse_base + (uint32_t)r * 4u, (uint32_t)lane));
+            const bool bad = __any_sync(FULL, lse != lse);
+            const float M = warp_max(lse);
+            const float wt = (lane < C && lse != -INFINITY) ? exp2f(lse - M) : 0.f;
+            const float wsum = warp_sum(wt);
+            // Issue every CTA's slice of the row before consuming any of them.
+            float4 v[16];
+            const uint32_t my = red_base + (uint32_t)r * AT_RED_STRIDE + (uint32_t)lane * 16u;
+#pragma unroll
+            for (int q = 0; q < 16; ++q)
+                if (q < C) v[q] = ld_cluster_v4(map_rank(my, (uint32_t)q));
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) {
+                const float wq = __shfl_sync(FULL, wt, q);   // 0 for q >= C and empty CTAs
+                if (q < C && wq != 0.f) {
+                    acc.x += wq * v[q].x;
+                    acc.y += wq * v[q].y;
+                    acc.z += wq * v[q].z;
+                    acc.w += wq * v[q].w;
+                }
+            }
+            const float inv = bad ? NAN : 1.0f / wsum;
+            const int i = r / a.G, h = g * a.G + r % a.G;
+            __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out) + (((size_t)b * a.N + i) * a.Hq + h) * 128;
+            uint2 pk;
+            pk.x = pack_bf16(acc.x * inv, acc.y * inv);
+            pk.y = pack_bf16(acc.z * inv, acc.w * inv);
+            reinterpret_cast<uint2*>(o)[lane] = pk;
+        }
+    }
+    cluster_sync();   // no CTA leaves while another may still read its rows
+}
+
+// ----------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn tensor_map_encoder();
+int make_map_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                uint64_t row_stride_bytes);
+
+// 3-D map over q[B*N][Hq][128] (bf16) with box {64 d, G heads, 128/G nodes}:
+// the box lands in smem as 128 rows (node-major, head-minor) of 64 d.
+static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G) {
+    EncodeTiledFn enc = tensor_map_encoder();
+    if (!enc) {
+        set_error("cuTensorMapEncodeTiled unavailable");
+        return GV_ERR_CUDA;
+    }
+    cuuint64_t dims[3] = {128, (cuuint64_t)Hq, (cuuint64_t)BN};
+    cuuint64_t strides[2] = {256, (cuuint64_t)Hq * 256};
+    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(128 / G)};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        set_error("cuTensorMapEncodeTiled (q) failed (%d)", (int)r);
+        return GV_ERR_CUDA;
+    }
+    return GV_OK;
+}
+
+static size_t attn_tc_smem(int mt) {
+    const int st = mt == 1 ? 4 : 3;
+    return 1024 + (size_t)mt * (AT_QTILE + 2 * AT_PTILE) + (size_t)st * AT_STAGE + 8 * (2 * st + 11) + 16;
+}
+
+// CTAs per cluster.  Wanted: enough clusters x CTAs to cover the SMs once
+// (at most 16, the largest cluster GB300 schedules), at least 4 for long
+// caches so that a long sequence of a ragged batch is not one CTA's serial
+// work.  When the whole grid fits in one wave, the size is lowered until
+// every cluster can be resident at once (GPC boundaries limit how many large
+// clusters of 1-CTA-per-SM kernels fit), since a cluster left for a second
+// wave doubles the layer's time.
+template <int MT>
+static int attn_tc_cluster(int units, int S_max, size_t smem) {
+    static int max_active[2][17] = {};
+    auto kern = attn_tc_kernel<MT>;
+    int want = (sm_count() + units - 1) / units;
+    if (S_max >= 4096 && want < 4) want = 4;
+    if (want > 16) want = 16;
+    if (want < 1) want = 1;
+    for (int c = want; c >= 1; --c) {
+        if (max_active[MT - 1][c] == 0) {
+            cudaLaunchConfig_t cfg{};
+            cfg.gridDim = dim3((unsigned)(c * units));
+            cfg.blockDim = dim3(64 + 128 * MT);
+            cfg.dynamicSmemBytes = smem;
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeClusterDimension;
+            attr[0].val.clusterDim.x = (unsigned)c;
+            attr[0].val.clusterDim.y = 1;
+            attr[0].val.clusterDim.z = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            int n = 0;
+            if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+                cudaGetLastError();
+                n = -1;
+            }
+            max_active[MT - 1][c] = n;
+        }
+        const int n = max_active[MT - 1][c];
+        if (n < 0) continue;                        // not schedulable at this size
+        if (units * c > sm_count() || n >= units) return c;
+    }
+    return 1;
+}
+
+template <int MT>
+static int launch_mt(const AttnArgs& a0, const CUtensorMap& mk, const CUtensorMap& mv,
+                     const CUtensorMap& mq, cudaStream_t st) {
+    const size_t smem = attn_tc_smem(MT);
+    auto kern = attn_tc_kernel<MT>;
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    const int units = a0.B * a0.Hkv;
+    AttnArgs a = a0;
+    a.csize = attn_tc_cluster<MT>(units, a.S_max, smem);
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((unsigned)(units * a.csize));
+    cfg.blockDim = dim3(64 + 128 * MT);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = (unsigned)a.csize;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mk, mv, mq, a);
+    if (e != cudaSuccess) {
+        set_error("attn_tc_kernel launch (cluster %d): %s", a.csize, cudaGetErrorString(e));
+        return GV_ERR_CUDA;
+    }
+    return GV_OK;
+}
+
+int launch_attn_tc(const AttnArgs& a, cudaStream_t st) {
+    CUtensorMap mk, mv, mq;
+    const uint64_t rows = (uint64_t)a.B * a.Hkv * a.S_max;
+    int rc = make_map_2d(&mk, a.cacheK, rows, 128, AT_BK, 256);
+    if (rc != GV_OK) return rc;
+    rc = make_map_2d(&mv, a.cacheV, rows, 128, AT_BK, 256);
+    if (rc != GV_OK) return rc;
+    rc = make_map_q(&mq, a.q, a.B * a.N, a.Hq, a.G);
+    if (rc != GV_OK) return rc;
+    return (a.R + 127) / 128 == 1 ? launch_mt<1>(a, mk, mv, mq, st) : launch_mt<2>(a, mk, mv, mq, st);
+}
+
+}  // namespace gv

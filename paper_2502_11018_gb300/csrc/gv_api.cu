@@ -77,36 +77,46 @@ int launch_lmhead_merge(SelectPartials, int, int, int32_t*, float*, float*, floa
 int lmhead_tc_grid(int slots_capacity);
 
 // ---------------------------------------------------------- attention plan --
-constexpr int KPS = 256;   // prefix keys per split
+constexpr int KPS_F32 = 256;   // prefix keys per split, CUDA-core path
 
 struct AttnPlan {
-    size_t q_rot, part_o, part_ml, counters, total;
-    int nsplit, q_rows_pad;
+    size_t q_rot, part_o, part_ml, total;
+    int nsplit, q_rows_pad, kps;
 };
 
-static bool attn_shape_ok(const gv_attn_shape* s) {
-    return s && s->B >= 1 && s->N >= 1 && s->N <= 64 && s->Hkv >= 1 && s->Hq >= s->Hkv &&
-           s->Hq % s->Hkv == 0 && (s->d == 64 || s->d == 128) && s->S_max >= 1 &&
-           (s->dt == GV_BF16 || s->dt == GV_F32) && s->rope_base > 0.0f &&
-           std::isfinite(s->rope_base);
+// Shapes the kernels handle: fp32 with d in {64, 128}; bf16 (tensor cores)
+// with d = 128, G = Hq / Hkv dividing 128 and at most 256 query rows (two
+// M = 128 tiles) per KV head.
+static int attn_shape_status(const gv_attn_shape* s) {
+    if (!s || s->B < 1 || s->Hkv < 1 || s->Hq < s->Hkv || s->Hq % s->Hkv != 0 || s->S_max < 1 ||
+        (s->dt != GV_BF16 && s->dt != GV_F32))
+        return GV_ERR_ARG;
+    if (s->N < 1 || s->N > 64) return GV_ERR_UNSUPPORTED;
+    if (s->dt == GV_F32 && !(s->d == 64 || s->d == 128)) return GV_ERR_UNSUPPORTED;
+    const int G = s->Hq / s->Hkv;
+    if (s->dt == GV_BF16 && (s->d != 128 || 128 % G != 0 || G * s->N > 256)) return GV_ERR_UNSUPPORTED;
+    return GV_OK;
 }
 
+// The fp32 path keeps rotated queries and per-split partials in the
+// workspace; the bf16 path reduces its splits on chip and needs none.
 static AttnPlan attn_plan(const gv_attn_shape* s) {
     AttnPlan p{};
     const int R = (s->Hq / s->Hkv) * s->N;
     p.q_rows_pad = (R + 127) / 128 * 128;
-    p.nsplit = (s->S_max + KPS - 1) / KPS + 1;
-    const size_t bh = (size_t)s->B * s->Hkv;
+    p.kps = KPS_F32;
+    p.nsplit = (s->S_max + KPS_F32 - 1) / KPS_F32 + 1;
     size_t off = 0;
-    p.q_rot = off;
-    off += align256(bh * p.q_rows_pad * s->d * sizeof(float));
-    p.part_o = off;
-    off += align256(bh * p.nsplit * R * s->d * sizeof(float));
-    p.part_ml = off;
-    off += align256(bh * p.nsplit * R * 2 * sizeof(float));
-    p.counters = off;
-    off += align256(bh * sizeof(unsigned));
-    p.total = off;
+    if (s->dt == GV_F32) {
+        const size_t bh = (size_t)s->B * s->Hkv;
+        p.q_rot = off;
+        off += align256(bh * p.q_rows_pad * s->d * sizeof(float));
+        p.part_o = off;
+        off += align256(bh * p.nsplit * R * s->d * sizeof(float));
+        p.part_ml = off;
+        off += align256(bh * p.nsplit * R * 2 * sizeof(float));
+    }
+    p.total = off > 0 ? off : 256;
     return p;
 }
 
@@ -177,30 +187,41 @@ int gv_tree_build(const int32_t* parents, const int32_t* prefix_len, int B, int 
                              as_stream(stream));
 }
 
+int gv_rope_table(const int32_t* pos, int B, int N, int d, float rope_base, float* rope,
+                  void* stream) {
+    clear_error();
+    GV_CHECK_ARG(pos && rope, "gv_rope_table: null pointer");
+    GV_CHECK_ARG(B >= 1 && N >= 1 && d >= 2 && d <= 256 && d % 2 == 0,
+                 "gv_rope_table: B=%d N=%d d=%d", B, N, d);
+    GV_CHECK_ARG(rope_base > 0.0f && std::isfinite(rope_base), "gv_rope_table: rope_base %g",
+                 (double)rope_base);
+    GV_CHECK_ARG(((uintptr_t)rope & 7u) == 0, "gv_rope_table: rope not 8-byte aligned");
+    return launch_rope_table(pos, B, N, d, rope_base, rope, as_stream(stream));
+}
+
 size_t gv_verify_attention_workspace(const gv_attn_shape* s) {
-    if (!attn_shape_ok(s)) return 0;
+    if (attn_shape_status(s) != GV_OK) return 0;
     return attn_plan(s).total;
 }
 
 int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new,
                         const void* v_new, const void* cacheK, const void* cacheV,
-                        const int32_t* prefix_len, const int32_t* pos, const uint64_t* anc,
+                        const int32_t* prefix_len, const float* rope, const uint64_t* anc,
                         void* treeK, void* treeV, void* out, void* workspace, size_t ws_bytes,
                         void* stream) {
     clear_error();
-    if (s && (s->N < 1 || s->N > 64)) {
-        set_error("gv_verify_attention: N=%d outside 1..64", s->N);
+    const int sst = attn_shape_status(s);
+    if (sst == GV_ERR_UNSUPPORTED) {
+        set_error("gv_verify_attention: unsupported shape (N=%d d=%d G*N=%d dt=%d); fp32 needs "
+                  "d in {64,128}, bf16 needs d=128 and G*N <= 256, N <= 64",
+                  s->N, s->d, (s->Hq / s->Hkv) * s->N, (int)s->dt);
         return GV_ERR_UNSUPPORTED;
     }
-    if (s && !(s->d == 64 || s->d == 128)) {
-        set_error("gv_verify_attention: head dim %d not in {64, 128}", s->d);
-        return GV_ERR_UNSUPPORTED;
-    }
-    GV_CHECK_ARG(attn_shape_ok(s), "gv_verify_attention: invalid shape");
-    const void* ptrs[] = {q, k_new, v_new, cacheK, cacheV, treeK, treeV, out};
+    GV_CHECK_ARG(sst == GV_OK, "gv_verify_attention: invalid shape");
+    const void* ptrs[] = {q, k_new, v_new, cacheK, cacheV, treeK, treeV, out, rope};
     for (const void* p : ptrs)
         GV_CHECK_ARG(p && aligned16(p), "gv_verify_attention: tensor null or not 16-byte aligned");
-    GV_CHECK_ARG(prefix_len && pos && anc, "gv_verify_attention: null index pointer");
+    GV_CHECK_ARG(prefix_len && anc, "gv_verify_attention: null index pointer");
     const AttnPlan plan = attn_plan(s);
     GV_CHECK_ARG(workspace && ((uintptr_t)workspace & 255u) == 0,
                  "gv_verify_attention: workspace null or not 256-byte aligned");
@@ -217,7 +238,6 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
     a.G = s->Hq / s->Hkv;
     a.R = a.G * s->N;
     a.q_rows_pad = plan.q_rows_pad;
-    a.rope_base = s->rope_base;
     a.scale = 1.0f / sqrtf((float)s->d);
     a.q = q;
     a.k_new = k_new;
@@ -225,7 +245,7 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
     a.cacheK = cacheK;
     a.cacheV = cacheV;
     a.prefix_len = prefix_len;
-    a.pos = pos;
+    a.rope = rope;
     a.anc = reinterpret_cast<const unsigned long long*>(anc);
     a.treeK = treeK;
     a.treeV = treeV;
@@ -233,19 +253,16 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
     a.q_rot = ws + plan.q_rot;
     a.part_o = reinterpret_cast<float*>(ws + plan.part_o);
     a.part_ml = reinterpret_cast<float*>(ws + plan.part_ml);
-    a.counters = reinterpret_cast<unsigned*>(ws + plan.counters);
     a.nsplit = plan.nsplit;
-    a.kps = KPS;
+    a.kps = plan.kps;
     cudaStream_t st = as_stream(stream);
     int rc;
     if (s->dt == GV_F32) {
-        if ((rc = launch_rope_tree<float, float>(a, st)) != GV_OK) return rc;
-        if ((rc = launch_attn_cc<float>(a, st)) != GV_OK) return rc;
-        return launch_attn_combine<float>(a, st);
+        if ((rc = launch_rope_tree_f32(a, st)) != GV_OK) return rc;
+        if ((rc = launch_attn_cc_f32(a, st)) != GV_OK) return rc;
+        return launch_attn_combine_f32(a, st);
     }
-    if ((rc = launch_rope_tree<__nv_bfloat16, float>(a, st)) != GV_OK) return rc;
-    if ((rc = launch_attn_cc<__nv_bfloat16>(a, st)) != GV_OK) return rc;
-    return launch_attn_combine<__nv_bfloat16>(a, st);
+    return launch_attn_tc(a, st);
 }
 
 size_t gv_lmhead_workspace(int rows, int H, int V, int dt, int mode, int k) {

@@ -31,7 +31,7 @@ GV_SELECT_TOPK = 1
 GV_SELECT_LOGITS = 2
 
 # Every symbol include/gv.h declares.
-EXPORTS = ("gv_tree_build", "gv_verify_attention_workspace", "gv_verify_attention",
+EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "gv_verify_attention",
            "gv_lmhead_workspace", "gv_lmhead_select", "gv_accept_workspace", "gv_accept",
            "gv_kv_compact", "gv_status_string", "gv_last_error", "gv_version")
 
@@ -45,7 +45,7 @@ class GvError(RuntimeError):
 class gv_attn_shape(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("N", ctypes.c_int), ("Hq", ctypes.c_int),
                 ("Hkv", ctypes.c_int), ("d", ctypes.c_int), ("S_max", ctypes.c_int),
-                ("rope_base", ctypes.c_float), ("dt", ctypes.c_int)]
+                ("dt", ctypes.c_int)]
 
 
 _lib = None
@@ -66,6 +66,7 @@ def lib():
     L = ctypes.CDLL(LIB_PATH)
     sig = {
         "gv_tree_build": ([_vp, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
+        "gv_rope_table": ([_vp, _i, _i, _i, _f, _vp, _vp], _i),
         "gv_verify_attention_workspace": ([ctypes.POINTER(gv_attn_shape)], _sz),
         "gv_verify_attention": ([ctypes.POINTER(gv_attn_shape)] + [_vp] * 12 + [_sz, _vp], _i),
         "gv_lmhead_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
@@ -135,20 +136,26 @@ def gv_tree_build(parents, prefix_len, depth, pos, anc, seq_status, stream=None)
         _ptr(pos, "pos"), _ptr(anc, "anc"), _ptr(seq_status, "seq_status"), _stream(stream)))
 
 
-def attn_shape(B, N, Hq, Hkv, d, S_max, rope_base, dt):
-    return gv_attn_shape(B, N, Hq, Hkv, d, S_max, float(rope_base), int(dt))
+def gv_rope_table(pos, d, rope_base, rope, stream=None):
+    B, N = pos.shape
+    return _check("gv_rope_table", lib().gv_rope_table(
+        _ptr(pos, "pos"), B, N, d, float(rope_base), _ptr(rope, "rope"), _stream(stream)))
+
+
+def attn_shape(B, N, Hq, Hkv, d, S_max, dt):
+    return gv_attn_shape(B, N, Hq, Hkv, d, S_max, int(dt))
 
 
 def gv_verify_attention_workspace(shape):
     return int(lib().gv_verify_attention_workspace(ctypes.byref(shape)))
 
 
-def gv_verify_attention(shape, q, k_new, v_new, cacheK, cacheV, prefix_len, pos, anc, treeK,
+def gv_verify_attention(shape, q, k_new, v_new, cacheK, cacheV, prefix_len, rope, anc, treeK,
                         treeV, out, workspace, stream=None):
     return _check("gv_verify_attention", lib().gv_verify_attention(
         ctypes.byref(shape), _ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"),
         _ptr(cacheK, "cacheK"), _ptr(cacheV, "cacheV"), _ptr(prefix_len, "prefix_len"),
-        _ptr(pos, "pos"), _ptr(anc, "anc"), _ptr(treeK, "treeK"), _ptr(treeV, "treeV"),
+        _ptr(rope, "rope"), _ptr(anc, "anc"), _ptr(treeK, "treeK"), _ptr(treeV, "treeV"),
         _ptr(out, "out"), _ptr(workspace, "workspace"), workspace.numel() * workspace.element_size(),
         _stream(stream)))
 

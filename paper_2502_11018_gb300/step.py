@@ -4,7 +4,7 @@
 five calls of include/gv.h in order on one stream (GRIFFIN Section 3: draft,
 then one verify forward over every draft token, then accept):
 
-1. ``gv_tree_build``;
+1. ``gv_tree_build`` and ``gv_rope_table`` (RoPE cos/sin shared by all layers);
 2. ``gv_verify_attention`` for every layer (per-layer tree K/V scratch);
 3. ``gv_lmhead_select`` (argmax for T = 0, fp32 logits + LSE for T > 0);
 4. ``gv_accept``;
@@ -38,10 +38,11 @@ class VerifyStep:
         self.pos = torch.zeros(B, N, **i32)
         self.anc = torch.zeros(B, N, dtype=torch.int64, device=dev)
         self.seq_status = torch.zeros(B, **i32)
+        self.rope = torch.zeros(B, N, d // 2, 2, dtype=torch.float32, device=dev)
         self.treeK = torch.zeros(L, B, Hkv, N, d, dtype=dt, device=dev)
         self.treeV = torch.zeros(L, B, Hkv, N, d, dtype=dt, device=dev)
         self.attn_out = torch.zeros(L, B, N, Hq, d, dtype=dt, device=dev)
-        self.shape = gv.attn_shape(B, N, Hq, Hkv, d, S_max, cfg["rope_base"], self.dt_code)
+        self.shape = gv.attn_shape(B, N, Hq, Hkv, d, S_max, self.dt_code)
         ws = gv.gv_verify_attention_workspace(self.shape)
         self.attn_ws = torch.empty(max(ws, 256), dtype=torch.uint8, device=dev)
         rows = B * N
@@ -71,11 +72,12 @@ class VerifyStep:
         i = self.inp
         gv.gv_tree_build(i.parents, i.prefix_len, self.depth, self.pos, self.anc, self.seq_status,
                          stream)
+        gv.gv_rope_table(self.pos, self.cfg["d"], self.cfg["rope_base"], self.rope, stream)
 
     def attention(self, layer, stream=None):
         i = self.inp
         gv.gv_verify_attention(self.shape, i.q[layer], i.k_new[layer], i.v_new[layer],
-                               i.cacheK[layer], i.cacheV[layer], i.prefix_len, self.pos, self.anc,
+                               i.cacheK[layer], i.cacheV[layer], i.prefix_len, self.rope, self.anc,
                                self.treeK[layer], self.treeV[layer], self.attn_out[layer],
                                self.attn_ws, stream)
 

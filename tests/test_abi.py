@@ -27,7 +27,7 @@ def declared_functions():
 
 def test_exports_match_header(lib):
     names = declared_functions()
-    assert len(names) >= 11
+    assert len(names) >= 12
     for n in names:
         assert hasattr(lib, n), n
     assert sorted(gv.EXPORTS) == names
@@ -48,10 +48,13 @@ def test_host_side_validation(lib):
     assert lib.gv_tree_build(nul, nul, 1, 0, nul, nul, nul, nul, nul) == gv.GV_ERR_INVALID_TREE
     assert lib.gv_tree_build(nul, nul, 1, 4, nul, nul, nul, nul, nul) == gv.GV_ERR_ARG
     assert "null" in gv.last_error()
-    shape = gv.attn_shape(1, 60, 32, 8, 96, 4224, 5e5, gv.GV_BF16)
+    shape = gv.attn_shape(1, 60, 32, 8, 96, 4224, gv.GV_BF16)
     assert lib.gv_verify_attention(ctypes.byref(shape), *([nul] * 12), 0, nul) == gv.GV_ERR_UNSUPPORTED
-    shape = gv.attn_shape(1, 60, 30, 8, 128, 4224, 5e5, gv.GV_BF16)
+    shape = gv.attn_shape(1, 60, 64, 8, 128, 4224, gv.GV_BF16)   # 480 query rows per KV head
+    assert lib.gv_verify_attention(ctypes.byref(shape), *([nul] * 12), 0, nul) == gv.GV_ERR_UNSUPPORTED
+    shape = gv.attn_shape(1, 60, 30, 8, 128, 4224, gv.GV_BF16)
     assert gv.gv_verify_attention_workspace(shape) == 0     # Hq not a multiple of Hkv
+    assert lib.gv_rope_table(nul, 1, 60, 128, 1e4, nul, nul) == gv.GV_ERR_ARG
     assert lib.gv_lmhead_select(nul, nul, 60, 4096, 1000, 0, 1, 17, *([nul] * 6), 0, nul) == gv.GV_ERR_ARG
     assert lib.gv_accept(1, 60, 6, 0, -1.0, *([nul] * 12), nul, 0, nul) == gv.GV_ERR_ARG
     assert lib.gv_kv_compact(1, 1, 60, 6, 8, 3, 100, 0, *([nul] * 9), nul) == gv.GV_ERR_ARG
@@ -59,7 +62,7 @@ def test_host_side_validation(lib):
 
 
 def test_workspace_queries(lib):
-    shape = gv.attn_shape(1, 60, 32, 8, 128, 4224, 5e5, gv.GV_BF16)
+    shape = gv.attn_shape(1, 60, 32, 8, 128, 4224, gv.GV_BF16)
     assert gv.gv_verify_attention_workspace(shape) > 0
     assert gv.gv_lmhead_workspace(60, 4096, 128256, gv.GV_BF16, gv.GV_SELECT_ARGMAX) > 0
     assert gv.gv_lmhead_workspace(60, 4096, 128256, gv.GV_BF16, gv.GV_SELECT_TOPK, 0) == 0

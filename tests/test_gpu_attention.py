@@ -25,10 +25,13 @@ CASES = [
     ("f32", 2, 60, 8, 2, 128, [300, 37], 5e5, 1.0),
     ("bf16", 1, 60, 32, 8, 128, [300], 5e5, 1.0),     # LLaMA-3-8B heads, short prefix
     ("bf16", 2, 17, 4, 4, 128, [127, 128], 1e4, 1.0),
-    ("bf16", 3, 64, 8, 1, 128, [1, 513, 1000], 1e6, 1.0),
-    ("bf16", 1, 1, 2, 2, 64, [0], 1e4, 1.0),
+    ("bf16", 3, 64, 8, 2, 128, [1, 513, 1000], 1e6, 1.0),   # 256 query rows per KV head
+    ("bf16", 1, 1, 2, 2, 128, [0], 1e4, 1.0),
     ("bf16", 2, 60, 8, 8, 128, [129, 2100], 1e4, 1.0),
-    ("bf16", 1, 61, 16, 4, 64, [777], 5e5, 1.0),
+    ("bf16", 1, 61, 16, 4, 128, [777], 5e5, 1.0),
+    ("bf16", 4, 60, 40, 40, 128, [64, 65, 255, 256], 1e4, 1.0),  # ragged batch, MHA
+    ("f32", 1, 1, 2, 2, 64, [0], 1e4, 1.0),
+    ("f32", 1, 61, 16, 4, 64, [777], 5e5, 1.0),
 ]
 
 
@@ -62,12 +65,14 @@ def run_gpu_attention(dev, parents, P, S_max, q, k, v, cK, cV, base):
     st = torch.zeros(B, dtype=torch.int32, device=dev)
     Pd = t(P)
     gv.gv_tree_build(t(parents), Pd, depth, pos, anc, st)
-    shape = gv.attn_shape(B, N, Hq, Hkv, d, S_max, base, gv.GV_BF16 if dt == torch.bfloat16 else gv.GV_F32)
+    rope = torch.zeros(B, N, d // 2, 2, dtype=torch.float32, device=dev)
+    gv.gv_rope_table(pos, d, base, rope)
+    shape = gv.attn_shape(B, N, Hq, Hkv, d, S_max, gv.GV_BF16 if dt == torch.bfloat16 else gv.GV_F32)
     ws = torch.full((gv.gv_verify_attention_workspace(shape),), 0xFF, dtype=torch.uint8, device=dev)
     tK = torch.zeros(B, Hkv, N, d, dtype=dt, device=dev)
     tV = torch.zeros_like(tK)
     out = torch.zeros(B, N, Hq, d, dtype=dt, device=dev)
-    gv.gv_verify_attention(shape, q.to(dev), k.to(dev), v.to(dev), cK.to(dev), cV.to(dev), Pd, pos,
+    gv.gv_verify_attention(shape, q.to(dev), k.to(dev), v.to(dev), cK.to(dev), cV.to(dev), Pd, rope,
                            anc, tK, tV, out, ws)
     torch.cuda.synchronize()
     return out, tK, tV, pos, anc
