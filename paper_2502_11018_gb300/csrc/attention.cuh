@@ -27,7 +27,8 @@ struct AttnArgs {
     void* q_rot;      // [B*Hkv][q_rows_pad][d]  rotated queries (fp32 or bf16)
     float* part_o;    // [B*Hkv][nsplit][R][d]   per-split partial outputs
     float* part_ml;   // [B*Hkv][nsplit][R][2] (m, l) on the CUDA-core path,
-                      // [B*Hkv][nsplit][R] log2-sum-exp on the tensor-core path
+                      // [B*Hkv][C][R] log2-sum-exp on the tensor-core path
+    void* part_bf16;  // [B*Hkv][C][R][d] bf16 normalised partial rows (tensor-core path)
     int nsplit;       // prefix splits + 1 tree split (CUDA-core path)
     int kps;          // prefix keys per split (CUDA-core path)
     int csize;        // CTAs per cluster, one cluster per (sequence, KV head) (tensor-core path)

@@ -25,23 +25,25 @@
 //                          always share one max), writes P = exp2(s - m) as
 //                          bf16 to one of two smem buffers
 //   O += P_j V_j           tcgen05.mma, P K-major, V MN-major (d contiguous)
-// Each CTA then leaves o = O / l and lse = m + log2(l) of its rows in its own
-// shared memory; after a cluster barrier every CTA reduces a 1/C share of the
-// rows across the cluster through distributed shared memory and writes the
-// final bf16 output.  No partial result goes through global memory.
+// Each CTA then writes o = O / l (bf16) and lse = m + log2(l) of its rows to
+// the workspace (they stay in L2); after a cluster barrier every CTA reduces
+// a 1/C share of the rows over the cluster's C partials and writes the final
+// bf16 output, so the split combine needs no extra launch.
 //
 // Warp roles: warp 0 issues the TMA loads (K/V blocks, raw Q tiles); warp 1
 // owns TMEM and issues the MMAs; warps 2.. (4 per M tile) rotate Q in place
 // (RoPE from the per-step table), build the tree K/V tile, and run the
 // softmax and the epilogue; all warps share the cluster reduction.
 //
-// Launch: cluster launch with programmatic dependent launch.  Before
-// griddepcontrol.wait a CTA only initialises barriers and TMEM and starts
-// streaming its K/V cache blocks (the cache is not written by the kernels it
-// overlaps); queries, RoPE table, ancestor masks and the output are touched
-// after it.  Every mbarrier wait is bounded; a CTA that gives up marks its
-// rows' lse NaN, which turns the affected outputs into NaN, and still
-// reaches both cluster barriers.
+// Launch: cluster launch (the cluster barrier orders the partial exchange and
+// guarantees the C CTAs are co-resident) with programmatic dependent launch.
+// Before griddepcontrol.wait a CTA only initialises barriers and TMEM, reads
+// step inputs written before the step's first attention launch (RoPE table,
+// ancestor masks, prefix lengths) and starts streaming two K/V cache blocks;
+// queries, tree keys/values, partials and the output are touched after it.
+// Every mbarrier wait is bounded; a CTA that gives up marks its rows' lse
+// NaN, which turns the affected outputs into NaN, and still reaches the
+// cluster barrier.
 #include "gv_internal.cuh"
 #include "attention.cuh"
 #include "sm103.cuh"
@@ -55,7 +57,6 @@ constexpr int AT_QTILE = 2 * AT_QHALF;      // one M tile of Q
 constexpr int AT_PTILE = 128 * 128;         // one M tile of P: 128 rows x 64 keys bf16
 constexpr int AT_KV_HALF = AT_BK * 128;     // 64 keys x 64 d bf16 (one swizzle sub-tile)
 constexpr int AT_STAGE = 4 * AT_KV_HALF;    // K (2 halves) + V (2 halves)
-constexpr int AT_RED_STRIDE = 512 + 16;     // bytes per fp32 row of the reduction buffer
 
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -78,23 +79,32 @@ __device__ __forceinline__ void cluster_sync() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
                  "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-// Shared::cluster address of the same smem location in CTA `rank`.
-__device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank) {
-    uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+// Packed fp32 pairs (one instruction for two lanes' worth of work) and the
+// three-input max of sm_100+.
+__device__ __forceinline__ uint64_t f32x2(float a, float b) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
     return r;
 }
-__device__ __forceinline__ float ld_cluster_f32(uint32_t addr) {
-    float v;
-    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+__device__ __forceinline__ float2 split_f32x2(uint64_t r) {
+    float2 v;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(v.x), "=f"(v.y) : "l"(r));
     return v;
 }
-__device__ __forceinline__ float4 ld_cluster_v4(uint32_t addr) {
-    float4 v;
-    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(addr));
-    return v;
+__device__ __forceinline__ uint64_t ffma_f32x2(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ uint64_t fadd_f32x2(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+    float m;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(m) : "f"(a), "f"(b), "f"(c));
+    return m;
 }
 __device__ __forceinline__ float fast_exp2(float x) {
     float y;
@@ -136,7 +146,8 @@ __device__ __forceinline__ void rope8(const uint4& lo, const uint4& hi, const fl
 template <int MT>
 __global__ void __launch_bounds__(64 + 128 * MT, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
-               const __grid_constant__ CUtensorMap map_q, AttnArgs a) {
+               const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_part,
+               AttnArgs a) {
     constexpr int NSM = 128 * MT;            // softmax threads
     constexpr int NTH = 64 + NSM;            // all threads
     constexpr int ST = MT == 1 ? 4 : 3;      // K/V stages
@@ -148,12 +159,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     // stream started, so it may be read before griddepcontrol.wait.
     const int P = min(max(a.prefix_len[b], 0), a.S_max);
     const int nb_pre = (P + AT_BK - 1) / AT_BK;
-    const int T = nb_pre + 1;                            // + the tree block
-    const int nblk = T > rank ? (T - 1 - rank) / C + 1 : 0;
-    const bool has_tree = nb_pre % C == rank;
+    // Prefix blocks go round robin from rank 0, so the highest ranks hold the
+    // fewest; the tree block goes to the last rank and runs first there.
+    const bool has_tree = rank == C - 1;
+    const int nblk = (nb_pre > rank ? (nb_pre - 1 - rank) / C + 1 : 0) + (has_tree ? 1 : 0);
     const int nb_per_tile = 128 / a.G;                   // nodes per M tile
-    // Prefix block index of this CTA's j-th block (the tree block, if owned,
-    // is j = 0 and returns -1).
+    const int R = a.G * a.N;                             // query rows of (b, g)
+    const int Rc = (R + C - 1) / C;                      // rows each CTA reduces
+    // Prefix block index of this CTA's j-th block (-1 for the tree block).
     auto prefix_block = [&](int j) -> int {
         if (has_tree) return j == 0 ? -1 : rank + C * (j - 1);
         return rank + C * j;
@@ -165,8 +178,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint8_t* sQ = smem;                                  // MT x 32 KB
     uint8_t* sP = sQ + MT * AT_QTILE;                    // 2 buffers x MT x 16 KB
     uint8_t* sKV = sP + 2 * MT * AT_PTILE;               // ST x 32 KB
-    uint8_t* sRed = sP;                                  // reduction rows (after the last PV)
-    float* sLse = reinterpret_cast<float*>(sRed + MT * 128 * AT_RED_STRIDE);
     uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + ST * AT_STAGE);
     uint64_t* kv_full = bars;
     uint64_t* kv_empty = kv_full + ST;
@@ -177,7 +188,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint64_t* q_raw = o_done + 2;
     uint64_t* q_full = q_raw + 1;
     uint64_t* drain = q_full + 1;
-    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+    uint64_t* rope_full = drain + 1;
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(rope_full + 1);
+    // The RoPE rows of sequence b (N x 64 (cos, sin) pairs) are staged in the
+    // P area, which is free until the first softmax block writes P.
+    const float4* sRope = reinterpret_cast<const float4*>(sP);
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -195,10 +210,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         mbar_init(q_raw, 1);
         mbar_init(q_full, 4 * MT);
         mbar_init(drain, 1);
+        mbar_init(rope_full, 1);
         *abort = 0;
         fence_mbar_init();
         if (nblk > 0) {
             prefetch_tmap(&map_q);
+            prefetch_tmap(&map_part);
             prefetch_tmap(&map_k);
             prefetch_tmap(&map_v);
         }
@@ -227,6 +244,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             if (lane == 0) {
                 const uint64_t pol_kv = policy_evict_first();
                 const uint64_t pol_q = policy_evict_last();
+                // RoPE rows first: written by a kernel that completed before
+                // the step's first attention launch, so safe before the wait.
+                mbar_arrive_expect_tx(rope_full, (uint32_t)a.N * 512u);
+                bulk_load(sP, reinterpret_cast<const char*>(a.rope) + (size_t)b * a.N * 512,
+                          (uint32_t)a.N * 512u, rope_full);
                 int issued[ST];
                 for (int q = 0; q < ST; ++q) issued[q] = -1;
                 bool q_issued = false;
@@ -243,7 +265,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 for (int j = 0; j < nblk; ++j) {
                     const int s = j % ST;
                     const uint32_t ph = (uint32_t)(j / ST) & 1u;
-                    if (j == ST) issue_q();          // the first ST blocks are in flight
+                    // Two K/V blocks stream before the dependency wait, then the
+                    // queries (on the critical path), then the remaining blocks.
+                    if (j == 2) issue_q();
                     const int k = prefix_block(j);
                     if (k < 0) continue;             // tree block: built by the softmax warps
                     if (!mbar_wait(&kv_empty[s], ph ^ 1u, abort)) break;
@@ -261,6 +285,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     for (int q = 0; q < ST; ++q)
                         if (issued[q] >= 0) mbar_wait_timeout_only(&kv_full[q], (uint32_t)issued[q]);
                     if (q_issued) mbar_wait_timeout_only(q_raw, 0);
+                    mbar_wait_timeout_only(rope_full, 0);
                 }
             }
         } else if (warp == 1) {
@@ -326,8 +351,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             }
         } else {
             // -------------------------- Q rotation, tree tile, softmax, epilogue
+            // The ancestor masks (like the RoPE rows the producer stages in
+            // smem) were written before the first attention launch of the
+            // step, so they are read before griddepcontrol.wait; the queries
+            // and tree keys/values come after it.
+            const unsigned long long anc_row =
+                (has_tree && row_ok) ? __ldg(a.anc + (size_t)b * a.N + node) : 0ull;
             grid_dep_wait();
-            const float4* rope_b = reinterpret_cast<const float4*>(a.rope) + (size_t)b * a.N * 32;
+            {
+                int w = 1;
+                if (lane == 0) w = mbar_wait(rope_full, 0, abort);
+                if (!__shfl_sync(FULL, w, 0)) ok = false;
+            }
             if (has_tree) {
                 // Rotated tree keys and the values into stage 0 (and into the
                 // tree K/V scratch in global memory for gv_kv_compact).
@@ -344,7 +379,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         vhi = __ldg(vr + 8 + c);
                         float4 cs[4];
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) cs[q] = __ldg(rope_b + (size_t)j * 32 + c * 4 + q);
+                        for (int q = 0; q < 4; ++q) cs[q] = sRope[j * 32 + c * 4 + q];
                         rope8(k0, k1, cs, klo, khi);
                         uint4* tk = reinterpret_cast<uint4*>(a.treeK) + ((size_t)bg * a.N + j) * 16;
                         uint4* tv = reinterpret_cast<uint4*>(a.treeV) + ((size_t)bg * a.N + j) * 16;
@@ -364,22 +399,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             }
             // RoPE of this thread's Q row, in place once the raw tile has landed.
             {
-                float4 cs[32];
-                if (row_ok) {
-#pragma unroll
-                    for (int q = 0; q < 32; ++q) cs[q] = __ldg(rope_b + (size_t)node * 32 + q);
-                }
                 int w = 1;
                 if (lane == 0) w = mbar_wait(q_raw, 0, abort);
                 w = __shfl_sync(FULL, w, 0);
                 uint8_t* qt = sQ + m * AT_QTILE;
-                if (w) {
+                if (w && ok) {
 #pragma unroll
                     for (int c = 0; c < 8; ++c) {
                         uint4* plo = reinterpret_cast<uint4*>(qt + sw128(row, c));
                         uint4* phi = reinterpret_cast<uint4*>(qt + AT_QHALF + sw128(row, c));
                         uint4 olo = make_uint4(0, 0, 0, 0), ohi = olo;
-                        if (row_ok) rope8(*plo, *phi, cs + 4 * c, olo, ohi);
+                        if (row_ok) {
+                            float4 cs[4];
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) cs[q] = sRope[node * 32 + c * 4 + q];
+                            rope8(*plo, *phi, cs, olo, ohi);
+                        }
                         *plo = olo;
                         *phi = ohi;
                     }
@@ -388,8 +423,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 __syncwarp();
                 if (lane == 0) mbar_arrive(q_full);
             }
-            const unsigned long long anc_row =
-                (has_tree && row_ok) ? __ldg(a.anc + (size_t)b * a.N + node) : 0ull;
             const float sl2 = a.scale * 1.4426950408889634f;     // scale * log2(e)
             for (int j = 0; j < nblk; ++j) {
                 const int buf = j & 1, s = j % ST;
@@ -412,26 +445,32 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&s_free[buf]);
-                // Branch-free validity mask of the block's 64 keys for this row.
+                // Keys of the block this row may see: all 64 of a full prefix
+                // block (the common, unmasked path), else a branch-free 64-bit
+                // mask (the prefix end, or the row's ancestor bitmask); masked
+                // scores become -inf and their exp2 is exactly 0.
                 const int k = prefix_block(j);
-                uint32_t vlo, vhi;
-                int nvalid = AT_BK;
-                if (k < 0) {
-                    vlo = (uint32_t)anc_row;
-                    vhi = (uint32_t)(anc_row >> 32);
-                } else {
-                    nvalid = min(AT_BK, P - k * AT_BK);
-                    vlo = nvalid >= 32 ? 0xFFFFFFFFu : ((1u << nvalid) - 1u);
-                    vhi = nvalid >= 64 ? 0xFFFFFFFFu : (nvalid > 32 ? ((1u << (nvalid - 32)) - 1u) : 0u);
-                }
-                float mx = -INFINITY;
+                const int nvalid = k < 0 ? a.N : min(AT_BK, P - k * AT_BK);
+                if (k < 0 || nvalid < AT_BK) {
+                    uint32_t vlo, vhi;
+                    if (k < 0) {
+                        vlo = (uint32_t)anc_row;
+                        vhi = (uint32_t)(anc_row >> 32);
+                    } else {
+                        vlo = nvalid >= 32 ? 0xFFFFFFFFu : ((1u << nvalid) - 1u);
+                        vhi = nvalid > 32 ? ((1u << (nvalid - 32)) - 1u) : 0u;
+                    }
 #pragma unroll
-                for (int c = 0; c < 64; ++c) {
-                    const uint32_t bit = c < 32 ? (vlo >> c) & 1u : (vhi >> (c - 32)) & 1u;
-                    const float x = bit ? __uint_as_float(sv[c]) * sl2 : -INFINITY;
-                    sv[c] = __float_as_uint(x);
-                    mx = fmaxf(mx, x);
+                    for (int c = 0; c < 64; ++c) {
+                        const uint32_t bit = c < 32 ? (vlo >> c) & 1u : (vhi >> (c - 32)) & 1u;
+                        sv[c] = bit ? sv[c] : __float_as_uint(-INFINITY);
+                    }
                 }
+                float mxs[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+                for (int c = 0; c < 64; c += 2)
+                    mxs[(c >> 1) & 3] = max3(mxs[(c >> 1) & 3], __uint_as_float(sv[c]), __uint_as_float(sv[c + 1]));
+                const float mx = max3(mxs[0], mxs[1], fmaxf(mxs[2], mxs[3])) * sl2;   // sl2 > 0
                 const float m_new = fmaxf(m_used, mx);
                 const bool need = m_new > m_used + 8.0f;     // also true the first time
                 float alpha = 1.0f;
@@ -439,18 +478,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     alpha = fast_exp2(m_used - m_new);       // 0 when m_used = -inf
                     m_used = m_new;
                 }
-                float ps[4] = {0.f, 0.f, 0.f, 0.f};
+                // p = 2^(s * sl2 - m); a row with no visible key so far keeps
+                // m = -inf and all its p are 0 (the offset is then irrelevant).
+                const float nmv = m_used == -INFINITY ? 0.f : -m_used;
+                const uint64_t sc2 = f32x2(sl2, sl2), nm2 = f32x2(nmv, nmv);
+                uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
                 uint32_t pk[32];
 #pragma unroll
                 for (int c = 0; c < 32; ++c) {
-                    // masked keys give 0 (also for a padding row whose max is -inf)
-                    const float x0 = __uint_as_float(sv[2 * c]), x1 = __uint_as_float(sv[2 * c + 1]);
-                    const float p0 = x0 == -INFINITY ? 0.f : fast_exp2(x0 - m_used);
-                    const float p1 = x1 == -INFINITY ? 0.f : fast_exp2(x1 - m_used);
-                    ps[c & 3] += p0 + p1;
+                    const float2 xa = split_f32x2(ffma_f32x2(
+                        f32x2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nm2));
+                    const float p0 = fast_exp2(xa.x), p1 = fast_exp2(xa.y);
+                    ps[c & 3] = fadd_f32x2(ps[c & 3], f32x2(p0, p1));
                     pk[c] = pack_bf16(p0, p1);
                 }
-                l = l * alpha + ((ps[0] + ps[1]) + (ps[2] + ps[3]));
+                const float2 psum = split_f32x2(fadd_f32x2(fadd_f32x2(ps[0], ps[1]), fadd_f32x2(ps[2], ps[3])));
+                l = l * alpha + (psum.x + psum.y);
                 const int pb = j & 1;
                 if (j >= 2) {
                     // P buffer pb was last read by PV_{j-2}.
@@ -513,17 +556,23 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         }
     }
 
-    // ---------------------------------------------- this CTA's partial rows
-    // Every MMA has completed once the final o_done phase (or the drain in the
-    // MMA thread) is observed; the P/K/V area is then reused for the rows.
+    // ------------------------------------------- exchange partial rows via L2
+    // Each CTA writes its rows' normalised partial o = O / l (bf16) and
+    // lse = m + log2(l) (fp32) to the workspace; after the cluster barrier
+    // CTA `rank` reduces rows [rank * Rc, (rank + 1) * Rc) over the C
+    // partials (read through L2, all loads of a row in flight at once).
+    int w = 0;
     if (warp >= 2) {
-        int w = ok && nblk > 0 ? 1 : 0;
+        w = ok && nblk > 0 ? 1 : 0;
         if (w && lane == 0)
             w = mbar_wait(&o_done[(nblk - 1) & 1], (uint32_t)((nblk - 1) >> 1) & 1u, abort);
         w = __shfl_sync(FULL, w, 0);
-        uint8_t* dst = sRed + (size_t)grow * AT_RED_STRIDE;
+        const bool mine = grow < R;
+        const size_t prow = ((size_t)bg * C + rank) * R + (mine ? grow : 0);
+        // Stage the bf16 row in the (now free) P area of this M tile with the
+        // 128-byte swizzle, so that a TMA tensor store writes whole rows.
+        uint8_t* stg = sP + m * AT_QTILE;
         if (w) {
-            __syncwarp();
             tc_fence_after();
             const uint32_t ocol = tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(m * 256 + 128);
             const float inv = 1.0f / l;
@@ -533,63 +582,86 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 tmem_ld32(ocol + c0, ov);
                 tmem_wait_ld();
 #pragma unroll
-                for (int e = 0; e < 32; e += 4)
-                    *reinterpret_cast<float4*>(dst + (c0 + e) * 4) =
-                        make_float4(__uint_as_float(ov[e]) * inv, __uint_as_float(ov[e + 1]) * inv,
-                                    __uint_as_float(ov[e + 2]) * inv, __uint_as_float(ov[e + 3]) * inv);
+                for (int e = 0; e < 32; e += 8) {
+                    const int chunk = (c0 + e) >> 3;   // 16-byte chunk of the 256-byte row
+                    *reinterpret_cast<uint4*>(stg + (chunk >> 3) * AT_QHALF + sw128(row, chunk & 7)) =
+                        make_uint4(
+                            pack_bf16(__uint_as_float(ov[e]) * inv, __uint_as_float(ov[e + 1]) * inv),
+                            pack_bf16(__uint_as_float(ov[e + 2]) * inv, __uint_as_float(ov[e + 3]) * inv),
+                            pack_bf16(__uint_as_float(ov[e + 4]) * inv, __uint_as_float(ov[e + 5]) * inv),
+                            pack_bf16(__uint_as_float(ov[e + 6]) * inv, __uint_as_float(ov[e + 7]) * inv));
+                }
             }
         }
         // lse: -inf for a CTA without blocks, NaN for one that gave up.
-        sLse[grow] = w ? m_used + log2f(l) : (nblk > 0 ? NAN : -INFINITY);
+        if (mine) a.part_ml[prow] = w ? m_used + log2f(l) : (nblk > 0 ? NAN : -INFINITY);
+        fence_proxy_async_smem();
+        named_bar_sync(1, NSM);
+        if (t == 0 && nblk > 0) {
+            // Rows past R fall outside the map's row extent and are not
+            // written; rows of a warp that gave up carry a NaN lse.
+            for (int mm = 0; mm < MT; ++mm) {
+                tma_store_3d(&map_part, sP + mm * AT_QTILE, 0, mm * 128, bg * C + rank);
+                tma_store_3d(&map_part, sP + mm * AT_QTILE + AT_QHALF, 64, mm * 128, bg * C + rank);
+            }
+            bulk_commit();
+            bulk_wait_all();
+            fence_proxy_async_global();
+        }
     }
+    __threadfence();
     tc_fence_before();
-    __syncthreads();
+    cluster_sync();
     tc_fence_after();
     if (warp == 1) tmem_dealloc(tmem, 256 * MT);
 
-    // ------------------------------------------ cluster reduction of the rows
-    cluster_sync();
+    // ----------------------------------------- reduce the rows this CTA owns
     grid_dep_wait();   // the output may be written only after the previous grid
-    {
-        const int R = a.G * a.N;
-        const int Rc = (R + C - 1) / C;
-        const int r_lo = rank * Rc, r_hi = min(R, r_lo + Rc);
-        const uint32_t red_base = smem_u32(sRed);
-        const uint32_t lse_base = smem_u32(sLse);
-        for (int r = r_lo + warp; r < r_hi; r += NTH / 32) {
-            float lse = -INFINITY;
-            if (lane < C) lse = ld_cluster_f32(map_rank(lse_base + (uint32_t)r * 4u, (uint32_t)lane));
-            const bool bad = __any_sync(FULL, lse != lse);
-            const float M = warp_max(lse);
-            const float wt = (lane < C && lse != -INFINITY) ? exp2f(lse - M) : 0.f;
-            const float wsum = warp_sum(wt);
-            // Issue every CTA's slice of the row before consuming any of them.
-            float4 v[16];
-            const uint32_t my = red_base + (uint32_t)r * AT_RED_STRIDE + (uint32_t)lane * 16u;
+    const int r_lo = rank * Rc, n_own = max(0, min(R, r_lo + Rc) - r_lo);
+    const size_t pbase = (size_t)bg * C * R;
+    const __nv_bfloat16* part = static_cast<const __nv_bfloat16*>(a.part_bf16);
+    // Two rows per warp per pass, every load of both rows issued before use.
+    for (int rr0 = warp * 2; rr0 < n_own; rr0 += 2 * (NTH / 32)) {
+        float lse[2];
+        uint2 v[2][16];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int r = r_lo + min(rr0 + u, n_own - 1);
+            lse[u] = lane < C ? __ldcg(a.part_ml + pbase + (size_t)lane * R + r) : -INFINITY;
 #pragma unroll
             for (int q = 0; q < 16; ++q)
-                if (q < C) v[q] = ld_cluster_v4(map_rank(my, (uint32_t)q));
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (q < C)
+                    v[u][q] = __ldcg(reinterpret_cast<const uint2*>(part + (pbase + (size_t)q * R + r) * 128) + lane);
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            if (rr0 + u >= n_own) break;
+            const int r = r_lo + rr0 + u;
+            const bool bad = __any_sync(FULL, lse[u] != lse[u]);
+            const float M = warp_max(lse[u]);
+            const float wt = (lane < C && lse[u] != -INFINITY) ? exp2f(lse[u] - M) : 0.f;
+            const float wsum = warp_sum(wt);
+            float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int q = 0; q < 16; ++q) {
                 const float wq = __shfl_sync(FULL, wt, q);   // 0 for q >= C and empty CTAs
                 if (q < C && wq != 0.f) {
-                    acc.x += wq * v[q].x;
-                    acc.y += wq * v[q].y;
-                    acc.z += wq * v[q].z;
-                    acc.w += wq * v[q].w;
+                    const float2 lo = unpack_bf16(v[u][q].x), hi = unpack_bf16(v[u][q].y);
+                    acc[0] += wq * lo.x;
+                    acc[1] += wq * lo.y;
+                    acc[2] += wq * hi.x;
+                    acc[3] += wq * hi.y;
                 }
             }
             const float inv = bad ? NAN : 1.0f / wsum;
             const int i = r / a.G, h = g * a.G + r % a.G;
             __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out) + (((size_t)b * a.N + i) * a.Hq + h) * 128;
             uint2 pk;
-            pk.x = pack_bf16(acc.x * inv, acc.y * inv);
-            pk.y = pack_bf16(acc.z * inv, acc.w * inv);
+            pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+            pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
             reinterpret_cast<uint2*>(o)[lane] = pk;
         }
     }
-    cluster_sync();   // no CTA leaves while another may still read its rows
 }
 
 // ----------------------------------------------------------------- host side
@@ -623,9 +695,31 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G) {
     return GV_OK;
 }
 
+// 3-D map over the bf16 partial rows [B*Hkv*16][R][128] with box
+// {64 d, 128 rows, 1}: rows of a 128-row store past R are clipped.
+static int make_map_part(CUtensorMap* map, void* part, int R, int units) {
+    EncodeTiledFn enc = tensor_map_encoder();
+    if (!enc) {
+        set_error("cuTensorMapEncodeTiled unavailable");
+        return GV_ERR_CUDA;
+    }
+    cuuint64_t dims[3] = {128, (cuuint64_t)R, (cuuint64_t)units * 16};
+    cuuint64_t strides[2] = {256, (cuuint64_t)R * 256};
+    cuuint32_t box[3] = {64, 128, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, part, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        set_error("cuTensorMapEncodeTiled (partials) failed (%d)", (int)r);
+        return GV_ERR_CUDA;
+    }
+    return GV_OK;
+}
+
 static size_t attn_tc_smem(int mt) {
     const int st = mt == 1 ? 4 : 3;
-    return 1024 + (size_t)mt * (AT_QTILE + 2 * AT_PTILE) + (size_t)st * AT_STAGE + 8 * (2 * st + 11) + 16;
+    return 1024 + (size_t)mt * (AT_QTILE + 2 * AT_PTILE) + (size_t)st * AT_STAGE + 8 * (2 * st + 12) + 16;
 }
 
 // CTAs per cluster.  Wanted: enough clusters x CTAs to cover the SMs once
@@ -672,7 +766,7 @@ static int attn_tc_cluster(int units, int S_max, size_t smem) {
 
 template <int MT>
 static int launch_mt(const AttnArgs& a0, const CUtensorMap& mk, const CUtensorMap& mv,
-                     const CUtensorMap& mq, cudaStream_t st) {
+                     const CUtensorMap& mq, const CUtensorMap& mp, cudaStream_t st) {
     const size_t smem = attn_tc_smem(MT);
     auto kern = attn_tc_kernel<MT>;
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -694,7 +788,7 @@ static int launch_mt(const AttnArgs& a0, const CUtensorMap& mk, const CUtensorMa
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mk, mv, mq, a);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mk, mv, mq, mp, a);
     if (e != cudaSuccess) {
         set_error("attn_tc_kernel launch (cluster %d): %s", a.csize, cudaGetErrorString(e));
         return GV_ERR_CUDA;
@@ -703,7 +797,7 @@ static int launch_mt(const AttnArgs& a0, const CUtensorMap& mk, const CUtensorMa
 }
 
 int launch_attn_tc(const AttnArgs& a, cudaStream_t st) {
-    CUtensorMap mk, mv, mq;
+    CUtensorMap mk, mv, mq, mp;
     const uint64_t rows = (uint64_t)a.B * a.Hkv * a.S_max;
     int rc = make_map_2d(&mk, a.cacheK, rows, 128, AT_BK, 256);
     if (rc != GV_OK) return rc;
@@ -711,7 +805,10 @@ int launch_attn_tc(const AttnArgs& a, cudaStream_t st) {
     if (rc != GV_OK) return rc;
     rc = make_map_q(&mq, a.q, a.B * a.N, a.Hq, a.G);
     if (rc != GV_OK) return rc;
-    return (a.R + 127) / 128 == 1 ? launch_mt<1>(a, mk, mv, mq, st) : launch_mt<2>(a, mk, mv, mq, st);
+    rc = make_map_part(&mp, a.part_bf16, a.R, a.B * a.Hkv);
+    if (rc != GV_OK) return rc;
+    return (a.R + 127) / 128 == 1 ? launch_mt<1>(a, mk, mv, mq, mp, st)
+                                  : launch_mt<2>(a, mk, mv, mq, mp, st);
 }
 
 }  // namespace gv

@@ -78,6 +78,7 @@ int lmhead_tc_grid(int slots_capacity);
 
 // ---------------------------------------------------------- attention plan --
 constexpr int KPS_F32 = 256;   // prefix keys per split, CUDA-core path
+constexpr int TC_MAX_CLUSTER = 16;   // largest cluster of the tensor-core attention
 
 struct AttnPlan {
     size_t q_rot, part_o, part_ml, total;
@@ -107,16 +108,23 @@ static AttnPlan attn_plan(const gv_attn_shape* s) {
     p.kps = KPS_F32;
     p.nsplit = (s->S_max + KPS_F32 - 1) / KPS_F32 + 1;
     size_t off = 0;
+    const size_t bh = (size_t)s->B * s->Hkv;
     if (s->dt == GV_F32) {
-        const size_t bh = (size_t)s->B * s->Hkv;
         p.q_rot = off;
         off += align256(bh * p.q_rows_pad * s->d * sizeof(float));
         p.part_o = off;
         off += align256(bh * p.nsplit * R * s->d * sizeof(float));
         p.part_ml = off;
         off += align256(bh * p.nsplit * R * 2 * sizeof(float));
+    } else {
+        // one bf16 partial row and one lse per (cluster CTA, query row); the
+        // cluster holds at most TC_MAX_CLUSTER CTAs
+        p.part_o = off;
+        off += align256(bh * TC_MAX_CLUSTER * R * s->d * 2);
+        p.part_ml = off;
+        off += align256(bh * TC_MAX_CLUSTER * R * sizeof(float));
     }
-    p.total = off > 0 ? off : 256;
+    p.total = off;
     return p;
 }
 
@@ -252,6 +260,7 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
     a.out = out;
     a.q_rot = ws + plan.q_rot;
     a.part_o = reinterpret_cast<float*>(ws + plan.part_o);
+    a.part_bf16 = ws + plan.part_o;
     a.part_ml = reinterpret_cast<float*>(ws + plan.part_ml);
     a.nsplit = plan.nsplit;
     a.kps = plan.kps;
