@@ -34,6 +34,10 @@ from paper_2502_11018_gb300 import gv, inputs  # noqa: E402
 
 METRIC = "verify steps/s and accepted tok/s (LLaMA-3-8B shape, 60-node tree); % HBM roofline"
 UNIT = "verify_steps/s"
+# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one
+# ncu capture of the kernel as it is now, keyed by (kernel, workload); a kernel
+# changed since its capture has no entry.
+TRAFFIC = {}
 
 
 def load_peaks():
@@ -66,6 +70,27 @@ def step_bytes(cfg, accept_len):
     compact = 2 * 2 * int(sum(accept_len)) * Hkv * d * es * L   # K,V rows read + written
     return {"attention": attn, "lmhead": lm, "compact": compact,
             "total": attn + lm + compact + B * N * 64}
+
+
+def attention_bytes(cfg):
+    """Algorithmic HBM bytes of one gv_verify_attention launch (one layer):
+    the prefix K/V read once, the tree's q/k/v read, the output and the rotated
+    tree K/V written, plus the per-node RoPE rows and ancestor masks."""
+    es = 2 if cfg["dtype"] == "bf16" else 4
+    B, N, Hq, Hkv, d = cfg["B"], cfg["N"], cfg["Hq"], cfg["Hkv"], cfg["d"]
+    b = sum(2 * P * Hkv * d * es for P in cfg["P"])
+    b += B * N * (Hq + 2 * Hkv) * d * es                  # q, k_new, v_new
+    b += B * N * Hq * d * es + 2 * B * N * Hkv * d * es    # out, tree K/V
+    b += B * N * (d // 2) * 2 * 4 + B * N * 8              # RoPE rows, ancestor masks
+    return b
+
+
+def launches_per_step(cfg):
+    """Kernels of this library one step launches: tree build, RoPE table, the
+    attention layers (one kernel each on the bf16 tensor-core path, rotate +
+    split + combine on the fp32 path), LM head + merge, accept, compaction."""
+    per_layer = 1 if cfg["dtype"] == "bf16" else 3
+    return 2 + per_layer * cfg["L"] + 2 + 1 + 1
 
 
 def lmhead_bytes(cfg):
@@ -264,8 +289,8 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--config", default="llama3_8b", choices=sorted(inputs.CONFIGS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--seed", type=int, default=1000)
@@ -326,10 +351,23 @@ def main():
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         t_max = float(t.item())
 
-    # Dominant kernel (LM head) timed alone on its own launch stream.
+    # The two kernels that dominate the step, each timed alone on the stream
+    # it is launched on: the LM head, and the attention layers in order (the
+    # 32 layers' caches cycle through far more than L2 holds).
     lm_ms = event_time_ms(step.lmhead, 20, stream)
+    L = cfg["L"]
+    attn_ms = event_time_ms(lambda: [step.attention(l) for l in range(L)], 5, stream) / L
     peaks = load_peaks()
     lm_gbs = lmhead_bytes(cfg) / (lm_ms * 1e-3) / 1e9
+    attn_gbs = attention_bytes(cfg) / (attn_ms * 1e-3) / 1e9
+    kernels = {
+        "lmhead_select": {"ms_per_launch": lm_ms, "launches_per_step": 1,
+                          "algorithmic_bytes": lmhead_bytes(cfg), "achieved_gbs": lm_gbs},
+        "verify_attention": {"ms_per_launch": attn_ms, "launches_per_step": L,
+                             "algorithmic_bytes": attention_bytes(cfg), "achieved_gbs": attn_gbs},
+    }
+    dom = max(kernels, key=lambda k: kernels[k]["ms_per_launch"] * kernels[k]["launches_per_step"])
+    dk = kernels[dom]
     sb = step_bytes(cfg, accept_len)
     step_gbs = sb["total"] / (t_max * 1e-3) / 1e9
 
@@ -337,7 +375,6 @@ def main():
     # copied in, step, result read back, every step.
     e2e = e2e_measure(step, inp, args.e2e_steps, stream)
 
-    launches_per_step = 1 + 3 * cfg["L"] + 2 + 1 + 1
     line = {
         "metric": METRIC, "value": world * 1000.0 / t_max, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max,
@@ -354,10 +391,12 @@ def main():
         "hbm_roofline": {"step_bytes": sb["total"], "achieved_gbs": step_gbs,
                          "peak_gbs": peaks["hbm_gbs"], "frac": step_gbs / peaks["hbm_gbs"],
                          "peak_source": peaks["source"]},
-        "roofline": {"kernel": "lmhead_select", "bound": "hbm", "achieved": lm_gbs,
-                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": lm_gbs / peaks["hbm_gbs"],
-                     "traffic": None, "ms_per_launch": lm_ms},
-        "gpu_launches": launches_per_step * args.steps,
+        "roofline": {"kernel": dom, "bound": "hbm", "achieved": dk["achieved_gbs"],
+                     "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": dk["achieved_gbs"] / peaks["hbm_gbs"], "traffic": TRAFFIC.get((dom, cfg["name"])),
+                     "ms_per_launch": dk["ms_per_launch"], "peak_source": peaks["source"]},
+        "kernels": kernels,
+        "gpu_launches": launches_per_step(cfg) * args.steps,
         "e2e": e2e,
         "clocks": clk,
     }
@@ -374,12 +413,19 @@ def run_kernel_only(args, cfg, dev):
     """Time one call of the verify path alone (one layer for attention), on a
     workload whose inputs hold only that call's tensors."""
     from paper_2502_11018_gb300.step import VerifyStep
-    layers = 1
+    # Attention cycles through all layers so that its caches are read from HBM.
+    layers = 1 if args.kernel == "lmhead" else cfg["L"]
     inp = inputs.make_step_inputs(cfg, args.seed, device=dev, layers=layers)
     step = VerifyStep(inp)
     step.tree()
     stream = torch.cuda.current_stream()
-    fn = step.lmhead if args.kernel == "lmhead" else (lambda: step.attention(0))
+    it = [0]
+
+    def attn():
+        step.attention(it[0] % layers)
+        it[0] += 1
+
+    fn = step.lmhead if args.kernel == "lmhead" else attn
     for _ in range(args.warmup):
         fn()
     torch.cuda.synchronize()
@@ -389,8 +435,7 @@ def run_kernel_only(args, cfg, dev):
     else:
         es = 2 if cfg["dtype"] == "bf16" else 4
         B, N, Hq, Hkv, d = cfg["B"], cfg["N"], cfg["Hq"], cfg["Hkv"], cfg["d"]
-        nbytes = sum(2 * P * Hkv * d * es for P in cfg["P"])
-        nbytes += B * N * (2 * Hq + 4 * Hkv) * d * es
+        nbytes = attention_bytes(cfg)
     peaks = load_peaks()
     gbs = nbytes / (ms * 1e-3) / 1e9
     print(json.dumps({"kernel": args.kernel, "workload": cfg["name"], "ms_per_call": ms,

@@ -58,6 +58,11 @@ constexpr int AT_PTILE = 128 * 128;         // one M tile of P: 128 rows x 64 ke
 constexpr int AT_KV_HALF = AT_BK * 128;     // 64 keys x 64 d bf16 (one swizzle sub-tile)
 constexpr int AT_STAGE = 4 * AT_KV_HALF;    // K (2 halves) + V (2 halves)
 
+// Makes generic-proxy shared-memory writes visible to the async proxy (the
+// tensor cores and TMA).  Writes of other threads are covered when they are
+// ordered before the fence by a barrier (__syncwarp, bar.sync), so each
+// hand-off below fences once, in the thread that signals, after the barrier:
+// the fence costs grow with the number of threads that execute it.
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -208,7 +213,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             mbar_init(&o_done[c], 1);
         }
         mbar_init(q_raw, 1);
-        mbar_init(q_full, 4 * MT);
+        mbar_init(q_full, 1);
         mbar_init(drain, 1);
         mbar_init(rope_full, 1);
         *abort = 0;
@@ -393,9 +398,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     *reinterpret_cast<uint4*>(st + 2 * AT_KV_HALF + sw128(j, c)) = vlo;
                     *reinterpret_cast<uint4*>(st + 3 * AT_KV_HALF + sw128(j, c)) = vhi;
                 }
-                fence_proxy_async_smem();
                 named_bar_sync(1, NSM);
-                if (t == 0) mbar_arrive(&kv_full[0]);
+                if (t == 0) {
+                    fence_proxy_async_smem();
+                    mbar_arrive(&kv_full[0]);
+                }
             }
             // RoPE of this thread's Q row, in place once the raw tile has landed.
             {
@@ -419,9 +426,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         *phi = ohi;
                     }
                 }
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(q_full);
+                named_bar_sync(1, NSM);
+                if (t == 0) {
+                    fence_proxy_async_smem();
+                    mbar_arrive(q_full);
+                }
             }
             const float sl2 = a.scale * 1.4426950408889634f;     // scale * log2(e)
             for (int j = 0; j < nblk; ++j) {
@@ -548,10 +557,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         }
                     }
                 }
-                fence_proxy_async_smem();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&p_full[pb]);
+                if (lane == 0) {
+                    fence_proxy_async_smem();
+                    mbar_arrive(&p_full[pb]);
+                }
             }
         }
     }
@@ -595,9 +606,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         }
         // lse: -inf for a CTA without blocks, NaN for one that gave up.
         if (mine) a.part_ml[prow] = w ? m_used + log2f(l) : (nblk > 0 ? NAN : -INFINITY);
-        fence_proxy_async_smem();
         named_bar_sync(1, NSM);
         if (t == 0 && nblk > 0) {
+            fence_proxy_async_smem();
             // Rows past R fall outside the map's row extent and are not
             // written; rows of a warp that gave up carry a NaN lse.
             for (int mm = 0; mm < MT; ++mm) {
