@@ -37,7 +37,10 @@ UNIT = "verify_steps/s"
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one
 # ncu capture of the kernel as it is now, keyed by (kernel, workload); a kernel
 # changed since its capture has no entry.
-TRAFFIC = {}
+TRAFFIC = {
+    # profiles/attn_tc_llama3_8b_layer.md
+    ("verify_attention", "llama3_8b"): 17630720,
+}
 
 
 def load_peaks():
@@ -250,6 +253,16 @@ def sample_size(cfg, est_full, budget_s):
     return ls, vs
 
 
+def bench_config(cfg, world):
+    """The `config` object of the JSON line (both arms)."""
+    return {"workload": cfg["name"], "batch": cfg["B"], "layers": cfg["L"],
+            "hidden": cfg["H"], "heads_q": cfg["Hq"], "heads_kv": cfg["Hkv"],
+            "head_dim": cfg["d"], "vocab": cfg["V"], "prefix": list(cfg["P"]),
+            "tree_nodes": cfg["N"], "tree_depth": cfg["D"],
+            "temperature": cfg.get("temperature", 0.0),
+            "l2": "working set above L2 (no flush needed)", "parallelism": f"replicas{world}"}
+
+
 def run_reference(args):
     """The reference arm: the float64 oracle on the host cores, each step a
     bounded sample of the workload sized so the whole run takes a few minutes."""
@@ -277,8 +290,7 @@ def run_reference(args):
             "warmup": args.warmup, "ms_per_step": 1000.0 * statistics.mean(vals),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded random weights, caches and draft trees)", "impl": "reference",
-            "config": {"workload": cfg["name"], "batch": cfg["B"], "layers": cfg["L"],
-                       "prefix": list(cfg["P"]), "tree_nodes": cfg["N"], "vocab": cfg["V"]},
+            "config": bench_config(cfg, args.gpus),
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                              "sample": desc},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -380,12 +392,7 @@ def main():
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg["dtype"],
         "data": "synthetic (seeded random weights, caches and draft trees)",
-        "config": {"workload": cfg["name"], "batch": cfg["B"], "layers": cfg["L"],
-                   "hidden": cfg["H"], "heads_q": cfg["Hq"], "heads_kv": cfg["Hkv"],
-                   "head_dim": cfg["d"], "vocab": cfg["V"], "prefix": list(cfg["P"]),
-                   "tree_nodes": cfg["N"], "tree_depth": cfg["D"],
-                   "temperature": cfg.get("temperature", 0.0),
-                   "l2": "working set above L2 (no flush needed)", "parallelism": f"replicas{world}"},
+        "config": bench_config(cfg, world),
         "accepted_tok_per_s": world * sum(accept_len) * 1000.0 / t_max,
         "accept_len": accept_len,
         "hbm_roofline": {"step_bytes": sb["total"], "achieved_gbs": step_gbs,

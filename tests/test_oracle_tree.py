@@ -6,11 +6,13 @@ from the root that propagates ancestor sets to children), and against the
 validity rules of the parent-array encoding.
 """
 
+import os
+
 import numpy as np
 import pytest
 
 import oracle
-from oracle.tree import tree_build, GV_ERR_INVALID_TREE
+from oracle.tree import tree_build, GV_OK, GV_ERR_INVALID_TREE
 from paper_2502_11018_gb300 import inputs
 
 
@@ -118,3 +120,31 @@ def test_generator_tree_shape():
             kids = [int(tokens[c]) for c in range(1, N) if parents[c] == u]
             assert len(kids) == len(set(kids))
     assert oracle.GV_OK == 0
+
+
+def _golden(name):
+    path = os.path.join(os.path.dirname(__file__), "golden", name)
+    vals = {}
+    with open(path) as f:
+        for line in f:
+            line = line.split("#", 1)[0].split()
+            if len(line) == 2:
+                vals[line[0]] = int(line[1])
+    return vals
+
+
+def test_paper_tree_configuration():
+    """The tree size and depth the paper prints (Appendix, draft tree
+    structure) yield, through the generator and the oracle, a valid tree of
+    exactly that many nodes whose deepest node sits at that depth, with
+    positions P + depth and one ancestor bit per level."""
+    g = _golden("draft_tree_config.txt")
+    N, D = g["draft_tokens"], g["depth"]
+    rng = np.random.default_rng(11)
+    parents, _ = inputs.make_tree(rng, N, D, 10, 32000)
+    P = 37
+    depth, pos, anc, st = tree_build(parents[None], [P])
+    assert st[0] == GV_OK and parents.shape == (N,)
+    assert depth.max() == D
+    np.testing.assert_array_equal(pos[0], P + depth[0])
+    assert all(bin(int(a)).count("1") == int(dd) + 1 for a, dd in zip(anc[0], depth[0]))
