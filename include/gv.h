@@ -163,12 +163,39 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
  *                          row_lse fp32[rows] = max + log(sum exp(l - max)).
  *   Unused outputs may be NULL.
  *   workspace >= gv_lmhead_workspace(rows, H, V, dt, mode, k) bytes.
- * H must be a multiple of 64 (bf16) or 4 (fp32); rows >= 1.
+ * H must be a multiple of 8 (bf16) or 4 (fp32); rows >= 1.
  */
 size_t gv_lmhead_workspace(int rows, int H, int V, int dt, int mode, int k);
 int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int dt, int mode,
                      int k, int32_t* ids, float* vals, float* logits, float* row_max,
                      float* row_lse, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * gv_lmhead_argmax_noalloc -- gv_lmhead_select(mode GV_SELECT_ARGMAX, bf16)
+ * without a workspace argument.  The paper has no counterpart: it exists for
+ * callers that cannot allocate or hold device memory of their own for
+ * scratch, e.g. an embedding runtime whose memory is fixed once at start-up,
+ * or a caller outside PyTorch's allocator that has only the inputs and
+ * outputs.  Same arithmetic and kernels as gv_lmhead_select; ids/vals equal.
+ *
+ *   h [rows][H] bf16, W [V][H] bf16, ids int32[rows], vals fp32[rows] (may
+ *   be NULL); 1 <= rows <= GV_NOALLOC_MAX_ROWS, H a multiple of 8.
+ *
+ * Scratch: a fixed 512 KB + 256 B array in the library's own device memory
+ * (a file-scope __device__ array, one per device, reserved when the library
+ * is loaded): per-CTA argmax partials of up to GV_NOALLOC_MAX_ROWS rows and
+ * an error word, which each call zeroes on the stream before its kernels.
+ * The first call on a device looks the array's address up
+ * (cudaGetSymbolAddress) and caches it; make that first call before any
+ * stream capture.  Nothing is allocated by any call.
+ * rows > GV_NOALLOC_MAX_ROWS returns GV_ERR_UNSUPPORTED (message in
+ * gv_last_error()), before anything is enqueued.
+ * Calls that overlap in time on one device (different streams, or host
+ * threads without ordering) share the scratch and race: serialise them.
+ */
+#define GV_NOALLOC_MAX_ROWS 256
+int gv_lmhead_argmax_noalloc(const void* h, const void* W, int rows, int H, int V,
+                             int32_t* ids, float* vals, void* stream);
 
 /*
  * gv_accept -- accept the longest verified root chain of each tree.

@@ -5,6 +5,7 @@
 #include <cstdio>
 #include <cstring>
 #include <cmath>
+#include <mutex>
 
 #include "gv_internal.cuh"
 #include "attention.cuh"
@@ -155,6 +156,47 @@ static LmPlan lm_plan(int rows, int V, int dt, int mode, int k) {
     off += 256;
     p.total = off;
     return p;
+}
+
+// ------------------------------------------- allocation-free LM head scratch --
+// gv_lmhead_argmax_noalloc keeps its scratch in the library's own device
+// memory: the argmax partials (value, id) of up to GV_NOALLOC_MAX_ROWS rows
+// for up to TC_SLOTS CTAs, then the error word of the bounded waits.
+constexpr size_t NOALLOC_ENTRIES = (size_t)TC_SLOTS * GV_NOALLOC_MAX_ROWS;
+constexpr size_t NOALLOC_ID_OFF = NOALLOC_ENTRIES * sizeof(float);
+constexpr size_t NOALLOC_ERR_OFF = NOALLOC_ID_OFF + NOALLOC_ENTRIES * sizeof(int);
+constexpr size_t NOALLOC_BYTES = NOALLOC_ERR_OFF + 256;
+__device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_BYTES];
+
+constexpr int NOALLOC_MAX_DEVICES = 64;
+static std::mutex g_noalloc_mu;
+static void* g_noalloc_addr[NOALLOC_MAX_DEVICES];
+
+// Address of the scratch on the current device, looked up once per device.
+static int noalloc_scratch(char** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) {
+        set_error("gv_lmhead_argmax_noalloc: cudaGetDevice: %s", cudaGetErrorString(e));
+        return GV_ERR_CUDA;
+    }
+    if (dev < 0 || dev >= NOALLOC_MAX_DEVICES) {
+        set_error("gv_lmhead_argmax_noalloc: device %d beyond the %d supported", dev,
+                  NOALLOC_MAX_DEVICES);
+        return GV_ERR_UNSUPPORTED;
+    }
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_addr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || !p) {
+            set_error("gv_lmhead_argmax_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+            return GV_ERR_CUDA;
+        }
+        g_noalloc_addr[dev] = p;
+    }
+    *out = static_cast<char*>(g_noalloc_addr[dev]);
+    return GV_OK;
 }
 
 }  // namespace gv
@@ -322,6 +364,39 @@ int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int d
     int rc = launch_lmhead_tc(h, W, rows, H, V, mode, plan.K, logits, part, err, st);
     if (rc != GV_OK) return rc;
     return launch_lmhead_merge(part, mode, plan.K, ids, vals, row_max, row_lse, err, st);
+}
+
+int gv_lmhead_argmax_noalloc(const void* h, const void* W, int rows, int H, int V, int32_t* ids,
+                             float* vals, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(rows >= 1 && H >= 1 && V >= 1, "gv_lmhead_argmax_noalloc: rows=%d H=%d V=%d",
+                 rows, H, V);
+    if (rows > GV_NOALLOC_MAX_ROWS) {
+        set_error("gv_lmhead_argmax_noalloc: rows=%d exceeds the fixed scratch (at most %d rows); "
+                  "use gv_lmhead_select with a workspace", rows, GV_NOALLOC_MAX_ROWS);
+        return GV_ERR_UNSUPPORTED;
+    }
+    GV_CHECK_ARG(h && W && aligned16(h) && aligned16(W),
+                 "gv_lmhead_argmax_noalloc: h/W null or not 16-byte aligned");
+    GV_CHECK_ARG(ids, "gv_lmhead_argmax_noalloc: ids output is null");
+    GV_CHECK_ARG(H % 8 == 0, "gv_lmhead_argmax_noalloc: H %% 8 != 0 (16-byte rows), H=%d", H);
+    char* ws = nullptr;
+    int rc = noalloc_scratch(&ws);
+    if (rc != GV_OK) return rc;
+    SelectPartials part;
+    part.val = reinterpret_cast<float*>(ws);
+    part.id = reinterpret_cast<int*>(ws + NOALLOC_ID_OFF);
+    part.m = nullptr;     // read and written only in GV_SELECT_LOGITS mode
+    part.s = nullptr;
+    part.slots = lmhead_tc_grid(TC_SLOTS);   // <= TC_SLOTS, so slots * rows fits
+    part.rows = rows;
+    part.K = 1;
+    int* err = reinterpret_cast<int*>(ws + NOALLOC_ERR_OFF);
+    cudaStream_t st = as_stream(stream);
+    if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return check_launch("memset");
+    rc = launch_lmhead_tc(h, W, rows, H, V, GV_SELECT_ARGMAX, 1, nullptr, part, err, st);
+    if (rc != GV_OK) return rc;
+    return launch_lmhead_merge(part, GV_SELECT_ARGMAX, 1, ids, vals, nullptr, nullptr, err, st);
 }
 
 size_t gv_accept_workspace(int B, int V, float temperature) {

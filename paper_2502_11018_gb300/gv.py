@@ -32,7 +32,8 @@ GV_SELECT_LOGITS = 2
 
 # Every symbol include/gv.h declares.
 EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "gv_verify_attention",
-           "gv_lmhead_workspace", "gv_lmhead_select", "gv_accept_workspace", "gv_accept",
+           "gv_lmhead_workspace", "gv_lmhead_select", "gv_lmhead_argmax_noalloc",
+           "gv_accept_workspace", "gv_accept",
            "gv_kv_compact", "gv_status_string", "gv_last_error", "gv_version")
 
 
@@ -72,6 +73,7 @@ def lib():
         "gv_lmhead_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
         "gv_lmhead_select": ([_vp, _vp, _i, _i, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp,
                               _sz, _vp], _i),
+        "gv_lmhead_argmax_noalloc": ([_vp, _vp, _i, _i, _i, _vp, _vp, _vp], _i),
         "gv_accept_workspace": ([_i, _i, _f], _sz),
         "gv_accept": ([_i, _i, _i, _i, _f] + [_vp] * 12 + [_vp, _sz, _vp], _i),
         "gv_kv_compact": ([_i] * 8 + [_vp] * 9 + [_vp], _i),
@@ -172,6 +174,20 @@ def gv_lmhead_select(h, W, mode, k, ids, vals, logits, row_max, row_lse, workspa
         _ptr(vals, "vals"), _ptr(logits, "logits"), _ptr(row_max, "row_max"),
         _ptr(row_lse, "row_lse"), _ptr(workspace, "workspace"),
         workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+GV_NOALLOC_MAX_ROWS = 256
+
+
+def gv_lmhead_argmax_noalloc(h, W, ids, vals=None, stream=None):
+    """Argmax LM head (bf16) that takes no workspace: its scratch is a fixed
+    array inside the library (rows <= GV_NOALLOC_MAX_ROWS; calls that overlap
+    in time on one device race)."""
+    rows, H = h.shape
+    V = W.shape[0]
+    return _check("gv_lmhead_argmax_noalloc", lib().gv_lmhead_argmax_noalloc(
+        _ptr(h, "h"), _ptr(W, "W"), rows, H, V, _ptr(ids, "ids"), _ptr(vals, "vals"),
+        _stream(stream)))
 
 
 def gv_accept_workspace(B, V, temperature):

@@ -56,6 +56,11 @@ def test_host_side_validation(lib):
     assert gv.gv_verify_attention_workspace(shape) == 0     # Hq not a multiple of Hkv
     assert lib.gv_rope_table(nul, 1, 60, 128, 1e4, nul, nul) == gv.GV_ERR_ARG
     assert lib.gv_lmhead_select(nul, nul, 60, 4096, 1000, 0, 1, 17, *([nul] * 6), 0, nul) == gv.GV_ERR_ARG
+    # The allocation-free argmax rejects row counts beyond its fixed scratch.
+    assert lib.gv_lmhead_argmax_noalloc(16, 16, gv.GV_NOALLOC_MAX_ROWS + 1, 4096, 1000, 16, nul,
+                                        nul) == gv.GV_ERR_UNSUPPORTED
+    assert "exceeds the fixed scratch" in gv.last_error()
+    assert lib.gv_lmhead_argmax_noalloc(nul, nul, 60, 4096, 1000, nul, nul, nul) == gv.GV_ERR_ARG
     assert lib.gv_accept(1, 60, 6, 0, -1.0, *([nul] * 12), nul, 0, nul) == gv.GV_ERR_ARG
     assert lib.gv_kv_compact(1, 1, 60, 6, 8, 3, 100, 0, *([nul] * 9), nul) == gv.GV_ERR_ARG
     assert "16-byte" in gv.last_error()
