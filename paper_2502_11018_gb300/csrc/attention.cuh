@@ -24,14 +24,13 @@ struct AttnArgs {
     void* treeV;
     void* out;
     // workspace pieces
-    void* q_rot;      // [B*Hkv][q_rows_pad][d]  rotated queries (fp32 or bf16)
-    float* part_o;    // [B*Hkv][nsplit][R][d]   per-split partial outputs
-    float* part_ml;   // [B*Hkv][nsplit][R][2] (m, l) on the CUDA-core path,
-                      // [B*Hkv][C][R] log2-sum-exp on the tensor-core path
-    void* part_bf16;  // [B*Hkv][C][R][d] bf16 normalised partial rows (tensor-core path)
+    void* q_rot;      // [B*Hkv][q_rows_pad][d]  rotated queries          (CUDA-core path)
+    float* part_o;    // [B*Hkv][nsplit][R][d]   per-split partial outputs (CUDA-core path)
+    float* part_ml;   // [B*Hkv][nsplit][R][2] (m, l)                  (CUDA-core path)
     int nsplit;       // prefix splits + 1 tree split (CUDA-core path)
     int kps;          // prefix keys per split (CUDA-core path)
-    int csize;        // CTAs per cluster, one cluster per (sequence, KV head) (tensor-core path)
+    int csize;        // CTAs per cluster (tensor-core path)
+    int tiles;        // clusters per (sequence, KV head), each on its own group of query rows
 };
 
 int launch_rope_table(const int32_t* pos, int B, int N, int d, float base, float* rope,

@@ -25,15 +25,17 @@
 //                          always share one max), writes P = exp2(s - m) as
 //                          bf16 to one of two smem buffers
 //   O += P_j V_j           tcgen05.mma, P K-major, V MN-major (d contiguous)
-// Each CTA then writes o = O / l (bf16) and lse = m + log2(l) of its rows to
-// the workspace (they stay in L2); after a cluster barrier every CTA reduces
-// a 1/C share of the rows over the cluster's C partials and writes the final
-// bf16 output, so the split combine needs no extra launch.
+// Each CTA then stages o = O / l (bf16) and lse = m + log2(l) of its rows in
+// its shared memory; after a cluster barrier it pushes to every CTA of the
+// cluster (bulk copies into distributed shared memory) the 1/C share of rows
+// that CTA merges, and every CTA merges its share over the C partials and
+// writes the final bf16 output: the split combine needs no extra launch and
+// no global scratch.
 //
 // Warp roles: warp 0 issues the TMA loads (K/V blocks, raw Q tiles); warp 1
 // owns TMEM and issues the MMAs; warps 2.. (4 per M tile) rotate Q in place
 // (RoPE from the per-step table), build the tree K/V tile, and run the
-// softmax and the epilogue; all warps share the cluster reduction.
+// softmax and the epilogue; all warps share the merge.
 //
 // Launch: cluster launch (the cluster barrier orders the partial exchange and
 // guarantees the C CTAs are co-resident) with programmatic dependent launch.
@@ -151,14 +153,17 @@ __device__ __forceinline__ void rope8(const uint4& lo, const uint4& hi, const fl
 template <int MT>
 __global__ void __launch_bounds__(64 + 128 * MT, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
-               const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_part,
-               AttnArgs a) {
+               const __grid_constant__ CUtensorMap map_q, AttnArgs a) {
     constexpr int NSM = 128 * MT;            // softmax threads
     constexpr int NTH = 64 + NSM;            // all threads
     constexpr int ST = MT == 1 ? 4 : 3;      // K/V stages
     const int C = a.csize;
     const int rank = (int)cluster_rank();
-    const int bg = blockIdx.x / C;
+    // Cluster -> (sequence b, KV head g, first M tile): the G * N query rows of
+    // (b, g) are cut into groups of MT tiles of 128, one cluster per group.
+    const int cl = blockIdx.x / C;
+    const int bg = cl / a.tiles;
+    const int tile0 = (cl % a.tiles) * MT;
     const int b = bg / a.Hkv, g = bg % a.Hkv;
     // prefix_len is a step input written before the previous kernel in the
     // stream started, so it may be read before griddepcontrol.wait.
@@ -169,8 +174,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     const bool has_tree = rank == C - 1;
     const int nblk = (nb_pre > rank ? (nb_pre - 1 - rank) / C + 1 : 0) + (has_tree ? 1 : 0);
     const int nb_per_tile = 128 / a.G;                   // nodes per M tile
-    const int R = a.G * a.N;                             // query rows of (b, g)
-    const int Rc = (R + C - 1) / C;                      // rows each CTA reduces
+    const int row0 = tile0 * 128;                        // first query row of this cluster
+    const int R = min(a.G * a.N - row0, MT * 128);       // query rows of this cluster
+    const int Rc = (R + C - 1) / C;                      // rows each CTA merges
+    const int slab_bytes = Rc * 256 + ((Rc + 3) & ~3) * 4;   // Rc bf16 rows + Rc lse (16-byte multiple)
+    const int r_own = min(R, rank * Rc + Rc) - rank * Rc;    // rows this CTA merges (<= 0: none)
     // Prefix block index of this CTA's j-th block (-1 for the tree block).
     auto prefix_block = [&](int j) -> int {
         if (has_tree) return j == 0 ? -1 : rank + C * (j - 1);
@@ -194,7 +202,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint64_t* q_full = q_raw + 1;
     uint64_t* drain = q_full + 1;
     uint64_t* rope_full = drain + 1;
-    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(rope_full + 1);
+    uint64_t* recv_full = rope_full + 1;
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(recv_full + 1);
     // The RoPE rows of sequence b (N x 64 (cos, sin) pairs) are staged in the
     // P area, which is free until the first softmax block writes P.
     const float4* sRope = reinterpret_cast<const float4*>(sP);
@@ -216,11 +225,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         mbar_init(q_full, 1);
         mbar_init(drain, 1);
         mbar_init(rope_full, 1);
+        mbar_init(recv_full, 1);
+        if (r_own > 0) mbar_arrive_expect_tx(recv_full, (uint32_t)(C * slab_bytes));
         *abort = 0;
         fence_mbar_init();
         if (nblk > 0) {
             prefetch_tmap(&map_q);
-            prefetch_tmap(&map_part);
             prefetch_tmap(&map_k);
             prefetch_tmap(&map_v);
         }
@@ -237,9 +247,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     const int m = (warp - 2) >> 2;                       // M tile of this warp
     const int sub = warp & 3;                            // TMEM lane quarter
     const int row = sub * 32 + lane;                     // row inside the M tile
-    const int node = m * nb_per_tile + row / a.G;        // tree node of this row
+    const int node = (tile0 + m) * nb_per_tile + row / a.G;   // tree node of this row
     const bool row_ok = warp >= 2 && node < a.N;
-    const int grow = m * 128 + row;                      // = node * G + head in group
+    const int grow = m * 128 + row;                      // row in the cluster; row0 + grow = node * G + head
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
 
@@ -261,7 +271,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     grid_dep_wait();
                     mbar_arrive_expect_tx(q_raw, MT * AT_QTILE);
                     for (int mm = 0; mm < MT; ++mm) {
-                        const int z = b * a.N + mm * nb_per_tile;
+                        const int z = b * a.N + (tile0 + mm) * nb_per_tile;
                         tma_load_3d(sQ + mm * AT_QTILE, &map_q, q_raw, 0, g * a.G, z, pol_q);
                         tma_load_3d(sQ + mm * AT_QTILE + AT_QHALF, &map_q, q_raw, 64, g * a.G, z, pol_q);
                     }
@@ -376,6 +386,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     const int j = e >> 3, c = e & 7;
                     uint4 klo = make_uint4(0, 0, 0, 0), khi = klo, vlo = klo, vhi = klo;
                     if (j < a.N) {
+                        // (every row group's cluster builds the tile; the first writes the scratch)
                         const size_t src = (((size_t)b * a.N + j) * a.Hkv + g) * 16;
                         const uint4* kr = reinterpret_cast<const uint4*>(a.k_new) + src;
                         const uint4* vr = reinterpret_cast<const uint4*>(a.v_new) + src;
@@ -388,10 +399,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         rope8(k0, k1, cs, klo, khi);
                         uint4* tk = reinterpret_cast<uint4*>(a.treeK) + ((size_t)bg * a.N + j) * 16;
                         uint4* tv = reinterpret_cast<uint4*>(a.treeV) + ((size_t)bg * a.N + j) * 16;
-                        tk[c] = klo;
-                        tk[8 + c] = khi;
-                        tv[c] = vlo;
-                        tv[8 + c] = vhi;
+                        if (tile0 == 0) {
+                            tk[c] = klo;
+                            tk[8 + c] = khi;
+                            tv[c] = vlo;
+                            tv[8 + c] = vhi;
+                        }
                     }
                     *reinterpret_cast<uint4*>(st + sw128(j, c)) = klo;
                     *reinterpret_cast<uint4*>(st + AT_KV_HALF + sw128(j, c)) = khi;
@@ -404,26 +417,35 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     mbar_arrive(&kv_full[0]);
                 }
             }
-            // RoPE of this thread's Q row, in place once the raw tile has landed.
+            // RoPE of this thread's Q row, in place once the raw tile has landed:
+            // all loads of the row first, the rotation in registers, then the
+            // stores (no store sits between two loads, so all loads overlap).
             {
-                int w = 1;
-                if (lane == 0) w = mbar_wait(q_raw, 0, abort);
-                w = __shfl_sync(FULL, w, 0);
+                const int w = mbar_wait(q_raw, 0, abort) ? 1 : 0;   // every lane observes the copy
                 uint8_t* qt = sQ + m * AT_QTILE;
-                if (w && ok) {
+                if (__all_sync(FULL, w) && ok) {
+                    uint4 lo[8], hi[8];
 #pragma unroll
                     for (int c = 0; c < 8; ++c) {
-                        uint4* plo = reinterpret_cast<uint4*>(qt + sw128(row, c));
-                        uint4* phi = reinterpret_cast<uint4*>(qt + AT_QHALF + sw128(row, c));
+                        lo[c] = *reinterpret_cast<const uint4*>(qt + sw128(row, c));
+                        hi[c] = *reinterpret_cast<const uint4*>(qt + AT_QHALF + sw128(row, c));
+                    }
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
                         uint4 olo = make_uint4(0, 0, 0, 0), ohi = olo;
                         if (row_ok) {
                             float4 cs[4];
 #pragma unroll
                             for (int q = 0; q < 4; ++q) cs[q] = sRope[node * 32 + c * 4 + q];
-                            rope8(*plo, *phi, cs, olo, ohi);
+                            rope8(lo[c], hi[c], cs, olo, ohi);
                         }
-                        *plo = olo;
-                        *phi = ohi;
+                        lo[c] = olo;
+                        hi[c] = ohi;
+                    }
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        *reinterpret_cast<uint4*>(qt + sw128(row, c)) = lo[c];
+                        *reinterpret_cast<uint4*>(qt + AT_QHALF + sw128(row, c)) = hi[c];
                     }
                 }
                 named_bar_sync(1, NSM);
@@ -567,112 +589,140 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         }
     }
 
-    // ------------------------------------------- exchange partial rows via L2
-    // Each CTA writes its rows' normalised partial o = O / l (bf16) and
-    // lse = m + log2(l) (fp32) to the workspace; after the cluster barrier
-    // CTA `rank` reduces rows [rank * Rc, (rank + 1) * Rc) over the C
-    // partials (read through L2, all loads of a row in flight at once).
-    int w = 0;
+    // ------------------------------- exchange partial rows through the cluster
+    // Each CTA stages its rows' normalised partial o = O / l (bf16) and
+    // lse = m + log2(l) (fp32) in its own (now free) Q and P areas as C slabs:
+    // slab q holds rows [q * Rc, (q + 1) * Rc), the rows CTA q merges, with
+    // the 16-byte chunks of row k of a slab rotated by (k & 15) so that the
+    // lanes of a warp store and load distinct banks.  After a cluster barrier
+    // (every CTA is past its main loop, so its K/V ring is idle) thread 0
+    // pushes slab q into the K/V ring of CTA q with one bulk shared::cta ->
+    // shared::cluster copy that completes on CTA q's `recv_full` barrier; CTA
+    // q merges its rows over the C slabs it received and writes the output.
+    // lse is -inf for a CTA without blocks and NaN for one that gave up.
+    uint8_t* stg = sQ;
     if (warp >= 2) {
-        w = ok && nblk > 0 ? 1 : 0;
+        int w = ok && nblk > 0 ? 1 : 0;
         if (w && lane == 0)
             w = mbar_wait(&o_done[(nblk - 1) & 1], (uint32_t)((nblk - 1) >> 1) & 1u, abort);
         w = __shfl_sync(FULL, w, 0);
         const bool mine = grow < R;
-        const size_t prow = ((size_t)bg * C + rank) * R + (mine ? grow : 0);
-        // Stage the bf16 row in the (now free) P area of this M tile with the
-        // 128-byte swizzle, so that a TMA tensor store writes whole rows.
-        uint8_t* stg = sP + m * AT_QTILE;
+        const int q = grow / Rc, k = grow - q * Rc;
+        uint8_t* slab = stg + (size_t)q * slab_bytes;
         if (w) {
             tc_fence_after();
             const uint32_t ocol = tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(m * 256 + 128);
             const float inv = 1.0f / l;
 #pragma unroll
-            for (int c0 = 0; c0 < 128; c0 += 32) {
-                uint32_t ov[32];
-                tmem_ld32(ocol + c0, ov);
+            for (int c0 = 0; c0 < 128; c0 += 64) {
+                uint32_t ov[64];
+                tmem_ld32(ocol + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[0]));
+                tmem_ld32(ocol + c0 + 32, *reinterpret_cast<uint32_t(*)[32]>(&ov[32]));
                 tmem_wait_ld();
+                if (mine) {
 #pragma unroll
-                for (int e = 0; e < 32; e += 8) {
-                    const int chunk = (c0 + e) >> 3;   // 16-byte chunk of the 256-byte row
-                    *reinterpret_cast<uint4*>(stg + (chunk >> 3) * AT_QHALF + sw128(row, chunk & 7)) =
-                        make_uint4(
-                            pack_bf16(__uint_as_float(ov[e]) * inv, __uint_as_float(ov[e + 1]) * inv),
-                            pack_bf16(__uint_as_float(ov[e + 2]) * inv, __uint_as_float(ov[e + 3]) * inv),
-                            pack_bf16(__uint_as_float(ov[e + 4]) * inv, __uint_as_float(ov[e + 5]) * inv),
-                            pack_bf16(__uint_as_float(ov[e + 6]) * inv, __uint_as_float(ov[e + 7]) * inv));
+                    for (int e = 0; e < 64; e += 8) {
+                        const int ch = (c0 + e) >> 3;   // 16-byte chunk of the 256-byte row
+                        *reinterpret_cast<uint4*>(slab + k * 256 + ((ch ^ (k & 15)) << 4)) =
+                            make_uint4(
+                                pack_bf16(__uint_as_float(ov[e]) * inv, __uint_as_float(ov[e + 1]) * inv),
+                                pack_bf16(__uint_as_float(ov[e + 2]) * inv, __uint_as_float(ov[e + 3]) * inv),
+                                pack_bf16(__uint_as_float(ov[e + 4]) * inv, __uint_as_float(ov[e + 5]) * inv),
+                                pack_bf16(__uint_as_float(ov[e + 6]) * inv, __uint_as_float(ov[e + 7]) * inv));
+                    }
                 }
             }
         }
-        // lse: -inf for a CTA without blocks, NaN for one that gave up.
-        if (mine) a.part_ml[prow] = w ? m_used + log2f(l) : (nblk > 0 ? NAN : -INFINITY);
-        named_bar_sync(1, NSM);
-        if (t == 0 && nblk > 0) {
-            fence_proxy_async_smem();
-            // Rows past R fall outside the map's row extent and are not
-            // written; rows of a warp that gave up carry a NaN lse.
-            for (int mm = 0; mm < MT; ++mm) {
-                tma_store_3d(&map_part, sP + mm * AT_QTILE, 0, mm * 128, bg * C + rank);
-                tma_store_3d(&map_part, sP + mm * AT_QTILE + AT_QHALF, 64, mm * 128, bg * C + rank);
+        if (mine) {
+            reinterpret_cast<float*>(slab + Rc * 256)[k] =
+                w ? m_used + log2f(l) : (nblk > 0 ? NAN : -INFINITY);
+            if (!w) {
+                // No partial (no blocks, or gave up): zeros, so that the
+                // merge may weight every slab without testing its weight.
+#pragma unroll
+                for (int ch = 0; ch < 16; ++ch)
+                    *reinterpret_cast<uint4*>(slab + k * 256 + (ch << 4)) = make_uint4(0, 0, 0, 0);
             }
-            bulk_commit();
-            bulk_wait_all();
-            fence_proxy_async_global();
         }
     }
-    __threadfence();
     tc_fence_before();
-    cluster_sync();
+    __syncthreads();
     tc_fence_after();
-    if (warp == 1) tmem_dealloc(tmem, 256 * MT);
-
-    // ----------------------------------------- reduce the rows this CTA owns
-    grid_dep_wait();   // the output may be written only after the previous grid
-    const int r_lo = rank * Rc, n_own = max(0, min(R, r_lo + Rc) - r_lo);
-    const size_t pbase = (size_t)bg * C * R;
-    const __nv_bfloat16* part = static_cast<const __nv_bfloat16*>(a.part_bf16);
-    // Two rows per warp per pass, every load of both rows issued before use.
-    for (int rr0 = warp * 2; rr0 < n_own; rr0 += 2 * (NTH / 32)) {
-        float lse[2];
-        uint2 v[2][16];
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int r = r_lo + min(rr0 + u, n_own - 1);
-            lse[u] = lane < C ? __ldcg(a.part_ml + pbase + (size_t)lane * R + r) : -INFINITY;
-#pragma unroll
-            for (int q = 0; q < 16; ++q)
-                if (q < C)
-                    v[u][q] = __ldcg(reinterpret_cast<const uint2*>(part + (pbase + (size_t)q * R + r) * 128) + lane);
+    if (*abort) {
+        // A role gave up, so a copy may have landed in the staging area after
+        // the rows were staged (each role drains its own copies before the
+        // barrier above): mark every row of this CTA invalid again.
+        if (warp >= 2 && grow < R) {
+            const int q = grow / Rc;
+            reinterpret_cast<float*>(stg + (size_t)q * slab_bytes + Rc * 256)[grow - q * Rc] = NAN;
         }
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            if (rr0 + u >= n_own) break;
-            const int r = r_lo + rr0 + u;
-            const bool bad = __any_sync(FULL, lse[u] != lse[u]);
-            const float M = warp_max(lse[u]);
-            const float wt = (lane < C && lse[u] != -INFINITY) ? exp2f(lse[u] - M) : 0.f;
-            const float wsum = warp_sum(wt);
-            float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-            for (int q = 0; q < 16; ++q) {
-                const float wq = __shfl_sync(FULL, wt, q);   // 0 for q >= C and empty CTAs
-                if (q < C && wq != 0.f) {
-                    const float2 lo = unpack_bf16(v[u][q].x), hi = unpack_bf16(v[u][q].y);
-                    acc[0] += wq * lo.x;
-                    acc[1] += wq * lo.y;
-                    acc[2] += wq * hi.x;
-                    acc[3] += wq * hi.y;
-                }
-            }
-            const float inv = bad ? NAN : 1.0f / wsum;
-            const int i = r / a.G, h = g * a.G + r % a.G;
-            __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out) + (((size_t)b * a.N + i) * a.Hq + h) * 128;
-            uint2 pk;
-            pk.x = pack_bf16(acc[0] * inv, acc[1] * inv);
-            pk.y = pack_bf16(acc[2] * inv, acc[3] * inv);
-            reinterpret_cast<uint2*>(o)[lane] = pk;
-        }
+        __syncthreads();
     }
+    if (warp == 1) tmem_dealloc(tmem, 256 * MT);
+    if (threadIdx.x == 0) fence_proxy_async_smem();   // the staged slabs, for the pushes
+    cluster_sync();
+    if (threadIdx.x == 0) {
+        const uint32_t dst = smem_u32(sKV) + (uint32_t)(rank * slab_bytes);
+        const uint32_t bar = smem_u32(recv_full);
+        for (int q = 0; q < C && q * Rc < R; ++q)
+            bulk_copy_to_cluster(mapa_cluster(dst, (uint32_t)q), stg + (size_t)q * slab_bytes,
+                                 (uint32_t)slab_bytes, mapa_cluster(bar, (uint32_t)q));
+    }
+
+    // ----------------------------------------- merge the rows this CTA owns
+    const int r_lo = rank * Rc, n_own = max(0, min(R, r_lo + Rc) - r_lo);
+    int got = 1;
+    if (n_own > 0) {
+        // Wait for all C slabs even if another role gave up: nothing may
+        // still be writing into this CTA's shared memory when it exits.
+        if (lane == 0) got = mbar_wait_timeout_only(recv_full, 0) ? 1 : 0;
+        got = __shfl_sync(FULL, got, 0);
+        if (!got) *abort = 1;
+    }
+    // Every push into this CTA has landed: release the other CTAs' exit.
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+    grid_dep_wait();   // the output may be written only after the previous grid
+    // One thread per (row, 16-byte chunk of d): C weights, C chunk loads and
+    // 8 FMAs per slab, all loads independent.
+    const uint8_t* recv = sKV;
+    for (int task = threadIdx.x; task < n_own * 16; task += NTH) {
+        const int k = task >> 4, ch = task & 15;
+        float lsv[16];
+        float M = -INFINITY;
+        bool bad = !got;
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+            lsv[q] = q < C ? reinterpret_cast<const float*>(recv + q * slab_bytes + Rc * 256)[k] : -INFINITY;
+            bad |= lsv[q] != lsv[q];
+            M = fmaxf(M, lsv[q]);
+        }
+        const int off = k * 256 + ((ch ^ (k & 15)) << 4);
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        float wsum = 0.f;
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+            if (q >= C) break;
+            const float wq = lsv[q] == -INFINITY ? 0.f : fast_exp2(lsv[q] - M);
+            const uint4 v = *reinterpret_cast<const uint4*>(recv + q * slab_bytes + off);
+            wsum += wq;
+            const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float2 f = unpack_bf16(u[e]);
+                acc[2 * e] = fmaf(wq, f.x, acc[2 * e]);
+                acc[2 * e + 1] = fmaf(wq, f.y, acc[2 * e + 1]);
+            }
+        }
+        const float inv = bad ? NAN : 1.0f / wsum;
+        const int r = row0 + r_lo + k;
+        const int i = r / a.G, h = g * a.G + r % a.G;
+        __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out) + (((size_t)b * a.N + i) * a.Hq + h) * 128;
+        reinterpret_cast<uint4*>(o)[ch] =
+            make_uint4(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv),
+                       pack_bf16(acc[4] * inv, acc[5] * inv), pack_bf16(acc[6] * inv, acc[7] * inv));
+    }
+    // The slabs this CTA pushed have landed once every CTA has arrived.
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 // ----------------------------------------------------------------- host side
@@ -706,34 +756,12 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G) {
     return GV_OK;
 }
 
-// 3-D map over the bf16 partial rows [B*Hkv*16][R][128] with box
-// {64 d, 128 rows, 1}: rows of a 128-row store past R are clipped.
-static int make_map_part(CUtensorMap* map, void* part, int R, int units) {
-    EncodeTiledFn enc = tensor_map_encoder();
-    if (!enc) {
-        set_error("cuTensorMapEncodeTiled unavailable");
-        return GV_ERR_CUDA;
-    }
-    cuuint64_t dims[3] = {128, (cuuint64_t)R, (cuuint64_t)units * 16};
-    cuuint64_t strides[2] = {256, (cuuint64_t)R * 256};
-    cuuint32_t box[3] = {64, 128, 1};
-    cuuint32_t estr[3] = {1, 1, 1};
-    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, part, dims, strides, box, estr,
-                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) {
-        set_error("cuTensorMapEncodeTiled (partials) failed (%d)", (int)r);
-        return GV_ERR_CUDA;
-    }
-    return GV_OK;
-}
-
 static size_t attn_tc_smem(int mt) {
     const int st = mt == 1 ? 4 : 3;
-    return 1024 + (size_t)mt * (AT_QTILE + 2 * AT_PTILE) + (size_t)st * AT_STAGE + 8 * (2 * st + 12) + 16;
+    return 1024 + (size_t)mt * (AT_QTILE + 2 * AT_PTILE) + (size_t)st * AT_STAGE + 8 * (2 * st + 13) + 16;
 }
 
-// CTAs per cluster.  Wanted: enough clusters x CTAs to cover the SMs once
+// CTAs per cluster.  Wanted: as many as fit the SMs in one wave
 // (at most 16, the largest cluster GB300 schedules), at least 4 for long
 // caches so that a long sequence of a ragged batch is not one CTA's serial
 // work.  When the whole grid fits in one wave, the size is lowered until
@@ -744,7 +772,7 @@ template <int MT>
 static int attn_tc_cluster(int units, int S_max, size_t smem) {
     static int max_active[2][17] = {};
     auto kern = attn_tc_kernel<MT>;
-    int want = (sm_count() + units - 1) / units;
+    int want = sm_count() / units;                  // one wave of 1-CTA-per-SM clusters
     if (S_max >= 4096 && want < 4) want = 4;
     if (want > 16) want = 16;
     if (want < 1) want = 1;
@@ -777,13 +805,14 @@ static int attn_tc_cluster(int units, int S_max, size_t smem) {
 
 template <int MT>
 static int launch_mt(const AttnArgs& a0, const CUtensorMap& mk, const CUtensorMap& mv,
-                     const CUtensorMap& mq, const CUtensorMap& mp, cudaStream_t st) {
+                     const CUtensorMap& mq, cudaStream_t st) {
     const size_t smem = attn_tc_smem(MT);
     auto kern = attn_tc_kernel<MT>;
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    const int units = a0.B * a0.Hkv;
     AttnArgs a = a0;
+    a.tiles = MT == 1 ? (a0.R + 127) / 128 : 1;
+    const int units = a0.B * a0.Hkv * a.tiles;
     a.csize = attn_tc_cluster<MT>(units, a.S_max, smem);
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3((unsigned)(units * a.csize));
@@ -799,7 +828,7 @@ static int launch_mt(const AttnArgs& a0, const CUtensorMap& mk, const CUtensorMa
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mk, mv, mq, mp, a);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mk, mv, mq, a);
     if (e != cudaSuccess) {
         set_error("attn_tc_kernel launch (cluster %d): %s", a.csize, cudaGetErrorString(e));
         return GV_ERR_CUDA;
@@ -807,8 +836,10 @@ static int launch_mt(const AttnArgs& a0, const CUtensorMap& mk, const CUtensorMa
     return GV_OK;
 }
 
+constexpr bool kRowSplit = true;
+
 int launch_attn_tc(const AttnArgs& a, cudaStream_t st) {
-    CUtensorMap mk, mv, mq, mp;
+    CUtensorMap mk, mv, mq;
     const uint64_t rows = (uint64_t)a.B * a.Hkv * a.S_max;
     int rc = make_map_2d(&mk, a.cacheK, rows, 128, AT_BK, 256);
     if (rc != GV_OK) return rc;
@@ -816,10 +847,11 @@ int launch_attn_tc(const AttnArgs& a, cudaStream_t st) {
     if (rc != GV_OK) return rc;
     rc = make_map_q(&mq, a.q, a.B * a.N, a.Hq, a.G);
     if (rc != GV_OK) return rc;
-    rc = make_map_part(&mp, a.part_bf16, a.R, a.B * a.Hkv);
-    if (rc != GV_OK) return rc;
-    return (a.R + 127) / 128 == 1 ? launch_mt<1>(a, mk, mv, mq, mp, st)
-                                  : launch_mt<2>(a, mk, mv, mq, mp, st);
+    // Query rows above 128 go to a second cluster of one-tile CTAs rather
+    // than a second M tile in the same CTAs: twice the SMs on the key blocks,
+    // half the rows in each cluster's exchange.
+    return kRowSplit || (a.R + 127) / 128 == 1 ? launch_mt<1>(a, mk, mv, mq, st)
+                                                : launch_mt<2>(a, mk, mv, mq, st);
 }
 
 }  // namespace gv

@@ -79,7 +79,6 @@ int lmhead_tc_grid(int slots_capacity);
 
 // ---------------------------------------------------------- attention plan --
 constexpr int KPS_F32 = 256;   // prefix keys per split, CUDA-core path
-constexpr int TC_MAX_CLUSTER = 16;   // largest cluster of the tensor-core attention
 
 struct AttnPlan {
     size_t q_rot, part_o, part_ml, total;
@@ -118,12 +117,7 @@ static AttnPlan attn_plan(const gv_attn_shape* s) {
         p.part_ml = off;
         off += align256(bh * p.nsplit * R * 2 * sizeof(float));
     } else {
-        // one bf16 partial row and one lse per (cluster CTA, query row); the
-        // cluster holds at most TC_MAX_CLUSTER CTAs
-        p.part_o = off;
-        off += align256(bh * TC_MAX_CLUSTER * R * s->d * 2);
-        p.part_ml = off;
-        off += align256(bh * TC_MAX_CLUSTER * R * sizeof(float));
+        off += 256;   // none used: the cluster merges its splits in shared memory
     }
     p.total = off;
     return p;
@@ -302,7 +296,6 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
     a.out = out;
     a.q_rot = ws + plan.q_rot;
     a.part_o = reinterpret_cast<float*>(ws + plan.part_o);
-    a.part_bf16 = ws + plan.part_o;
     a.part_ml = reinterpret_cast<float*>(ws + plan.part_ml);
     a.nsplit = plan.nsplit;
     a.kps = plan.kps;
