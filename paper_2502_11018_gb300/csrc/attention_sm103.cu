@@ -5,47 +5,50 @@
 // to the nodes on its own root chain (Section 4.1: rejecting a token drops
 // its subtree, so the ancestor set is exactly what node i may see).
 //
-// One thread-block cluster of C CTAs per (sequence b, KV head g).  The keys
-// of (b, g) are cut into 64-key blocks: ceil(P_b / 64) prefix blocks and one
-// tree block (the N <= 64 tree keys, masked per query row by its ancestor
-// bitmask).  CTA `rank` of the cluster takes blocks rank, rank + C, ...; the
-// CTA that owns the tree block runs it first.  All G * N query rows of KV
-// head g share every K/V block; row r = i * G + hl holds node i and query
-// head g * G + hl, and 128 rows form one MMA M tile (MT = 1 or 2 tiles).
+// Query rows: row r = i * G + hl of KV head g holds tree node i and query
+// head g * G + hl; all G * N rows of (b, g) share every K/V block (GQA), and
+// each 128 of them form one MMA M tile.  One thread-block cluster of C CTAs
+// per (sequence b, KV head g, M tile).  The keys of (b, g) are cut into
+// 64-key blocks: ceil(P_b / 64) prefix blocks and one tree block (the N <= 64
+// tree keys, masked per query row by its ancestor bitmask).  CTA `rank` of
+// the cluster takes blocks rank, rank + C, ...; the CTA that owns the tree
+// block runs it first.
 //
 // Per block j of a CTA:
 //   S_j = Q K_j^T          tcgen05.mma, Q and K K-major 128B-swizzled in smem,
 //                          fp32 S in TMEM (two buffers: S_{j+1} overlaps the
 //                          softmax of block j)
-//   softmax                one thread per query row reads its S row from TMEM,
-//                          masks with a branch-free 64-bit validity mask
-//                          (prefix end, or the row's ancestor bitmask), keeps a
-//                          running max in the log2 domain and rescales O only
-//                          when the max grew by more than 2^8 (exact: O and l
-//                          always share one max), writes P = exp2(s - m) as
-//                          bf16 to one of two smem buffers
-//   O += P_j V_j           tcgen05.mma, P K-major, V MN-major (d contiguous)
-// Each CTA then stages o = O / l (bf16) and lse = m + log2(l) of its rows in
-// its shared memory; after a cluster barrier it pushes to every CTA of the
-// cluster (bulk copies into distributed shared memory) the 1/C share of rows
-// that CTA merges, and every CTA merges its share over the C partials and
-// writes the final bf16 output: the split combine needs no extra launch and
-// no global scratch.
+//   softmax                two threads per query row, one per 32-key half of
+//                          the block, read their S row half from TMEM, mask
+//                          with a branch-free validity mask (prefix end, or
+//                          the row's ancestor bitmask), keep a running max in
+//                          the log2 domain and rescale their O only when the
+//                          max grew by more than 2^8 (exact: O and l always
+//                          share one max), and write P = exp2(s - m) as bf16
+//                          to one of two smem buffers
+//   O_h += P_j,h V_j,h     tcgen05.mma, P K-major, V MN-major (d contiguous),
+//                          one accumulator per key half h
+// Each CTA then merges its two halves and stages o = O / l (bf16) and
+// lse = m + log2(l) of its rows in its shared memory; after a cluster barrier
+// it pushes to every CTA of the cluster (bulk copies into distributed shared
+// memory) the 1/C share of rows that CTA merges, and every CTA merges its
+// share over the C partials and writes the final bf16 output: the split
+// combine needs no extra launch and no global scratch.
 //
-// Warp roles: warp 0 issues the TMA loads (K/V blocks, raw Q tiles); warp 1
-// owns TMEM and issues the MMAs; warps 2.. (4 per M tile) rotate Q in place
+// Warp roles: warp 0 issues the TMA loads (RoPE rows, K/V blocks, raw Q
+// tile); warp 1 owns TMEM and issues the MMAs; warps 2..9 rotate Q in place
 // (RoPE from the per-step table), build the tree K/V tile, and run the
-// softmax and the epilogue; all warps share the merge.
+// softmax and the staging; all warps share the merge.
 //
 // Launch: cluster launch (the cluster barrier orders the partial exchange and
 // guarantees the C CTAs are co-resident) with programmatic dependent launch.
 // Before griddepcontrol.wait a CTA only initialises barriers and TMEM, reads
 // step inputs written before the step's first attention launch (RoPE table,
 // ancestor masks, prefix lengths) and starts streaming two K/V cache blocks;
-// queries, tree keys/values, partials and the output are touched after it.
-// Every mbarrier wait is bounded; a CTA that gives up marks its rows' lse
-// NaN, which turns the affected outputs into NaN, and still reaches the
-// cluster barrier.
+// queries, tree keys/values and the output are touched after it.  Every
+// mbarrier wait is bounded; a CTA that gives up marks its rows' lse NaN,
+// which turns the affected outputs into NaN, and still reaches the cluster
+// barriers.
 #include "gv_internal.cuh"
 #include "attention.cuh"
 #include "sm103.cuh"
@@ -150,20 +153,28 @@ __device__ __forceinline__ void rope8(const uint4& lo, const uint4& hi, const fl
     }
 }
 
-template <int MT>
-__global__ void __launch_bounds__(64 + 128 * MT, 1)
+// Softmax warps 2..9: warp w reads TMEM lane quarter (w & 3), i.e. query
+// rows 32 * (w & 3) .. + 31, and key half h = (w - 2) >> 2 (keys 32h .. 32h+31)
+// of every 64-key block.  Each (row, half) keeps its own running max, sum and
+// O accumulator O_h in TMEM -- a two-way split of the keys inside the CTA --
+// so each thread handles 32 scores per block; the halves are merged when the
+// CTA's partial row is staged.
+constexpr int AT_NSM = 256;               // softmax threads: 128 rows x 2 key halves
+constexpr int AT_NTH = 64 + AT_NSM;       // + TMA producer warp + MMA warp
+constexpr int AT_ST = 4;                  // K/V stages
+constexpr uint32_t AT_TMEM_COLS = 512;    // S double buffer [0,128), O_0 [128,256), O_1 [256,384)
+
+__global__ void __launch_bounds__(AT_NTH, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
                const __grid_constant__ CUtensorMap map_q, AttnArgs a) {
-    constexpr int NSM = 128 * MT;            // softmax threads
-    constexpr int NTH = 64 + NSM;            // all threads
-    constexpr int ST = MT == 1 ? 4 : 3;      // K/V stages
+    constexpr int NSM = AT_NSM, NTH = AT_NTH, ST = AT_ST;
     const int C = a.csize;
     const int rank = (int)cluster_rank();
-    // Cluster -> (sequence b, KV head g, first M tile): the G * N query rows of
-    // (b, g) are cut into groups of MT tiles of 128, one cluster per group.
+    // Cluster -> (sequence b, KV head g, M tile): the G * N query rows of
+    // (b, g) are cut into tiles of 128, one cluster per tile.
     const int cl = blockIdx.x / C;
     const int bg = cl / a.tiles;
-    const int tile0 = (cl % a.tiles) * MT;
+    const int tile0 = cl % a.tiles;
     const int b = bg / a.Hkv, g = bg % a.Hkv;
     // prefix_len is a step input written before the previous kernel in the
     // stream started, so it may be read before griddepcontrol.wait.
@@ -175,7 +186,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     const int nblk = (nb_pre > rank ? (nb_pre - 1 - rank) / C + 1 : 0) + (has_tree ? 1 : 0);
     const int nb_per_tile = 128 / a.G;                   // nodes per M tile
     const int row0 = tile0 * 128;                        // first query row of this cluster
-    const int R = min(a.G * a.N - row0, MT * 128);       // query rows of this cluster
+    const int R = min(a.G * a.N - row0, 128);            // query rows of this cluster
     const int Rc = (R + C - 1) / C;                      // rows each CTA merges
     const int slab_bytes = Rc * 256 + ((Rc + 3) & ~3) * 4;   // Rc bf16 rows + Rc lse (16-byte multiple)
     const int r_own = min(R, rank * Rc + Rc) - rank * Rc;    // rows this CTA merges (<= 0: none)
@@ -188,10 +199,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
-    uint8_t* sQ = smem;                                  // MT x 32 KB
-    uint8_t* sP = sQ + MT * AT_QTILE;                    // 2 buffers x MT x 16 KB
-    uint8_t* sKV = sP + 2 * MT * AT_PTILE;               // ST x 32 KB
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + ST * AT_STAGE);
+    uint8_t* sQ = smem;                                  // 32 KB
+    uint8_t* sP = sQ + AT_QTILE;                         // 2 buffers x 16 KB
+    uint8_t* sKV = sP + 2 * AT_PTILE;                    // ST x 32 KB
+    float2* sML = reinterpret_cast<float2*>(sKV + ST * AT_STAGE);   // [2][128] (m, l) per key half
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sML + 2 * 128);
     uint64_t* kv_full = bars;
     uint64_t* kv_empty = kv_full + ST;
     uint64_t* s_full = kv_empty + ST;
@@ -217,8 +229,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         }
         for (int c = 0; c < 2; ++c) {
             mbar_init(&s_full[c], 1);
-            mbar_init(&s_free[c], 4 * MT);
-            mbar_init(&p_full[c], 4 * MT);
+            mbar_init(&s_free[c], NSM / 32);
+            mbar_init(&p_full[c], NSM / 32);
             mbar_init(&o_done[c], 1);
         }
         mbar_init(q_raw, 1);
@@ -235,21 +247,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             prefetch_tmap(&map_v);
         }
     }
-    if (warp == 1) tmem_alloc(tmem_holder, 256 * MT);
+    if (warp == 1) tmem_alloc(tmem_holder, AT_TMEM_COLS);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
     grid_dep_launch();
 
-    // Row owned by a softmax thread (valid for warps >= 2).
+    // Row and key half of a softmax thread (valid for warps >= 2).
     const int t = threadIdx.x - 64;
-    const int m = (warp - 2) >> 2;                       // M tile of this warp
+    const int kh = warp >= 2 ? (warp - 2) >> 2 : 0;     // key half
     const int sub = warp & 3;                            // TMEM lane quarter
-    const int row = sub * 32 + lane;                     // row inside the M tile
-    const int node = (tile0 + m) * nb_per_tile + row / a.G;   // tree node of this row
+    const int row = sub * 32 + lane;                     // query row in the cluster's tile
+    const int node = tile0 * nb_per_tile + row / a.G;    // tree node of this row
     const bool row_ok = warp >= 2 && node < a.N;
-    const int grow = m * 128 + row;                      // row in the cluster; row0 + grow = node * G + head
+    const uint32_t lane_base = tmem + ((uint32_t)(sub * 32) << 16);
+    const uint32_t ocol_self = lane_base + 128u + 128u * (uint32_t)kh;   // O of this key half
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
 
@@ -269,12 +282,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 bool q_issued = false;
                 auto issue_q = [&]() {
                     grid_dep_wait();
-                    mbar_arrive_expect_tx(q_raw, MT * AT_QTILE);
-                    for (int mm = 0; mm < MT; ++mm) {
-                        const int z = b * a.N + (tile0 + mm) * nb_per_tile;
-                        tma_load_3d(sQ + mm * AT_QTILE, &map_q, q_raw, 0, g * a.G, z, pol_q);
-                        tma_load_3d(sQ + mm * AT_QTILE + AT_QHALF, &map_q, q_raw, 64, g * a.G, z, pol_q);
-                    }
+                    mbar_arrive_expect_tx(q_raw, AT_QTILE);
+                    const int z = b * a.N + tile0 * nb_per_tile;
+                    tma_load_3d(sQ, &map_q, q_raw, 0, g * a.G, z, pol_q);
+                    tma_load_3d(sQ + AT_QHALF, &map_q, q_raw, 64, g * a.G, z, pol_q);
                     q_issued = true;
                 };
                 for (int j = 0; j < nblk; ++j) {
@@ -319,15 +330,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     // 1 KB per 8 keys), the two 64-wide halves of d LBO = 8 KB apart.
                     uint64_t vdesc = sdesc_kmajor_sw128(smem_u32(sKV + sp * AT_STAGE + 2 * AT_KV_HALF));
                     vdesc = (vdesc & ~(0x3FFFull << 16)) | ((uint64_t)(AT_KV_HALF >> 4) << 16);
+                    const uint64_t pdesc = sdesc_kmajor_sw128(smem_u32(sP + pb * AT_PTILE));
+                    // Keys 0..31 (K steps 0, 1) into O_0, keys 32..63 into O_1.
 #pragma unroll
-                    for (int mm = 0; mm < MT; ++mm) {
-                        const uint64_t pdesc =
-                            sdesc_kmajor_sw128(smem_u32(sP + (pb * MT + mm) * AT_PTILE));
-#pragma unroll
-                        for (int kk = 0; kk < AT_BK / 16; ++kk)
-                            mma_bf16(tmem + (uint32_t)(mm * 256 + 128), pdesc + 2u * kk,
-                                     vdesc + (uint64_t)(kk * 128), idesc_o, (jj | kk) != 0);
-                    }
+                    for (int kk = 0; kk < AT_BK / 16; ++kk)
+                        mma_bf16(tmem + 128u + 128u * (uint32_t)(kk >> 1), pdesc + 2u * kk,
+                                 vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (kk & 1));
                     mma_commit(&kv_empty[sp]);
                     mma_commit(&o_done[pb]);
                     return true;
@@ -342,17 +350,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     tc_fence_after();
                     const uint32_t kbase = smem_u32(sKV + s * AT_STAGE);
 #pragma unroll
-                    for (int mm = 0; mm < MT; ++mm) {
+                    for (int kb = 0; kb < 2; ++kb) {
+                        const uint64_t qdesc = sdesc_kmajor_sw128(smem_u32(sQ + kb * AT_QHALF));
+                        const uint64_t kdesc = sdesc_kmajor_sw128(kbase + kb * AT_KV_HALF);
 #pragma unroll
-                        for (int kb = 0; kb < 2; ++kb) {
-                            const uint64_t qdesc =
-                                sdesc_kmajor_sw128(smem_u32(sQ + mm * AT_QTILE + kb * AT_QHALF));
-                            const uint64_t kdesc = sdesc_kmajor_sw128(kbase + kb * AT_KV_HALF);
-#pragma unroll
-                            for (int kk = 0; kk < 4; ++kk)
-                                mma_bf16(tmem + (uint32_t)(mm * 256 + buf * AT_BK), qdesc + 2u * kk,
-                                         kdesc + 2u * kk, idesc_s, (kb | kk) != 0);
-                        }
+                        for (int kk = 0; kk < 4; ++kk)
+                            mma_bf16(tmem + (uint32_t)(buf * AT_BK), qdesc + 2u * kk, kdesc + 2u * kk,
+                                     idesc_s, (kb | kk) != 0);
                     }
                     mma_commit(&s_full[buf]);
                     if (j >= 1 && !issue_pv(j - 1)) {
@@ -386,7 +390,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     const int j = e >> 3, c = e & 7;
                     uint4 klo = make_uint4(0, 0, 0, 0), khi = klo, vlo = klo, vhi = klo;
                     if (j < a.N) {
-                        // (every row group's cluster builds the tile; the first writes the scratch)
+                        // (every row tile's cluster builds the tile; the first writes the scratch)
                         const size_t src = (((size_t)b * a.N + j) * a.Hkv + g) * 16;
                         const uint4* kr = reinterpret_cast<const uint4*>(a.k_new) + src;
                         const uint4* vr = reinterpret_cast<const uint4*>(a.v_new) + src;
@@ -417,35 +421,34 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     mbar_arrive(&kv_full[0]);
                 }
             }
-            // RoPE of this thread's Q row, in place once the raw tile has landed:
-            // all loads of the row first, the rotation in registers, then the
-            // stores (no store sits between two loads, so all loads overlap).
+            // RoPE of this thread's half of its Q row (16-byte chunks 4 kh ..
+            // 4 kh + 3 of both d halves), in place once the raw tile has
+            // landed: loads first, the rotation in registers, then the stores.
             {
                 const int w = mbar_wait(q_raw, 0, abort) ? 1 : 0;   // every lane observes the copy
-                uint8_t* qt = sQ + m * AT_QTILE;
                 if (__all_sync(FULL, w) && ok) {
-                    uint4 lo[8], hi[8];
+                    uint4 lo[4], hi[4];
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        lo[c] = *reinterpret_cast<const uint4*>(qt + sw128(row, c));
-                        hi[c] = *reinterpret_cast<const uint4*>(qt + AT_QHALF + sw128(row, c));
+                    for (int c = 0; c < 4; ++c) {
+                        lo[c] = *reinterpret_cast<const uint4*>(sQ + sw128(row, 4 * kh + c));
+                        hi[c] = *reinterpret_cast<const uint4*>(sQ + AT_QHALF + sw128(row, 4 * kh + c));
                     }
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) {
+                    for (int c = 0; c < 4; ++c) {
                         uint4 olo = make_uint4(0, 0, 0, 0), ohi = olo;
                         if (row_ok) {
                             float4 cs[4];
 #pragma unroll
-                            for (int q = 0; q < 4; ++q) cs[q] = sRope[node * 32 + c * 4 + q];
+                            for (int q = 0; q < 4; ++q) cs[q] = sRope[node * 32 + (4 * kh + c) * 4 + q];
                             rope8(lo[c], hi[c], cs, olo, ohi);
                         }
                         lo[c] = olo;
                         hi[c] = ohi;
                     }
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        *reinterpret_cast<uint4*>(qt + sw128(row, c)) = lo[c];
-                        *reinterpret_cast<uint4*>(qt + AT_QHALF + sw128(row, c)) = hi[c];
+                    for (int c = 0; c < 4; ++c) {
+                        *reinterpret_cast<uint4*>(sQ + sw128(row, 4 * kh + c)) = lo[c];
+                        *reinterpret_cast<uint4*>(sQ + AT_QHALF + sw128(row, 4 * kh + c)) = hi[c];
                     }
                 }
                 named_bar_sync(1, NSM);
@@ -465,41 +468,35 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 }
                 __syncwarp();
                 tc_fence_after();
-                uint32_t sv[64];
-                const uint32_t scol =
-                    tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(m * 256 + buf * AT_BK);
-                tmem_ld32(scol, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
-                tmem_ld32(scol + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+                uint32_t sv[32];
+                tmem_ld32(lane_base + (uint32_t)(buf * AT_BK + 32 * kh), sv);
                 tmem_wait_ld();
 #pragma unroll
-                for (int c = 0; c < 64; ++c) asm volatile("" : "+r"(sv[c]));  // uses stay after the wait
+                for (int c = 0; c < 32; ++c) asm volatile("" : "+r"(sv[c]));  // uses stay after the wait
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&s_free[buf]);
-                // Keys of the block this row may see: all 64 of a full prefix
-                // block (the common, unmasked path), else a branch-free 64-bit
-                // mask (the prefix end, or the row's ancestor bitmask); masked
-                // scores become -inf and their exp2 is exactly 0.
+                // Keys of the block this row may see: all of a full prefix block
+                // (the common, unmasked path), else a branch-free mask (the
+                // prefix end, or the row's ancestor bitmask); masked scores
+                // become -inf and their exp2 is exactly 0.
                 const int k = prefix_block(j);
                 const int nvalid = k < 0 ? a.N : min(AT_BK, P - k * AT_BK);
                 if (k < 0 || nvalid < AT_BK) {
-                    uint32_t vlo, vhi;
+                    uint32_t vbits;
                     if (k < 0) {
-                        vlo = (uint32_t)anc_row;
-                        vhi = (uint32_t)(anc_row >> 32);
+                        vbits = (uint32_t)(anc_row >> (32 * kh));
                     } else {
-                        vlo = nvalid >= 32 ? 0xFFFFFFFFu : ((1u << nvalid) - 1u);
-                        vhi = nvalid > 32 ? ((1u << (nvalid - 32)) - 1u) : 0u;
+                        const int nv = nvalid - 32 * kh;     // valid keys of this half
+                        vbits = nv >= 32 ? 0xFFFFFFFFu : (nv <= 0 ? 0u : ((1u << nv) - 1u));
                     }
 #pragma unroll
-                    for (int c = 0; c < 64; ++c) {
-                        const uint32_t bit = c < 32 ? (vlo >> c) & 1u : (vhi >> (c - 32)) & 1u;
-                        sv[c] = bit ? sv[c] : __float_as_uint(-INFINITY);
-                    }
+                    for (int c = 0; c < 32; ++c)
+                        sv[c] = (vbits >> c) & 1u ? sv[c] : __float_as_uint(-INFINITY);
                 }
                 float mxs[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-                for (int c = 0; c < 64; c += 2)
+                for (int c = 0; c < 32; c += 2)
                     mxs[(c >> 1) & 3] = max3(mxs[(c >> 1) & 3], __uint_as_float(sv[c]), __uint_as_float(sv[c + 1]));
                 const float mx = max3(mxs[0], mxs[1], fmaxf(mxs[2], mxs[3])) * sl2;   // sl2 > 0
                 const float m_new = fmaxf(m_used, mx);
@@ -514,9 +511,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 const float nmv = m_used == -INFINITY ? 0.f : -m_used;
                 const uint64_t sc2 = f32x2(sl2, sl2), nm2 = f32x2(nmv, nmv);
                 uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
-                uint32_t pk[32];
+                uint32_t pk[16];
 #pragma unroll
-                for (int c = 0; c < 32; ++c) {
+                for (int c = 0; c < 16; ++c) {
                     const float2 xa = split_f32x2(ffma_f32x2(
                         f32x2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nm2));
                     const float p0 = fast_exp2(xa.x), p1 = fast_exp2(xa.y);
@@ -535,7 +532,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     }
                 }
                 if (j >= 1 && __any_sync(FULL, need)) {
-                    // Rescale O: PV_{j-1} must have landed first.
+                    // Rescale O of this half: PV_{j-1} must have landed first.
                     if (lane == 0)
                         w = mbar_wait(&o_done[(j - 1) & 1], (uint32_t)((j - 1) >> 1) & 1u, abort);
                     if (!__shfl_sync(FULL, w, 0)) {
@@ -544,11 +541,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     }
                     __syncwarp();
                     tc_fence_after();
-                    const uint32_t ocol = tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(m * 256 + 128);
 #pragma unroll
                     for (int c0 = 0; c0 < 128; c0 += 32) {
                         uint32_t ov[32];
-                        tmem_ld32(ocol + c0, ov);
+                        tmem_ld32(ocol_self + c0, ov);
                         tmem_wait_ld();
                         uint32_t lo[16], hi[16];
 #pragma unroll
@@ -556,17 +552,17 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                             lo[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
                             hi[e] = __float_as_uint(__uint_as_float(ov[16 + e]) * alpha);
                         }
-                        tmem_st16(ocol + c0, lo);
-                        tmem_st16(ocol + c0 + 16, hi);
+                        tmem_st16(ocol_self + c0, lo);
+                        tmem_st16(ocol_self + c0 + 16, hi);
                     }
                     tmem_wait_st();
                 }
-                uint8_t* pt = sP + (pb * MT + m) * AT_PTILE;
+                uint8_t* pt = sP + pb * AT_PTILE;
 #pragma unroll
-                for (int c = 0; c < 8; ++c)
-                    *reinterpret_cast<uint4*>(pt + sw128(row, c)) =
+                for (int c = 0; c < 4; ++c)
+                    *reinterpret_cast<uint4*>(pt + sw128(row, 4 * kh + c)) =
                         make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-                if (k >= 0 && nvalid < AT_BK && m == 0) {
+                if (k >= 0 && nvalid < AT_BK && kh == 0) {
                     // Zero the V rows past the prefix end (they may hold anything).
                     int w2 = 1;
                     if (lane == 0) w2 = mbar_wait(&kv_full[s], (uint32_t)(j / ST) & 1u, abort);
@@ -590,58 +586,76 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     }
 
     // ------------------------------- exchange partial rows through the cluster
-    // Each CTA stages its rows' normalised partial o = O / l (bf16) and
-    // lse = m + log2(l) (fp32) in its own (now free) Q and P areas as C slabs:
-    // slab q holds rows [q * Rc, (q + 1) * Rc), the rows CTA q merges, with
-    // the 16-byte chunks of row k of a slab rotated by (k & 15) so that the
-    // lanes of a warp store and load distinct banks.  After a cluster barrier
-    // (every CTA is past its main loop, so its K/V ring is idle) thread 0
-    // pushes slab q into the K/V ring of CTA q with one bulk shared::cta ->
-    // shared::cluster copy that completes on CTA q's `recv_full` barrier; CTA
-    // q merges its rows over the C slabs it received and writes the output.
-    // lse is -inf for a CTA without blocks and NaN for one that gave up.
+    // Each CTA merges its two key halves and stages its rows' normalised
+    // partial o = O / l (bf16) and lse = m + log2(l) (fp32) in its own (now
+    // free) Q and P areas as C slabs: slab q holds rows [q * Rc, (q + 1) * Rc),
+    // the rows CTA q merges, with the 16-byte chunks of row k of a slab rotated
+    // by (k & 15) so that the lanes of a warp store and load distinct banks.
+    // After a cluster barrier (every CTA is past its main loop, so its K/V ring
+    // is idle) thread 0 pushes slab q into the K/V ring of CTA q with one bulk
+    // shared::cta -> shared::cluster copy that completes on CTA q's
+    // `recv_full` barrier; CTA q merges its rows over the C slabs it received
+    // and writes the output.  lse is -inf for a CTA without blocks and NaN for
+    // one that gave up.
     uint8_t* stg = sQ;
+    int w = 0;
     if (warp >= 2) {
-        int w = ok && nblk > 0 ? 1 : 0;
+        w = ok && nblk > 0 ? 1 : 0;
         if (w && lane == 0)
             w = mbar_wait(&o_done[(nblk - 1) & 1], (uint32_t)((nblk - 1) >> 1) & 1u, abort);
         w = __shfl_sync(FULL, w, 0);
-        const bool mine = grow < R;
-        const int q = grow / Rc, k = grow - q * Rc;
+        sML[kh * 128 + row] = make_float2(m_used, l);
+    }
+    // The halves' (m, l) and the last PV are visible after this barrier; the
+    // CTA's partial is valid only if every softmax warp finished.
+    w = __syncthreads_and(warp < 2 || w);
+    if (warp >= 2) {
+        const bool mine = row < R;
+        const int q = row / Rc, k = row - q * Rc;
         uint8_t* slab = stg + (size_t)q * slab_bytes;
+        const float2 other = sML[(1 - kh) * 128 + row];
+        const float M = fmaxf(m_used, other.x);
+        const float ws = m_used == -INFINITY ? 0.f : fast_exp2(m_used - M);
+        const float wo = other.x == -INFINITY ? 0.f : fast_exp2(other.x - M);
+        const float ltot = l * ws + other.y * wo;
         if (w) {
+            // This thread writes d columns [64 kh, 64 kh + 64) of the row:
+            // O_kh and O_{1-kh} there, weighted by their halves' max offsets.
             tc_fence_after();
-            const uint32_t ocol = tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(m * 256 + 128);
-            const float inv = 1.0f / l;
+            const uint32_t ocol_other = lane_base + 128u + 128u * (uint32_t)(1 - kh);
+            const float inv = ltot > 0.f ? 1.0f / ltot : 0.f;
+            const float as = ws * inv, ao = wo * inv;
 #pragma unroll
-            for (int c0 = 0; c0 < 128; c0 += 64) {
-                uint32_t ov[64];
-                tmem_ld32(ocol + c0, *reinterpret_cast<uint32_t(*)[32]>(&ov[0]));
-                tmem_ld32(ocol + c0 + 32, *reinterpret_cast<uint32_t(*)[32]>(&ov[32]));
+            for (int c0 = 0; c0 < 64; c0 += 32) {
+                uint32_t os[32], oo[32];
+                tmem_ld32(ocol_self + (uint32_t)(64 * kh + c0), os);
+                tmem_ld32(ocol_other + (uint32_t)(64 * kh + c0), oo);
                 tmem_wait_ld();
                 if (mine) {
 #pragma unroll
-                    for (int e = 0; e < 64; e += 8) {
-                        const int ch = (c0 + e) >> 3;   // 16-byte chunk of the 256-byte row
+                    for (int e = 0; e < 32; e += 8) {
+                        const int ch = (64 * kh + c0 + e) >> 3;   // 16-byte chunk of the 256-byte row
+                        float v[8];
+#pragma unroll
+                        for (int u = 0; u < 8; ++u)
+                            v[u] = __uint_as_float(os[e + u]) * as + __uint_as_float(oo[e + u]) * ao;
                         *reinterpret_cast<uint4*>(slab + k * 256 + ((ch ^ (k & 15)) << 4)) =
-                            make_uint4(
-                                pack_bf16(__uint_as_float(ov[e]) * inv, __uint_as_float(ov[e + 1]) * inv),
-                                pack_bf16(__uint_as_float(ov[e + 2]) * inv, __uint_as_float(ov[e + 3]) * inv),
-                                pack_bf16(__uint_as_float(ov[e + 4]) * inv, __uint_as_float(ov[e + 5]) * inv),
-                                pack_bf16(__uint_as_float(ov[e + 6]) * inv, __uint_as_float(ov[e + 7]) * inv));
+                            make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]),
+                                       pack_bf16(v[4], v[5]), pack_bf16(v[6], v[7]));
                     }
                 }
             }
         }
         if (mine) {
-            reinterpret_cast<float*>(slab + Rc * 256)[k] =
-                w ? m_used + log2f(l) : (nblk > 0 ? NAN : -INFINITY);
+            if (kh == 0)
+                reinterpret_cast<float*>(slab + Rc * 256)[k] =
+                    w ? (ltot > 0.f ? M + log2f(ltot) : -INFINITY) : (nblk > 0 ? NAN : -INFINITY);
             if (!w) {
                 // No partial (no blocks, or gave up): zeros, so that the
                 // merge may weight every slab without testing its weight.
 #pragma unroll
-                for (int ch = 0; ch < 16; ++ch)
-                    *reinterpret_cast<uint4*>(slab + k * 256 + (ch << 4)) = make_uint4(0, 0, 0, 0);
+                for (int ch = 0; ch < 8; ++ch)
+                    *reinterpret_cast<uint4*>(slab + k * 256 + ((8 * kh + ch) << 4)) = make_uint4(0, 0, 0, 0);
             }
         }
     }
@@ -652,13 +666,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         // A role gave up, so a copy may have landed in the staging area after
         // the rows were staged (each role drains its own copies before the
         // barrier above): mark every row of this CTA invalid again.
-        if (warp >= 2 && grow < R) {
-            const int q = grow / Rc;
-            reinterpret_cast<float*>(stg + (size_t)q * slab_bytes + Rc * 256)[grow - q * Rc] = NAN;
+        if (warp >= 2 && kh == 0 && row < R) {
+            const int q = row / Rc;
+            reinterpret_cast<float*>(stg + (size_t)q * slab_bytes + Rc * 256)[row - q * Rc] = NAN;
         }
         __syncthreads();
     }
-    if (warp == 1) tmem_dealloc(tmem, 256 * MT);
+    if (warp == 1) tmem_dealloc(tmem, AT_TMEM_COLS);
     if (threadIdx.x == 0) fence_proxy_async_smem();   // the staged slabs, for the pushes
     cluster_sync();
     if (threadIdx.x == 0) {
@@ -756,31 +770,29 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G) {
     return GV_OK;
 }
 
-static size_t attn_tc_smem(int mt) {
-    const int st = mt == 1 ? 4 : 3;
-    return 1024 + (size_t)mt * (AT_QTILE + 2 * AT_PTILE) + (size_t)st * AT_STAGE + 8 * (2 * st + 13) + 16;
+static size_t attn_tc_smem() {
+    return 1024 + (size_t)AT_QTILE + 2 * AT_PTILE + (size_t)AT_ST * AT_STAGE + 2 * 128 * sizeof(float2) +
+           8 * (2 * AT_ST + 13) + 16;
 }
 
-// CTAs per cluster.  Wanted: as many as fit the SMs in one wave
-// (at most 16, the largest cluster GB300 schedules), at least 4 for long
-// caches so that a long sequence of a ragged batch is not one CTA's serial
-// work.  When the whole grid fits in one wave, the size is lowered until
-// every cluster can be resident at once (GPC boundaries limit how many large
-// clusters of 1-CTA-per-SM kernels fit), since a cluster left for a second
-// wave doubles the layer's time.
-template <int MT>
+// CTAs per cluster.  Wanted: as many as fit the SMs in one wave (at most 16,
+// the largest cluster GB300 schedules), at least 4 for long caches so that a
+// long sequence of a ragged batch is not one CTA's serial work.  When the
+// whole grid fits in one wave, the size is lowered until every cluster can be
+// resident at once (GPC boundaries limit how many large clusters of
+// 1-CTA-per-SM kernels fit), since a cluster left for a second wave doubles
+// the layer's time.
 static int attn_tc_cluster(int units, int S_max, size_t smem) {
-    static int max_active[2][17] = {};
-    auto kern = attn_tc_kernel<MT>;
+    static int max_active[17] = {};
     int want = sm_count() / units;                  // one wave of 1-CTA-per-SM clusters
     if (S_max >= 4096 && want < 4) want = 4;
     if (want > 16) want = 16;
     if (want < 1) want = 1;
     for (int c = want; c >= 1; --c) {
-        if (max_active[MT - 1][c] == 0) {
+        if (max_active[c] == 0) {
             cudaLaunchConfig_t cfg{};
             cfg.gridDim = dim3((unsigned)(c * units));
-            cfg.blockDim = dim3(64 + 128 * MT);
+            cfg.blockDim = dim3(AT_NTH);
             cfg.dynamicSmemBytes = smem;
             cudaLaunchAttribute attr[1];
             attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -790,33 +802,39 @@ static int attn_tc_cluster(int units, int S_max, size_t smem) {
             cfg.attrs = attr;
             cfg.numAttrs = 1;
             int n = 0;
-            if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+            if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel, &cfg) != cudaSuccess) {
                 cudaGetLastError();
                 n = -1;
             }
-            max_active[MT - 1][c] = n;
+            max_active[c] = n;
         }
-        const int n = max_active[MT - 1][c];
+        const int n = max_active[c];
         if (n < 0) continue;                        // not schedulable at this size
         if (units * c > sm_count() || n >= units) return c;
     }
     return 1;
 }
 
-template <int MT>
-static int launch_mt(const AttnArgs& a0, const CUtensorMap& mk, const CUtensorMap& mv,
-                     const CUtensorMap& mq, cudaStream_t st) {
-    const size_t smem = attn_tc_smem(MT);
-    auto kern = attn_tc_kernel<MT>;
-    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
+    CUtensorMap mk, mv, mq;
+    const uint64_t rows = (uint64_t)a0.B * a0.Hkv * a0.S_max;
+    int rc = make_map_2d(&mk, a0.cacheK, rows, 128, AT_BK, 256);
+    if (rc != GV_OK) return rc;
+    rc = make_map_2d(&mv, a0.cacheV, rows, 128, AT_BK, 256);
+    if (rc != GV_OK) return rc;
+    rc = make_map_q(&mq, a0.q, a0.B * a0.N, a0.Hq, a0.G);
+    if (rc != GV_OK) return rc;
+    const size_t smem = attn_tc_smem();
+    cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    // Every 128 query rows of a (sequence, KV head) get their own cluster.
     AttnArgs a = a0;
-    a.tiles = MT == 1 ? (a0.R + 127) / 128 : 1;
+    a.tiles = (a0.R + 127) / 128;
     const int units = a0.B * a0.Hkv * a.tiles;
-    a.csize = attn_tc_cluster<MT>(units, a.S_max, smem);
+    a.csize = attn_tc_cluster(units, a.S_max, smem);
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3((unsigned)(units * a.csize));
-    cfg.blockDim = dim3(64 + 128 * MT);
+    cfg.blockDim = dim3(AT_NTH);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
     cudaLaunchAttribute attr[2];
@@ -828,30 +846,12 @@ static int launch_mt(const AttnArgs& a0, const CUtensorMap& mk, const CUtensorMa
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, mk, mv, mq, a);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, attn_tc_kernel, mk, mv, mq, a);
     if (e != cudaSuccess) {
         set_error("attn_tc_kernel launch (cluster %d): %s", a.csize, cudaGetErrorString(e));
         return GV_ERR_CUDA;
     }
     return GV_OK;
-}
-
-constexpr bool kRowSplit = true;
-
-int launch_attn_tc(const AttnArgs& a, cudaStream_t st) {
-    CUtensorMap mk, mv, mq;
-    const uint64_t rows = (uint64_t)a.B * a.Hkv * a.S_max;
-    int rc = make_map_2d(&mk, a.cacheK, rows, 128, AT_BK, 256);
-    if (rc != GV_OK) return rc;
-    rc = make_map_2d(&mv, a.cacheV, rows, 128, AT_BK, 256);
-    if (rc != GV_OK) return rc;
-    rc = make_map_q(&mq, a.q, a.B * a.N, a.Hq, a.G);
-    if (rc != GV_OK) return rc;
-    // Query rows above 128 go to a second cluster of one-tile CTAs rather
-    // than a second M tile in the same CTAs: twice the SMs on the key blocks,
-    // half the rows in each cluster's exchange.
-    return kRowSplit || (a.R + 127) / 128 == 1 ? launch_mt<1>(a, mk, mv, mq, st)
-                                                : launch_mt<2>(a, mk, mv, mq, st);
 }
 
 }  // namespace gv
