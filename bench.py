@@ -91,9 +91,9 @@ def attention_bytes(cfg):
 
 def launches_per_step(cfg):
     """Kernels of this library one step launches: tree build, RoPE table, the
-    attention layers (one kernel each on the bf16 tensor-core path, rotate +
+    attention layers (split attention + merge on the bf16 tensor-core path, rotate +
     split + combine on the fp32 path), LM head + merge, accept, compaction."""
-    per_layer = 1 if cfg["dtype"] == "bf16" else 3
+    per_layer = 2 if cfg["dtype"] == "bf16" else 3
     return 2 + per_layer * cfg["L"] + 2 + 1 + 1
 
 

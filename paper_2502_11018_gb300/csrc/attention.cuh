@@ -27,10 +27,12 @@ struct AttnArgs {
     void* q_rot;      // [B*Hkv][q_rows_pad][d]  rotated queries          (CUDA-core path)
     float* part_o;    // [B*Hkv][nsplit][R][d]   per-split partial outputs (CUDA-core path)
     float* part_ml;   // [B*Hkv][nsplit][R][2] (m, l)                  (CUDA-core path)
+                      // [units][csize][128] lse                       (tensor-core path)
+    void* part_o_bf16;  // [units][csize][128][d] bf16 rows, chunks rotated (tensor-core path)
     int nsplit;       // prefix splits + 1 tree split (CUDA-core path)
     int kps;          // prefix keys per split (CUDA-core path)
-    int csize;        // CTAs per cluster (tensor-core path)
-    int tiles;        // clusters per (sequence, KV head), each on its own group of query rows
+    int csize;        // key splits (CTAs) per unit (tensor-core path)
+    int tiles;        // M tiles of 128 query rows per (sequence, KV head); unit = (b, g, tile)
 };
 
 int launch_rope_table(const int32_t* pos, int B, int N, int d, float base, float* rope,
@@ -39,5 +41,6 @@ int launch_rope_tree_f32(const AttnArgs& a, cudaStream_t st);
 int launch_attn_combine_f32(const AttnArgs& a, cudaStream_t st);
 int launch_attn_cc_f32(const AttnArgs& a, cudaStream_t st);
 int launch_attn_tc(const AttnArgs& a, cudaStream_t st);
+int attn_tc_splits(int units, int S_max);
 
 }  // namespace gv

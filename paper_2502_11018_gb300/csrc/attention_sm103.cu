@@ -7,12 +7,12 @@
 //
 // Query rows: row r = i * G + hl of KV head g holds tree node i and query
 // head g * G + hl; all G * N rows of (b, g) share every K/V block (GQA), and
-// each 128 of them form one MMA M tile.  One thread-block cluster of C CTAs
-// per (sequence b, KV head g, M tile).  The keys of (b, g) are cut into
+// each 128 of them form one MMA M tile.  A unit = (sequence b, KV head g, M
+// tile); each unit gets C CTAs (key splits).  The keys of (b, g) are cut into
 // 64-key blocks: ceil(P_b / 64) prefix blocks and one tree block (the N <= 64
-// tree keys, masked per query row by its ancestor bitmask).  CTA `rank` of
-// the cluster takes blocks rank, rank + C, ...; the CTA that owns the tree
-// block runs it first.
+// tree keys, masked per query row by its ancestor bitmask).  The last split
+// runs the tree block first and then the last prefix blocks; the others take
+// the remaining prefix blocks round robin.
 //
 // Per block j of a CTA:
 //   S_j = Q K_j^T          tcgen05.mma, Q and K K-major 128B-swizzled in smem,
@@ -28,27 +28,24 @@
 //                          to one of two smem buffers
 //   O_h += P_j,h V_j,h     tcgen05.mma, P K-major, V MN-major (d contiguous),
 //                          one accumulator per key half h
-// Each CTA then merges its two halves and stages o = O / l (bf16) and
-// lse = m + log2(l) of its rows in its shared memory; after a cluster barrier
-// it pushes to every CTA of the cluster (bulk copies into distributed shared
-// memory) the 1/C share of rows that CTA merges, and every CTA merges its
-// share over the C partials and writes the final bf16 output: the split
-// combine needs no extra launch and no global scratch.
+// Each CTA then merges its two halves and writes o = O / l (bf16) and
+// lse = m + log2(l) of its rows to the workspace (L2-resident), and
+// attn_merge_kernel, launched right behind it, combines the C splits of every
+// row into the bf16 output.  No CTA waits for another, so the splits need no
+// cluster co-scheduling and the grid fills the SMs.
 //
 // Warp roles: warp 0 issues the TMA loads (RoPE rows, K/V blocks, raw Q
 // tile); warp 1 owns TMEM and issues the MMAs; warps 2..9 rotate Q in place
 // (RoPE from the per-step table), build the tree K/V tile, and run the
-// softmax and the staging; all warps share the merge.
+// softmax and the staging.
 //
-// Launch: cluster launch (the cluster barrier orders the partial exchange and
-// guarantees the C CTAs are co-resident) with programmatic dependent launch.
-// Before griddepcontrol.wait a CTA only initialises barriers and TMEM, reads
-// step inputs written before the step's first attention launch (RoPE table,
-// ancestor masks, prefix lengths) and starts streaming two K/V cache blocks;
-// queries, tree keys/values and the output are touched after it.  Every
-// mbarrier wait is bounded; a CTA that gives up marks its rows' lse NaN,
-// which turns the affected outputs into NaN, and still reaches the cluster
-// barriers.
+// Both kernels use programmatic dependent launch.  Before griddepcontrol.wait
+// a CTA only initialises barriers and TMEM, reads step inputs written before
+// the step's first attention launch (RoPE table, ancestor masks, prefix
+// lengths) and starts streaming two K/V cache blocks; queries, tree
+// keys/values, the workspace and the output are touched after it.  Every
+// mbarrier wait is bounded; a CTA that gives up writes NaN lse for its rows,
+// which turns the affected outputs into NaN.
 #include "gv_internal.cuh"
 #include "attention.cuh"
 #include "sm103.cuh"
@@ -79,15 +76,6 @@ __device__ __forceinline__ void grid_dep_wait() {
 }
 __device__ __forceinline__ void grid_dep_launch() {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ uint32_t cluster_rank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-__device__ __forceinline__ void cluster_sync() {
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
-                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 // Packed fp32 pairs (one instruction for two lanes' worth of work) and the
 // three-input max of sm_100+.
@@ -166,13 +154,14 @@ constexpr uint32_t AT_TMEM_COLS = 512;    // S double buffer [0,128), O_0 [128,2
 
 __global__ void __launch_bounds__(AT_NTH, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
-               const __grid_constant__ CUtensorMap map_q, AttnArgs a) {
-    constexpr int NSM = AT_NSM, NTH = AT_NTH, ST = AT_ST;
-    const int C = a.csize;
-    const int rank = (int)cluster_rank();
-    // Cluster -> (sequence b, KV head g, M tile): the G * N query rows of
-    // (b, g) are cut into tiles of 128, one cluster per tile.
+               const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_rope,
+               AttnArgs a) {
+    constexpr int NSM = AT_NSM, ST = AT_ST;
+    const int C = a.csize;                     // key splits per unit
+    // CTA -> unit (sequence b, KV head g, M tile of 128 query rows) and key
+    // split `rank` of that unit.
     const int cl = blockIdx.x / C;
+    const int rank = blockIdx.x - cl * C;
     const int bg = cl / a.tiles;
     const int tile0 = cl % a.tiles;
     const int b = bg / a.Hkv, g = bg % a.Hkv;
@@ -180,20 +169,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     // stream started, so it may be read before griddepcontrol.wait.
     const int P = min(max(a.prefix_len[b], 0), a.S_max);
     const int nb_pre = (P + AT_BK - 1) / AT_BK;
-    // Prefix blocks go round robin from rank 0, so the highest ranks hold the
-    // fewest; the tree block goes to the last rank and runs first there.
+    // The tree block goes to the last split and runs first there; it counts
+    // as two blocks (its tile is built from the tree's keys and values on the
+    // critical path).  The last split takes the last nt prefix blocks, the
+    // other splits the first `rest` blocks round robin.
     const bool has_tree = rank == C - 1;
-    const int nblk = (nb_pre > rank ? (nb_pre - 1 - rank) / C + 1 : 0) + (has_tree ? 1 : 0);
+    const int per = (nb_pre + 2 + C - 1) / C;
+    const int nt = C == 1 ? nb_pre : max(0, min(nb_pre, per - 2));
+    const int rest = nb_pre - nt;
+    const int nblk = has_tree ? nt + 1 : (rest > rank ? (rest - 1 - rank) / (C - 1) + 1 : 0);
     const int nb_per_tile = 128 / a.G;                   // nodes per M tile
     const int row0 = tile0 * 128;                        // first query row of this cluster
-    const int R = min(a.G * a.N - row0, 128);            // query rows of this cluster
-    const int Rc = (R + C - 1) / C;                      // rows each CTA merges
-    const int slab_bytes = Rc * 256 + ((Rc + 3) & ~3) * 4;   // Rc bf16 rows + Rc lse (16-byte multiple)
-    const int r_own = min(R, rank * Rc + Rc) - rank * Rc;    // rows this CTA merges (<= 0: none)
+    const int R = min(a.G * a.N - row0, 128);            // query rows of this unit
     // Prefix block index of this CTA's j-th block (-1 for the tree block).
     auto prefix_block = [&](int j) -> int {
-        if (has_tree) return j == 0 ? -1 : rank + C * (j - 1);
-        return rank + C * j;
+        if (has_tree) return j == 0 ? -1 : rest + (j - 1);
+        return rank + (C - 1) * j;
     };
 
     extern __shared__ uint8_t smem_raw[];
@@ -214,11 +205,16 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint64_t* q_full = q_raw + 1;
     uint64_t* drain = q_full + 1;
     uint64_t* rope_full = drain + 1;
-    uint64_t* recv_full = rope_full + 1;
-    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(recv_full + 1);
-    // The RoPE rows of sequence b (N x 64 (cos, sin) pairs) are staged in the
-    // P area, which is free until the first softmax block writes P.
-    const float4* sRope = reinterpret_cast<const float4*>(sP);
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(rope_full + 1);
+    // The RoPE rows of sequence b (N x 64 (cos, sin) pairs, 512 B per node)
+    // are staged in the P area, which is free until the first softmax block
+    // writes P, as four 128B-swizzled column boxes of 32 floats x N rows (8 KB
+    // apart): the lanes of a warp read the same pairs of 8 consecutive nodes
+    // from 8 different banks.  (cos, sin) of pairs 8c + 2q, 8c + 2q + 1:
+    auto rope_cs = [&](int n, int c, int q) -> float4 {
+        return *reinterpret_cast<const float4*>(sP + (c >> 1) * 8192 + n * 128 +
+                                                (((4 * (c & 1) + q) ^ (n & 7)) << 4));
+    };
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -237,12 +233,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         mbar_init(q_full, 1);
         mbar_init(drain, 1);
         mbar_init(rope_full, 1);
-        mbar_init(recv_full, 1);
-        if (r_own > 0) mbar_arrive_expect_tx(recv_full, (uint32_t)(C * slab_bytes));
         *abort = 0;
         fence_mbar_init();
         if (nblk > 0) {
             prefetch_tmap(&map_q);
+            prefetch_tmap(&map_rope);
             prefetch_tmap(&map_k);
             prefetch_tmap(&map_v);
         }
@@ -275,8 +270,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 // RoPE rows first: written by a kernel that completed before
                 // the step's first attention launch, so safe before the wait.
                 mbar_arrive_expect_tx(rope_full, (uint32_t)a.N * 512u);
-                bulk_load(sP, reinterpret_cast<const char*>(a.rope) + (size_t)b * a.N * 512,
-                          (uint32_t)a.N * 512u, rope_full);
+                for (int cb = 0; cb < 4; ++cb)
+                    tma_load_2d(sP + cb * 8192, &map_rope, rope_full, cb * 32, b * a.N, pol_q);
                 int issued[ST];
                 for (int q = 0; q < ST; ++q) issued[q] = -1;
                 bool q_issued = false;
@@ -399,7 +394,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         vhi = __ldg(vr + 8 + c);
                         float4 cs[4];
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) cs[q] = sRope[j * 32 + c * 4 + q];
+                        for (int q = 0; q < 4; ++q) cs[q] = rope_cs(j, c, q);
                         rope8(k0, k1, cs, klo, khi);
                         uint4* tk = reinterpret_cast<uint4*>(a.treeK) + ((size_t)bg * a.N + j) * 16;
                         uint4* tv = reinterpret_cast<uint4*>(a.treeV) + ((size_t)bg * a.N + j) * 16;
@@ -439,7 +434,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         if (row_ok) {
                             float4 cs[4];
 #pragma unroll
-                            for (int q = 0; q < 4; ++q) cs[q] = sRope[node * 32 + (4 * kh + c) * 4 + q];
+                            for (int q = 0; q < 4; ++q) cs[q] = rope_cs(node, 4 * kh + c, q);
                             rope8(lo[c], hi[c], cs, olo, ohi);
                         }
                         lo[c] = olo;
@@ -585,19 +580,16 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         }
     }
 
-    // ------------------------------- exchange partial rows through the cluster
-    // Each CTA merges its two key halves and stages its rows' normalised
-    // partial o = O / l (bf16) and lse = m + log2(l) (fp32) in its own (now
-    // free) Q and P areas as C slabs: slab q holds rows [q * Rc, (q + 1) * Rc),
-    // the rows CTA q merges, with the 16-byte chunks of row k of a slab rotated
-    // by (k & 15) so that the lanes of a warp store and load distinct banks.
-    // After a cluster barrier (every CTA is past its main loop, so its K/V ring
-    // is idle) thread 0 pushes slab q into the K/V ring of CTA q with one bulk
-    // shared::cta -> shared::cluster copy that completes on CTA q's
-    // `recv_full` barrier; CTA q merges its rows over the C slabs it received
-    // and writes the output.  lse is -inf for a CTA without blocks and NaN for
+    // ------------------------------------------------ partial rows to the workspace
+    // The two key halves of every row are merged, and the row's normalised
+    // partial o = O / l (bf16, the 16-byte chunks of row r rotated by r & 15
+    // so that the lanes of a warp store distinct banks) and lse = m + log2(l)
+    // are staged in the (now free) Q and P areas, then written to the
+    // workspace with one bulk copy each; attn_merge_kernel combines the C
+    // splits of every row.  lse is -inf for a CTA without blocks and NaN for
     // one that gave up.
-    uint8_t* stg = sQ;
+    uint8_t* stg = sQ;                                  // R rows x 256 B
+    float* stg_lse = reinterpret_cast<float*>(sP);      // R floats
     int w = 0;
     if (warp >= 2) {
         w = ok && nblk > 0 ? 1 : 0;
@@ -609,15 +601,17 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     // The halves' (m, l) and the last PV are visible after this barrier; the
     // CTA's partial is valid only if every softmax warp finished.
     w = __syncthreads_and(warp < 2 || w);
+    // The workspace may still be read by the previous grid (the merge of the
+    // previous call): wait for it before writing (a no-op if already done).
+    grid_dep_wait();
     if (warp >= 2) {
         const bool mine = row < R;
-        const int q = row / Rc, k = row - q * Rc;
-        uint8_t* slab = stg + (size_t)q * slab_bytes;
         const float2 other = sML[(1 - kh) * 128 + row];
         const float M = fmaxf(m_used, other.x);
         const float ws = m_used == -INFINITY ? 0.f : fast_exp2(m_used - M);
         const float wo = other.x == -INFINITY ? 0.f : fast_exp2(other.x - M);
         const float ltot = l * ws + other.y * wo;
+        uint8_t* srow = stg + row * 256;
         if (w) {
             // This thread writes d columns [64 kh, 64 kh + 64) of the row:
             // O_kh and O_{1-kh} there, weighted by their halves' max offsets.
@@ -639,7 +633,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
 #pragma unroll
                         for (int u = 0; u < 8; ++u)
                             v[u] = __uint_as_float(os[e + u]) * as + __uint_as_float(oo[e + u]) * ao;
-                        *reinterpret_cast<uint4*>(slab + k * 256 + ((ch ^ (k & 15)) << 4)) =
+                        *reinterpret_cast<uint4*>(srow + ((ch ^ (row & 15)) << 4)) =
                             make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]),
                                        pack_bf16(v[4], v[5]), pack_bf16(v[6], v[7]));
                     }
@@ -648,14 +642,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         }
         if (mine) {
             if (kh == 0)
-                reinterpret_cast<float*>(slab + Rc * 256)[k] =
-                    w ? (ltot > 0.f ? M + log2f(ltot) : -INFINITY) : (nblk > 0 ? NAN : -INFINITY);
+                stg_lse[row] = w ? (ltot > 0.f ? M + log2f(ltot) : -INFINITY) : (nblk > 0 ? NAN : -INFINITY);
             if (!w) {
                 // No partial (no blocks, or gave up): zeros, so that the
-                // merge may weight every slab without testing its weight.
+                // merge may weight every split without testing its weight.
 #pragma unroll
                 for (int ch = 0; ch < 8; ++ch)
-                    *reinterpret_cast<uint4*>(slab + k * 256 + ((8 * kh + ch) << 4)) = make_uint4(0, 0, 0, 0);
+                    *reinterpret_cast<uint4*>(srow + ((8 * kh + ch) << 4)) = make_uint4(0, 0, 0, 0);
             }
         }
     }
@@ -666,60 +659,62 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         // A role gave up, so a copy may have landed in the staging area after
         // the rows were staged (each role drains its own copies before the
         // barrier above): mark every row of this CTA invalid again.
-        if (warp >= 2 && kh == 0 && row < R) {
-            const int q = row / Rc;
-            reinterpret_cast<float*>(stg + (size_t)q * slab_bytes + Rc * 256)[row - q * Rc] = NAN;
-        }
+        if (warp >= 2 && kh == 0 && row < R) stg_lse[row] = NAN;
         __syncthreads();
     }
     if (warp == 1) tmem_dealloc(tmem, AT_TMEM_COLS);
-    if (threadIdx.x == 0) fence_proxy_async_smem();   // the staged slabs, for the pushes
-    cluster_sync();
     if (threadIdx.x == 0) {
-        const uint32_t dst = smem_u32(sKV) + (uint32_t)(rank * slab_bytes);
-        const uint32_t bar = smem_u32(recv_full);
-        for (int q = 0; q < C && q * Rc < R; ++q)
-            bulk_copy_to_cluster(mapa_cluster(dst, (uint32_t)q), stg + (size_t)q * slab_bytes,
-                                 (uint32_t)slab_bytes, mapa_cluster(bar, (uint32_t)q));
+        fence_proxy_async_smem();   // the staged rows, for the bulk copies
+        const size_t split = (size_t)cl * C + rank;
+        bulk_store(static_cast<uint8_t*>(a.part_o_bf16) + split * 128 * 256, stg, (uint32_t)R * 256u);
+        bulk_store(a.part_ml + split * 128, stg_lse, (uint32_t)((R + 3) & ~3) * 4u);
+        bulk_commit();
+        bulk_wait_all();            // written before the grid completes
     }
+}
 
-    // ----------------------------------------- merge the rows this CTA owns
-    const int r_lo = rank * Rc, n_own = max(0, min(R, r_lo + Rc) - r_lo);
-    int got = 1;
-    if (n_own > 0) {
-        // Wait for all C slabs even if another role gave up: nothing may
-        // still be writing into this CTA's shared memory when it exits.
-        if (lane == 0) got = mbar_wait_timeout_only(recv_full, 0) ? 1 : 0;
-        got = __shfl_sync(FULL, got, 0);
-        if (!got) *abort = 1;
+// Combines the C key splits of every query row: one thread per (row, 16-byte
+// chunk of d), weights 2^(lse_s - max lse) over the splits, bf16 output.
+// Launched right after attn_tc_kernel with programmatic dependent launch; it
+// reads the partials after griddepcontrol.wait.
+constexpr int AM_ROWS = 8;                  // rows per CTA (x 16 chunks = 128 threads)
+
+__global__ void __launch_bounds__(AM_ROWS * 16)
+attn_merge_kernel(AttnArgs a) {
+    grid_dep_launch();
+    const int C = a.csize;
+    const int cl = blockIdx.x / (128 / AM_ROWS);         // unit
+    const int row = (blockIdx.x % (128 / AM_ROWS)) * AM_ROWS + (threadIdx.x >> 4);
+    const int ch = threadIdx.x & 15;
+    const int bg = cl / a.tiles, tile0 = cl % a.tiles;
+    const int b = bg / a.Hkv, g = bg % a.Hkv;
+    const int r = tile0 * 128 + row;                    // query row of (b, g)
+    if (row >= 128 || r >= a.G * a.N) return;
+    grid_dep_wait();
+    const size_t split0 = (size_t)cl * C;
+    float lsv[16];
+    float M = -INFINITY;
+    bool bad = false;
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+        lsv[q] = q < C ? __ldcg(a.part_ml + (split0 + q) * 128 + row) : -INFINITY;
+        bad |= lsv[q] != lsv[q];
+        M = fmaxf(M, lsv[q]);
     }
-    // Every push into this CTA has landed: release the other CTAs' exit.
-    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
-    grid_dep_wait();   // the output may be written only after the previous grid
-    // One thread per (row, 16-byte chunk of d): C weights, C chunk loads and
-    // 8 FMAs per slab, all loads independent.
-    const uint8_t* recv = sKV;
-    for (int task = threadIdx.x; task < n_own * 16; task += NTH) {
-        const int k = task >> 4, ch = task & 15;
-        float lsv[16];
-        float M = -INFINITY;
-        bool bad = !got;
+    const uint8_t* po = static_cast<const uint8_t*>(a.part_o_bf16);
+    const size_t off = (size_t)row * 256 + ((ch ^ (row & 15)) << 4);
+    uint4 v[16];
 #pragma unroll
-        for (int q = 0; q < 16; ++q) {
-            lsv[q] = q < C ? reinterpret_cast<const float*>(recv + q * slab_bytes + Rc * 256)[k] : -INFINITY;
-            bad |= lsv[q] != lsv[q];
-            M = fmaxf(M, lsv[q]);
-        }
-        const int off = k * 256 + ((ch ^ (k & 15)) << 4);
-        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        float wsum = 0.f;
+    for (int q = 0; q < 16; ++q)
+        if (q < C) v[q] = __ldcg(reinterpret_cast<const uint4*>(po + (split0 + q) * 128 * 256 + off));
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    float wsum = 0.f;
 #pragma unroll
-        for (int q = 0; q < 16; ++q) {
-            if (q >= C) break;
+    for (int q = 0; q < 16; ++q) {
+        if (q < C) {
             const float wq = lsv[q] == -INFINITY ? 0.f : fast_exp2(lsv[q] - M);
-            const uint4 v = *reinterpret_cast<const uint4*>(recv + q * slab_bytes + off);
             wsum += wq;
-            const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+            const uint32_t u[4] = {v[q].x, v[q].y, v[q].z, v[q].w};
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const float2 f = unpack_bf16(u[e]);
@@ -727,16 +722,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 acc[2 * e + 1] = fmaf(wq, f.y, acc[2 * e + 1]);
             }
         }
-        const float inv = bad ? NAN : 1.0f / wsum;
-        const int r = row0 + r_lo + k;
-        const int i = r / a.G, h = g * a.G + r % a.G;
-        __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out) + (((size_t)b * a.N + i) * a.Hq + h) * 128;
-        reinterpret_cast<uint4*>(o)[ch] =
-            make_uint4(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv),
-                       pack_bf16(acc[4] * inv, acc[5] * inv), pack_bf16(acc[6] * inv, acc[7] * inv));
     }
-    // The slabs this CTA pushed have landed once every CTA has arrived.
-    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+    const float inv = bad ? NAN : 1.0f / wsum;
+    const int i = r / a.G, h = g * a.G + r % a.G;
+    __nv_bfloat16* o = static_cast<__nv_bfloat16*>(a.out) + (((size_t)b * a.N + i) * a.Hq + h) * 128;
+    reinterpret_cast<uint4*>(o)[ch] =
+        make_uint4(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv),
+                   pack_bf16(acc[4] * inv, acc[5] * inv), pack_bf16(acc[6] * inv, acc[7] * inv));
 }
 
 // ----------------------------------------------------------------- host side
@@ -772,51 +764,48 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G) {
 
 static size_t attn_tc_smem() {
     return 1024 + (size_t)AT_QTILE + 2 * AT_PTILE + (size_t)AT_ST * AT_STAGE + 2 * 128 * sizeof(float2) +
-           8 * (2 * AT_ST + 13) + 16;
+           8 * (2 * AT_ST + 12) + 16;
 }
 
-// CTAs per cluster.  Wanted: as many as fit the SMs in one wave (at most 16,
-// the largest cluster GB300 schedules), at least 4 for long caches so that a
-// long sequence of a ragged batch is not one CTA's serial work.  When the
-// whole grid fits in one wave, the size is lowered until every cluster can be
-// resident at once (GPC boundaries limit how many large clusters of
-// 1-CTA-per-SM kernels fit), since a cluster left for a second wave doubles
-// the layer's time.
-static int attn_tc_cluster(int units, int S_max, size_t smem) {
-    static int max_active[17] = {};
-    int want = sm_count() / units;                  // one wave of 1-CTA-per-SM clusters
-    if (S_max >= 4096 && want < 4) want = 4;
-    if (want > 16) want = 16;
-    if (want < 1) want = 1;
-    for (int c = want; c >= 1; --c) {
-        if (max_active[c] == 0) {
-            cudaLaunchConfig_t cfg{};
-            cfg.gridDim = dim3((unsigned)(c * units));
-            cfg.blockDim = dim3(AT_NTH);
-            cfg.dynamicSmemBytes = smem;
-            cudaLaunchAttribute attr[1];
-            attr[0].id = cudaLaunchAttributeClusterDimension;
-            attr[0].val.clusterDim.x = (unsigned)c;
-            attr[0].val.clusterDim.y = 1;
-            attr[0].val.clusterDim.z = 1;
-            cfg.attrs = attr;
-            cfg.numAttrs = 1;
-            int n = 0;
-            if (cudaOccupancyMaxActiveClusters(&n, attn_tc_kernel, &cfg) != cudaSuccess) {
-                cudaGetLastError();
-                n = -1;
-            }
-            max_active[c] = n;
-        }
-        const int n = max_active[c];
-        if (n < 0) continue;                        // not schedulable at this size
-        if (units * c > sm_count() || n >= units) return c;
+// Key splits per unit (CTAs per (sequence, KV head, M tile)): as many as fit
+// the SMs in one wave of 1-CTA-per-SM CTAs, at most 16, and at least 4 for
+// long caches so that a long sequence of a ragged batch is not one CTA's
+// serial work; never more than the blocks a unit can have.  The workspace
+// plan uses the same count.
+int attn_tc_splits(int units, int S_max) {
+    int c = sm_count() / units;
+    if (S_max >= 4096 && c < 4) c = 4;
+    const int blocks = (S_max + AT_BK - 1) / AT_BK + 1;   // most 64-key blocks a unit can have
+    if (c > blocks) c = blocks;
+    if (c > 16) c = 16;
+    if (c < 1) c = 1;
+    return c;
+}
+
+// 2-D map over the RoPE table rope[B*N][128] (fp32) with box {32 floats,
+// N rows}, 128B-swizzled.
+static int make_map_rope(CUtensorMap* map, const float* rope, int BN, int N) {
+    EncodeTiledFn enc = tensor_map_encoder();
+    if (!enc) {
+        set_error("cuTensorMapEncodeTiled unavailable");
+        return GV_ERR_CUDA;
     }
-    return 1;
+    cuuint64_t dims[2] = {128, (cuuint64_t)BN};
+    cuuint64_t strides[1] = {512};
+    cuuint32_t box[2] = {32, (cuuint32_t)N};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(rope), dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        set_error("cuTensorMapEncodeTiled (rope) failed (%d)", (int)r);
+        return GV_ERR_CUDA;
+    }
+    return GV_OK;
 }
 
 int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
-    CUtensorMap mk, mv, mq;
+    CUtensorMap mk, mv, mq, mr;
     const uint64_t rows = (uint64_t)a0.B * a0.Hkv * a0.S_max;
     int rc = make_map_2d(&mk, a0.cacheK, rows, 128, AT_BK, 256);
     if (rc != GV_OK) return rc;
@@ -824,31 +813,35 @@ int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
     if (rc != GV_OK) return rc;
     rc = make_map_q(&mq, a0.q, a0.B * a0.N, a0.Hq, a0.G);
     if (rc != GV_OK) return rc;
+    rc = make_map_rope(&mr, a0.rope, a0.B * a0.N, a0.N);
+    if (rc != GV_OK) return rc;
     const size_t smem = attn_tc_smem();
     cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    // Every 128 query rows of a (sequence, KV head) get their own cluster.
-    AttnArgs a = a0;
-    a.tiles = (a0.R + 127) / 128;
-    const int units = a0.B * a0.Hkv * a.tiles;
-    a.csize = attn_tc_cluster(units, a.S_max, smem);
+    const int units = a0.B * a0.Hkv * a0.tiles;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
     cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3((unsigned)(units * a.csize));
+    cfg.gridDim = dim3((unsigned)(units * a0.csize));
     cfg.blockDim = dim3(AT_NTH);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[2];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    attr[1].id = cudaLaunchAttributeClusterDimension;
-    attr[1].val.clusterDim.x = (unsigned)a.csize;
-    attr[1].val.clusterDim.y = 1;
-    attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 2;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, attn_tc_kernel, mk, mv, mq, a);
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, attn_tc_kernel, mk, mv, mq, mr, a0);
     if (e != cudaSuccess) {
-        set_error("attn_tc_kernel launch (cluster %d): %s", a.csize, cudaGetErrorString(e));
+        set_error("attn_tc_kernel launch: %s", cudaGetErrorString(e));
+        return GV_ERR_CUDA;
+    }
+    cudaLaunchConfig_t mcfg{};
+    mcfg.gridDim = dim3((unsigned)(units * (128 / AM_ROWS)));
+    mcfg.blockDim = dim3(AM_ROWS * 16);
+    mcfg.stream = st;
+    mcfg.attrs = attr;
+    mcfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&mcfg, attn_merge_kernel, a0);
+    if (e != cudaSuccess) {
+        set_error("attn_merge_kernel launch: %s", cudaGetErrorString(e));
         return GV_ERR_CUDA;
     }
     return GV_OK;

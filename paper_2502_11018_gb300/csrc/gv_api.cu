@@ -83,6 +83,7 @@ constexpr int KPS_F32 = 256;   // prefix keys per split, CUDA-core path
 struct AttnPlan {
     size_t q_rot, part_o, part_ml, total;
     int nsplit, q_rows_pad, kps;
+    int tiles, csize;   // tensor-core path: M tiles per (b, g), key splits per unit
 };
 
 // Shapes the kernels handle: fp32 with d in {64, 128}; bf16 (tensor cores)
@@ -100,7 +101,8 @@ static int attn_shape_status(const gv_attn_shape* s) {
 }
 
 // The fp32 path keeps rotated queries and per-split partials in the
-// workspace; the bf16 path reduces its splits on chip and needs none.
+// workspace; the bf16 path keeps one bf16 partial row and one lse per (unit,
+// key split, row of the unit's 128-row tile), for its merge kernel.
 static AttnPlan attn_plan(const gv_attn_shape* s) {
     AttnPlan p{};
     const int R = (s->Hq / s->Hkv) * s->N;
@@ -117,7 +119,14 @@ static AttnPlan attn_plan(const gv_attn_shape* s) {
         p.part_ml = off;
         off += align256(bh * p.nsplit * R * 2 * sizeof(float));
     } else {
-        off += 256;   // none used: the cluster merges its splits in shared memory
+        p.tiles = (R + 127) / 128;
+        const int units = s->B * s->Hkv * p.tiles;
+        p.csize = attn_tc_splits(units, s->S_max);
+        const size_t nrows = (size_t)units * p.csize * 128;
+        p.part_o = off;
+        off += align256(nrows * 128 * 2);
+        p.part_ml = off;
+        off += align256(nrows * sizeof(float));
     }
     p.total = off;
     return p;
@@ -297,6 +306,9 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
     a.q_rot = ws + plan.q_rot;
     a.part_o = reinterpret_cast<float*>(ws + plan.part_o);
     a.part_ml = reinterpret_cast<float*>(ws + plan.part_ml);
+    a.part_o_bf16 = ws + plan.part_o;
+    a.tiles = plan.tiles;
+    a.csize = plan.csize;
     a.nsplit = plan.nsplit;
     a.kps = plan.kps;
     cudaStream_t st = as_stream(stream);
