@@ -16,8 +16,8 @@
 //
 // Per block j of a CTA:
 //   S_j = Q K_j^T          tcgen05.mma, Q and K K-major 128B-swizzled in smem,
-//                          fp32 S in TMEM (two buffers: S_{j+1} overlaps the
-//                          softmax of block j)
+//                          fp32 S in TMEM (three buffers: S_{j+1} and S_{j+2}
+//                          are computed during the softmax of block j)
 //   softmax                two threads per query row, one per 32-key half of
 //                          the block, read their S row half from TMEM, mask
 //                          with a branch-free validity mask (prefix end, or
@@ -150,7 +150,9 @@ __device__ __forceinline__ void rope8(const uint4& lo, const uint4& hi, const fl
 constexpr int AT_NSM = 256;               // softmax threads: 128 rows x 2 key halves
 constexpr int AT_NTH = 64 + AT_NSM;       // + TMA producer warp + MMA warp
 constexpr int AT_ST = 4;                  // K/V stages
-constexpr uint32_t AT_TMEM_COLS = 512;    // S double buffer [0,128), O_0 [128,256), O_1 [256,384)
+constexpr int AT_SB = 3;                  // S buffers in TMEM
+constexpr uint32_t AT_OCOL = 256;         // O_h at columns [256 + 128 h, 384 + 128 h)
+constexpr uint32_t AT_TMEM_COLS = 512;    // S buffers [0, 192), O_0, O_1
 
 __global__ void __launch_bounds__(AT_NTH, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
@@ -198,8 +200,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint64_t* kv_full = bars;
     uint64_t* kv_empty = kv_full + ST;
     uint64_t* s_full = kv_empty + ST;
-    uint64_t* s_free = s_full + 2;
-    uint64_t* p_full = s_free + 2;
+    uint64_t* s_free = s_full + AT_SB;
+    uint64_t* p_full = s_free + AT_SB;
     uint64_t* o_done = p_full + 2;
     uint64_t* q_raw = o_done + 2;
     uint64_t* q_full = q_raw + 1;
@@ -223,9 +225,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             mbar_init(&kv_full[s], 1);
             mbar_init(&kv_empty[s], 1);
         }
-        for (int c = 0; c < 2; ++c) {
+        for (int c = 0; c < AT_SB; ++c) {
             mbar_init(&s_full[c], 1);
             mbar_init(&s_free[c], NSM / 32);
+        }
+        for (int c = 0; c < 2; ++c) {
             mbar_init(&p_full[c], NSM / 32);
             mbar_init(&o_done[c], 1);
         }
@@ -257,7 +261,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     const int node = tile0 * nb_per_tile + row / a.G;    // tree node of this row
     const bool row_ok = warp >= 2 && node < a.N;
     const uint32_t lane_base = tmem + ((uint32_t)(sub * 32) << 16);
-    const uint32_t ocol_self = lane_base + 128u + 128u * (uint32_t)kh;   // O of this key half
+    const uint32_t ocol_self = lane_base + AT_OCOL + 128u * (uint32_t)kh;   // O of this key half
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
 
@@ -316,33 +320,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 const uint32_t idesc_o = idesc_bf16(128, 128, /*b_mn_major=*/true);
                 bool mok = mbar_wait(q_full, 0, abort);
                 tc_fence_after();
-                auto issue_pv = [&](int jj) -> bool {
-                    const int pb = jj & 1;
-                    if (!mbar_wait(&p_full[pb], (uint32_t)(jj >> 1) & 1u, abort)) return false;
-                    tc_fence_after();
-                    const int sp = jj % ST;
-                    // V as the MN-major B operand: rows = keys (128 B apart, SBO =
-                    // 1 KB per 8 keys), the two 64-wide halves of d LBO = 8 KB apart.
-                    uint64_t vdesc = sdesc_kmajor_sw128(smem_u32(sKV + sp * AT_STAGE + 2 * AT_KV_HALF));
-                    vdesc = (vdesc & ~(0x3FFFull << 16)) | ((uint64_t)(AT_KV_HALF >> 4) << 16);
-                    const uint64_t pdesc = sdesc_kmajor_sw128(smem_u32(sP + pb * AT_PTILE));
-                    // Keys 0..31 (K steps 0, 1) into O_0, keys 32..63 into O_1.
-#pragma unroll
-                    for (int kk = 0; kk < AT_BK / 16; ++kk)
-                        mma_bf16(tmem + 128u + 128u * (uint32_t)(kk >> 1), pdesc + 2u * kk,
-                                 vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (kk & 1));
-                    mma_commit(&kv_empty[sp]);
-                    mma_commit(&o_done[pb]);
-                    return true;
-                };
-                for (int j = 0; mok && j < nblk; ++j) {
-                    const int s = j % ST, buf = j & 1;
-                    if (!mbar_wait(&kv_full[s], (uint32_t)(j / ST) & 1u, abort) ||
-                        !mbar_wait(&s_free[buf], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort)) {
-                        mok = false;
-                        break;
-                    }
-                    tc_fence_after();
+                // S_j = Q K_j^T into S buffer j % 3, as soon as block j's K/V
+                // has landed and softmax j - 3 has read that buffer.
+                auto issue_s = [&](int jj) {
+                    const int s = jj % ST, buf = jj % AT_SB;
                     const uint32_t kbase = smem_u32(sKV + s * AT_STAGE);
 #pragma unroll
                     for (int kb = 0; kb < 2; ++kb) {
@@ -354,12 +335,48 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                                      idesc_s, (kb | kk) != 0);
                     }
                     mma_commit(&s_full[buf]);
-                    if (j >= 1 && !issue_pv(j - 1)) {
+                };
+                // O_h += P_j,h V_j,h once softmax j has written P_j.
+                auto issue_pv = [&](int jj) {
+                    const int pb = jj & 1, sp = jj % ST;
+                    // V as the MN-major B operand: rows = keys (128 B apart, SBO =
+                    // 1 KB per 8 keys), the two 64-wide halves of d LBO = 8 KB apart.
+                    uint64_t vdesc = sdesc_kmajor_sw128(smem_u32(sKV + sp * AT_STAGE + 2 * AT_KV_HALF));
+                    vdesc = (vdesc & ~(0x3FFFull << 16)) | ((uint64_t)(AT_KV_HALF >> 4) << 16);
+                    const uint64_t pdesc = sdesc_kmajor_sw128(smem_u32(sP + pb * AT_PTILE));
+                    // Keys 0..31 (K steps 0, 1) into O_0, keys 32..63 into O_1.
+#pragma unroll
+                    for (int kk = 0; kk < AT_BK / 16; ++kk)
+                        mma_bf16(tmem + AT_OCOL + 128u * (uint32_t)(kk >> 1), pdesc + 2u * kk,
+                                 vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (kk & 1));
+                    mma_commit(&kv_empty[sp]);
+                    mma_commit(&o_done[pb]);
+                };
+                // Issue whichever is ready (S first: the softmax waits on it),
+                // polling without blocking; give up after WAIT_TIMEOUT_NS
+                // without progress.
+                int ns = 0, np = 0;
+                unsigned long long t_last = globaltimer();
+                while (mok && np < nblk) {
+                    bool prog = false;
+                    if (ns < nblk && mbar_test_wait(&kv_full[ns % ST], (uint32_t)(ns / ST) & 1u) &&
+                        mbar_test_wait(&s_free[ns % AT_SB], ((uint32_t)(ns / AT_SB) & 1u) ^ 1u)) {
+                        tc_fence_after();
+                        issue_s(ns++);
+                        prog = true;
+                    }
+                    if (np < ns && mbar_test_wait(&p_full[np & 1], (uint32_t)(np >> 1) & 1u)) {
+                        tc_fence_after();
+                        issue_pv(np++);
+                        prog = true;
+                    }
+                    if (prog) {
+                        t_last = globaltimer();
+                    } else if (*abort || globaltimer() - t_last > WAIT_TIMEOUT_NS) {
+                        *abort = 1;
                         mok = false;
-                        break;
                     }
                 }
-                if (mok) issue_pv(nblk - 1);
                 mma_commit(drain);
                 mbar_wait_timeout_only(drain, 0);
             }
@@ -454,9 +471,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             }
             const float sl2 = a.scale * 1.4426950408889634f;     // scale * log2(e)
             for (int j = 0; j < nblk; ++j) {
-                const int buf = j & 1, s = j % ST;
+                const int buf = j % AT_SB, s = j % ST;
                 int w = 1;
-                if (lane == 0) w = mbar_wait(&s_full[buf], (uint32_t)(j >> 1) & 1u, abort);
+                if (lane == 0) w = mbar_wait(&s_full[buf], (uint32_t)(j / AT_SB) & 1u, abort);
                 if (!__shfl_sync(FULL, w, 0)) {
                     ok = false;
                     break;
@@ -616,7 +633,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             // This thread writes d columns [64 kh, 64 kh + 64) of the row:
             // O_kh and O_{1-kh} there, weighted by their halves' max offsets.
             tc_fence_after();
-            const uint32_t ocol_other = lane_base + 128u + 128u * (uint32_t)(1 - kh);
+            const uint32_t ocol_other = lane_base + AT_OCOL + 128u * (uint32_t)(1 - kh);
             const float inv = ltot > 0.f ? 1.0f / ltot : 0.f;
             const float as = ws * inv, ao = wo * inv;
 #pragma unroll
@@ -764,7 +781,7 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G) {
 
 static size_t attn_tc_smem() {
     return 1024 + (size_t)AT_QTILE + 2 * AT_PTILE + (size_t)AT_ST * AT_STAGE + 2 * 128 * sizeof(float2) +
-           8 * (2 * AT_ST + 12) + 16;
+           8 * (2 * AT_ST + 2 * AT_SB + 8) + 16;
 }
 
 // Key splits per unit (CTAs per (sequence, KV head, M tile)): as many as fit
