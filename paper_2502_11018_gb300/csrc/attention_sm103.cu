@@ -149,7 +149,7 @@ __device__ __forceinline__ void rope8(const uint4& lo, const uint4& hi, const fl
 // CTA's partial row is staged.
 constexpr int AT_NSM = 256;               // softmax threads: 128 rows x 2 key halves
 constexpr int AT_NTH = 64 + AT_NSM;       // + TMA producer warp + MMA warp
-constexpr int AT_ST = 4;                  // K/V stages
+constexpr int AT_ST = 5;                  // K/V stages
 constexpr int AT_SB = 3;                  // S buffers in TMEM
 constexpr uint32_t AT_OCOL = 256;         // O_h at columns [256 + 128 h, 384 + 128 h)
 constexpr uint32_t AT_TMEM_COLS = 512;    // S buffers [0, 192), O_0, O_1
@@ -195,8 +195,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint8_t* sQ = smem;                                  // 32 KB
     uint8_t* sP = sQ + AT_QTILE;                         // 2 buffers x 16 KB
     uint8_t* sKV = sP + 2 * AT_PTILE;                    // ST x 32 KB
-    float2* sML = reinterpret_cast<float2*>(sKV + ST * AT_STAGE);   // [2][128] (m, l) per key half
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sML + 2 * 128);
+    // [2][128] (m, l) per key half, in the P area once the last PV is done
+    float2* sML = reinterpret_cast<float2*>(sP + 4096);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + ST * AT_STAGE);
     uint64_t* kv_full = bars;
     uint64_t* kv_empty = kv_full + ST;
     uint64_t* s_full = kv_empty + ST;
@@ -281,7 +282,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 bool q_issued = false;
                 auto issue_q = [&]() {
                     grid_dep_wait();
-                    mbar_arrive_expect_tx(q_raw, AT_QTILE);
+                    // The box holds min(128 / G, N) nodes (the rows of nodes past
+                    // it are never valid query rows).
+                    mbar_arrive_expect_tx(q_raw, (uint32_t)(256 * a.G * min(nb_per_tile, a.N)));
                     const int z = b * a.N + tile0 * nb_per_tile;
                     tma_load_3d(sQ, &map_q, q_raw, 0, g * a.G, z, pol_q);
                     tma_load_3d(sQ + AT_QHALF, &map_q, q_raw, 64, g * a.G, z, pol_q);
@@ -686,7 +689,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         bulk_store(static_cast<uint8_t*>(a.part_o_bf16) + split * 128 * 256, stg, (uint32_t)R * 256u);
         bulk_store(a.part_ml + split * 128, stg_lse, (uint32_t)((R + 3) & ~3) * 4u);
         bulk_commit();
-        bulk_wait_all();            // written before the grid completes
+        bulk_wait_read();           // the staging smem may be released; the writes
+                                    // are visible to the grids that depend on this one
     }
 }
 
@@ -757,9 +761,10 @@ EncodeTiledFn tensor_map_encoder();
 int make_map_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
                 uint64_t row_stride_bytes);
 
-// 3-D map over q[B*N][Hq][128] (bf16) with box {64 d, G heads, 128/G nodes}:
-// the box lands in smem as 128 rows (node-major, head-minor) of 64 d.
-static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G) {
+// 3-D map over q[B*N][Hq][128] (bf16) with box {64 d, G heads, min(128/G, N)
+// nodes}: the box lands in smem as up to 128 rows (node-major, head-minor) of
+// 64 d.
+static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G, int N) {
     EncodeTiledFn enc = tensor_map_encoder();
     if (!enc) {
         set_error("cuTensorMapEncodeTiled unavailable");
@@ -767,7 +772,7 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G) {
     }
     cuuint64_t dims[3] = {128, (cuuint64_t)Hq, (cuuint64_t)BN};
     cuuint64_t strides[2] = {256, (cuuint64_t)Hq * 256};
-    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(128 / G)};
+    cuuint32_t box[3] = {64, (cuuint32_t)G, (cuuint32_t)(128 / G < N ? 128 / G : N)};
     cuuint32_t estr[3] = {1, 1, 1};
     CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(q), dims, strides,
                      box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -780,8 +785,7 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G) {
 }
 
 static size_t attn_tc_smem() {
-    return 1024 + (size_t)AT_QTILE + 2 * AT_PTILE + (size_t)AT_ST * AT_STAGE + 2 * 128 * sizeof(float2) +
-           8 * (2 * AT_ST + 2 * AT_SB + 8) + 16;
+    return 1024 + (size_t)AT_QTILE + 2 * AT_PTILE + (size_t)AT_ST * AT_STAGE + 8 * (2 * AT_ST + 2 * AT_SB + 8) + 16;
 }
 
 // Key splits per unit (CTAs per (sequence, KV head, M tile)): as many as fit
@@ -828,7 +832,7 @@ int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
     if (rc != GV_OK) return rc;
     rc = make_map_2d(&mv, a0.cacheV, rows, 128, AT_BK, 256);
     if (rc != GV_OK) return rc;
-    rc = make_map_q(&mq, a0.q, a0.B * a0.N, a0.Hq, a0.G);
+    rc = make_map_q(&mq, a0.q, a0.B * a0.N, a0.Hq, a0.G, a0.N);
     if (rc != GV_OK) return rc;
     rc = make_map_rope(&mr, a0.rope, a0.B * a0.N, a0.N);
     if (rc != GV_OK) return rc;
