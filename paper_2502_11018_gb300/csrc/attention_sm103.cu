@@ -713,6 +713,7 @@ attn_merge_kernel(AttnArgs a) {
     if (row >= 128 || r >= a.G * a.N) return;
     grid_dep_wait();
     const size_t split0 = (size_t)cl * C;
+    // All loads first (the lse of every split, then its 16-byte chunk).
     float lsv[16];
     float M = -INFINITY;
     bool bad = false;

@@ -54,7 +54,7 @@ def _case(dtype, B, N, Hq, Hkv, d, P, base, std, seed):
     return parents, np.array(P, dtype=np.int32), S_max, q, k, v, cK, cV
 
 
-def run_gpu_attention(dev, parents, P, S_max, q, k, v, cK, cV, base):
+def run_gpu_attention(dev, parents, P, S_max, q, k, v, cK, cV, base, ws=None):
     B, N, Hq, d = q.shape
     Hkv = k.shape[2]
     dt = q.dtype
@@ -68,7 +68,8 @@ def run_gpu_attention(dev, parents, P, S_max, q, k, v, cK, cV, base):
     rope = torch.zeros(B, N, d // 2, 2, dtype=torch.float32, device=dev)
     gv.gv_rope_table(pos, d, base, rope)
     shape = gv.attn_shape(B, N, Hq, Hkv, d, S_max, gv.GV_BF16 if dt == torch.bfloat16 else gv.GV_F32)
-    ws = torch.full((gv.gv_verify_attention_workspace(shape),), 0xFF, dtype=torch.uint8, device=dev)
+    if ws is None:
+        ws = torch.full((gv.gv_verify_attention_workspace(shape),), 0xFF, dtype=torch.uint8, device=dev)
     tK = torch.zeros(B, Hkv, N, d, dtype=dt, device=dev)
     tV = torch.zeros_like(tK)
     out = torch.zeros(B, N, Hq, d, dtype=dt, device=dev)
@@ -94,10 +95,15 @@ def test_attention_parity(case):
     np.testing.assert_array_equal(f64(tV), rV)
 
 
-def test_attention_repeatable_with_dirty_workspace():
-    """Two calls (the second on a workspace the first left behind) agree bitwise."""
+def test_attention_repeatable_on_reused_workspace():
+    """Three calls on one workspace that starts dirty (each on what the
+    previous left behind) agree bitwise and with the oracle."""
     dev = device()
     parents, P, S_max, q, k, v, cK, cV = _case("bf16", 2, 60, 32, 8, 128, [700, 1500], 5e5, 1.0, 7)
-    o1, _, _, _, _ = run_gpu_attention(dev, parents, P, S_max, q, k, v, cK, cV, 5e5)
-    o2, _, _, _, _ = run_gpu_attention(dev, parents, P, S_max, q, k, v, cK, cV, 5e5)
-    assert torch.equal(o1, o2)
+    shape = gv.attn_shape(2, 60, 32, 8, 128, S_max, gv.GV_BF16)
+    ws = torch.full((gv.gv_verify_attention_workspace(shape),), 0xFF, dtype=torch.uint8, device=dev)
+    outs = [run_gpu_attention(dev, parents, P, S_max, q, k, v, cK, cV, 5e5, ws)[0] for _ in range(3)]
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+    ro, _, _ = oracle.tree_attention(f64(q), f64(k), f64(v), f64(cK), f64(cV), P,
+                                     oracle.tree_build(parents, P)[1], oracle.tree_build(parents, P)[2], 5e5)
+    assert rel_err(f64(outs[2]), ro) <= TOL_ATTN["bf16"]
