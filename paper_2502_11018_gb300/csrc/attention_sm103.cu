@@ -25,9 +25,9 @@
 //                          the log2 domain and rescale their O only when the
 //                          max grew by more than 2^8 (exact: O and l always
 //                          share one max), and write P = exp2(s - m) as bf16
-//                          to one of two smem buffers
-//   O_h += P_j,h V_j,h     tcgen05.mma, P K-major, V MN-major (d contiguous),
-//                          one accumulator per key half h
+//                          back to TMEM, over the first half of its own S columns
+//   O_h += P_j,h V_j,h     tcgen05.mma with A = P read from TMEM, V MN-major
+//                          in smem (d contiguous), one accumulator per key half h
 // Each CTA then merges its two halves and writes o = O / l (bf16) and
 // lse = m + log2(l) of its rows to the workspace (L2-resident), and
 // attn_merge_kernel, launched right behind it, combines the C splits of every
@@ -201,8 +201,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint64_t* kv_full = bars;
     uint64_t* kv_empty = kv_full + ST;
     uint64_t* s_full = kv_empty + ST;
-    uint64_t* s_free = s_full + AT_SB;
-    uint64_t* p_full = s_free + AT_SB;
+    uint64_t* p_full = s_full + AT_SB;
     uint64_t* o_done = p_full + 2;
     uint64_t* q_raw = o_done + 2;
     uint64_t* q_full = q_raw + 1;
@@ -226,10 +225,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             mbar_init(&kv_full[s], 1);
             mbar_init(&kv_empty[s], 1);
         }
-        for (int c = 0; c < AT_SB; ++c) {
-            mbar_init(&s_full[c], 1);
-            mbar_init(&s_free[c], NSM / 32);
-        }
+        for (int c = 0; c < AT_SB; ++c) mbar_init(&s_full[c], 1);
         for (int c = 0; c < 2; ++c) {
             mbar_init(&p_full[c], NSM / 32);
             mbar_init(&o_done[c], 1);
@@ -339,31 +335,36 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     }
                     mma_commit(&s_full[buf]);
                 };
-                // O_h += P_j,h V_j,h once softmax j has written P_j.
+                // O_h += P_j,h V_j,h once softmax j has written P_j, with P
+                // read from TMEM: the softmax stores P_j,h (bf16 pairs, 16
+                // columns) over the first half of its own S_j,h columns.
                 auto issue_pv = [&](int jj) {
-                    const int pb = jj & 1, sp = jj % ST;
+                    const int pb = jj & 1, sp = jj % ST, buf = jj % AT_SB;
                     // V as the MN-major B operand: rows = keys (128 B apart, SBO =
                     // 1 KB per 8 keys), the two 64-wide halves of d LBO = 8 KB apart.
                     uint64_t vdesc = sdesc_kmajor_sw128(smem_u32(sKV + sp * AT_STAGE + 2 * AT_KV_HALF));
                     vdesc = (vdesc & ~(0x3FFFull << 16)) | ((uint64_t)(AT_KV_HALF >> 4) << 16);
-                    const uint64_t pdesc = sdesc_kmajor_sw128(smem_u32(sP + pb * AT_PTILE));
-                    // Keys 0..31 (K steps 0, 1) into O_0, keys 32..63 into O_1.
+                    // Keys 0..31 (K steps 0, 1) into O_0, keys 32..63 into O_1;
+                    // one K step of 16 keys is 8 TMEM columns of P.
 #pragma unroll
                     for (int kk = 0; kk < AT_BK / 16; ++kk)
-                        mma_bf16(tmem + AT_OCOL + 128u * (uint32_t)(kk >> 1), pdesc + 2u * kk,
-                                 vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (kk & 1));
+                        mma_bf16_ta(tmem + AT_OCOL + 128u * (uint32_t)(kk >> 1),
+                                    tmem + (uint32_t)(buf * AT_BK + 32 * (kk >> 1) + 8 * (kk & 1)),
+                                    vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (kk & 1));
                     mma_commit(&kv_empty[sp]);
                     mma_commit(&o_done[pb]);
                 };
                 // Issue whichever is ready (S first: the softmax waits on it),
                 // polling without blocking; give up after WAIT_TIMEOUT_NS
-                // without progress.
+                // without progress.  S_j reuses the TMEM of S_{j-3} / P_{j-3}:
+                // it is issued after PV_{j-3}, and the tensor pipe runs the
+                // MMAs of this thread in order.
                 int ns = 0, np = 0;
                 unsigned long long t_last = globaltimer();
                 while (mok && np < nblk) {
                     bool prog = false;
-                    if (ns < nblk && mbar_test_wait(&kv_full[ns % ST], (uint32_t)(ns / ST) & 1u) &&
-                        mbar_test_wait(&s_free[ns % AT_SB], ((uint32_t)(ns / AT_SB) & 1u) ^ 1u)) {
+                    if (ns < nblk && np > ns - AT_SB &&
+                        mbar_test_wait(&kv_full[ns % ST], (uint32_t)(ns / ST) & 1u)) {
                         tc_fence_after();
                         issue_s(ns++);
                         prog = true;
@@ -488,9 +489,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 tmem_wait_ld();
 #pragma unroll
                 for (int c = 0; c < 32; ++c) asm volatile("" : "+r"(sv[c]));  // uses stay after the wait
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&s_free[buf]);
                 // Keys of the block this row may see: all of a full prefix block
                 // (the common, unmasked path), else a branch-free mask (the
                 // prefix end, or the row's ancestor bitmask); masked scores
@@ -538,14 +536,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 const float2 psum = split_f32x2(fadd_f32x2(fadd_f32x2(ps[0], ps[1]), fadd_f32x2(ps[2], ps[3])));
                 l = l * alpha + (psum.x + psum.y);
                 const int pb = j & 1;
-                if (j >= 2) {
-                    // P buffer pb was last read by PV_{j-2}.
-                    if (lane == 0) w = mbar_wait(&o_done[pb], ((uint32_t)(j >> 1) & 1u) ^ 1u, abort);
-                    if (!__shfl_sync(FULL, w, 0)) {
-                        ok = false;
-                        break;
-                    }
-                }
                 if (j >= 1 && __any_sync(FULL, need)) {
                     // Rescale O of this half: PV_{j-1} must have landed first.
                     if (lane == 0)
@@ -572,12 +562,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     }
                     tmem_wait_st();
                 }
-                uint8_t* pt = sP + pb * AT_PTILE;
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-                    *reinterpret_cast<uint4*>(pt + sw128(row, 4 * kh + c)) =
-                        make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-                if (k >= 0 && nvalid < AT_BK && kh == 0) {
+                // P over the first 16 of this half's 32 S columns.
+                tmem_st16(lane_base + (uint32_t)(buf * AT_BK + 32 * kh), pk);
+                const bool zero_v = k >= 0 && nvalid < AT_BK;
+                if (zero_v && kh == 0) {
                     // Zero the V rows past the prefix end (they may hold anything).
                     int w2 = 1;
                     if (lane == 0) w2 = mbar_wait(&kv_full[s], (uint32_t)(j / ST) & 1u, abort);
@@ -590,10 +578,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         }
                     }
                 }
+                tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) {
-                    fence_proxy_async_smem();
+                    if (zero_v) fence_proxy_async_smem();   // the zeroed V rows, for the MMA
                     mbar_arrive(&p_full[pb]);
                 }
             }
@@ -786,7 +775,7 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G, in
 }
 
 static size_t attn_tc_smem() {
-    return 1024 + (size_t)AT_QTILE + 2 * AT_PTILE + (size_t)AT_ST * AT_STAGE + 8 * (2 * AT_ST + 2 * AT_SB + 8) + 16;
+    return 1024 + (size_t)AT_QTILE + 2 * AT_PTILE + (size_t)AT_ST * AT_STAGE + 8 * (2 * AT_ST + AT_SB + 8) + 16;
 }
 
 // Key splits per unit (CTAs per (sequence, KV head, M tile)): as many as fit
