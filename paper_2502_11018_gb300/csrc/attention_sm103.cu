@@ -42,7 +42,7 @@
 // Both kernels use programmatic dependent launch.  Before griddepcontrol.wait
 // a CTA only initialises barriers and TMEM, reads step inputs written before
 // the step's first attention launch (RoPE table, ancestor masks, prefix
-// lengths) and starts streaming two K/V cache blocks; queries, tree
+// lengths) and fills its K/V ring from the cache; queries, tree
 // keys/values, the workspace and the output are touched after it.  Every
 // mbarrier wait is bounded; a CTA that gives up writes NaN lse for its rows,
 // which turns the affected outputs into NaN.
@@ -289,9 +289,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 for (int j = 0; j < nblk; ++j) {
                     const int s = j % ST;
                     const uint32_t ph = (uint32_t)(j / ST) & 1u;
-                    // Two K/V blocks stream before the dependency wait, then the
-                    // queries (on the critical path), then the remaining blocks.
-                    if (j == 2) issue_q();
+                    // The first fill of the K/V ring streams before the
+                    // dependency wait (the previous grid is still finishing),
+                    // then the queries, then the remaining blocks.
+                    if (j == ST) issue_q();
                     const int k = prefix_block(j);
                     if (k < 0) continue;             // tree block: built by the softmax warps
                     if (!mbar_wait(&kv_empty[s], ph ^ 1u, abort)) break;
@@ -345,12 +346,15 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     uint64_t vdesc = sdesc_kmajor_sw128(smem_u32(sKV + sp * AT_STAGE + 2 * AT_KV_HALF));
                     vdesc = (vdesc & ~(0x3FFFull << 16)) | ((uint64_t)(AT_KV_HALF >> 4) << 16);
                     // Keys 0..31 (K steps 0, 1) into O_0, keys 32..63 into O_1;
-                    // one K step of 16 keys is 8 TMEM columns of P.
+                    // one K step of 16 keys is 8 TMEM columns of P.  The two
+                    // accumulators alternate, so consecutive MMAs are independent.
 #pragma unroll
-                    for (int kk = 0; kk < AT_BK / 16; ++kk)
-                        mma_bf16_ta(tmem + AT_OCOL + 128u * (uint32_t)(kk >> 1),
-                                    tmem + (uint32_t)(buf * AT_BK + 32 * (kk >> 1) + 8 * (kk & 1)),
+                    for (int i = 0; i < AT_BK / 16; ++i) {
+                        const int h = i & 1, kk = 2 * h + (i >> 1);
+                        mma_bf16_ta(tmem + AT_OCOL + 128u * (uint32_t)h,
+                                    tmem + (uint32_t)(buf * AT_BK + 32 * h + 8 * (kk & 1)),
                                     vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (kk & 1));
+                    }
                     mma_commit(&kv_empty[sp]);
                     mma_commit(&o_done[pb]);
                 };
