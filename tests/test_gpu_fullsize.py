@@ -1,7 +1,9 @@
 """Full-size parity: the whole benchmark step -- every layer, the benchmark
 seed, the CUDA graph bench.py replays -- on the LLaMA-3-8B workload (32
-layers, prefix 4096, vocabulary 128256, greedy) and the Mixtral-attention
-workload (32 layers, prefix 16384, temperature 1).
+layers, prefix 4096, vocabulary 128256, greedy; the benchmark's own
+workload), the LLaMA-2-7B and the batch-4 LLaMA-2-13B workloads (greedy; the
+latter with ragged prefixes up to 8192 and more CTAs than SMs), and the
+Mixtral-attention workload (32 layers, prefix 16384, temperature 1).
 
 The float64 oracle cannot redo all 32 layers in seconds, so it checks samples
 that it can compute one by one: the first, a middle and the last layer's
@@ -80,14 +82,15 @@ def _check_tree_attention_compaction(cfg, inp, step, layers, keep, P):
     return parents, path, alen
 
 
-def test_fullsize_llama3_8b_greedy():
-    cfg, inp, step, layers, keep, P, D = _run_bench_step("llama3_8b")
+@pytest.mark.parametrize("name", ["llama3_8b", "llama2_7b", "llama2_13b_b4"])
+def test_fullsize_greedy(name):
+    cfg, inp, step, layers, keep, P, D = _run_bench_step(name)
     parents, path, alen = _check_tree_attention_compaction(cfg, inp, step, layers, keep, P)
     ids = step.ids.cpu().numpy()
     # Every row's argmax is the planted token (margin > 1 by construction) ...
     np.testing.assert_array_equal(ids, inp.planted.cpu().numpy().reshape(-1))
     # ... and, on a sample of rows, the float64 LM head's argmax.
-    rows = [0, 1, 17, 31, 45, ids.size - 1]
+    rows = sorted({0, 1, 17, 31, 45, ids.size // 2, ids.size - 1})
     h = f64(inp.h)[rows]
     W = f64(inp.W)
     ref_ids, _ = oracle.select_argmax(oracle.lmhead_logits(h, W))
