@@ -9,7 +9,7 @@
 // head g * G + hl; all G * N rows of (b, g) share every K/V block (GQA), and
 // each 128 of them form one MMA M tile.  A unit = (sequence b, KV head g, M
 // tile); each unit gets C CTAs (key splits).  The keys of (b, g) are cut into
-// 64-key blocks: ceil(P_b / 64) prefix blocks and one tree block (the N <= 64
+// 128-key blocks: ceil(P_b / 128) prefix blocks and one tree block (the N <= 64
 // tree keys, masked per query row by its ancestor bitmask).  The last split
 // runs the tree block first and then the last prefix blocks; the others take
 // the remaining prefix blocks round robin.
@@ -18,7 +18,7 @@
 //   S_j = Q K_j^T          tcgen05.mma, Q and K K-major 128B-swizzled in smem,
 //                          fp32 S in TMEM (three buffers: S_{j+1} and S_{j+2}
 //                          are computed during the softmax of block j)
-//   softmax                two threads per query row, one per 32-key half of
+//   softmax                two threads per query row, one per 64-key half of
 //                          the block, read their S row half from TMEM, mask
 //                          with a branch-free validity mask (prefix end, or
 //                          the row's ancestor bitmask), keep a running max in
@@ -53,11 +53,12 @@
 namespace gv {
 using namespace sm103;
 
-constexpr int AT_BK = 64;                   // keys per block
+constexpr int AT_BK = 128;                  // keys per block
+constexpr int AT_HK = AT_BK / 2;            // keys per half (one softmax thread)
 constexpr int AT_QHALF = 128 * 128;         // one M tile, 64 of the 128 d columns (bf16)
 constexpr int AT_QTILE = 2 * AT_QHALF;      // one M tile of Q
-constexpr int AT_PTILE = 128 * 128;         // one M tile of P: 128 rows x 64 keys bf16
-constexpr int AT_KV_HALF = AT_BK * 128;     // 64 keys x 64 d bf16 (one swizzle sub-tile)
+constexpr int AT_PTILE = 128 * 128;         // half of the scratch area (RoPE rows, epilogue)
+constexpr int AT_KV_HALF = AT_BK * 128;     // 128 keys x 64 d bf16 (one swizzle sub-tile)
 constexpr int AT_STAGE = 4 * AT_KV_HALF;    // K (2 halves) + V (2 halves)
 
 // Makes generic-proxy shared-memory writes visible to the async proxy (the
@@ -142,17 +143,17 @@ __device__ __forceinline__ void rope8(const uint4& lo, const uint4& hi, const fl
 }
 
 // Softmax warps 2..9: warp w reads TMEM lane quarter (w & 3), i.e. query
-// rows 32 * (w & 3) .. + 31, and key half h = (w - 2) >> 2 (keys 32h .. 32h+31)
-// of every 64-key block.  Each (row, half) keeps its own running max, sum and
+// rows 32 * (w & 3) .. + 31, and key half h = (w - 2) >> 2 (keys 64h .. 64h+63)
+// of every 128-key block.  Each (row, half) keeps its own running max, sum and
 // O accumulator O_h in TMEM -- a two-way split of the keys inside the CTA --
-// so each thread handles 32 scores per block; the halves are merged when the
+// so each thread handles 64 scores per block; the halves are merged when the
 // CTA's partial row is staged.
 constexpr int AT_NSM = 256;               // softmax threads: 128 rows x 2 key halves
 constexpr int AT_NTH = 64 + AT_NSM;       // + TMA producer warp + MMA warp
-constexpr int AT_ST = 5;                  // K/V stages
-constexpr int AT_SB = 3;                  // S buffers in TMEM
+constexpr int AT_ST = 2;                  // K/V stages (64 KB each)
+constexpr int AT_SB = 2;                  // S buffers in TMEM (128 columns each)
 constexpr uint32_t AT_OCOL = 256;         // O_h at columns [256 + 128 h, 384 + 128 h)
-constexpr uint32_t AT_TMEM_COLS = 512;    // S buffers [0, 192), O_0, O_1
+constexpr uint32_t AT_TMEM_COLS = 512;    // S buffers [0, 256), O_0, O_1
 
 __global__ void __launch_bounds__(AT_NTH, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
@@ -345,15 +346,15 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     // 1 KB per 8 keys), the two 64-wide halves of d LBO = 8 KB apart.
                     uint64_t vdesc = sdesc_kmajor_sw128(smem_u32(sKV + sp * AT_STAGE + 2 * AT_KV_HALF));
                     vdesc = (vdesc & ~(0x3FFFull << 16)) | ((uint64_t)(AT_KV_HALF >> 4) << 16);
-                    // Keys 0..31 (K steps 0, 1) into O_0, keys 32..63 into O_1;
+                    // Keys 0..63 (K steps 0..3) into O_0, keys 64..127 into O_1;
                     // one K step of 16 keys is 8 TMEM columns of P.  The two
                     // accumulators alternate, so consecutive MMAs are independent.
 #pragma unroll
                     for (int i = 0; i < AT_BK / 16; ++i) {
-                        const int h = i & 1, kk = 2 * h + (i >> 1);
+                        const int h = i & 1, s4 = i >> 1, kk = 4 * h + s4;
                         mma_bf16_ta(tmem + AT_OCOL + 128u * (uint32_t)h,
-                                    tmem + (uint32_t)(buf * AT_BK + 32 * h + 8 * (kk & 1)),
-                                    vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (kk & 1));
+                                    tmem + (uint32_t)(buf * AT_BK + AT_HK * h + 8 * s4),
+                                    vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (s4 != 0));
                     }
                     mma_commit(&kv_empty[sp]);
                     mma_commit(&o_done[pb]);
@@ -488,11 +489,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 }
                 __syncwarp();
                 tc_fence_after();
-                uint32_t sv[32];
-                tmem_ld32(lane_base + (uint32_t)(buf * AT_BK + 32 * kh), sv);
+                uint32_t sv[AT_HK];
+                tmem_ld32(lane_base + (uint32_t)(buf * AT_BK + AT_HK * kh), *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+                tmem_ld32(lane_base + (uint32_t)(buf * AT_BK + AT_HK * kh + 32),
+                          *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
                 tmem_wait_ld();
 #pragma unroll
-                for (int c = 0; c < 32; ++c) asm volatile("" : "+r"(sv[c]));  // uses stay after the wait
+                for (int c = 0; c < AT_HK; ++c) asm volatile("" : "+r"(sv[c]));  // uses stay after the wait
                 // Keys of the block this row may see: all of a full prefix block
                 // (the common, unmasked path), else a branch-free mask (the
                 // prefix end, or the row's ancestor bitmask); masked scores
@@ -500,20 +503,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 const int k = prefix_block(j);
                 const int nvalid = k < 0 ? a.N : min(AT_BK, P - k * AT_BK);
                 if (k < 0 || nvalid < AT_BK) {
-                    uint32_t vbits;
+                    // (the tree keys are nodes 0..N-1 <= 63: the first half)
+                    unsigned long long vbits;
                     if (k < 0) {
-                        vbits = (uint32_t)(anc_row >> (32 * kh));
+                        vbits = kh == 0 ? anc_row : 0ull;
                     } else {
-                        const int nv = nvalid - 32 * kh;     // valid keys of this half
-                        vbits = nv >= 32 ? 0xFFFFFFFFu : (nv <= 0 ? 0u : ((1u << nv) - 1u));
+                        const int nv = nvalid - AT_HK * kh;  // valid keys of this half
+                        vbits = nv >= 64 ? ~0ull : (nv <= 0 ? 0ull : ((1ull << nv) - 1ull));
                     }
+                    const uint32_t vlo = (uint32_t)vbits, vhi = (uint32_t)(vbits >> 32);
 #pragma unroll
-                    for (int c = 0; c < 32; ++c)
-                        sv[c] = (vbits >> c) & 1u ? sv[c] : __float_as_uint(-INFINITY);
+                    for (int c = 0; c < AT_HK; ++c)
+                        sv[c] = ((c < 32 ? vlo >> c : vhi >> (c - 32)) & 1u) ? sv[c] : __float_as_uint(-INFINITY);
                 }
                 float mxs[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-                for (int c = 0; c < 32; c += 2)
+                for (int c = 0; c < AT_HK; c += 2)
                     mxs[(c >> 1) & 3] = max3(mxs[(c >> 1) & 3], __uint_as_float(sv[c]), __uint_as_float(sv[c + 1]));
                 const float mx = max3(mxs[0], mxs[1], fmaxf(mxs[2], mxs[3])) * sl2;   // sl2 > 0
                 const float m_new = fmaxf(m_used, mx);
@@ -528,9 +533,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 const float nmv = m_used == -INFINITY ? 0.f : -m_used;
                 const uint64_t sc2 = f32x2(sl2, sl2), nm2 = f32x2(nmv, nmv);
                 uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
-                uint32_t pk[16];
+                uint32_t pk[AT_HK / 2];
 #pragma unroll
-                for (int c = 0; c < 16; ++c) {
+                for (int c = 0; c < AT_HK / 2; ++c) {
                     const float2 xa = split_f32x2(ffma_f32x2(
                         f32x2(__uint_as_float(sv[2 * c]), __uint_as_float(sv[2 * c + 1])), sc2, nm2));
                     const float p0 = fast_exp2(xa.x), p1 = fast_exp2(xa.y);
@@ -566,8 +571,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     }
                     tmem_wait_st();
                 }
-                // P over the first 16 of this half's 32 S columns.
-                tmem_st16(lane_base + (uint32_t)(buf * AT_BK + 32 * kh), pk);
+                // P over the first 32 of this half's 64 S columns.
+                tmem_st16(lane_base + (uint32_t)(buf * AT_BK + AT_HK * kh), *reinterpret_cast<uint32_t(*)[16]>(&pk[0]));
+                tmem_st16(lane_base + (uint32_t)(buf * AT_BK + AT_HK * kh + 16),
+                          *reinterpret_cast<uint32_t(*)[16]>(&pk[16]));
                 const bool zero_v = k >= 0 && nvalid < AT_BK;
                 if (zero_v && kh == 0) {
                     // Zero the V rows past the prefix end (they may hold anything).
@@ -790,7 +797,7 @@ static size_t attn_tc_smem() {
 int attn_tc_splits(int units, int S_max) {
     int c = sm_count() / units;
     if (S_max >= 4096 && c < 4) c = 4;
-    const int blocks = (S_max + AT_BK - 1) / AT_BK + 1;   // most 64-key blocks a unit can have
+    const int blocks = (S_max + AT_BK - 1) / AT_BK + 1;   // most blocks a unit can have
     if (c > blocks) c = blocks;
     if (c > 16) c = 16;
     if (c < 1) c = 1;
