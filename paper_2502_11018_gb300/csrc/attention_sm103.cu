@@ -40,10 +40,10 @@
 // softmax and the staging.
 //
 // Both kernels use programmatic dependent launch.  Before griddepcontrol.wait
-// a CTA only initialises barriers and TMEM, reads step inputs written before
-// the step's first attention launch (RoPE table, ancestor masks, prefix
-// lengths) and fills its K/V ring from the cache; queries, tree
-// keys/values, the workspace and the output are touched after it.  Every
+// a CTA only initialises barriers and TMEM, reads step inputs written two
+// launches before the step's first attention launch (ancestor masks, prefix
+// lengths) and fills its K/V ring from the cache; the RoPE table, queries,
+// tree keys/values, the workspace and the output are touched after it.  Every
 // mbarrier wait is bounded; a CTA that gives up writes NaN lse for its rows,
 // which turns the affected outputs into NaN.
 #include "gv_internal.cuh"
@@ -57,7 +57,6 @@ constexpr int AT_BK = 128;                  // keys per block
 constexpr int AT_HK = AT_BK / 2;            // keys per half (one softmax thread)
 constexpr int AT_QHALF = 128 * 128;         // one M tile, 64 of the 128 d columns (bf16)
 constexpr int AT_QTILE = 2 * AT_QHALF;      // one M tile of Q
-constexpr int AT_PTILE = 128 * 128;         // half of the scratch area (RoPE rows, epilogue)
 constexpr int AT_KV_HALF = AT_BK * 128;     // 128 keys x 64 d bf16 (one swizzle sub-tile)
 constexpr int AT_STAGE = 4 * AT_KV_HALF;    // K (2 halves) + V (2 halves)
 
@@ -150,15 +149,14 @@ __device__ __forceinline__ void rope8(const uint4& lo, const uint4& hi, const fl
 // CTA's partial row is staged.
 constexpr int AT_NSM = 256;               // softmax threads: 128 rows x 2 key halves
 constexpr int AT_NTH = 64 + AT_NSM;       // + TMA producer warp + MMA warp
-constexpr int AT_ST = 2;                  // K/V stages (64 KB each)
+constexpr int AT_ST = 3;                  // K/V stages (64 KB each)
 constexpr int AT_SB = 2;                  // S buffers in TMEM (128 columns each)
 constexpr uint32_t AT_OCOL = 256;         // O_h at columns [256 + 128 h, 384 + 128 h)
 constexpr uint32_t AT_TMEM_COLS = 512;    // S buffers [0, 256), O_0, O_1
 
 __global__ void __launch_bounds__(AT_NTH, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
-               const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_rope,
-               AttnArgs a) {
+               const __grid_constant__ CUtensorMap map_q, AttnArgs a) {
     constexpr int NSM = AT_NSM, ST = AT_ST;
     const int C = a.csize;                     // key splits per unit
     // CTA -> unit (sequence b, KV head g, M tile of 128 query rows) and key
@@ -194,10 +192,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
     uint8_t* sQ = smem;                                  // 32 KB
-    uint8_t* sP = sQ + AT_QTILE;                         // 2 buffers x 16 KB
-    uint8_t* sKV = sP + 2 * AT_PTILE;                    // ST x 32 KB
+    uint8_t* sKV = sQ + AT_QTILE;                        // ST x 64 KB
     // [2][128] (m, l) per key half, in the P area once the last PV is done
-    float2* sML = reinterpret_cast<float2*>(sP + 4096);
+    float2* sML = reinterpret_cast<float2*>(sKV);    // [2][128] (m, l), once the ring is idle
     uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + ST * AT_STAGE);
     uint64_t* kv_full = bars;
     uint64_t* kv_empty = kv_full + ST;
@@ -207,17 +204,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint64_t* q_raw = o_done + 2;
     uint64_t* q_full = q_raw + 1;
     uint64_t* drain = q_full + 1;
-    uint64_t* rope_full = drain + 1;
-    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(rope_full + 1);
-    // The RoPE rows of sequence b (N x 64 (cos, sin) pairs, 512 B per node)
-    // are staged in the P area, which is free until the first softmax block
-    // writes P, as four 128B-swizzled column boxes of 32 floats x N rows (8 KB
-    // apart): the lanes of a warp read the same pairs of 8 consecutive nodes
-    // from 8 different banks.  (cos, sin) of pairs 8c + 2q, 8c + 2q + 1:
-    auto rope_cs = [&](int n, int c, int q) -> float4 {
-        return *reinterpret_cast<const float4*>(sP + (c >> 1) * 8192 + n * 128 +
-                                                (((4 * (c & 1) + q) ^ (n & 7)) << 4));
-    };
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+    // (cos, sin) of pairs 8c + 2q, 8c + 2q + 1 of node n of sequence b, read
+    // from the per-step RoPE table (L2-resident: every CTA of the sequence
+    // reads the same N x 512 B).
+    const float4* rope_b = reinterpret_cast<const float4*>(a.rope) + (size_t)b * a.N * 32;
+    auto rope_cs = [&](int n, int c, int q) -> float4 { return __ldg(rope_b + n * 32 + c * 4 + q); };
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -234,12 +226,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         mbar_init(q_raw, 1);
         mbar_init(q_full, 1);
         mbar_init(drain, 1);
-        mbar_init(rope_full, 1);
         *abort = 0;
         fence_mbar_init();
         if (nblk > 0) {
             prefetch_tmap(&map_q);
-            prefetch_tmap(&map_rope);
             prefetch_tmap(&map_k);
             prefetch_tmap(&map_v);
         }
@@ -269,11 +259,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             if (lane == 0) {
                 const uint64_t pol_kv = policy_evict_first();
                 const uint64_t pol_q = policy_evict_last();
-                // RoPE rows first: written by a kernel that completed before
-                // the step's first attention launch, so safe before the wait.
-                mbar_arrive_expect_tx(rope_full, (uint32_t)a.N * 512u);
-                for (int cb = 0; cb < 4; ++cb)
-                    tma_load_2d(sP + cb * 8192, &map_rope, rope_full, cb * 32, b * a.N, pol_q);
                 int issued[ST];
                 for (int q = 0; q < ST; ++q) issued[q] = -1;
                 bool q_issued = false;
@@ -311,7 +296,6 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     for (int q = 0; q < ST; ++q)
                         if (issued[q] >= 0) mbar_wait_timeout_only(&kv_full[q], (uint32_t)issued[q]);
                     if (q_issued) mbar_wait_timeout_only(q_raw, 0);
-                    mbar_wait_timeout_only(rope_full, 0);
                 }
             }
         } else if (warp == 1) {
@@ -391,18 +375,21 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             }
         } else {
             // -------------------------- Q rotation, tree tile, softmax, epilogue
-            // The ancestor masks (like the RoPE rows the producer stages in
-            // smem) were written before the first attention launch of the
-            // step, so they are read before griddepcontrol.wait; the queries
-            // and tree keys/values come after it.
+            // The ancestor masks were written two launches before the step's
+            // first attention launch, so they are read before
+            // griddepcontrol.wait; the RoPE table, the queries and the tree
+            // keys/values come after it.
             const unsigned long long anc_row =
                 (has_tree && row_ok) ? __ldg(a.anc + (size_t)b * a.N + node) : 0ull;
             grid_dep_wait();
-            {
-                int w = 1;
-                if (lane == 0) w = mbar_wait(rope_full, 0, abort);
-                if (!__shfl_sync(FULL, w, 0)) ok = false;
-            }
+            // This row's RoPE pairs (chunks 4 kh .. 4 kh + 3), in flight while
+            // the queries land.
+            float4 rcs[16];
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    rcs[4 * c + q] = row_ok ? rope_cs(node, 4 * kh + c, q) : make_float4(0.f, 0.f, 0.f, 0.f);
             if (has_tree) {
                 // Rotated tree keys and the values into stage 0 (and into the
                 // tree K/V scratch in global memory for gv_kv_compact).
@@ -457,12 +444,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
                         uint4 olo = make_uint4(0, 0, 0, 0), ohi = olo;
-                        if (row_ok) {
-                            float4 cs[4];
-#pragma unroll
-                            for (int q = 0; q < 4; ++q) cs[q] = rope_cs(node, 4 * kh + c, q);
-                            rope8(lo[c], hi[c], cs, olo, ohi);
-                        }
+                        if (row_ok) rope8(lo[c], hi[c], &rcs[4 * c], olo, ohi);
                         lo[c] = olo;
                         hi[c] = ohi;
                     }
@@ -609,7 +591,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     // splits of every row.  lse is -inf for a CTA without blocks and NaN for
     // one that gave up.
     uint8_t* stg = sQ;                                  // R rows x 256 B
-    float* stg_lse = reinterpret_cast<float*>(sP);      // R floats
+    float* stg_lse = reinterpret_cast<float*>(sKV + 4096);   // R floats, once the ring is idle
     int w = 0;
     if (warp >= 2) {
         w = ok && nblk > 0 ? 1 : 0;
@@ -786,7 +768,7 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G, in
 }
 
 static size_t attn_tc_smem() {
-    return 1024 + (size_t)AT_QTILE + 2 * AT_PTILE + (size_t)AT_ST * AT_STAGE + 8 * (2 * AT_ST + AT_SB + 8) + 16;
+    return 1024 + (size_t)AT_QTILE + (size_t)AT_ST * AT_STAGE + 8 * (2 * AT_ST + AT_SB + 7) + 16;
 }
 
 // Key splits per unit (CTAs per (sequence, KV head, M tile)): as many as fit
@@ -804,38 +786,14 @@ int attn_tc_splits(int units, int S_max) {
     return c;
 }
 
-// 2-D map over the RoPE table rope[B*N][128] (fp32) with box {32 floats,
-// N rows}, 128B-swizzled.
-static int make_map_rope(CUtensorMap* map, const float* rope, int BN, int N) {
-    EncodeTiledFn enc = tensor_map_encoder();
-    if (!enc) {
-        set_error("cuTensorMapEncodeTiled unavailable");
-        return GV_ERR_CUDA;
-    }
-    cuuint64_t dims[2] = {128, (cuuint64_t)BN};
-    cuuint64_t strides[1] = {512};
-    cuuint32_t box[2] = {32, (cuuint32_t)N};
-    cuuint32_t estr[2] = {1, 1};
-    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(rope), dims, strides,
-                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) {
-        set_error("cuTensorMapEncodeTiled (rope) failed (%d)", (int)r);
-        return GV_ERR_CUDA;
-    }
-    return GV_OK;
-}
-
 int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
-    CUtensorMap mk, mv, mq, mr;
+    CUtensorMap mk, mv, mq;
     const uint64_t rows = (uint64_t)a0.B * a0.Hkv * a0.S_max;
     int rc = make_map_2d(&mk, a0.cacheK, rows, 128, AT_BK, 256);
     if (rc != GV_OK) return rc;
     rc = make_map_2d(&mv, a0.cacheV, rows, 128, AT_BK, 256);
     if (rc != GV_OK) return rc;
     rc = make_map_q(&mq, a0.q, a0.B * a0.N, a0.Hq, a0.G, a0.N);
-    if (rc != GV_OK) return rc;
-    rc = make_map_rope(&mr, a0.rope, a0.B * a0.N, a0.N);
     if (rc != GV_OK) return rc;
     const size_t smem = attn_tc_smem();
     cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -850,7 +808,7 @@ int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, attn_tc_kernel, mk, mv, mq, mr, a0);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, attn_tc_kernel, mk, mv, mq, a0);
     if (e != cudaSuccess) {
         set_error("attn_tc_kernel launch: %s", cudaGetErrorString(e));
         return GV_ERR_CUDA;
