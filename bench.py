@@ -475,30 +475,22 @@ def run_kernel_only(args, cfg, dev):
 
 
 def e2e_measure(step, inp, steps, stream):
-    """Same metric through VerifyStep with host buffers: the step's inputs
-    (tree, tokens, per-layer q/k/v, hidden states, uniforms) are copied from
-    pinned host memory, the step runs, and the accepted tokens are read back."""
-    names = ["parents", "tokens", "prefix_len", "q", "k_new", "v_new", "h"]
-    if inp.draft_logits is not None:
-        names += ["draft_logits", "u_acc", "u_res"]
+    """Same metric through VerifyStep with host buffers: every step copies its
+    inputs (tree, tokens, per-layer q/k/v, hidden states, uniforms) from pinned
+    host memory -- the per-layer ones on a side stream, overlapping the earlier
+    layers -- runs, and reads the accepted tokens back (one CUDA graph)."""
+    names = [n for n in step.HOST_INPUTS if getattr(inp, n) is not None]
     host = {n: getattr(inp, n).cpu().pin_memory() for n in names}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
     outs = [step.accept_len, step.out_tokens, step.path]
     d2h = sum(t.numel() * t.element_size() for t in outs)
     pinned_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
-
-    def one():
-        for n in names:
-            getattr(inp, n).copy_(host[n], non_blocking=True)
-        step.replay()
-        for dst, src in zip(pinned_out, outs):
-            dst.copy_(src, non_blocking=True)
-
-    one()
+    g = step.capture_from_host(host, pinned_out)
+    g.replay()
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(steps):
-        one()
+        g.replay()
         torch.cuda.current_stream().synchronize()
     dt = (time.perf_counter() - t0) / steps
     return {"value": 1.0 / dt, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,

@@ -130,3 +130,79 @@ class VerifyStep:
 
     def replay(self):
         self.graph.replay()
+
+    # ------------------------------------------------ steps fed from the host --
+    # Per-layer inputs a layer waits for, grouped so that each group's copies
+    # finish before the compute reaches it: the first layers wait for their
+    # own copies, later groups double in size (the copies run ahead of the
+    # attention layers, which take several times longer than one layer's
+    # copy).
+    @staticmethod
+    def _copy_groups(L):
+        starts, s = [], 0
+        while s < L:
+            starts.append(s)
+            s = 1 if s == 0 else 2 * s
+        return [(a, min(b, L)) for a, b in zip(starts, starts[1:] + [L])]
+
+    HOST_INPUTS = ("parents", "tokens", "prefix_len", "q", "k_new", "v_new", "h",
+                   "draft_logits", "u_acc", "u_res")
+
+    def run_from_host(self, host, host_out, stream, copy_stream):
+        """The step with its inputs copied from pinned host memory and its
+        result (accept_len, out_tokens, path) copied back.  The tree inputs
+        are copied on ``stream`` before the tree build; the per-layer q, k_new,
+        v_new and the hidden states (and the sampling inputs) on
+        ``copy_stream``, so that they stream in while the earlier layers run.
+        """
+        i = self.inp
+        L = self.cfg["L"]
+        with torch.cuda.stream(stream):
+            for n in ("parents", "tokens", "prefix_len"):
+                getattr(i, n).copy_(host[n], non_blocking=True)
+        copy_stream.wait_stream(stream)
+        groups = self._copy_groups(L)
+        ready = []
+        with torch.cuda.stream(copy_stream):
+            for a, b in groups:
+                for n in ("q", "k_new", "v_new"):
+                    getattr(i, n)[a:b].copy_(host[n][a:b], non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(copy_stream)
+                ready.append(ev)
+            for n in ("h", "draft_logits", "u_acc", "u_res"):
+                if getattr(i, n) is not None and n in host:
+                    getattr(i, n).copy_(host[n], non_blocking=True)
+            late = torch.cuda.Event()
+            late.record(copy_stream)
+        self.tree(stream)
+        first = {a: ev for (a, _), ev in zip(groups, ready)}
+        for layer in range(L):
+            if layer in first:
+                stream.wait_event(first[layer])
+            self.attention(layer, stream)
+        stream.wait_event(late)
+        self.lmhead(stream)
+        self.accept(stream)
+        self.compact(stream)
+        with torch.cuda.stream(stream):
+            for dst, src in zip(host_out, (self.accept_len, self.out_tokens, self.path)):
+                dst.copy_(src, non_blocking=True)
+
+    def capture_from_host(self, host, host_out):
+        """Capture ``run_from_host`` into a CUDA graph (after one eager run);
+        ``host`` maps input names to pinned host tensors shaped like the
+        device inputs, ``host_out`` holds pinned tensors for accept_len,
+        out_tokens and path."""
+        main, side = torch.cuda.Stream(), torch.cuda.Stream()
+        main.wait_stream(torch.cuda.current_stream())
+        self.run_from_host(host, host_out, main, side)
+        main.wait_stream(side)
+        torch.cuda.current_stream().wait_stream(main)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=main):
+            self.run_from_host(host, host_out, main, side)
+            main.wait_stream(side)
+        self.host_graph = g
+        return g

@@ -100,3 +100,38 @@ def test_step_graph_replay_matches_eager():
     assert torch.equal(step.ids, eager[1])
     assert torch.equal(step.path, eager[2])
     assert torch.equal(step.out_tokens, eager[3])
+
+
+@pytest.mark.parametrize("name,layers", [("llama3_8b", 5), ("mixtral_attn", 3)])
+def test_step_from_host_matches_device(name, layers):
+    """The host-fed graph (per-layer inputs copied on a side stream while the
+    earlier layers run) gives the same bits as the step on device inputs;
+    the device inputs are overwritten after capture, so the replay must copy
+    them."""
+    dev = device()
+    cfg = inputs.config(name)
+    inp = inputs.make_step_inputs(cfg, 11, device="cpu", layers=layers)
+    ref = VerifyStep(to_device(inp, dev))
+    ref.run()
+    torch.cuda.synchronize()
+    step = VerifyStep(to_device(inp, dev))
+    host = {n: getattr(inp, n).pin_memory() for n in step.HOST_INPUTS if getattr(inp, n) is not None}
+    outs = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+            for t in (step.accept_len, step.out_tokens, step.path)]
+    g = step.capture_from_host(host, outs)
+    for n in ("q", "k_new", "v_new", "h"):
+        getattr(step.inp, n).zero_()
+    step.inp.tokens.fill_(-1)
+    for o in outs:
+        o.fill_(-7)
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(step.attn_out, ref.attn_out)
+    assert torch.equal(step.treeK, ref.treeK) and torch.equal(step.treeV, ref.treeV)
+    if ref.ids is not None:
+        assert torch.equal(step.ids, ref.ids)
+    else:
+        assert torch.equal(step.logits, ref.logits)
+    assert torch.equal(outs[0], ref.accept_len.cpu())
+    assert torch.equal(outs[1], ref.out_tokens.cpu())
+    assert torch.equal(outs[2], ref.path.cpu())
