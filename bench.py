@@ -479,12 +479,9 @@ def e2e_measure(step, inp, steps, stream):
     inputs (tree, tokens, per-layer q/k/v, hidden states, uniforms) from pinned
     host memory -- the per-layer ones on a side stream, overlapping the earlier
     layers -- runs, and reads the accepted tokens back (one CUDA graph)."""
-    names = [n for n in step.HOST_INPUTS if getattr(inp, n) is not None]
-    host = {n: getattr(inp, n).cpu().pin_memory() for n in names}
+    host, pinned_out = step.host_buffers()
     h2d = sum(t.numel() * t.element_size() for t in host.values())
-    outs = [step.accept_len, step.out_tokens, step.path]
-    d2h = sum(t.numel() * t.element_size() for t in outs)
-    pinned_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
+    d2h = pinned_out.numel() * pinned_out.element_size()
     g = step.capture_from_host(host, pinned_out)
     g.replay()
     torch.cuda.synchronize()

@@ -59,9 +59,12 @@ class VerifyStep:
             self.row_lse = torch.zeros(rows, dtype=torch.float32, device=dev)
         lw = gv.gv_lmhead_workspace(rows, H, V, self.dt_code, self.lm_mode, 1)
         self.lm_ws = torch.empty(max(lw, 256), dtype=torch.uint8, device=dev)
-        self.path = torch.zeros(B, D + 1, **i32)
-        self.accept_len = torch.zeros(B, **i32)
-        self.out_tokens = torch.zeros(B, D + 1, **i32)
+        # The step's result (accept_len, out_tokens, path) in one buffer, so
+        # that a host-fed step reads it back with one copy.
+        self.result = torch.zeros(B + 2 * B * (D + 1), **i32)
+        self.accept_len = self.result[:B]
+        self.out_tokens = self.result[B:B + B * (D + 1)].view(B, D + 1)
+        self.path = self.result[B + B * (D + 1):].view(B, D + 1)
         aw = gv.gv_accept_workspace(B, V, self.T)
         self.acc_ws = torch.empty(max(aw, 256), dtype=torch.uint8, device=dev)
         self.new_len = torch.zeros(B, **i32)
@@ -145,32 +148,59 @@ class VerifyStep:
             s = 1 if s == 0 else 2 * s
         return [(a, min(b, L)) for a, b in zip(starts, starts[1:] + [L])]
 
-    HOST_INPUTS = ("parents", "tokens", "prefix_len", "q", "k_new", "v_new", "h",
-                   "draft_logits", "u_acc", "u_res")
+    HOST_INPUTS = ("parents", "tokens", "prefix_len", "qkv", "h", "draft_logits", "u_acc", "u_res")
 
-    def run_from_host(self, host, host_out, stream, copy_stream):
-        """The step with its inputs copied from pinned host memory and its
-        result (accept_len, out_tokens, path) copied back.  The tree inputs
-        are copied on ``stream`` before the tree build; the per-layer q, k_new,
-        v_new and the hidden states (and the sampling inputs) on
-        ``copy_stream``, so that they stream in while the earlier layers run.
-        """
+    def host_buffers(self):
+        """Pinned host buffers for a host-fed step, filled from the current
+        device inputs: the caller writes each step's inputs into them before
+        the replay of ``capture_from_host``'s graph.  The per-layer q, k_new
+        and v_new are packed as ``qkv[L][q | k_new | v_new]`` (one copy per
+        group of layers); the step's device q, k_new and v_new become views
+        of a device buffer with the same layout.  Returns (inputs by name,
+        result buffer shaped like ``self.result``)."""
         i = self.inp
         L = self.cfg["L"]
+        nq, nk = i.q[0].numel(), i.k_new[0].numel()
+        qkv = torch.empty(L, nq + 2 * nk, dtype=i.q.dtype, device=i.q.device)
+        qkv[:, :nq].copy_(i.q.reshape(L, nq))
+        qkv[:, nq:nq + nk].copy_(i.k_new.reshape(L, nk))
+        qkv[:, nq + nk:].copy_(i.v_new.reshape(L, nk))
+        i.q = qkv[:, :nq].view(i.q.shape)
+        i.k_new = qkv[:, nq:nq + nk].view(i.k_new.shape)
+        i.v_new = qkv[:, nq + nk:].view(i.v_new.shape)
+        self.qkv = qkv
+        host = {"qkv": qkv.cpu().pin_memory()}
+        for n in self.HOST_INPUTS:
+            if n != "qkv" and getattr(i, n) is not None:
+                host[n] = getattr(i, n).cpu().pin_memory()
+        out = torch.empty(self.result.shape, dtype=self.result.dtype, pin_memory=True)
+        return host, out
+
+    def run_from_host(self, host, host_out, stream, copy_stream):
+        """The step with its inputs copied from the pinned buffers of
+        ``host_buffers`` and its result (``self.result``: accept_len,
+        out_tokens, path) copied back to ``host_out``.  The tree inputs are
+        copied on ``stream`` before the tree build; the packed per-layer
+        q, k_new, v_new, then the tokens, hidden states and sampling inputs on
+        ``copy_stream`` after them, so that they stream in while the earlier
+        layers run."""
+        i = self.inp
+        L = self.cfg["L"]
+        # The tree inputs first: the copy engine serves copies in order, so
+        # the per-layer copies are queued only after them.
         with torch.cuda.stream(stream):
-            for n in ("parents", "tokens", "prefix_len"):
+            for n in ("parents", "prefix_len"):
                 getattr(i, n).copy_(host[n], non_blocking=True)
         copy_stream.wait_stream(stream)
         groups = self._copy_groups(L)
         ready = []
         with torch.cuda.stream(copy_stream):
             for a, b in groups:
-                for n in ("q", "k_new", "v_new"):
-                    getattr(i, n)[a:b].copy_(host[n][a:b], non_blocking=True)
+                self.qkv[a:b].copy_(host["qkv"][a:b], non_blocking=True)
                 ev = torch.cuda.Event()
                 ev.record(copy_stream)
                 ready.append(ev)
-            for n in ("h", "draft_logits", "u_acc", "u_res"):
+            for n in ("tokens", "h", "draft_logits", "u_acc", "u_res"):
                 if getattr(i, n) is not None and n in host:
                     getattr(i, n).copy_(host[n], non_blocking=True)
             late = torch.cuda.Event()
@@ -186,14 +216,11 @@ class VerifyStep:
         self.accept(stream)
         self.compact(stream)
         with torch.cuda.stream(stream):
-            for dst, src in zip(host_out, (self.accept_len, self.out_tokens, self.path)):
-                dst.copy_(src, non_blocking=True)
+            host_out.copy_(self.result, non_blocking=True)
 
     def capture_from_host(self, host, host_out):
-        """Capture ``run_from_host`` into a CUDA graph (after one eager run);
-        ``host`` maps input names to pinned host tensors shaped like the
-        device inputs, ``host_out`` holds pinned tensors for accept_len,
-        out_tokens and path."""
+        """Capture ``run_from_host`` into a CUDA graph (after one eager run)
+        over the buffers ``host_buffers`` returned."""
         main, side = torch.cuda.Stream(), torch.cuda.Stream()
         main.wait_stream(torch.cuda.current_stream())
         self.run_from_host(host, host_out, main, side)

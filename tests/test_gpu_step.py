@@ -115,15 +115,12 @@ def test_step_from_host_matches_device(name, layers):
     ref.run()
     torch.cuda.synchronize()
     step = VerifyStep(to_device(inp, dev))
-    host = {n: getattr(inp, n).pin_memory() for n in step.HOST_INPUTS if getattr(inp, n) is not None}
-    outs = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
-            for t in (step.accept_len, step.out_tokens, step.path)]
-    g = step.capture_from_host(host, outs)
+    host, res = step.host_buffers()
+    g = step.capture_from_host(host, res)
     for n in ("q", "k_new", "v_new", "h"):
         getattr(step.inp, n).zero_()
     step.inp.tokens.fill_(-1)
-    for o in outs:
-        o.fill_(-7)
+    res.fill_(-7)
     g.replay()
     torch.cuda.synchronize()
     assert torch.equal(step.attn_out, ref.attn_out)
@@ -132,6 +129,7 @@ def test_step_from_host_matches_device(name, layers):
         assert torch.equal(step.ids, ref.ids)
     else:
         assert torch.equal(step.logits, ref.logits)
-    assert torch.equal(outs[0], ref.accept_len.cpu())
-    assert torch.equal(outs[1], ref.out_tokens.cpu())
-    assert torch.equal(outs[2], ref.path.cpu())
+    B, D = cfg["B"], cfg["D"]
+    assert torch.equal(res[:B], ref.accept_len.cpu())
+    assert torch.equal(res[B:B + B * (D + 1)].view(B, D + 1), ref.out_tokens.cpu())
+    assert torch.equal(res[B + B * (D + 1):].view(B, D + 1), ref.path.cpu())
