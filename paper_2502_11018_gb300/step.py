@@ -140,13 +140,17 @@ class VerifyStep:
     # own copies, later groups double in size (the copies run ahead of the
     # attention layers, which take several times longer than one layer's
     # copy).
-    @staticmethod
-    def _copy_groups(L):
-        starts, s = [], 0
-        while s < L:
-            starts.append(s)
-            s = 1 if s == 0 else 2 * s
-        return [(a, min(b, L)) for a, b in zip(starts, starts[1:] + [L])]
+    COPY_GROUP_CAP = 0    # largest group (layers); 0: no cap
+
+    @classmethod
+    def _copy_groups(cls, L):
+        out, a, size = [], 0, 1
+        while a < L:
+            b = min(L, a + size)
+            out.append((a, b))
+            a = b
+            size = 2 * size if cls.COPY_GROUP_CAP <= 0 else min(cls.COPY_GROUP_CAP, 2 * size)
+        return out
 
     HOST_INPUTS = ("parents", "tokens", "prefix_len", "qkv", "h", "draft_logits", "u_acc", "u_res")
 
