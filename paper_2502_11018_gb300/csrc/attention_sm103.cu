@@ -17,18 +17,20 @@
 // Per block j of a CTA:
 //   S_j = Q K_j^T          tcgen05.mma, Q and K K-major 128B-swizzled in smem,
 //                          fp32 S in TMEM (three buffers: S_{j+1} and S_{j+2}
-//                          are computed during the softmax of block j)
+//                          can be computed during the softmax of block j)
 //   softmax                two threads per query row, one per 64-key half of
 //                          the block, read their S row half from TMEM, mask
 //                          with a branch-free validity mask (prefix end, or
-//                          the row's ancestor bitmask), keep a running max in
-//                          the log2 domain and rescale their O only when the
-//                          max grew by more than 2^8 (exact: O and l always
-//                          share one max), and write P = exp2(s - m) as bf16
-//                          back to TMEM, over the first half of its own S columns
-//   O_h += P_j,h V_j,h     tcgen05.mma with A = P read from TMEM, V MN-major
-//                          in smem (d contiguous), one accumulator per key half h
-// Each CTA then merges its two halves and writes o = O / l (bf16) and
+//                          the row's ancestor bitmask), exchange their half
+//                          maxima through shared memory, keep the row's
+//                          running max in the log2 domain and rescale O only
+//                          when the max grew by more than 2^8 (exact: O and l
+//                          always share one max), and write P = exp2(s - m) as
+//                          bf16 back to TMEM, over the first half of its own S
+//                          columns
+//   O += P_j V_j           tcgen05.mma with A = P read from TMEM, V MN-major
+//                          in smem (d contiguous), one accumulator per row tile
+// Each CTA then writes o = O / l (bf16) and
 // lse = m + log2(l) of its rows to the workspace (L2-resident), and
 // attn_merge_kernel, launched right behind it, combines the C splits of every
 // row into the bf16 output.  No CTA waits for another, so the splits need no
@@ -70,6 +72,20 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 }
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+// Named barrier of two warps (64 threads) that also returns whether every
+// thread passed a nonzero flag.
+__device__ __forceinline__ bool pair_bar_and(int id, int flag) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.s32 q, %2, 0;\n\t"
+        "bar.red.and.pred p, %1, 64, q;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(r)
+        : "r"(id), "r"(flag)
+        : "memory");
+    return r != 0;
 }
 __device__ __forceinline__ void grid_dep_wait() {
     asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -143,16 +159,17 @@ __device__ __forceinline__ void rope8(const uint4& lo, const uint4& hi, const fl
 
 // Softmax warps 2..9: warp w reads TMEM lane quarter (w & 3), i.e. query
 // rows 32 * (w & 3) .. + 31, and key half h = (w - 2) >> 2 (keys 64h .. 64h+63)
-// of every 128-key block.  Each (row, half) keeps its own running max, sum and
-// O accumulator O_h in TMEM -- a two-way split of the keys inside the CTA --
-// so each thread handles 64 scores per block; the halves are merged when the
-// CTA's partial row is staged.
+// of every 128-key block, so each thread handles 64 scores per block.  The
+// two threads of a row (warps w and w + 4) share the row's running max --
+// they exchange their half maxima every block -- and one O accumulator; each
+// keeps the sum of its own half, and the sums are added when the CTA's
+// partial row is staged.
 constexpr int AT_NSM = 256;               // softmax threads: 128 rows x 2 key halves
 constexpr int AT_NTH = 64 + AT_NSM;       // + TMA producer warp + MMA warp
 constexpr int AT_ST = 3;                  // K/V stages (64 KB each)
-constexpr int AT_SB = 2;                  // S buffers in TMEM (128 columns each)
-constexpr uint32_t AT_OCOL = 256;         // O_h at columns [256 + 128 h, 384 + 128 h)
-constexpr uint32_t AT_TMEM_COLS = 512;    // S buffers [0, 256), O_0, O_1
+constexpr int AT_SB = 3;                  // S buffers in TMEM (128 columns each)
+constexpr uint32_t AT_OCOL = 384;         // O at columns [384, 512)
+constexpr uint32_t AT_TMEM_COLS = 512;    // S buffers [0, 384), O
 
 __global__ void __launch_bounds__(AT_NTH, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
@@ -200,8 +217,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     uint64_t* kv_empty = kv_full + ST;
     uint64_t* s_full = kv_empty + ST;
     uint64_t* p_full = s_full + AT_SB;
-    uint64_t* o_done = p_full + 2;
-    uint64_t* q_raw = o_done + 2;
+    uint64_t* o_done = p_full + AT_SB;
+    uint64_t* q_raw = o_done + AT_SB;
     uint64_t* q_full = q_raw + 1;
     uint64_t* drain = q_full + 1;
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
@@ -211,6 +228,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     const float4* rope_b = reinterpret_cast<const float4*>(a.rope) + (size_t)b * a.N * 32;
     auto rope_cs = [&](int n, int c, int q) -> float4 { return __ldg(rope_b + n * 32 + c * 4 + q); };
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
+    // Half maxima of the current block, [block parity][key half][row], rounded
+    // up to bf16 (both threads of a row then compute the same row max).
+    __nv_bfloat16* sMX = reinterpret_cast<__nv_bfloat16*>(reinterpret_cast<uint8_t*>(tmem_holder) + 16);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
@@ -218,8 +238,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             mbar_init(&kv_full[s], 1);
             mbar_init(&kv_empty[s], 1);
         }
-        for (int c = 0; c < AT_SB; ++c) mbar_init(&s_full[c], 1);
-        for (int c = 0; c < 2; ++c) {
+        for (int c = 0; c < AT_SB; ++c) {
+            mbar_init(&s_full[c], 1);
             mbar_init(&p_full[c], NSM / 32);
             mbar_init(&o_done[c], 1);
         }
@@ -249,7 +269,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     const int node = tile0 * nb_per_tile + row / a.G;    // tree node of this row
     const bool row_ok = warp >= 2 && node < a.N;
     const uint32_t lane_base = tmem + ((uint32_t)(sub * 32) << 16);
-    const uint32_t ocol_self = lane_base + AT_OCOL + 128u * (uint32_t)kh;   // O of this key half
+    const uint32_t ocol_self = lane_base + AT_OCOL + 64u * (uint32_t)kh;   // this thread's d columns of O
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
 
@@ -321,25 +341,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     }
                     mma_commit(&s_full[buf]);
                 };
-                // O_h += P_j,h V_j,h once softmax j has written P_j, with P
-                // read from TMEM: the softmax stores P_j,h (bf16 pairs, 16
-                // columns) over the first half of its own S_j,h columns.
+                // O += P_j V_j once softmax j has written P_j, with P read
+                // from TMEM: the softmax stores the P of each key half (bf16
+                // pairs, 16 columns) over the first half of that half's 64 S
+                // columns.
                 auto issue_pv = [&](int jj) {
-                    const int pb = jj & 1, sp = jj % ST, buf = jj % AT_SB;
+                    const int pb = jj % AT_SB, sp = jj % ST, buf = jj % AT_SB;
                     // V as the MN-major B operand: rows = keys (128 B apart, SBO =
                     // 1 KB per 8 keys), the two 64-wide halves of d LBO = 8 KB apart.
                     uint64_t vdesc = sdesc_kmajor_sw128(smem_u32(sKV + sp * AT_STAGE + 2 * AT_KV_HALF));
                     vdesc = (vdesc & ~(0x3FFFull << 16)) | ((uint64_t)(AT_KV_HALF >> 4) << 16);
-                    // Keys 0..63 (K steps 0..3) into O_0, keys 64..127 into O_1;
-                    // one K step of 16 keys is 8 TMEM columns of P.  The two
-                    // accumulators alternate, so consecutive MMAs are independent.
+                    // One K step of 16 keys is 8 TMEM columns of P: keys 16 kk ..
+                    // of half kk / 4 start at column 64 (kk / 4) + 8 (kk % 4).
 #pragma unroll
-                    for (int i = 0; i < AT_BK / 16; ++i) {
-                        const int h = i & 1, s4 = i >> 1, kk = 4 * h + s4;
-                        mma_bf16_ta(tmem + AT_OCOL + 128u * (uint32_t)h,
-                                    tmem + (uint32_t)(buf * AT_BK + AT_HK * h + 8 * s4),
-                                    vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (s4 != 0));
-                    }
+                    for (int kk = 0; kk < AT_BK / 16; ++kk)
+                        mma_bf16_ta(tmem + AT_OCOL, tmem + (uint32_t)(buf * AT_BK + AT_HK * (kk >> 2) + 8 * (kk & 3)),
+                                    vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (kk != 0));
                     mma_commit(&kv_empty[sp]);
                     mma_commit(&o_done[pb]);
                 };
@@ -358,7 +375,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         issue_s(ns++);
                         prog = true;
                     }
-                    if (np < ns && mbar_test_wait(&p_full[np & 1], (uint32_t)(np >> 1) & 1u)) {
+                    if (np < ns && mbar_test_wait(&p_full[np % AT_SB], (uint32_t)(np / AT_SB) & 1u)) {
                         tc_fence_after();
                         issue_pv(np++);
                         prog = true;
@@ -463,12 +480,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             const float sl2 = a.scale * 1.4426950408889634f;     // scale * log2(e)
             for (int j = 0; j < nblk; ++j) {
                 const int buf = j % AT_SB, s = j % ST;
-                int w = 1;
-                if (lane == 0) w = mbar_wait(&s_full[buf], (uint32_t)(j / AT_SB) & 1u, abort);
-                if (!__shfl_sync(FULL, w, 0)) {
-                    ok = false;
-                    break;
-                }
+                int w = ok ? 1 : 0;
+                if (w && lane == 0) w = mbar_wait(&s_full[buf], (uint32_t)(j / AT_SB) & 1u, abort);
+                w = __shfl_sync(FULL, w, 0);
                 __syncwarp();
                 tc_fence_after();
                 uint32_t sv[AT_HK];
@@ -502,7 +516,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
 #pragma unroll
                 for (int c = 0; c < AT_HK; c += 2)
                     mxs[(c >> 1) & 3] = max3(mxs[(c >> 1) & 3], __uint_as_float(sv[c]), __uint_as_float(sv[c + 1]));
-                const float mx = max3(mxs[0], mxs[1], fmaxf(mxs[2], mxs[3])) * sl2;   // sl2 > 0
+                // This half's max, rounded up to bf16, to the row's other
+                // thread (warp w +- 4, same lane) through shared memory; the
+                // barrier of the pair also agrees on whether both got S_j.
+                const __nv_bfloat16 mh =
+                    __float2bfloat16_ru(max3(mxs[0], mxs[1], fmaxf(mxs[2], mxs[3])) * sl2);   // sl2 > 0
+                __nv_bfloat16* mslot = sMX + (j & 1) * 256;
+                mslot[kh * 128 + row] = mh;
+                if (!pair_bar_and(2 + sub, w)) {
+                    ok = false;
+                    break;
+                }
+                const float mx = fmaxf(__bfloat162float(mh), __bfloat162float(mslot[(1 - kh) * 128 + row]));
                 const float m_new = fmaxf(m_used, mx);
                 const bool need = m_new > m_used + 8.0f;     // also true the first time
                 float alpha = 1.0f;
@@ -526,32 +551,35 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 }
                 const float2 psum = split_f32x2(fadd_f32x2(fadd_f32x2(ps[0], ps[1]), fadd_f32x2(ps[2], ps[3])));
                 l = l * alpha + (psum.x + psum.y);
-                const int pb = j & 1;
+                const int pb = j % AT_SB;
                 if (j >= 1 && __any_sync(FULL, need)) {
-                    // Rescale O of this half: PV_{j-1} must have landed first.
+                    // Rescale this thread's 64 columns of O (the row's other
+                    // thread takes the other 64, with the same alpha): PV_{j-1}
+                    // must have landed first.  A failed wait is seen by both
+                    // threads of the row at the next block's pair barrier.
                     if (lane == 0)
-                        w = mbar_wait(&o_done[(j - 1) & 1], (uint32_t)((j - 1) >> 1) & 1u, abort);
-                    if (!__shfl_sync(FULL, w, 0)) {
-                        ok = false;
-                        break;
-                    }
-                    __syncwarp();
-                    tc_fence_after();
+                        w = mbar_wait(&o_done[(j - 1) % AT_SB], (uint32_t)((j - 1) / AT_SB) & 1u, abort);
+                    if (__shfl_sync(FULL, w, 0)) {
+                        __syncwarp();
+                        tc_fence_after();
 #pragma unroll
-                    for (int c0 = 0; c0 < 128; c0 += 32) {
-                        uint32_t ov[32];
-                        tmem_ld32(ocol_self + c0, ov);
-                        tmem_wait_ld();
-                        uint32_t lo[16], hi[16];
+                        for (int c0 = 0; c0 < 64; c0 += 32) {
+                            uint32_t ov[32];
+                            tmem_ld32(ocol_self + c0, ov);
+                            tmem_wait_ld();
+                            uint32_t lo[16], hi[16];
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            lo[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
-                            hi[e] = __float_as_uint(__uint_as_float(ov[16 + e]) * alpha);
+                            for (int e = 0; e < 16; ++e) {
+                                lo[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
+                                hi[e] = __float_as_uint(__uint_as_float(ov[16 + e]) * alpha);
+                            }
+                            tmem_st16(ocol_self + c0, lo);
+                            tmem_st16(ocol_self + c0 + 16, hi);
                         }
-                        tmem_st16(ocol_self + c0, lo);
-                        tmem_st16(ocol_self + c0 + 16, hi);
+                        tmem_wait_st();
+                    } else {
+                        ok = false;
                     }
-                    tmem_wait_st();
                 }
                 // P over the first 32 of this half's 64 S columns.
                 tmem_st16(lane_base + (uint32_t)(buf * AT_BK + AT_HK * kh), *reinterpret_cast<uint32_t(*)[16]>(&pk[0]));
@@ -583,8 +611,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     }
 
     // ------------------------------------------------ partial rows to the workspace
-    // The two key halves of every row are merged, and the row's normalised
-    // partial o = O / l (bf16, the 16-byte chunks of row r rotated by r & 15
+    // The row's normalised partial o = O / l, l the sum of both key halves'
+    // sums (bf16, the 16-byte chunks of row r rotated by r & 15
     // so that the lanes of a warp store distinct banks) and lse = m + log2(l)
     // are staged in the (now free) Q and P areas, then written to the
     // workspace with one bulk copy each; attn_merge_kernel combines the C
@@ -596,7 +624,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     if (warp >= 2) {
         w = ok && nblk > 0 ? 1 : 0;
         if (w && lane == 0)
-            w = mbar_wait(&o_done[(nblk - 1) & 1], (uint32_t)((nblk - 1) >> 1) & 1u, abort);
+            w = mbar_wait(&o_done[(nblk - 1) % AT_SB], (uint32_t)((nblk - 1) / AT_SB) & 1u, abort);
         w = __shfl_sync(FULL, w, 0);
         sML[kh * 128 + row] = make_float2(m_used, l);
     }
@@ -609,23 +637,17 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     if (warp >= 2) {
         const bool mine = row < R;
         const float2 other = sML[(1 - kh) * 128 + row];
-        const float M = fmaxf(m_used, other.x);
-        const float ws = m_used == -INFINITY ? 0.f : fast_exp2(m_used - M);
-        const float wo = other.x == -INFINITY ? 0.f : fast_exp2(other.x - M);
-        const float ltot = l * ws + other.y * wo;
+        const float M = m_used;                 // the row's max, shared by its halves
+        const float ltot = l + other.y;
         uint8_t* srow = stg + row * 256;
         if (w) {
-            // This thread writes d columns [64 kh, 64 kh + 64) of the row:
-            // O_kh and O_{1-kh} there, weighted by their halves' max offsets.
+            // This thread writes d columns [64 kh, 64 kh + 64) of the row.
             tc_fence_after();
-            const uint32_t ocol_other = lane_base + AT_OCOL + 128u * (uint32_t)(1 - kh);
             const float inv = ltot > 0.f ? 1.0f / ltot : 0.f;
-            const float as = ws * inv, ao = wo * inv;
 #pragma unroll
             for (int c0 = 0; c0 < 64; c0 += 32) {
-                uint32_t os[32], oo[32];
-                tmem_ld32(ocol_self + (uint32_t)(64 * kh + c0), os);
-                tmem_ld32(ocol_other + (uint32_t)(64 * kh + c0), oo);
+                uint32_t os[32];
+                tmem_ld32(ocol_self + (uint32_t)c0, os);
                 tmem_wait_ld();
                 if (mine) {
 #pragma unroll
@@ -633,8 +655,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         const int ch = (64 * kh + c0 + e) >> 3;   // 16-byte chunk of the 256-byte row
                         float v[8];
 #pragma unroll
-                        for (int u = 0; u < 8; ++u)
-                            v[u] = __uint_as_float(os[e + u]) * as + __uint_as_float(oo[e + u]) * ao;
+                        for (int u = 0; u < 8; ++u) v[u] = __uint_as_float(os[e + u]) * inv;
                         *reinterpret_cast<uint4*>(srow + ((ch ^ (row & 15)) << 4)) =
                             make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]),
                                        pack_bf16(v[4], v[5]), pack_bf16(v[6], v[7]));
@@ -768,7 +789,8 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G, in
 }
 
 static size_t attn_tc_smem() {
-    return 1024 + (size_t)AT_QTILE + (size_t)AT_ST * AT_STAGE + 8 * (2 * AT_ST + AT_SB + 7) + 16;
+    return 1024 + (size_t)AT_QTILE + (size_t)AT_ST * AT_STAGE + 8 * (2 * AT_ST + 3 * AT_SB + 3) + 16 +
+           2 * 2 * 128 * sizeof(__nv_bfloat16);
 }
 
 // Key splits per unit (CTAs per (sequence, KV head, M tile)): as many as fit
