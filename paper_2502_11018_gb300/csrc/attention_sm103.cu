@@ -36,8 +36,9 @@
 // row into the bf16 output.  No CTA waits for another, so the splits need no
 // cluster co-scheduling and the grid fills the SMs.
 //
-// Warp roles: warp 0 issues the TMA loads (RoPE rows, K/V blocks, raw Q
-// tile); warp 1 owns TMEM and issues the MMAs; warps 2..9 rotate Q in place
+// Warp roles: warp 0 issues the TMA loads (lane 0 the K halves of the
+// blocks and the raw Q tile, lane 1 the V halves); warp 1 owns TMEM and
+// issues the MMAs; warps 2..9 rotate Q in place
 // (RoPE from the per-step table), build the tree K/V tile, and run the
 // softmax and the staging.
 //
@@ -213,9 +214,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     // [2][128] (m, l) per key half, in the P area once the last PV is done
     float2* sML = reinterpret_cast<float2*>(sKV);    // [2][128] (m, l), once the ring is idle
     uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + ST * AT_STAGE);
-    uint64_t* kv_full = bars;
-    uint64_t* kv_empty = kv_full + ST;
-    uint64_t* s_full = kv_empty + ST;
+    // K and V of a stage land and are released separately: S_j frees K_j,
+    // PV_j frees V_j, so the next K block can stream in during PV_j.
+    uint64_t* k_full = bars;
+    uint64_t* v_full = k_full + ST;
+    uint64_t* k_empty = v_full + ST;
+    uint64_t* v_empty = k_empty + ST;
+    uint64_t* s_full = v_empty + ST;
     uint64_t* p_full = s_full + AT_SB;
     uint64_t* o_done = p_full + AT_SB;
     uint64_t* q_raw = o_done + AT_SB;
@@ -235,8 +240,10 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
         for (int s = 0; s < ST; ++s) {
-            mbar_init(&kv_full[s], 1);
-            mbar_init(&kv_empty[s], 1);
+            mbar_init(&k_full[s], 1);
+            mbar_init(&v_full[s], 1);
+            mbar_init(&k_empty[s], 1);
+            mbar_init(&v_empty[s], 1);
         }
         for (int c = 0; c < AT_SB; ++c) {
             mbar_init(&s_full[c], 1);
@@ -276,7 +283,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     if (nblk > 0) {
         if (warp == 0) {
             // ----------------------------------------------------- TMA producer
-            if (lane == 0) {
+            // Lane 0 streams the K halves of the blocks (and the queries),
+            // lane 1 the V halves, each as soon as its half of the stage is free.
+            if (lane < 2) {
+                const bool isk = lane == 0;
+                uint64_t* full = isk ? k_full : v_full;
+                uint64_t* empty = isk ? k_empty : v_empty;
+                const CUtensorMap* map = isk ? &map_k : &map_v;
+                const int off = isk ? 0 : 2 * AT_KV_HALF;
                 const uint64_t pol_kv = policy_evict_first();
                 const uint64_t pol_q = policy_evict_last();
                 int issued[ST];
@@ -298,23 +312,21 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     // The first fill of the K/V ring streams before the
                     // dependency wait (the previous grid is still finishing),
                     // then the queries, then the remaining blocks.
-                    if (j == ST) issue_q();
+                    if (isk && j == ST) issue_q();
                     const int k = prefix_block(j);
                     if (k < 0) continue;             // tree block: built by the softmax warps
-                    if (!mbar_wait(&kv_empty[s], ph ^ 1u, abort)) break;
-                    mbar_arrive_expect_tx(&kv_full[s], AT_STAGE);
-                    uint8_t* st = sKV + s * AT_STAGE;
+                    if (!mbar_wait(&empty[s], ph ^ 1u, abort)) break;
+                    mbar_arrive_expect_tx(&full[s], 2 * AT_KV_HALF);
+                    uint8_t* st = sKV + s * AT_STAGE + off;
                     const int y = bg * a.S_max + k * AT_BK;
-                    tma_load_2d(st, &map_k, &kv_full[s], 0, y, pol_kv);
-                    tma_load_2d(st + AT_KV_HALF, &map_k, &kv_full[s], 64, y, pol_kv);
-                    tma_load_2d(st + 2 * AT_KV_HALF, &map_v, &kv_full[s], 0, y, pol_kv);
-                    tma_load_2d(st + 3 * AT_KV_HALF, &map_v, &kv_full[s], 64, y, pol_kv);
+                    tma_load_2d(st, map, &full[s], 0, y, pol_kv);
+                    tma_load_2d(st + AT_KV_HALF, map, &full[s], 64, y, pol_kv);
                     issued[s] = (int)ph;
                 }
-                if (!q_issued && !*abort) issue_q();
+                if (isk && !q_issued && !*abort) issue_q();
                 if (*abort) {
                     for (int q = 0; q < ST; ++q)
-                        if (issued[q] >= 0) mbar_wait_timeout_only(&kv_full[q], (uint32_t)issued[q]);
+                        if (issued[q] >= 0) mbar_wait_timeout_only(&full[q], (uint32_t)issued[q]);
                     if (q_issued) mbar_wait_timeout_only(q_raw, 0);
                 }
             }
@@ -325,8 +337,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 const uint32_t idesc_o = idesc_bf16(128, 128, /*b_mn_major=*/true);
                 bool mok = mbar_wait(q_full, 0, abort);
                 tc_fence_after();
-                // S_j = Q K_j^T into S buffer j % 3, as soon as block j's K/V
-                // has landed and softmax j - 3 has read that buffer.
+                // S_j = Q K_j^T into S buffer j % 3, as soon as block j's K
+                // has landed and PV_{j-3} has consumed that buffer.
                 auto issue_s = [&](int jj) {
                     const int s = jj % ST, buf = jj % AT_SB;
                     const uint32_t kbase = smem_u32(sKV + s * AT_STAGE);
@@ -339,6 +351,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                             mma_bf16(tmem + (uint32_t)(buf * AT_BK), qdesc + 2u * kk, kdesc + 2u * kk,
                                      idesc_s, (kb | kk) != 0);
                     }
+                    mma_commit(&k_empty[s]);
                     mma_commit(&s_full[buf]);
                 };
                 // O += P_j V_j once softmax j has written P_j, with P read
@@ -357,7 +370,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                     for (int kk = 0; kk < AT_BK / 16; ++kk)
                         mma_bf16_ta(tmem + AT_OCOL, tmem + (uint32_t)(buf * AT_BK + AT_HK * (kk >> 2) + 8 * (kk & 3)),
                                     vdesc + (uint64_t)(kk * 128), idesc_o, (jj != 0) || (kk != 0));
-                    mma_commit(&kv_empty[sp]);
+                    mma_commit(&v_empty[sp]);
                     mma_commit(&o_done[pb]);
                 };
                 // Issue whichever is ready (S first: the softmax waits on it),
@@ -370,12 +383,13 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 while (mok && np < nblk) {
                     bool prog = false;
                     if (ns < nblk && np > ns - AT_SB &&
-                        mbar_test_wait(&kv_full[ns % ST], (uint32_t)(ns / ST) & 1u)) {
+                        mbar_test_wait(&k_full[ns % ST], (uint32_t)(ns / ST) & 1u)) {
                         tc_fence_after();
                         issue_s(ns++);
                         prog = true;
                     }
-                    if (np < ns && mbar_test_wait(&p_full[np % AT_SB], (uint32_t)(np / AT_SB) & 1u)) {
+                    if (np < ns && mbar_test_wait(&p_full[np % AT_SB], (uint32_t)(np / AT_SB) & 1u) &&
+                        mbar_test_wait(&v_full[np % ST], (uint32_t)(np / ST) & 1u)) {
                         tc_fence_after();
                         issue_pv(np++);
                         prog = true;
@@ -443,7 +457,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 named_bar_sync(1, NSM);
                 if (t == 0) {
                     fence_proxy_async_smem();
-                    mbar_arrive(&kv_full[0]);
+                    mbar_arrive(&k_full[0]);
+                    mbar_arrive(&v_full[0]);
                 }
             }
             // RoPE of this thread's half of its Q row (16-byte chunks 4 kh ..
@@ -589,7 +604,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 if (zero_v && kh == 0) {
                     // Zero the V rows past the prefix end (they may hold anything).
                     int w2 = 1;
-                    if (lane == 0) w2 = mbar_wait(&kv_full[s], (uint32_t)(j / ST) & 1u, abort);
+                    if (lane == 0) w2 = mbar_wait(&v_full[s], (uint32_t)(j / ST) & 1u, abort);
                     if (__shfl_sync(FULL, w2, 0)) {
                         uint8_t* vt = sKV + s * AT_STAGE + 2 * AT_KV_HALF;
                         for (int e = row; e < (AT_BK - nvalid) * 16; e += 128) {
@@ -789,7 +804,7 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G, in
 }
 
 static size_t attn_tc_smem() {
-    return 1024 + (size_t)AT_QTILE + (size_t)AT_ST * AT_STAGE + 8 * (2 * AT_ST + 3 * AT_SB + 3) + 16 +
+    return 1024 + (size_t)AT_QTILE + (size_t)AT_ST * AT_STAGE + 8 * (4 * AT_ST + 3 * AT_SB + 3) + 16 +
            2 * 2 * 128 * sizeof(__nv_bfloat16);
 }
 
