@@ -206,9 +206,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         return rank + (C - 1) * j;
     };
 
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                               ~static_cast<uintptr_t>(1023));
+    // The 128B-swizzled tiles need 1024-byte alignment; the dynamic shared
+    // memory of a kernel without static shared memory starts there (checked
+    // below: a CTA whose base is not aligned gives up, with NaN rows).  No
+    // slack is allocated, so that one merge CTA fits on the SM beside this one.
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = smem_raw;
     uint8_t* sQ = smem;                                  // 32 KB
     uint8_t* sKV = sQ + AT_QTILE;                        // ST x 64 KB
     // [2][128] (m, l) per key half, in the P area once the last PV is done
@@ -253,7 +256,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         mbar_init(q_raw, 1);
         mbar_init(q_full, 1);
         mbar_init(drain, 1);
-        *abort = 0;
+        *abort = (smem_u32(smem_raw) & 1023u) != 0 ? 1 : 0;
         fence_mbar_init();
         if (nblk > 0) {
             prefetch_tmap(&map_q);
@@ -716,14 +719,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
 // chunk of d), weights 2^(lse_s - max lse) over the splits, bf16 output.
 // Launched right after attn_tc_kernel with programmatic dependent launch; it
 // reads the partials after griddepcontrol.wait.
-constexpr int AM_ROWS = 8;                  // rows per CTA (x 16 chunks = 128 threads)
+constexpr int AM_ROWS = 16;                 // rows per CTA (x 16 chunks = 256 threads)
 
 __global__ void __launch_bounds__(AM_ROWS * 16)
 attn_merge_kernel(AttnArgs a) {
     grid_dep_launch();
     const int C = a.csize;
-    const int cl = blockIdx.x / (128 / AM_ROWS);         // unit
-    const int row = (blockIdx.x % (128 / AM_ROWS)) * AM_ROWS + (threadIdx.x >> 4);
+    // ceil(min(128, G N) / AM_ROWS) CTAs per unit: one merge CTA per SM fits
+    // beside an attention CTA, so a grid of at most one CTA per SM is resident
+    // (and waiting) before the attention grid ends.
+    const int per_unit = (min(128, a.G * a.N) + AM_ROWS - 1) / AM_ROWS;
+    const int cl = blockIdx.x / per_unit;                // unit
+    const int row = (blockIdx.x % per_unit) * AM_ROWS + (threadIdx.x >> 4);
     const int ch = threadIdx.x & 15;
     const int bg = cl / a.tiles, tile0 = cl % a.tiles;
     const int b = bg / a.Hkv, g = bg % a.Hkv;
@@ -804,7 +811,7 @@ static int make_map_q(CUtensorMap* map, const void* q, int BN, int Hq, int G, in
 }
 
 static size_t attn_tc_smem() {
-    return 1024 + (size_t)AT_QTILE + (size_t)AT_ST * AT_STAGE + 8 * (4 * AT_ST + 3 * AT_SB + 3) + 16 +
+    return (size_t)AT_QTILE + (size_t)AT_ST * AT_STAGE + 8 * (4 * AT_ST + 3 * AT_SB + 3) + 16 +
            2 * 2 * 128 * sizeof(__nv_bfloat16);
 }
 
@@ -851,7 +858,8 @@ int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
         return GV_ERR_CUDA;
     }
     cudaLaunchConfig_t mcfg{};
-    mcfg.gridDim = dim3((unsigned)(units * (128 / AM_ROWS)));
+    const int rmax = a0.G * a0.N < 128 ? a0.G * a0.N : 128;
+    mcfg.gridDim = dim3((unsigned)(units * ((rmax + AM_ROWS - 1) / AM_ROWS)));
     mcfg.blockDim = dim3(AM_ROWS * 16);
     mcfg.stream = st;
     mcfg.attrs = attr;
