@@ -28,6 +28,8 @@ accept_greedy_kernel(int B, int N, int D, const int32_t* __restrict__ tokens,
                      const int32_t* __restrict__ choice, int32_t* __restrict__ path,
                      int32_t* __restrict__ accept_len, int32_t* __restrict__ out_tokens,
                      int32_t* __restrict__ seq_status) {
+    pdl_wait();
+    pdl_trigger();
     const int b = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (b >= B) return;
@@ -123,6 +125,8 @@ accept_sample_kernel(int B, int N, int D, int V, float invT, const int32_t* __re
     __shared__ int s_emit[65];
     __shared__ float red[33];
     __shared__ float s_scan[SAMPLE_THREADS];
+    pdl_wait();
+    pdl_trigger();
     __shared__ int s_pick;
     const int b = blockIdx.x;
     const int tid = threadIdx.x;
@@ -283,13 +287,13 @@ int launch_accept(int B, int N, int D, int V, float temperature, const int32_t* 
     if (temperature == 0.0f) {
         const int warps_per_block = 4;
         const int blocks = (B + warps_per_block - 1) / warps_per_block;
-        accept_greedy_kernel<<<blocks, 32 * warps_per_block, 0, st>>>(
-            B, N, D, tokens, a, depth, choice, path, accept_len, out_tokens, seq_status);
+        launch_pdl(accept_greedy_kernel, dim3(blocks), dim3(32 * warps_per_block), 0, st, B, N, D, tokens,
+                   a, depth, choice, path, accept_len, out_tokens, seq_status);
         return check_launch("accept_greedy_kernel");
     }
-    accept_sample_kernel<<<B, SAMPLE_THREADS, 0, st>>>(
-        B, N, D, V, 1.0f / temperature, tokens, a, depth, target_logits, draft_logits, u_acc, u_res,
-        path, accept_len, out_tokens, seq_status, static_cast<float*>(workspace));
+    launch_pdl(accept_sample_kernel, dim3(B), dim3(SAMPLE_THREADS), 0, st, B, N, D, V, 1.0f / temperature,
+               tokens, a, depth, target_logits, draft_logits, u_acc, u_res, path, accept_len, out_tokens,
+               seq_status, static_cast<float*>(workspace));
     return check_launch("accept_sample_kernel");
 }
 

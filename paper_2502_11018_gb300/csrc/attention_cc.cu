@@ -29,10 +29,12 @@ rope_table_kernel(const int32_t* __restrict__ pos, int B, int N, int d, double b
                   float2* __restrict__ rope) {
     const int half = d >> 1;
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= B * N * half) return;
     const int j = idx % half;
+    const double theta = pow(base, -2.0 * (double)j / (double)d);   // (before the wait)
+    pdl_wait();
+    pdl_trigger();
+    if (idx >= B * N * half) return;
     const int bi = idx / half;
-    const double theta = pow(base, -2.0 * (double)j / (double)d);
     double sn, cs;
     sincos((double)pos[bi] * theta, &sn, &cs);
     rope[idx] = make_float2((float)cs, (float)sn);
@@ -41,8 +43,8 @@ rope_table_kernel(const int32_t* __restrict__ pos, int B, int N, int d, double b
 int launch_rope_table(const int32_t* pos, int B, int N, int d, float base, float* rope,
                       cudaStream_t st) {
     const int total = B * N * (d / 2);
-    rope_table_kernel<<<(total + 63) / 64, 64, 0, st>>>(pos, B, N, d, (double)base,
-                                                        reinterpret_cast<float2*>(rope));
+    launch_pdl(rope_table_kernel, dim3((total + 63) / 64), dim3(64), 0, st, pos, B, N, d, (double)base,
+               reinterpret_cast<float2*>(rope));
     return check_launch("rope_table_kernel");
 }
 

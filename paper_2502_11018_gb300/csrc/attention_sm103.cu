@@ -88,12 +88,6 @@ __device__ __forceinline__ bool pair_bar_and(int id, int flag) {
         : "memory");
     return r != 0;
 }
-__device__ __forceinline__ void grid_dep_wait() {
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-}
-__device__ __forceinline__ void grid_dep_launch() {
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
 // Packed fp32 pairs (one instruction for two lanes' worth of work) and the
 // three-input max of sm_100+.
 __device__ __forceinline__ uint64_t f32x2(float a, float b) {
@@ -269,7 +263,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
-    grid_dep_launch();
+    pdl_trigger();
 
     // Row and key half of a softmax thread (valid for warps >= 2).
     const int t = threadIdx.x - 64;
@@ -300,7 +294,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                 for (int q = 0; q < ST; ++q) issued[q] = -1;
                 bool q_issued = false;
                 auto issue_q = [&]() {
-                    grid_dep_wait();
+                    pdl_wait();
                     // The box holds min(128 / G, N) nodes (the rows of nodes past
                     // it are never valid query rows).
                     mbar_arrive_expect_tx(q_raw, (uint32_t)(256 * a.G * min(nb_per_tile, a.N)));
@@ -415,7 +409,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             // keys/values come after it.
             const unsigned long long anc_row =
                 (has_tree && row_ok) ? __ldg(a.anc + (size_t)b * a.N + node) : 0ull;
-            grid_dep_wait();
+            pdl_wait();
             // This row's RoPE pairs (chunks 4 kh .. 4 kh + 3), in flight while
             // the queries land.
             float4 rcs[16];
@@ -651,7 +645,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     w = __syncthreads_and(warp < 2 || w);
     // The workspace may still be read by the previous grid (the merge of the
     // previous call): wait for it before writing (a no-op if already done).
-    grid_dep_wait();
+    pdl_wait();
     if (warp >= 2) {
         const bool mine = row < R;
         const float2 other = sML[(1 - kh) * 128 + row];
@@ -723,7 +717,7 @@ constexpr int AM_ROWS = 16;                 // rows per CTA (x 16 chunks = 256 t
 
 __global__ void __launch_bounds__(AM_ROWS * 16)
 attn_merge_kernel(AttnArgs a) {
-    grid_dep_launch();
+    pdl_trigger();
     const int C = a.csize;
     // ceil(min(128, G N) / AM_ROWS) CTAs per unit: one merge CTA per SM fits
     // beside an attention CTA, so a grid of at most one CTA per SM is resident
@@ -736,7 +730,7 @@ attn_merge_kernel(AttnArgs a) {
     const int b = bg / a.Hkv, g = bg % a.Hkv;
     const int r = tile0 * 128 + row;                    // query row of (b, g)
     if (row >= 128 || r >= a.G * a.N) return;
-    grid_dep_wait();
+    pdl_wait();
     const size_t split0 = (size_t)cl * C;
     // All loads first (the lse of every split, then its 16-byte chunk).
     float lsv[16];
@@ -842,29 +836,15 @@ int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
     const size_t smem = attn_tc_smem();
     cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     const int units = a0.B * a0.Hkv * a0.tiles;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3((unsigned)(units * a0.csize));
-    cfg.blockDim = dim3(AT_NTH);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = st;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, attn_tc_kernel, mk, mv, mq, a0);
+    cudaError_t e = launch_pdl(attn_tc_kernel, dim3((unsigned)(units * a0.csize)), dim3(AT_NTH), smem, st,
+                               mk, mv, mq, a0);
     if (e != cudaSuccess) {
         set_error("attn_tc_kernel launch: %s", cudaGetErrorString(e));
         return GV_ERR_CUDA;
     }
-    cudaLaunchConfig_t mcfg{};
     const int rmax = a0.G * a0.N < 128 ? a0.G * a0.N : 128;
-    mcfg.gridDim = dim3((unsigned)(units * ((rmax + AM_ROWS - 1) / AM_ROWS)));
-    mcfg.blockDim = dim3(AM_ROWS * 16);
-    mcfg.stream = st;
-    mcfg.attrs = attr;
-    mcfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&mcfg, attn_merge_kernel, a0);
+    e = launch_pdl(attn_merge_kernel, dim3((unsigned)(units * ((rmax + AM_ROWS - 1) / AM_ROWS))),
+                   dim3(AM_ROWS * 16), 0, st, a0);
     if (e != cudaSuccess) {
         set_error("attn_merge_kernel launch: %s", cudaGetErrorString(e));
         return GV_ERR_CUDA;

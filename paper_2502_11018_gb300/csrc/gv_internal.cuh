@@ -33,6 +33,36 @@ int sm_count();
 // Compute capability major*10+minor of the current device.
 int device_cc();
 
+// ---- programmatic dependent launch -------------------------------------------
+// The step's kernels are launched with programmatic stream serialization, so a
+// kernel's CTAs can be resident (and run their prologue) while the previous
+// kernel of the stream finishes.  A kernel calls pdl_wait() before it reads
+// anything an earlier kernel of the stream wrote, or writes anything one may
+// still read: it returns once those grids have completed and their memory is
+// visible.  pdl_trigger() lets the next kernel's CTAs launch; kernels that
+// trigger only after their own pdl_wait() keep the ordering transitive (the
+// next kernel starts after the previous one has completed).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, Args... args) {
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // ---- device helpers ---------------------------------------------------------
 constexpr unsigned FULL = 0xffffffffu;
 

@@ -17,6 +17,8 @@ kv_compact_kernel(int L, int B, int N, int W, int Hkv, int S_max, int row_vec,
                   const int32_t* __restrict__ path, const int32_t* __restrict__ accept_len,
                   const int32_t* __restrict__ prefix_len, int32_t* __restrict__ new_len,
                   int32_t* __restrict__ seq_status) {
+    pdl_wait();
+    pdl_trigger();
     // Status / new_len: decided by block 0 from the same inputs every copying
     // thread tests, so the status write never changes another thread's choice.
     if (blockIdx.x == 0) {
@@ -74,10 +76,10 @@ int launch_kv_compact(int L, int B, int N, int D, int Hkv, int d, int S_max, int
     const size_t cap = (size_t)sm_count() * 8;
     if (blocks > cap) blocks = cap;
     if (blocks < 1) blocks = 1;
-    kv_compact_kernel<<<(unsigned)blocks, 256, 0, st>>>(
-        L, B, N, W, Hkv, S_max, row_vec, static_cast<const uint4*>(treeK),
-        static_cast<const uint4*>(treeV), static_cast<uint4*>(cacheK), static_cast<uint4*>(cacheV),
-        path, accept_len, prefix_len, new_len, seq_status);
+    launch_pdl(kv_compact_kernel, dim3((unsigned)blocks), dim3(256), 0, st, L, B, N, W, Hkv, S_max, row_vec,
+               static_cast<const uint4*>(treeK), static_cast<const uint4*>(treeV),
+               static_cast<uint4*>(cacheK), static_cast<uint4*>(cacheV), path, accept_len, prefix_len,
+               new_len, seq_status);
     return check_launch("kv_compact_kernel");
 }
 

@@ -135,6 +135,8 @@ lmhead_merge_kernel(SelectPartials part, int mode, int K, int32_t* __restrict__ 
     __shared__ float sv[8][16];
     __shared__ int si[8][16];
     __shared__ float red[33];
+    pdl_wait();
+    pdl_trigger();
     const int r = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int rows = part.rows;
@@ -235,7 +237,8 @@ lmhead_merge_kernel(SelectPartials part, int mode, int K, int32_t* __restrict__ 
 
 int launch_lmhead_merge(SelectPartials part, int mode, int K, int32_t* ids, float* vals,
                         float* row_max, float* row_lse, const int* err, cudaStream_t st) {
-    lmhead_merge_kernel<<<part.rows, 256, 0, st>>>(part, mode, K, ids, vals, row_max, row_lse, err);
+    launch_pdl(lmhead_merge_kernel, dim3(part.rows), dim3(256), 0, st, part, mode, K, ids, vals, row_max,
+               row_lse, err);
     return check_launch("lmhead_merge_kernel");
 }
 

@@ -96,8 +96,27 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
             uint32_t ph = 0;
             int issued[8];   // parity of the last load issued into each stage, or -1
             for (int q = 0; q < 8; ++q) issued[q] = -1;
+            // The first ring fill of W (a weight: no kernel of the stream
+            // writes it) streams before the dependency wait; the hidden rows,
+            // written upstream, are loaded after it.
+            const int t0 = blockIdx.x;
+            const int pre = t0 < a.n_tiles ? (a.stages < a.kblocks ? a.stages : a.kblocks) : 0;
+            for (int q = 0; q < pre; ++q) {
+                mbar_arrive_expect_tx(&full[q], tx);
+                tma_load_2d(stage_base + (size_t)q * a.stage_bytes + a.mt * LM_A_TILE_BYTES, &tmap_w, &full[q],
+                            q * 64, t0 * a.BN, pol_w);
+                issued[q] = 0;
+            }
+            pdl_wait();
+            pdl_trigger();
+            for (int q = 0; q < pre; ++q)
+                for (int m = 0; m < a.mt; ++m)
+                    tma_load_2d(stage_base + (size_t)q * a.stage_bytes + m * LM_A_TILE_BYTES, &tmap_h,
+                                &full[q], q * 64, m * 128, pol_h);
+            s = pre % a.stages;
+            ph = pre == a.stages ? 1u : 0u;
             for (int t = blockIdx.x; t < a.n_tiles; t += gridDim.x) {
-                for (int kb = 0; kb < a.kblocks; ++kb) {
+                for (int kb = t == t0 ? pre : 0; kb < a.kblocks; ++kb) {
                     if (!mbar_wait(&empty[s], ph ^ 1u, abort)) goto producer_done;
                     mbar_arrive_expect_tx(&full[s], tx);
                     uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
@@ -164,6 +183,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
         // ----------------------------------------------------------- epilogue
         const int sub = warp & 3;                 // TMEM lane quarter this warp may access
         const int row_in_tile = sub * 32 + lane;
+        pdl_wait();   // (before this role's global writes: logits, partials)
         float lv[2][KM];
         int li[2][KM];
         float rm[2], rs[2];
@@ -381,11 +401,11 @@ int launch_lmhead_tc(const void* h, const void* W, int rows, int H, int V, int m
         if (mode == GV_SELECT_TOPK) {
             cudaFuncSetAttribute(lmhead_tc_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)smem);
-            lmhead_tc_kernel<16><<<grid, LM_THREADS, smem, st>>>(mh, mw, a);
+            launch_pdl(lmhead_tc_kernel<16>, dim3(grid), dim3(LM_THREADS), smem, st, mh, mw, a);
         } else {
             cudaFuncSetAttribute(lmhead_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)smem);
-            lmhead_tc_kernel<1><<<grid, LM_THREADS, smem, st>>>(mh, mw, a);
+            launch_pdl(lmhead_tc_kernel<1>, dim3(grid), dim3(LM_THREADS), smem, st, mh, mw, a);
         }
         rc = check_launch("lmhead_tc_kernel");
         if (rc != GV_OK) return rc;

@@ -15,6 +15,8 @@ tree_build_kernel(const int32_t* __restrict__ parents, const int32_t* __restrict
                   unsigned long long* __restrict__ anc, int32_t* __restrict__ seq_status) {
     __shared__ int s_jump[64];
     __shared__ unsigned long long s_set[64];
+    pdl_wait();
+    pdl_trigger();
     const int b = blockIdx.x;
     const int i = threadIdx.x;
     int jump = -1;
@@ -54,8 +56,8 @@ tree_build_kernel(const int32_t* __restrict__ parents, const int32_t* __restrict
 int launch_tree_build(const int32_t* parents, const int32_t* prefix_len, int B, int N,
                       int32_t* depth, int32_t* pos, uint64_t* anc, int32_t* seq_status,
                       cudaStream_t st) {
-    tree_build_kernel<<<B, 64, 0, st>>>(parents, prefix_len, N, depth, pos,
-                                        reinterpret_cast<unsigned long long*>(anc), seq_status);
+    launch_pdl(tree_build_kernel, dim3(B), dim3(64), 0, st, parents, prefix_len, N, depth, pos,
+               reinterpret_cast<unsigned long long*>(anc), seq_status);
     return check_launch("tree_build_kernel");
 }
 
