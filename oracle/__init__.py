@@ -18,7 +18,11 @@ What it computes (GRIFFIN, arXiv 2502.11018):
 * the rule of Section 4.1 that rejecting a draft token discards every later
   token of its draft sequence (the whole subtree);
 * losslessness (Section 5): greedy acceptance reproduces greedy decoding, and
-  temperature-1 acceptance reproduces the target distribution.
+  temperature-1 acceptance reproduces the target distribution;
+* the token-alignable training objective of the draft model (Section 4.1,
+  Eqs. 2-5 and the loss of the Implementation Details appendix: top-k
+  predictable masks, chain alignment masks, masked per-sequence loss) in
+  ``tat``.
 
 Every function works in float64 with plain loops or single library
 primitives (a matmul, a sort), in the order the definition states.
@@ -35,3 +39,4 @@ from .lmhead import lmhead_logits, select_argmax, select_topk, row_logsumexp  # 
 from .accept import accept_greedy, accept_sampling  # noqa: F401
 from .compact import kv_compact  # noqa: F401
 from .step import verify_step  # noqa: F401
+from .tat import predictable_mask, alignment_mask, token_loss, feature_loss, tat_pass  # noqa: F401
