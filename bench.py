@@ -322,9 +322,11 @@ def main():
     ap.add_argument("--seed", type=int, default=1000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention"],
+    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention", "tat"],
                     help="step: the benchmark; lmhead / attention: time that call alone "
-                         "(a small, self-contained launch sequence for profiler captures)")
+                         "(a small, self-contained launch sequence for profiler captures); "
+                         "tat: one token-alignable training pass (gv_tat_loss) on a "
+                         "4 x 2048-token batch, vocabulary 32000")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
 
@@ -348,6 +350,9 @@ def main():
     gv.lib()
 
     from paper_2502_11018_gb300.step import VerifyStep
+    if args.kernel == "tat":
+        run_tat(args, dev)
+        return
     cfg = inputs.config(args.config)
     if args.kernel != "step":
         run_kernel_only(args, cfg, dev)
@@ -472,6 +477,51 @@ def run_kernel_only(args, cfg, dev):
                       "ms_per_call_graph": ms_graph, "algorithmic_bytes": nbytes,
                       "achieved_gbs_graph": gbs_graph,
                       "frac_of_measured_hbm_graph": gbs_graph / peaks["hbm_gbs"]}), flush=True)
+
+
+def tat_bytes(cfg):
+    """Algorithmic bytes of one token-alignable training pass: every logit and
+    both feature rows read once, the tokens, the earlier passes' masks, and
+    the per-position outputs (two masks, the loss) plus the sequence losses."""
+    B, T, V, H, n = cfg["B"], cfg["T"], cfg["V"], cfg["H"], cfg["n"]
+    el = 2 if cfg["logits"] == "bf16" else 4
+    ef = 2 if cfg["feat"] == "bf16" else 4
+    rows = B * T
+    return rows * (V * el + 2 * H * ef + 4 + (n - 1) + 1 + 1 + 4) + 4 * B
+
+
+def run_tat(args, dev):
+    """One token-alignable training pass over the LLaMA-2-7B-sized batch, timed
+    from a CUDA graph of back-to-back calls (the 1.2 GB of inputs are far above
+    L2, so every call reads them from HBM)."""
+    cfg = inputs.TAT_CONFIGS["tat_llama2_7b"]
+    inp = inputs.make_tat_inputs(cfg, args.seed, device=dev)
+    B, T = cfg["B"], cfg["T"]
+    mbar = torch.zeros((B, T), dtype=torch.uint8, device=dev)
+    mask = torch.zeros((B, T), dtype=torch.uint8, device=dev)
+    ell = torch.zeros((B, T), dtype=torch.float32, device=dev)
+    seq = torch.zeros((B,), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def call():
+        gv.gv_tat_loss(inp.logits, inp.tokens, inp.feat_draft, inp.feat_target, cfg["k"], cfg["n"],
+                       inp.mbar_prev, mbar, mask, ell, seq)
+
+    for _ in range(args.warmup):
+        call()
+    torch.cuda.synchronize()
+    reps = max(3, min(args.steps, 200))
+    g = graph_of(lambda: [call() for _ in range(4)])
+    g.replay()
+    torch.cuda.synchronize()
+    ms = event_time_ms(g.replay, reps, stream) / 4
+    nbytes = tat_bytes(cfg)
+    peaks = load_peaks()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    print(json.dumps({"kernel": "tat", "workload": "tat_llama2_7b", "config": cfg, "ms_per_call_graph": ms,
+                      "algorithmic_bytes": nbytes, "achieved_gbs_graph": gbs,
+                      "frac_of_measured_hbm_graph": gbs / peaks["hbm_gbs"],
+                      "rows_per_s": B * T / (ms * 1e-3)}), flush=True)
 
 
 def e2e_measure(step, inp, steps, stream):

@@ -15,6 +15,11 @@
  *                        rejection sampling (T > 0)
  *   gv_kv_compact        commit the accepted chain's K/V into the cache
  *
+ * and, for training the draft model (Section 4.1):
+ *
+ *   gv_tat_loss          top-k predictable masks, chain alignment masks and
+ *                        the masked loss of one token-alignable training pass
+ *
  * Conventions shared by every call:
  *  - Every pointer argument is DEVICE memory owned by the caller, unless the
  *    argument says otherwise.  The library never allocates on these paths:
@@ -256,6 +261,36 @@ int gv_kv_compact(int L, int B, int N, int D, int Hkv, int d, int S_max, int dt,
                   const void* treeK, const void* treeV, void* cacheK, void* cacheV,
                   const int32_t* path, const int32_t* accept_len, const int32_t* prefix_len,
                   int32_t* new_len, int32_t* seq_status, void* stream);
+
+/*
+ * gv_tat_loss -- the draft model's token-alignable training objective for
+ * training pass n (Section 4.1, Eqs. 2-5; per-step loss of the Implementation
+ * Details appendix).  Not part of the verify step: a data-parallel pass over
+ * the draft model's logits for a batch of training sequences.
+ *
+ *   logits      [B][T][V]    draft logits Xd_t                  (logits_dt)
+ *   tokens      int32 [B][T] ground-truth tokens x_t, 0 <= x_t < V
+ *   feat_draft  [B][T][H]    draft features Fd_t                (feat_dt)
+ *   feat_target [B][T][H]    target features Ft_t               (feat_dt)
+ *   mbar_prev   uint8 [n-1][B][T]  predictable masks of passes 1 .. n-1
+ *                            (the mbar outputs of those passes); NULL iff n == 1
+ *   mbar        uint8 [B][T] out: 1 iff x_t is among the top-k of Xd_t (ties
+ *                            toward the lower id)
+ *   mask        uint8 [B][T] out: alignment mask m_t (Eq. 3, along the draft
+ *                            chain): prod_{j=1}^{n-1} mbar_prev[j-1][b][t-n+j],
+ *                            0 for t < n-1, 1 everywhere when n == 1
+ *   ell         fp32 [B][T]  out: lam_tok * (logsumexp(Xd_t) - Xd_t[x_t])
+ *                            + lam_feat * ||Fd_t - Ft_t||_1
+ *   seq_loss    fp32 [B]     out: sum_t m_t ell_t / sum_t m_t (Eq. 5), 0 when
+ *                            no position is aligned; NaN when a token of the
+ *                            sequence is outside [0, V) (its ell is NaN)
+ * The paper's defaults are k = 3, lam_tok = 1, lam_feat = 0.1.  1 <= k <= V,
+ * n >= 1, T >= 1, V >= 1, H >= 0.  Output buffers must not overlap the inputs.
+ */
+int gv_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* feat_draft,
+                const void* feat_target, int feat_dt, int B, int T, int V, int H, int k, int n,
+                const uint8_t* mbar_prev, float lambda_tok, float lambda_feat, uint8_t* mbar,
+                uint8_t* mask, float* ell, float* seq_loss, void* stream);
 
 /* Static name of a status code. */
 const char* gv_status_string(int status);

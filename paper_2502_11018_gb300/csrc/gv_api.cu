@@ -63,6 +63,10 @@ static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 // Kernel launchers defined in the other translation units.
 int launch_tree_build(const int32_t*, const int32_t*, int, int, int32_t*, int32_t*, uint64_t*,
                       int32_t*, cudaStream_t);
+int launch_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* fd,
+                    const void* ft, int feat_dt, int B, int T, int V, int H, int k, int n,
+                    const uint8_t* mbar_prev, float lam_tok, float lam_feat, uint8_t* mbar,
+                    uint8_t* mask, float* ell, float* seq_loss, cudaStream_t st);
 int launch_kv_compact(int, int, int, int, int, int, int, int, const void*, const void*, void*,
                       void*, const int32_t*, const int32_t*, const int32_t*, int32_t*, int32_t*,
                       cudaStream_t);
@@ -458,6 +462,23 @@ int gv_kv_compact(int L, int B, int N, int D, int Hkv, int d, int S_max, int dt,
                  "gv_kv_compact: null index pointer");
     return launch_kv_compact(L, B, N, D, Hkv, d, S_max, esize, treeK, treeV, cacheK, cacheV, path,
                              accept_len, prefix_len, new_len, seq_status, as_stream(stream));
+}
+
+int gv_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* feat_draft,
+                const void* feat_target, int feat_dt, int B, int T, int V, int H, int k, int n,
+                const uint8_t* mbar_prev, float lambda_tok, float lambda_feat, uint8_t* mbar,
+                uint8_t* mask, float* ell, float* seq_loss, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(B >= 1 && T >= 1 && V >= 1 && H >= 0 && n >= 1 && k >= 1 && k <= V,
+                 "gv_tat_loss: bad sizes (B %d, T %d, V %d, H %d, k %d, n %d)", B, T, V, H, k, n);
+    GV_CHECK_ARG((long long)B * T <= 0x7fffffffLL, "gv_tat_loss: B * T too large");
+    GV_CHECK_ARG(logits_dt == GV_BF16 || logits_dt == GV_F32, "gv_tat_loss: logits dtype %d", logits_dt);
+    GV_CHECK_ARG(feat_dt == GV_BF16 || feat_dt == GV_F32, "gv_tat_loss: feature dtype %d", feat_dt);
+    GV_CHECK_ARG(logits && tokens && mbar && mask && ell && seq_loss, "gv_tat_loss: null pointer");
+    GV_CHECK_ARG(H == 0 || (feat_draft && feat_target), "gv_tat_loss: null feature pointer");
+    GV_CHECK_ARG((n == 1) == (mbar_prev == nullptr), "gv_tat_loss: mbar_prev must be NULL iff n == 1");
+    return launch_tat_loss(logits, logits_dt, tokens, feat_draft, feat_target, feat_dt, B, T, V, H, k, n,
+                           mbar_prev, lambda_tok, lambda_feat, mbar, mask, ell, seq_loss, as_stream(stream));
 }
 
 }  // extern "C"

@@ -34,7 +34,7 @@ GV_SELECT_LOGITS = 2
 EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "gv_verify_attention",
            "gv_lmhead_workspace", "gv_lmhead_select", "gv_lmhead_argmax_noalloc",
            "gv_accept_workspace", "gv_accept",
-           "gv_kv_compact", "gv_status_string", "gv_last_error", "gv_version")
+           "gv_kv_compact", "gv_tat_loss", "gv_status_string", "gv_last_error", "gv_version")
 
 
 class GvError(RuntimeError):
@@ -77,6 +77,8 @@ def lib():
         "gv_accept_workspace": ([_i, _i, _f], _sz),
         "gv_accept": ([_i, _i, _i, _i, _f] + [_vp] * 12 + [_vp, _sz, _vp], _i),
         "gv_kv_compact": ([_i] * 8 + [_vp] * 9 + [_vp], _i),
+        "gv_tat_loss": ([_vp, _i, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, _i, _vp, _f, _f,
+                         _vp, _vp, _vp, _vp, _vp], _i),
         "gv_status_string": ([_i], ctypes.c_char_p),
         "gv_last_error": ([], ctypes.c_char_p),
         "gv_version": ([], _i),
@@ -217,3 +219,18 @@ def gv_kv_compact(D, treeK, treeV, cacheK, cacheV, path, accept_len, prefix_len,
         _ptr(cacheK, "cacheK"), _ptr(cacheV, "cacheV"), _ptr(path, "path"),
         _ptr(accept_len, "accept_len"), _ptr(prefix_len, "prefix_len"), _ptr(new_len, "new_len"),
         _ptr(seq_status, "seq_status"), _stream(stream)))
+
+
+def gv_tat_loss(logits, tokens, feat_draft, feat_target, k, n, mbar_prev, mbar, mask, ell, seq_loss,
+                lambda_tok=1.0, lambda_feat=0.1, stream=None):
+    """One token-alignable training pass (see include/gv.h).  logits [B][T][V],
+    tokens int32 [B][T], features [B][T][H], mbar_prev uint8 [n-1][B][T] or
+    None (n == 1); outputs mbar, mask uint8 [B][T], ell fp32 [B][T],
+    seq_loss fp32 [B]."""
+    B, T, V = logits.shape
+    H = feat_draft.shape[2]
+    return _check("gv_tat_loss", lib().gv_tat_loss(
+        _ptr(logits, "logits"), dtype_code(logits), _ptr(tokens, "tokens"), _ptr(feat_draft, "feat_draft"),
+        _ptr(feat_target, "feat_target"), dtype_code(feat_draft), B, T, V, H, k, n,
+        _ptr(mbar_prev, "mbar_prev"), float(lambda_tok), float(lambda_feat), _ptr(mbar, "mbar"),
+        _ptr(mask, "mask"), _ptr(ell, "ell"), _ptr(seq_loss, "seq_loss"), _stream(stream)))

@@ -299,3 +299,60 @@ def make_step_inputs(cfg, seed, device="cpu", layers=None):
                       prefix_len=i32(np.array(cfg["P"], dtype=np.int32)), planted=i32(planted),
                       q=q, k_new=k_new, v_new=v_new, cacheK=cacheK, cacheV=cacheV,
                       h=h, W=W, draft_logits=draft_logits, u_acc=u_acc, u_res=u_res)
+
+
+# --------------------------------------------------------------------------
+# Token-alignable training pass (Section 4.1): draft logits over training
+# sequences, ground-truth tokens, draft / target features and the earlier
+# passes' predictable masks.  Shapes follow the paper's training setup for a
+# LLaMA-2-7B-sized drafter (vocabulary 32000, hidden 4096, N = 3 passes, top-3
+# alignment); ShareGPT itself is not used: seeded random values of the same
+# shapes stand in for it.
+# --------------------------------------------------------------------------
+
+TAT_CONFIGS = {
+    # ragged sizes (no 16-byte multiple rows), every pass
+    "tat_small": dict(B=2, T=37, V=1001, H=72, k=3, n=3, logits="f32", feat="bf16"),
+    # a training batch of 4 sequences x 2048 tokens, fp32 logits
+    "tat_llama2_7b": dict(B=4, T=2048, V=32000, H=4096, k=3, n=3, logits="f32", feat="bf16"),
+}
+
+
+@dataclass
+class TatInputs:
+    cfg: dict
+    logits: torch.Tensor        # [B][T][V]
+    tokens: torch.Tensor        # int32 [B][T]
+    feat_draft: torch.Tensor    # [B][T][H]
+    feat_target: torch.Tensor   # [B][T][H]
+    mbar_prev: torch.Tensor     # uint8 [n-1][B][T] (None for n = 1)
+
+
+def make_tat_inputs(cfg, seed, device="cpu", p_plant=0.7, p_prev=0.7):
+    """Seeded inputs of one training pass.  Logits ~ N(0, 1); for a fraction
+    ``p_plant`` of the positions the ground-truth token is the one at rank
+    0..4 of its row (ranks 3 and 4 fall outside a top-3), else a uniform
+    token, so that the predictable mask is mixed; features ~ N(0, 1); the
+    earlier passes' masks are Bernoulli(``p_prev``)."""
+    B, T, V, H, n = cfg["B"], cfg["T"], cfg["V"], cfg["H"], cfg["n"]
+    ldt = torch.bfloat16 if cfg["logits"] == "bf16" else torch.float32
+    fdt = torch.bfloat16 if cfg["feat"] == "bf16" else torch.float32
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(int(seed))
+    rng = np.random.default_rng(seed)
+    logits = torch.randn((B * T, V), generator=gen, dtype=torch.float32).to(ldt)
+    tokens = rng.integers(0, V, size=B * T)
+    plant = rng.random(B * T) < p_plant
+    ranks = rng.integers(0, 5, size=B * T)
+    top = torch.topk(logits.float(), k=min(5, V), dim=1).indices.numpy()
+    for r in np.nonzero(plant)[0]:
+        tokens[r] = top[r, min(ranks[r], top.shape[1] - 1)]
+    fd = torch.randn((B, T, H), generator=gen, dtype=torch.float32).to(fdt)
+    ft = torch.randn((B, T, H), generator=gen, dtype=torch.float32).to(fdt)
+    prev = None
+    if n > 1:
+        prev = torch.from_numpy((rng.random((n - 1, B, T)) < p_prev).astype(np.uint8))
+    return TatInputs(cfg=dict(cfg), logits=logits.view(B, T, V).to(device),
+                     tokens=torch.from_numpy(tokens.astype(np.int32)).view(B, T).to(device),
+                     feat_draft=fd.to(device), feat_target=ft.to(device),
+                     mbar_prev=None if prev is None else prev.to(device))

@@ -64,6 +64,12 @@ def test_host_side_validation(lib):
     assert lib.gv_accept(1, 60, 6, 0, -1.0, *([nul] * 12), nul, 0, nul) == gv.GV_ERR_ARG
     assert lib.gv_kv_compact(1, 1, 60, 6, 8, 3, 100, 0, *([nul] * 9), nul) == gv.GV_ERR_ARG
     assert "16-byte" in gv.last_error()
+    # token-alignable loss: k beyond the vocabulary, mbar_prev given for n = 1
+    assert lib.gv_tat_loss(16, gv.GV_F32, 16, 16, 16, gv.GV_BF16, 2, 8, 10, 64, 11, 1, nul, 1.0, 0.1,
+                           16, 16, 16, 16, nul) == gv.GV_ERR_ARG
+    assert lib.gv_tat_loss(16, gv.GV_F32, 16, 16, 16, gv.GV_BF16, 2, 8, 10, 64, 3, 1, 16, 1.0, 0.1,
+                           16, 16, 16, 16, nul) == gv.GV_ERR_ARG
+    assert "mbar_prev" in gv.last_error()
 
 
 def test_workspace_queries(lib):
