@@ -518,10 +518,25 @@ def run_tat(args, dev):
     nbytes = tat_bytes(cfg)
     peaks = load_peaks()
     gbs = nbytes / (ms * 1e-3) / 1e9
-    print(json.dumps({"kernel": "tat", "workload": "tat_llama2_7b", "config": cfg, "ms_per_call_graph": ms,
-                      "algorithmic_bytes": nbytes, "achieved_gbs_graph": gbs,
-                      "frac_of_measured_hbm_graph": gbs / peaks["hbm_gbs"],
-                      "rows_per_s": B * T / (ms * 1e-3)}), flush=True)
+    line = {"kernel": "tat", "workload": "tat_llama2_7b", "config": cfg, "ms_per_call_graph": ms,
+            "algorithmic_bytes": nbytes, "achieved_gbs_graph": gbs,
+            "frac_of_measured_hbm_graph": gbs / peaks["hbm_gbs"], "rows_per_s": B * T / (ms * 1e-3)}
+    if not args.no_cpu_baseline:
+        # The float64 oracle on the host cores, on the first 256 positions of
+        # every sequence (the alignment mask needs whole chains), scaled to
+        # the whole pass.
+        import oracle
+        ts = 256
+        f = lambda t: t[:, :ts].detach().cpu().double().numpy()
+        t0 = time.perf_counter()
+        oracle.tat_pass(f(inp.logits), inp.tokens[:, :ts].cpu().numpy(), f(inp.feat_draft), f(inp.feat_target),
+                        cfg["k"], cfg["n"], inp.mbar_prev[:, :, :ts].cpu().numpy())
+        sec = (time.perf_counter() - t0) * (T / ts)
+        line["cpu_baseline"] = {"value": B * T / sec, "unit": "rows/s", "cores": os.cpu_count(),
+                                "kind": "oracle",
+                                "sample": f"float64 numpy oracle on {B} x {ts} of the {B} x {T} positions, "
+                                          f"scaled linearly ({sec:.2f} s per pass)"}
+    print(json.dumps(line), flush=True)
 
 
 def e2e_measure(step, inp, steps, stream):
