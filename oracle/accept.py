@@ -30,6 +30,13 @@ distribution at that node:
 4. When no child of ``u`` is accepted (or ``u`` is a leaf) the bonus token is
    the inverse-CDF draw of the current ``p`` at ``u_res[u]``: the smallest
    ``v`` with ``sum_{w <= v} p(w) > u_res[u] * sum_w p(w)``.
+
+Variant without a draft distribution (``draft_logits`` None): the children are
+deterministic proposals (EAGLE-style top-k drafts), so ``q(x)`` is taken as 1
+for every drafted token.  Step 3 then accepts ``c`` when ``u_acc[c] <= p(x)``,
+and a rejection sets ``p(x) = 0`` and renormalises ``p`` (kept unchanged if
+nothing is left).  With distinct children this draws the emitted token from
+``p`` exactly (sampling without replacement), so it is lossless too.
 """
 
 import numpy as np
@@ -108,6 +115,17 @@ def _inverse_cdf(p, u):
     return v, margin
 
 
+def _residual(p, q, x):
+    """The unnormalised distribution after a rejected draft token ``x``:
+    ``max(p - q, 0)``, or ``p`` with ``p(x) = 0`` when there is no draft
+    distribution (``q`` None)."""
+    if q is None:
+        r = p.copy()
+        r[x] = 0.0
+        return r
+    return np.maximum(p - q, 0.0)
+
+
 def accept_sampling(parents, tokens, target_logits, draft_logits, u_acc, u_res, D,
                     temperature=1.0, seq_status=None):
     """Temperature sampling acceptance; returns ``(path, accept_len, out_tokens,
@@ -136,19 +154,20 @@ def accept_sampling(parents, tokens, target_logits, draft_logits, u_acc, u_res, 
         emitted = []
         while True:
             p = _softmax(target_logits[b, u], temperature)
-            q = _softmax(draft_logits[b, u], temperature)
+            q = None if draft_logits is None else _softmax(draft_logits[b, u], temperature)
             nxt = None
             for c in _children(parents[b], u):
                 x = int(tokens[b, c])
-                if q[x] == 0.0:
+                qx = 1.0 if q is None else q[x]
+                if qx == 0.0:
                     nxt = c
                     break
-                ratio = p[x] / q[x]
+                ratio = p[x] / qx
                 min_margin[b] = min(min_margin[b], abs(float(u_acc[b, c]) - ratio))
                 if float(u_acc[b, c]) <= ratio:
                     nxt = c
                     break
-                r = np.maximum(p - q, 0.0)
+                r = _residual(p, q, x)
                 s = r.sum()
                 if s > 0.0:
                     p = r / s
@@ -180,11 +199,12 @@ def check_sampling_trail(parents_row, tokens_row, target_logits_row, draft_logit
     ambiguous = 0
     for step, u in enumerate(trail):
         p = _softmax(target_logits_row[u], temperature)
-        q = _softmax(draft_logits_row[u], temperature)
+        q = None if draft_logits_row is None else _softmax(draft_logits_row[u], temperature)
         nxt = trail[step + 1] if step + 1 < len(trail) else None
         for c in _children(parents_row, u):
             x = int(tokens_row[c])
-            ratio = np.inf if q[x] == 0.0 else p[x] / q[x]
+            qx = 1.0 if q is None else q[x]
+            ratio = np.inf if qx == 0.0 else p[x] / qx
             ua = float(u_acc_row[c])
             if abs(ua - ratio) <= tol:
                 ambiguous += 1
@@ -194,7 +214,7 @@ def check_sampling_trail(parents_row, tokens_row, target_logits_row, draft_logit
                 break
             if not ua > ratio - tol:
                 return False, ambiguous
-            r = np.maximum(p - q, 0.0)
+            r = _residual(p, q, x)
             s = r.sum()
             if s > 0.0:
                 p = r / s

@@ -122,8 +122,9 @@ def _softmax(z):
     return e / e.sum()
 
 
-def _trials(seed, n, tgt, drf):
-    """Seeded trials: children drawn from q at the parent (the drafter)."""
+def _trials(seed, n, tgt, drf, T=1.0):
+    """Seeded trials: children drawn from q at the parent (the drafter), at
+    temperature T."""
     rng = np.random.default_rng(seed)
     N = len(SHAPE)
     parents = np.tile(SHAPE, (n, 1))
@@ -135,7 +136,7 @@ def _trials(seed, n, tgt, drf):
         for i in range(N):
             if i > 0:
                 par = SHAPE[i]
-                qd = _softmax(drf[paths[par]])
+                qd = _softmax(drf[paths[par]] / T)
                 tokens[b, i] = rng.choice(V1, p=qd)
                 paths[i] = paths[par] + (int(tokens[b, i]),)
             key = paths[i] if len(paths[i]) < 2 else None
@@ -232,3 +233,60 @@ def test_trail_checker_accepts_oracle_and_rejects_others():
             ok2, _ = check_sampling_trail(parents[b], tokens[b], tl[b], dl[b], ua[b], ur[b], trail, alt)
             wrong += not ok2
     assert wrong > 200
+
+
+def test_sampling_lossless_at_temperature_07():
+    # T != 1: children drawn from softmax(draft / T), emitted tokens follow
+    # softmax(target / T).
+    T = 0.7
+    tgt, drf = _tables(41)
+    parents, tokens, tl, dl, ua, ur = _trials(42, 20000, tgt, drf, T=T)
+    path, alen, out, st, margin = accept_sampling(parents, tokens, tl, dl, ua, ur, 2, T)
+    first, _ = _first_two(out, alen)
+    assert _chi2_p(first, _softmax(tgt[()] / T)) > 1e-3
+    # ... and not softmax(target) at T = 1
+    assert _chi2_p(first, _softmax(tgt[()])) < 1e-3
+
+
+def test_draftless_variant_hand_example():
+    # No draft distribution: q(x) = 1 for drafted tokens, a rejection zeroes p(x).
+    # Root p = [0.5, 0.3, 0.2]; children 1, 2 (leaves) carry tokens 0, 1.
+    parents = np.array([[-1, 0, 0]])
+    tokens = np.array([[0, 0, 1]])
+    tl = np.zeros((1, 3, 3))
+    tl[0, 0] = np.log([0.5, 0.3, 0.2])
+    tl[0, 2] = np.log([0.1, 0.2, 0.7])
+    tl[0, 1] = np.log([0.2, 0.2, 0.6])
+    # child 1: u = 0.6 > p(0) = 0.5 -> rejected, p -> [0, 0.6, 0.4];
+    # child 2: u = 0.55 <= 0.6 -> accepted; leaf 2 draws its bonus from its
+    # own p at u_res = 0.25: CDF [0.1, 0.3, 1.0] -> token 1.
+    ua = np.array([[0.0, 0.6, 0.55]])
+    ur = np.array([[0.9, 0.0, 0.25]])
+    path, alen, out, st, _ = accept_sampling(parents, tokens, tl, None, ua, ur, 1, 1.0)
+    assert path[0].tolist() == [0, 2] and alen[0] == 2 and out[0].tolist() == [1, 1]
+    # both rejected (0.7 > 0.6): p -> [0, 0, 1], the bonus is token 2 whatever u_res
+    ua[0, 2] = 0.7
+    path, alen, out, st, _ = accept_sampling(parents, tokens, tl, None, ua, ur, 1, 1.0)
+    assert path[0].tolist() == [0, -1] and alen[0] == 1 and out[0].tolist() == [2, -1]
+
+
+def test_draftless_variant_lossless():
+    # Deterministic distinct drafts (the root's children carry tokens 0, 1, 2,
+    # as a top-3 proposal would): the first emitted token follows p exactly.
+    V = 6
+    rng = np.random.default_rng(51)
+    z = rng.normal(scale=1.3, size=V)
+    n = 20000
+    parents = np.tile(np.array([-1, 0, 0, 0]), (n, 1))
+    tokens = np.tile(np.array([0, 2, 0, 5]), (n, 1))
+    tl = np.zeros((n, 4, V))
+    tl[:, :, :] = z
+    ua = rng.random((n, 4))
+    ur = rng.random((n, 4))
+    path, alen, out, st, _ = accept_sampling(parents, tokens, tl, None, ua, ur, 1, 1.0)
+    assert (st == 0).all()
+    assert _chi2_p(out[:, 0], _softmax(z)) > 1e-3
+    # the same trials under the draft-distribution rule with q = p would accept
+    # the first child always: a different distribution
+    path2, alen2, out2, _, _ = accept_sampling(parents, tokens, tl, tl, ua, ur, 1, 1.0)
+    assert (out2[:, 0] == 2).all()
