@@ -218,12 +218,16 @@ int gv_lmhead_argmax_noalloc(const void* h, const void* W, int rows, int H, int 
  *   p <- max(p - q, 0) / sum(max(p - q, 0)) (kept if that sum is 0); when no
  *   child is accepted the bonus token is the smallest v with
  *   sum_{w<=v} p(w) > u_res[b][u] * sum(p).
+ * temperature > 0 and draft_logits == NULL: the drafts are deterministic
+ *   proposals (top-k, EAGLE style): q(x_c) is taken as 1, so c is accepted
+ *   when u_acc[b][c] <= p(x_c), and a rejection sets p(x_c) = 0 and
+ *   renormalises p (kept if nothing is left); the bonus is drawn as above.
  *
  *   tokens        int32 [B][N]      draft token per node (tokens[b][0] = root)
  *   anc, depth    from gv_tree_build
  *   choice        int32 [B*N]       target argmax per node (T == 0; else NULL)
  *   target_logits fp32  [B][N][V]   (T > 0; else NULL)
- *   draft_logits  fp32  [B][N][V]   (T > 0; else NULL)
+ *   draft_logits  fp32  [B][N][V]   (T > 0, or NULL for the q = 1 rule; NULL for T == 0)
  *   u_acc, u_res  fp32  [B][N]      uniforms in [0, 1) (T > 0; else NULL)
  *   path          int32 [B][D+1]    out: accepted chain, root first, -1 padded
  *   accept_len    int32 [B]         out: entries of path (1 .. D+1)

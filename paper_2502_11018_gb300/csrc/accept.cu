@@ -164,24 +164,27 @@ accept_sample_kernel(int B, int N, int D, int V, float invT, const int32_t* __re
     const int seg = (V + blockDim.x - 1) / blockDim.x;
     const int v_lo = min(V, tid * seg), v_hi = min(V, v_lo + seg);
 #pragma unroll 1
+    // Without draft logits the drafts are deterministic proposals: q(x) = 1
+    // for a drafted token, and a rejection zeroes p(x) (q = 0 elsewhere).
+    const bool has_q = dlog != nullptr;
     while (true) {
         const float* T = tlog + (base + u) * (size_t)V;
-        const float* Q = dlog + (base + u) * (size_t)V;
+        const float* Q = has_q ? dlog + (base + u) * (size_t)V : nullptr;
         float tm = -INFINITY, qm = -INFINITY;
         for (int v = v_lo; v < v_hi; ++v) {
             tm = fmaxf(tm, T[v] * invT);
-            qm = fmaxf(qm, Q[v] * invT);
+            if (has_q) qm = fmaxf(qm, Q[v] * invT);
         }
         tm = block_reduce(tm, true, red);
-        qm = block_reduce(qm, true, red);
+        if (has_q) qm = block_reduce(qm, true, red);
         float ts = 0.f, qs = 0.f;
         for (int v = v_lo; v < v_hi; ++v) {
             ts += __expf(T[v] * invT - tm);
-            qs += __expf(Q[v] * invT - qm);
+            if (has_q) qs += __expf(Q[v] * invT - qm);
         }
         ts = block_reduce(ts, false, red);
-        qs = block_reduce(qs, false, red);
-        const float tinv = 1.0f / ts, qinv = 1.0f / qs;
+        if (has_q) qs = block_reduce(qs, false, red);
+        const float tinv = 1.0f / ts, qinv = has_q ? 1.0f / qs : 0.f;
         // p(v) = exp(T[v]/T - tm) / ts while mode == 0, else wbuf[cur][v] / wsum.
         int mode = 0, cur = 0;
         float wsum = 1.0f;
@@ -191,7 +194,7 @@ accept_sample_kernel(int B, int N, int D, int V, float invT, const int32_t* __re
             if (s_par[c] != u) continue;
             const int x = tokens[base + c];
             const float px = mode == 0 ? __expf(T[x] * invT - tm) * tinv : wbuf[cur][x] / wsum;
-            const float qx = __expf(Q[x] * invT - qm) * qinv;
+            const float qx = has_q ? __expf(Q[x] * invT - qm) * qinv : 1.0f;
             if (qx == 0.0f || u_acc[base + c] <= px / qx) {
                 next = c;
                 break;
@@ -201,7 +204,7 @@ accept_sample_kernel(int B, int N, int D, int V, float invT, const int32_t* __re
             const float winv = 1.0f / wsum;
             for (int v = v_lo; v < v_hi; ++v) {
                 const float pv = mode == 0 ? __expf(T[v] * invT - tm) * tinv : wbuf[cur][v] * winv;
-                const float r = fmaxf(pv - __expf(Q[v] * invT - qm) * qinv, 0.0f);
+                const float r = has_q ? fmaxf(pv - __expf(Q[v] * invT - qm) * qinv, 0.0f) : (v == x ? 0.0f : pv);
                 dst[v] = r;
                 part += r;
             }

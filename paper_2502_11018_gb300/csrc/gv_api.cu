@@ -433,8 +433,8 @@ int gv_accept(int B, int N, int D, int V, float temperature, const int32_t* toke
         GV_CHECK_ARG(choice, "gv_accept: greedy acceptance needs choice");
     } else {
         GV_CHECK_ARG(V >= 1, "gv_accept: V=%d", V);
-        GV_CHECK_ARG(target_logits && draft_logits && u_acc && u_res,
-                     "gv_accept: sampling needs logits and uniforms");
+        GV_CHECK_ARG(target_logits && u_acc && u_res,
+                     "gv_accept: sampling needs target logits and uniforms");
         GV_CHECK_ARG(workspace && ws_bytes >= gv_accept_workspace(B, V, temperature),
                      "gv_accept: workspace too small");
     }

@@ -107,8 +107,11 @@ def test_accept_greedy_depth_over_D():
     assert (path.cpu() == -1).all() and (out.cpu() == -1).all()
 
 
-@pytest.mark.parametrize("seed,V", [(0, 1000), (1, 32000), (2, 7)])
-def test_accept_sampling_parity(seed, V):
+@pytest.mark.parametrize("seed,V,T,with_q", [(0, 1000, 1.0, True), (1, 32000, 1.0, True), (2, 7, 1.0, True),
+                                             (3, 1000, 0.7, True), (4, 1000, 1.0, False),
+                                             (5, 32000, 0.7, False), (6, 7, 1.3, False)])
+def test_accept_sampling_parity(seed, V, T, with_q):
+    # with_q False: no draft distribution (q = 1 for drafted tokens).
     dev = device()
     rng = np.random.default_rng(seed)
     gen = torch.Generator().manual_seed(seed)
@@ -128,19 +131,20 @@ def test_accept_sampling_parity(seed, V):
     path = torch.zeros(B, D + 1, dtype=torch.int32, device=dev)
     alen = torch.zeros(B, dtype=torch.int32, device=dev)
     out = torch.zeros(B, D + 1, dtype=torch.int32, device=dev)
-    ws = torch.empty(gv.gv_accept_workspace(B, V, 1.0), dtype=torch.uint8, device=dev)
-    gv.gv_accept(D, 1.0, t(tokens), anc, depth, None, tl.to(dev), dl.to(dev), ua.to(dev),
+    ws = torch.empty(gv.gv_accept_workspace(B, V, T), dtype=torch.uint8, device=dev)
+    gv.gv_accept(D, T, t(tokens), anc, depth, None, tl.to(dev), dl.to(dev) if with_q else None, ua.to(dev),
                  ur.to(dev), path, alen, out, st, ws)
     torch.cuda.synchronize()
-    rp, ra, ro, rs, margin = oracle.accept_sampling(parents, tokens, f64(tl), f64(dl), f64(ua),
-                                                    f64(ur), D, 1.0)
+    dl64 = f64(dl) if with_q else None
+    rp, ra, ro, rs, margin = oracle.accept_sampling(parents, tokens, f64(tl), dl64, f64(ua),
+                                                    f64(ur), D, T)
     gp, ga, go = path.cpu().numpy(), alen.cpu().numpy(), out.cpu().numpy()
     assert (st.cpu().numpy() == 0).all()
     exact = 0
     for b in range(B):
         trail = gp[b, :ga[b]].tolist()
-        ok, amb = check_sampling_trail(parents[b], tokens[b], f64(tl[b]), f64(dl[b]), f64(ua[b]),
-                                       f64(ur[b]), trail, int(go[b, ga[b] - 1]), 1.0, tol=1e-5)
+        ok, amb = check_sampling_trail(parents[b], tokens[b], f64(tl[b]), None if dl64 is None else dl64[b],
+                                       f64(ua[b]), f64(ur[b]), trail, int(go[b, ga[b] - 1]), T, tol=1e-5)
         assert ok, (b, trail)
         assert go[b, :ga[b] - 1].tolist() == [int(tokens[b, j]) for j in trail[1:]]
         if margin[b] > 1e-4:
