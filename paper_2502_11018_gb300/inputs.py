@@ -41,6 +41,12 @@ CONFIGS = {
     "llama2_13b_b4": dict(dtype="bf16", B=4, L=40, H=5120, Hq=40, Hkv=40, d=128, V=32000,
                           P=(1024, 3072, 6144, 8192), N=60, D=6, branch=10,
                           rope_base=10000.0, std_w=0.02, std_kv=1.0, temperature=0.0),
+    # Batched chain speculation (the paper's vLLM throughput appendix): LLaMA-3-8B
+    # shape, 16 sequences, each a chain of 2 drafts after the root token
+    # (N = 3, D = 2), ragged chat-length prefixes, greedy acceptance.
+    "llama3_8b_chain_b16": dict(dtype="bf16", B=16, L=32, H=4096, Hq=32, Hkv=8, d=128, V=128256,
+                                P=(512, 768, 1024, 1536), N=3, D=2, branch=1,
+                                rope_base=500000.0, std_w=0.02, std_kv=1.0, temperature=0.0),
     # Mixtral-8x7B attention shape, long context, temperature-1 acceptance.
     "mixtral_attn": dict(dtype="bf16", B=1, L=32, H=4096, Hq=32, Hkv=8, d=128, V=32000,
                          P=(16384,), N=60, D=8, branch=10, rope_base=1000000.0,

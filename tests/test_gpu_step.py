@@ -23,7 +23,7 @@ from gpu_util import device, f64, rel_err, to_device, TOL_ATTN, TOL_ROT
 pytestmark = pytest.mark.gpu
 
 STEPS = [("tiny_f32", 1, 1), ("tiny_f32", 1, 2), ("llama2_7b", 1, 3), ("llama3_8b", 2, 4),
-         ("llama2_13b_b4", 1, 5), ("mixtral_attn", 1, 6)]
+         ("llama2_13b_b4", 1, 5), ("mixtral_attn", 1, 6), ("llama3_8b_chain_b16", 1, 7)]
 
 
 def check_step(inp, step, ref, graph=False):
