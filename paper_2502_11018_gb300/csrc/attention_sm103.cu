@@ -166,6 +166,9 @@ constexpr int AT_SB = 3;                  // S buffers in TMEM (128 columns each
 constexpr uint32_t AT_OCOL = 384;         // O at columns [384, 512)
 constexpr uint32_t AT_TMEM_COLS = 512;    // S buffers [0, 384), O
 
+// DIRECT: a single key split (C == 1) writes the final rows to the output
+// itself (no partials, no merge kernel).
+template <bool DIRECT>
 __global__ void __launch_bounds__(AT_NTH, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
                const __grid_constant__ CUtensorMap map_q, AttnArgs a) {
@@ -652,6 +655,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         const float M = m_used;                 // the row's max, shared by its halves
         const float ltot = l + other.y;
         uint8_t* srow = stg + row * 256;
+        // With a single key split the row is final: it goes straight to the
+        // output ([B][N][Hq][d], bf16) and no merge kernel runs.
+        uint4* orow = nullptr;
+        if (DIRECT && mine) {
+            const int r = row0 + row, i = r / a.G, h = g * a.G + r % a.G;
+            orow = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) +
+                                            (((size_t)b * a.N + i) * a.Hq + h) * 128);
+        }
         if (w) {
             // This thread writes d columns [64 kh, 64 kh + 64) of the row.
             tc_fence_after();
@@ -668,14 +679,23 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         float v[8];
 #pragma unroll
                         for (int u = 0; u < 8; ++u) v[u] = __uint_as_float(os[e + u]) * inv;
-                        *reinterpret_cast<uint4*>(srow + ((ch ^ (row & 15)) << 4)) =
-                            make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]),
-                                       pack_bf16(v[4], v[5]), pack_bf16(v[6], v[7]));
+                        const uint4 pv = make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]),
+                                                    pack_bf16(v[4], v[5]), pack_bf16(v[6], v[7]));
+                        if (DIRECT)
+                            orow[ch] = pv;
+                        else
+                            *reinterpret_cast<uint4*>(srow + ((ch ^ (row & 15)) << 4)) = pv;
                     }
                 }
             }
         }
-        if (mine) {
+        if (DIRECT && mine && !w) {
+            // (the single split owns the tree block, so it gave up)
+            const uint32_t nan2 = pack_bf16(NAN, NAN);
+#pragma unroll
+            for (int ch = 0; ch < 8; ++ch) orow[8 * kh + ch] = make_uint4(nan2, nan2, nan2, nan2);
+        }
+        if (mine && !DIRECT) {
             if (kh == 0)
                 stg_lse[row] = w ? (ltot > 0.f ? M + log2f(ltot) : -INFINITY) : (nblk > 0 ? NAN : -INFINITY);
             if (!w) {
@@ -694,11 +714,18 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
         // A role gave up, so a copy may have landed in the staging area after
         // the rows were staged (each role drains its own copies before the
         // barrier above): mark every row of this CTA invalid again.
-        if (warp >= 2 && kh == 0 && row < R) stg_lse[row] = NAN;
+        if (warp >= 2 && kh == 0 && row < R && !DIRECT) stg_lse[row] = NAN;
+        if (warp >= 2 && row < R && DIRECT) {
+            const int r = row0 + row, i = r / a.G, h = g * a.G + r % a.G;
+            uint4* orow = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) +
+                                                   (((size_t)b * a.N + i) * a.Hq + h) * 128);
+            const uint32_t nan2 = pack_bf16(NAN, NAN);
+            for (int ch = 0; ch < 8; ++ch) orow[8 * kh + ch] = make_uint4(nan2, nan2, nan2, nan2);
+        }
         __syncthreads();
     }
     if (warp == 1) tmem_dealloc(tmem, AT_TMEM_COLS);
-    if (threadIdx.x == 0) {
+    if (threadIdx.x == 0 && !DIRECT) {
         fence_proxy_async_smem();   // the staged rows, for the bulk copies
         const size_t split = (size_t)cl * C + rank;
         bulk_store(static_cast<uint8_t*>(a.part_o_bf16) + split * 128 * 256, stg, (uint32_t)R * 256u);
@@ -834,14 +861,19 @@ int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
     rc = make_map_q(&mq, a0.q, a0.B * a0.N, a0.Hq, a0.G, a0.N);
     if (rc != GV_OK) return rc;
     const size_t smem = attn_tc_smem();
-    cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaFuncSetAttribute(attn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaFuncSetAttribute(attn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     const int units = a0.B * a0.Hkv * a0.tiles;
-    cudaError_t e = launch_pdl(attn_tc_kernel, dim3((unsigned)(units * a0.csize)), dim3(AT_NTH), smem, st,
-                               mk, mv, mq, a0);
+    cudaError_t e = a0.csize == 1
+                        ? launch_pdl(attn_tc_kernel<true>, dim3((unsigned)units), dim3(AT_NTH), smem, st, mk, mv,
+                                     mq, a0)
+                        : launch_pdl(attn_tc_kernel<false>, dim3((unsigned)(units * a0.csize)), dim3(AT_NTH), smem,
+                                     st, mk, mv, mq, a0);
     if (e != cudaSuccess) {
         set_error("attn_tc_kernel launch: %s", cudaGetErrorString(e));
         return GV_ERR_CUDA;
     }
+    if (a0.csize == 1) return GV_OK;   // the split kernel wrote the output
     const int rmax = a0.G * a0.N < 128 ? a0.G * a0.N : 128;
     e = launch_pdl(attn_merge_kernel, dim3((unsigned)(units * ((rmax + AM_ROWS - 1) / AM_ROWS))),
                    dim3(AM_ROWS * 16), 0, st, a0);
