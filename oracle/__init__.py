@@ -22,7 +22,9 @@ What it computes (GRIFFIN, arXiv 2502.11018):
 * the token-alignable training objective of the draft model (Section 4.1,
   Eqs. 2-5 and the loss of the Implementation Details appendix: top-k
   predictable masks, chain alignment masks, masked per-sequence loss) in
-  ``tat``.
+  ``tat``;
+* the target model's decoder layers around the tree attention (RMSNorm,
+  projections, SwiGLU MLP, residuals) in ``layer``.
 
 Every function works in float64 with plain loops or single library
 primitives (a matmul, a sort), in the order the definition states.
@@ -40,3 +42,4 @@ from .accept import accept_greedy, accept_sampling  # noqa: F401
 from .compact import kv_compact  # noqa: F401
 from .step import verify_step  # noqa: F401
 from .tat import predictable_mask, alignment_mask, token_loss, feature_loss, tat_pass  # noqa: F401
+from .layer import rmsnorm, linear, silu, swiglu, decoder_layer  # noqa: F401
