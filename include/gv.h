@@ -15,6 +15,12 @@
  *                        rejection sampling (T > 0)
  *   gv_kv_compact        commit the accepted chain's K/V into the cache
  *
+ * the target model's layer body around the attention (the rest of the verify
+ * forward pass of Section 3, for LLaMA-style targets):
+ *
+ *   gv_rmsnorm           RMSNorm of the node rows
+ *   gv_linear            skinny projection x W^T with a fused epilogue
+ *
  * and, for training the draft model (Section 4.1):
  *
  *   gv_tat_loss          top-k predictable masks, chain alignment masks and
@@ -72,6 +78,13 @@ typedef enum {
     GV_SELECT_TOPK = 1,       /* ids[rows][k], vals[rows][k], k <= 16          */
     GV_SELECT_LOGITS = 2      /* logits[rows][V] fp32, row_max[rows], row_lse[rows] */
 } gv_select_mode;
+
+/* Epilogues of gv_linear. */
+typedef enum {
+    GV_LINEAR_STORE = 0,   /* out = x W^T                                   */
+    GV_LINEAR_ADD = 1,     /* out = residual + x W^T (out may be residual)  */
+    GV_LINEAR_SWIGLU = 2   /* out = silu(x Wg^T) * (x Wu^T), W = [Wg ; Wu]  */
+} gv_linear_epilogue;
 
 /* Shape of one attention layer of the verify pass. */
 typedef struct {
@@ -295,6 +308,34 @@ int gv_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const 
                 const void* feat_target, int feat_dt, int B, int T, int V, int H, int k, int n,
                 const uint8_t* mbar_prev, float lambda_tok, float lambda_feat, uint8_t* mbar,
                 uint8_t* mask, float* ell, float* seq_loss, void* stream);
+
+/*
+ * gv_rmsnorm -- out[r] = x[r] / sqrt(mean(x[r]^2) + eps) * w (the target
+ * layer's input and post-attention norms, and the final norm before the LM
+ * head).  bf16 x, w, out [rows][H] / [H]; fp32 arithmetic; H % 8 == 0,
+ * 16-byte aligned pointers; out may equal x.
+ */
+int gv_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, void* stream);
+
+/*
+ * gv_linear -- a projection of the node rows, out = epilogue(x W^T): the
+ * Q/K/V, O, gate/up and down projections of the target layer.  The weight is
+ * streamed once from HBM (tensor cores, K split across CTAs when the output is
+ * narrow); fp32 accumulation; bf16 in and out.
+ *
+ *   x         bf16 [rows][K]           node rows, 1 <= rows <= 256
+ *   W         bf16 [N][K]              N = n_out, or 2 * n_out for
+ *                                      GV_LINEAR_SWIGLU (gate rows, then up rows)
+ *   residual  bf16 [rows][n_out]       GV_LINEAR_ADD only (else NULL); out may be
+ *                                      the same buffer
+ *   out       bf16 [rows][n_out]
+ *   workspace >= gv_linear_workspace(rows, K, n_out, epilogue) bytes
+ * K % 8 == 0, n_out % 8 == 0, 16-byte aligned pointers.  A bounded wait that
+ * gives up turns the affected outputs into NaN.
+ */
+size_t gv_linear_workspace(int rows, int K, int n_out, int epilogue);
+int gv_linear(const void* x, const void* W, int rows, int K, int n_out, int epilogue,
+              const void* residual, void* out, void* workspace, size_t ws_bytes, void* stream);
 
 /* Static name of a status code. */
 const char* gv_status_string(int status);

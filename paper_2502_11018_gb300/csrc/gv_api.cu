@@ -63,6 +63,10 @@ static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 // Kernel launchers defined in the other translation units.
 int launch_tree_build(const int32_t*, const int32_t*, int, int, int32_t*, int32_t*, uint64_t*,
                       int32_t*, cudaStream_t);
+size_t linear_workspace_bytes(int rows, int K, int N);
+int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int epi, const void* residual,
+                  void* out, void* workspace, cudaStream_t st);
+int launch_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, cudaStream_t st);
 int launch_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* fd,
                     const void* ft, int feat_dt, int B, int T, int V, int H, int k, int n,
                     const uint8_t* mbar_prev, float lam_tok, float lam_feat, uint8_t* mbar,
@@ -462,6 +466,40 @@ int gv_kv_compact(int L, int B, int N, int D, int Hkv, int d, int S_max, int dt,
                  "gv_kv_compact: null index pointer");
     return launch_kv_compact(L, B, N, D, Hkv, d, S_max, esize, treeK, treeV, cacheK, cacheV, path,
                              accept_len, prefix_len, new_len, seq_status, as_stream(stream));
+}
+
+size_t gv_linear_workspace(int rows, int K, int n_out, int epilogue) {
+    if (rows < 1 || rows > 256 || K < 8 || n_out < 8) return 0;
+    if (epilogue < GV_LINEAR_STORE || epilogue > GV_LINEAR_SWIGLU) return 0;
+    const int N = epilogue == GV_LINEAR_SWIGLU ? 2 * n_out : n_out;
+    return align256(linear_workspace_bytes(rows, K, N));
+}
+
+int gv_linear(const void* x, const void* W, int rows, int K, int n_out, int epilogue,
+              const void* residual, void* out, void* workspace, size_t ws_bytes, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(rows >= 1 && rows <= 256, "gv_linear: rows=%d outside 1..256", rows);
+    GV_CHECK_ARG(K >= 8 && K % 8 == 0 && n_out >= 8 && n_out % 8 == 0,
+                 "gv_linear: K=%d and n_out=%d must be positive multiples of 8", K, n_out);
+    GV_CHECK_ARG(epilogue >= GV_LINEAR_STORE && epilogue <= GV_LINEAR_SWIGLU, "gv_linear: epilogue %d",
+                 epilogue);
+    GV_CHECK_ARG(x && W && out && workspace, "gv_linear: null pointer");
+    GV_CHECK_ARG(aligned16(x) && aligned16(W) && aligned16(out), "gv_linear: pointers not 16-byte aligned");
+    GV_CHECK_ARG((epilogue == GV_LINEAR_ADD) == (residual != nullptr),
+                 "gv_linear: residual is required by GV_LINEAR_ADD and only by it");
+    GV_CHECK_ARG(!residual || aligned16(residual), "gv_linear: residual not 16-byte aligned");
+    GV_CHECK_ARG(ws_bytes >= gv_linear_workspace(rows, K, n_out, epilogue) && aligned16(workspace),
+                 "gv_linear: workspace too small or misaligned");
+    return launch_linear(x, W, rows, K, n_out, epilogue, residual, out, workspace, as_stream(stream));
+}
+
+int gv_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(rows >= 1 && H >= 8 && H % 8 == 0, "gv_rmsnorm: rows=%d H=%d (H a multiple of 8)", rows, H);
+    GV_CHECK_ARG(std::isfinite(eps) && eps >= 0.0f, "gv_rmsnorm: eps %g", (double)eps);
+    GV_CHECK_ARG(x && w && out, "gv_rmsnorm: null pointer");
+    GV_CHECK_ARG(aligned16(x) && aligned16(w) && aligned16(out), "gv_rmsnorm: pointers not 16-byte aligned");
+    return launch_rmsnorm(x, w, rows, H, eps, out, as_stream(stream));
 }
 
 int gv_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* feat_draft,

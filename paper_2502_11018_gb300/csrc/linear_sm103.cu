@@ -1,0 +1,414 @@
+// gv_linear / gv_rmsnorm: the target model's projections and norms around the
+// tree attention (the decoder layer of the verify forward, GRIFFIN Section 3),
+// bf16 on sm_103a.
+//
+// The projections of a verify step are skinny: the R = B * N <= 256 tree
+// nodes times a weight W[N][K] that is read once from HBM (4096 x 4096 up to
+// 28672 x 4096 per matrix), so the kernel is a weight stream with the node
+// rows resident, like the LM head: TMA brings k-blocks of 64 of the node rows
+// (one or two M tiles of 128) and of BN weight rows into a ring of shared
+// memory stages, one lane issues tcgen05.mma into a double-buffered TMEM
+// accumulator, and four epilogue warps write the tile's fp32 sums.  A work
+// unit is (weight tile of BN rows, K split); the split count and BN are chosen
+// so that the units fill the SMs in as few waves as possible, and the fp32
+// partial sums of every split go to the workspace.  gemm_reduce_kernel then
+// adds the splits and applies the epilogue (store, residual add, or SwiGLU
+// over the gate and up halves), writing bf16.
+#include "gv_internal.cuh"
+#include "sm103.cuh"
+
+namespace gv {
+using namespace sm103;
+
+int make_map_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                uint64_t row_stride_bytes);
+
+constexpr int GM_THREADS = 192;
+constexpr int GM_A_TILE = 128 * 128;    // 128 rows x 64 bf16
+
+struct GemmArgs {
+    int rows, mt;            // node rows (<= 256) and M tiles
+    int N, K;                // weight rows (GEMM output columns) and inner size
+    int BN, n_tiles, KS, kblocks, units;
+    int stages, stage_bytes;
+    uint32_t tmem_cols;
+    float* part;             // [KS][rows][N] fp32
+};
+
+__global__ void __launch_bounds__(GM_THREADS, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_w,
+               GemmArgs a) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* stage_base = smem_raw;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw + (size_t)a.stages * a.stage_bytes);
+    uint64_t* full = bars;
+    uint64_t* empty = bars + a.stages;
+    uint64_t* tfull = empty + a.stages;
+    uint64_t* tempty = tfull + 2;
+    uint64_t* drain = tempty + 2;
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+    volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < a.stages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int c = 0; c < 2; ++c) {
+            mbar_init(&tfull[c], 1);
+            mbar_init(&tempty[c], 4);
+        }
+        mbar_init(drain, 1);
+        // (the 128B-swizzled stages need a 1024-byte aligned base)
+        *abort = (smem_u32(smem_raw) & 1023u) != 0 ? 1 : 0;
+        fence_mbar_init();
+        prefetch_tmap(&tmap_x);
+        prefetch_tmap(&tmap_w);
+    }
+    if (warp == 1) tmem_alloc(tmem_holder, a.tmem_cols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+    const int acc_cols = a.mt * a.BN;
+    // k-block range of split ks (the splits differ by at most one block)
+    auto kb_lo = [&](int ks) { return (int)(((long)a.kblocks * ks) / a.KS); };
+
+    if (warp == 0) {
+        // ------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            const uint64_t pol_w = policy_evict_first();
+            const uint64_t pol_x = policy_evict_last();
+            const uint32_t tx = (uint32_t)(a.mt * GM_A_TILE + a.BN * 128);
+            int s = 0;
+            uint32_t ph = 0;
+            int issued[8];
+            for (int q = 0; q < 8; ++q) issued[q] = -1;
+            // The first ring fill of W (a weight: no kernel of the stream
+            // writes it) streams before the dependency wait; the node rows,
+            // written upstream, are loaded after it.
+            const int u0 = blockIdx.x;
+            int pre = 0;
+            if (u0 < a.units) {
+                const int nt = u0 / a.KS, ks = u0 % a.KS;
+                const int lo = kb_lo(ks), hi = kb_lo(ks + 1);
+                pre = min(a.stages, hi - lo);
+                for (int q = 0; q < pre; ++q) {
+                    mbar_arrive_expect_tx(&full[q], tx);
+                    tma_load_2d(stage_base + (size_t)q * a.stage_bytes + a.mt * GM_A_TILE, &tmap_w, &full[q],
+                                (lo + q) * 64, nt * a.BN, pol_w);
+                    issued[q] = 0;
+                }
+            }
+            pdl_wait();
+            pdl_trigger();
+            if (u0 < a.units) {
+                const int lo = kb_lo(u0 % a.KS);
+                for (int q = 0; q < pre; ++q)
+                    for (int m = 0; m < a.mt; ++m)
+                        tma_load_2d(stage_base + (size_t)q * a.stage_bytes + m * GM_A_TILE, &tmap_x, &full[q],
+                                    (lo + q) * 64, m * 128, pol_x);
+            }
+            s = pre % a.stages;
+            ph = pre == a.stages ? 1u : 0u;
+            for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
+                const int nt = u / a.KS, ks = u % a.KS;
+                const int lo = kb_lo(ks), hi = kb_lo(ks + 1);
+                for (int kb = lo + (u == u0 ? pre : 0); kb < hi; ++kb) {
+                    if (!mbar_wait(&empty[s], ph ^ 1u, abort)) goto producer_done;
+                    mbar_arrive_expect_tx(&full[s], tx);
+                    uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
+                    for (int m = 0; m < a.mt; ++m)
+                        tma_load_2d(st + m * GM_A_TILE, &tmap_x, &full[s], kb * 64, m * 128, pol_x);
+                    tma_load_2d(st + a.mt * GM_A_TILE, &tmap_w, &full[s], kb * 64, nt * a.BN, pol_w);
+                    issued[s] = (int)ph;
+                    if (++s == a.stages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+            }
+        producer_done:
+            if (*abort) {
+                for (int q = 0; q < a.stages; ++q)
+                    if (issued[q] >= 0) mbar_wait_timeout_only(&full[q], (uint32_t)issued[q]);
+            }
+        }
+    } else if (warp == 1) {
+        // -------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(128, a.BN);
+            int s = 0;
+            uint32_t ph = 0;
+            int i = 0;
+            for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++i) {
+                const int ks = u % a.KS;
+                const int lo = kb_lo(ks), hi = kb_lo(ks + 1);
+                const int acc = i & 1;
+                if (!mbar_wait(&tempty[acc], ((uint32_t)(i >> 1) & 1u) ^ 1u, abort)) break;
+                tc_fence_after();
+                const uint32_t d_base = tmem + (uint32_t)(acc * acc_cols);
+                bool ok = true;
+                for (int kb = lo; kb < hi; ++kb) {
+                    if (!mbar_wait(&full[s], ph, abort)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
+                    const uint64_t bdesc = sdesc_kmajor_sw128(smem_u32(st + a.mt * GM_A_TILE));
+                    for (int m = 0; m < a.mt; ++m) {
+                        const uint64_t adesc = sdesc_kmajor_sw128(smem_u32(st + m * GM_A_TILE));
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk)
+                            mma_bf16(d_base + (uint32_t)(m * a.BN), adesc + 2u * kk, bdesc + 2u * kk, idesc,
+                                     (kb != lo || kk != 0) ? 1u : 0u);
+                    }
+                    mma_commit(&empty[s]);
+                    if (++s == a.stages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                mma_commit(&tfull[acc]);
+            }
+            mma_commit(drain);
+            mbar_wait_timeout_only(drain, 0);
+        }
+    } else {
+        // ----------------------------------------------------------- epilogue
+        const int sub = warp & 3;                 // TMEM lane quarter this warp may access
+        const int row_in_tile = sub * 32 + lane;
+        pdl_wait();   // (before this role's global writes)
+        // Once a wait gives up, this CTA's remaining tiles get NaN partials,
+        // so that the reduction turns the affected outputs into NaN.
+        bool failed = false;
+        int i = 0;
+        for (int u = blockIdx.x; u < a.units; u += gridDim.x, ++i) {
+            const int nt = u / a.KS, ks = u % a.KS;
+            const int acc = i & 1;
+            if (!failed) {
+                int ok = 1;
+                if (lane == 0) ok = mbar_wait(&tfull[acc], (uint32_t)(i >> 1) & 1u, abort);
+                failed = __shfl_sync(FULL, ok, 0) == 0;
+            }
+            __syncwarp();
+            tc_fence_after();
+            const int n0 = nt * a.BN;
+            for (int m = 0; m < a.mt; ++m) {
+                const int r = m * 128 + row_in_tile;
+                float* dst = a.part + ((size_t)ks * a.rows + r) * a.N;
+                for (int c0 = 0; c0 < a.BN; c0 += 32) {
+                    uint32_t v[32];
+                    if (!failed) {
+                        tmem_ld32(tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * acc_cols + m * a.BN + c0),
+                                  v);
+                        tmem_wait_ld();
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(NAN);
+                    }
+                    if (r < a.rows) {
+                        const int n = n0 + c0;
+                        if (n + 32 <= a.N && (a.N & 3) == 0) {
+#pragma unroll
+                            for (int j = 0; j < 32; j += 4)
+                                *reinterpret_cast<float4*>(dst + n + j) =
+                                    make_float4(__uint_as_float(v[j]), __uint_as_float(v[j + 1]),
+                                                __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
+                        } else {
+                            for (int j = 0; j < 32 && n + j < a.N; ++j) dst[n + j] = __uint_as_float(v[j]);
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0 && !failed) mbar_arrive(&tempty[acc]);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, a.tmem_cols);
+}
+
+// Adds the K splits of 8 consecutive output columns of one row and applies
+// the epilogue; one thread per (row, 8 columns), bf16 16-byte stores (NaN
+// partials of a GEMM that gave up propagate to the outputs).
+__global__ void __launch_bounds__(256)
+gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int n_out, int epi,
+                   const __nv_bfloat16* residual, __nv_bfloat16* out) {
+    pdl_wait();
+    pdl_trigger();
+    const int per_row = n_out / 8;
+    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= rows * per_row) return;
+    const int r = idx / per_row, c = (idx - r * per_row) * 8;
+    float acc[8], up[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] = up[e] = 0.f;
+    for (int ks = 0; ks < KS; ++ks) {
+        const float* p = part + ((size_t)ks * rows + r) * N;
+        const float4 a0 = *reinterpret_cast<const float4*>(p + c);
+        const float4 a1 = *reinterpret_cast<const float4*>(p + c + 4);
+        acc[0] += a0.x; acc[1] += a0.y; acc[2] += a0.z; acc[3] += a0.w;
+        acc[4] += a1.x; acc[5] += a1.y; acc[6] += a1.z; acc[7] += a1.w;
+        if (epi == GV_LINEAR_SWIGLU) {
+            const float4 b0 = *reinterpret_cast<const float4*>(p + n_out + c);
+            const float4 b1 = *reinterpret_cast<const float4*>(p + n_out + c + 4);
+            up[0] += b0.x; up[1] += b0.y; up[2] += b0.z; up[3] += b0.w;
+            up[4] += b1.x; up[5] += b1.y; up[6] += b1.z; up[7] += b1.w;
+        }
+    }
+    float o[8];
+    if (epi == GV_LINEAR_SWIGLU) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) o[e] = acc[e] / (1.0f + __expf(-acc[e])) * up[e];
+    } else if (epi == GV_LINEAR_ADD) {
+        const uint4 rv = *reinterpret_cast<const uint4*>(residual + (size_t)r * n_out + c);
+        const uint32_t w[4] = {rv.x, rv.y, rv.z, rv.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            o[2 * e] = acc[2 * e] + __uint_as_float(w[e] << 16);
+            o[2 * e + 1] = acc[2 * e + 1] + __uint_as_float(w[e] & 0xffff0000u);
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) o[e] = acc[e];
+    }
+    uint32_t pk[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        __nv_bfloat162 h2 = __floats2bfloat162_rn(o[2 * e], o[2 * e + 1]);
+        pk[e] = *reinterpret_cast<uint32_t*>(&h2);
+    }
+    *reinterpret_cast<uint4*>(out + (size_t)r * n_out + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+}
+
+// RMSNorm of one row per CTA: out = x / sqrt(mean(x^2) + eps) * w, fp32 math,
+// bf16 in and out (16-byte vectors; H % 8 == 0).
+__global__ void __launch_bounds__(256)
+rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ w, int H, float eps,
+               __nv_bfloat16* __restrict__ out) {
+    __shared__ float red[8];
+    pdl_wait();
+    pdl_trigger();
+    const int r = blockIdx.x, tid = threadIdx.x;
+    const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)r * H);
+    float ss = 0.f;
+    for (int i = tid; i < H / 8; i += blockDim.x) {
+        const uint4 v = xr[i];
+        const uint32_t q[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float lo = __uint_as_float(q[e] << 16), hi = __uint_as_float(q[e] & 0xffff0000u);
+            ss += lo * lo + hi * hi;
+        }
+    }
+    ss = warp_sum(ss);
+    if ((tid & 31) == 0) red[tid >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) tot += red[k];
+    const float inv = rsqrtf(tot / (float)H + eps);
+    const uint4* wr = reinterpret_cast<const uint4*>(w);
+    uint4* orow = reinterpret_cast<uint4*>(out + (size_t)r * H);
+    for (int i = tid; i < H / 8; i += blockDim.x) {
+        const uint4 v = xr[i], g = wr[i];
+        const uint32_t q[4] = {v.x, v.y, v.z, v.w}, gw[4] = {g.x, g.y, g.z, g.w};
+        uint32_t pk[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float lo = __uint_as_float(q[e] << 16) * inv * __uint_as_float(gw[e] << 16);
+            const float hi = __uint_as_float(q[e] & 0xffff0000u) * inv * __uint_as_float(gw[e] & 0xffff0000u);
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(lo, hi);
+            pk[e] = *reinterpret_cast<uint32_t*>(&h2);
+        }
+        orow[i] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    }
+}
+
+// ----------------------------------------------------------------- host side
+// (BN, KS) minimising ceil(units / SMs) * per-unit cost, with a unit's cost
+// counted in weight rows streamed per k-block plus a fixed and an epilogue
+// share; larger BN on ties.
+struct GemmPlan {
+    int BN, KS, n_tiles, kblocks, units, grid;
+};
+
+static GemmPlan gemm_plan(int rows, int N, int K) {
+    const int mt = (rows + 127) / 128;
+    const int sms = sm_count();
+    GemmPlan best{};
+    long best_cost = -1;
+    const int kblocks = (K + 63) / 64;
+    for (int bn = 64; bn <= 256 && 2 * mt * bn <= 512; bn += 32) {
+        const int tiles = (N + bn - 1) / bn;
+        for (int ks = 1; ks <= kblocks && ks <= 32; ++ks) {
+            const long units = (long)tiles * ks;
+            const long waves = (units + sms - 1) / sms;
+            const long kb_per = (kblocks + ks - 1) / ks;
+            const long cost = waves * (kb_per * (bn + 8) + 3L * bn * mt);
+            if (best_cost < 0 || cost < best_cost || (cost == best_cost && bn > best.BN)) {
+                best_cost = cost;
+                best = GemmPlan{bn, ks, tiles, kblocks, (int)units, 0};
+            }
+        }
+    }
+    best.grid = best.units < sms ? best.units : sms;
+    return best;
+}
+
+size_t linear_workspace_bytes(int rows, int K, int N) {
+    const GemmPlan p = gemm_plan(rows, N, K);
+    return (size_t)p.KS * rows * N * sizeof(float);
+}
+
+int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int epi, const void* residual,
+                  void* out, void* workspace, cudaStream_t st) {
+    const int N = epi == GV_LINEAR_SWIGLU ? 2 * n_out : n_out;
+    const GemmPlan p = gemm_plan(rows, N, K);
+    GemmArgs a{};
+    a.rows = rows;
+    a.mt = (rows + 127) / 128;
+    a.N = N;
+    a.K = K;
+    a.BN = p.BN;
+    a.n_tiles = p.n_tiles;
+    a.KS = p.KS;
+    a.kblocks = p.kblocks;
+    a.units = p.units;
+    a.stage_bytes = a.mt * GM_A_TILE + a.BN * 128;
+    constexpr int SMEM_BUDGET = 220 * 1024;
+    a.stages = (SMEM_BUDGET - 2048) / a.stage_bytes;
+    if (a.stages > 8) a.stages = 8;
+    const int cols = 2 * a.mt * a.BN;
+    a.tmem_cols = cols <= 32 ? 32 : cols <= 64 ? 64 : cols <= 128 ? 128 : cols <= 256 ? 256 : 512;
+    a.part = static_cast<float*>(workspace);
+    CUtensorMap mx, mw;
+    int rc = make_map_2d(&mx, x, (uint64_t)rows, (uint64_t)K, 128, (uint64_t)K * 2);
+    if (rc != GV_OK) return rc;
+    rc = make_map_2d(&mw, W, (uint64_t)N, (uint64_t)K, (uint32_t)a.BN, (uint64_t)K * 2);
+    if (rc != GV_OK) return rc;
+    const size_t smem = (size_t)a.stages * a.stage_bytes + 8 * (2 * a.stages + 5) + 16;
+    cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    launch_pdl(gemm_tc_kernel, dim3(p.grid), dim3(GM_THREADS), smem, st, mx, mw, a);
+    rc = check_launch("gemm_tc_kernel");
+    if (rc != GV_OK) return rc;
+    const int items = rows * (n_out / 8);
+    launch_pdl(gemm_reduce_kernel, dim3((items + 255) / 256), dim3(256), 0, st, (const float*)a.part, a.KS, rows,
+               N, n_out, epi, static_cast<const __nv_bfloat16*>(residual), static_cast<__nv_bfloat16*>(out));
+    return check_launch("gemm_reduce_kernel");
+}
+
+int launch_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, cudaStream_t st) {
+    launch_pdl(rmsnorm_kernel, dim3(rows), dim3(256), 0, st, static_cast<const __nv_bfloat16*>(x),
+               static_cast<const __nv_bfloat16*>(w), H, eps, static_cast<__nv_bfloat16*>(out));
+    return check_launch("rmsnorm_kernel");
+}
+
+}  // namespace gv

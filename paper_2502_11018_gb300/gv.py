@@ -29,12 +29,14 @@ GV_F32 = 1
 GV_SELECT_ARGMAX = 0
 GV_SELECT_TOPK = 1
 GV_SELECT_LOGITS = 2
+GV_LINEAR_STORE, GV_LINEAR_ADD, GV_LINEAR_SWIGLU = 0, 1, 2
 
 # Every symbol include/gv.h declares.
 EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "gv_verify_attention",
            "gv_lmhead_workspace", "gv_lmhead_select", "gv_lmhead_argmax_noalloc",
            "gv_accept_workspace", "gv_accept",
-           "gv_kv_compact", "gv_tat_loss", "gv_status_string", "gv_last_error", "gv_version")
+           "gv_kv_compact", "gv_rmsnorm", "gv_linear_workspace", "gv_linear", "gv_tat_loss",
+           "gv_status_string", "gv_last_error", "gv_version")
 
 
 class GvError(RuntimeError):
@@ -77,6 +79,9 @@ def lib():
         "gv_accept_workspace": ([_i, _i, _f], _sz),
         "gv_accept": ([_i, _i, _i, _i, _f] + [_vp] * 12 + [_vp, _sz, _vp], _i),
         "gv_kv_compact": ([_i] * 8 + [_vp] * 9 + [_vp], _i),
+        "gv_rmsnorm": ([_vp, _vp, _i, _i, _f, _vp, _vp], _i),
+        "gv_linear_workspace": ([_i, _i, _i, _i], _sz),
+        "gv_linear": ([_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _sz, _vp], _i),
         "gv_tat_loss": ([_vp, _i, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, _i, _vp, _f, _f,
                          _vp, _vp, _vp, _vp, _vp], _i),
         "gv_status_string": ([_i], ctypes.c_char_p),
@@ -234,3 +239,24 @@ def gv_tat_loss(logits, tokens, feat_draft, feat_target, k, n, mbar_prev, mbar, 
         _ptr(feat_target, "feat_target"), dtype_code(feat_draft), B, T, V, H, k, n,
         _ptr(mbar_prev, "mbar_prev"), float(lambda_tok), float(lambda_feat), _ptr(mbar, "mbar"),
         _ptr(mask, "mask"), _ptr(ell, "ell"), _ptr(seq_loss, "seq_loss"), _stream(stream)))
+
+
+def gv_rmsnorm(x, w, out, eps=1e-5, stream=None):
+    """RMSNorm of the rows of x [rows][H] with weight w [H] into out (bf16)."""
+    rows, H = x.shape
+    return _check("gv_rmsnorm", lib().gv_rmsnorm(_ptr(x, "x"), _ptr(w, "w"), rows, H, float(eps),
+                                                 _ptr(out, "out"), _stream(stream)))
+
+
+def gv_linear_workspace(rows, K, n_out, epilogue=0):
+    return int(lib().gv_linear_workspace(rows, K, n_out, epilogue))
+
+
+def gv_linear(x, W, out, epilogue=0, residual=None, workspace=None, stream=None):
+    """out [rows][n_out] = epilogue(x W^T) (see include/gv.h)."""
+    rows, K = x.shape
+    n_out = out.shape[1]
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    return _check("gv_linear", lib().gv_linear(
+        _ptr(x, "x"), _ptr(W, "W"), rows, K, n_out, int(epilogue), _ptr(residual, "residual"), _ptr(out, "out"),
+        _ptr(workspace, "workspace"), ws_bytes, _stream(stream)))

@@ -70,6 +70,13 @@ def test_host_side_validation(lib):
     assert lib.gv_tat_loss(16, gv.GV_F32, 16, 16, 16, gv.GV_BF16, 2, 8, 10, 64, 3, 1, 16, 1.0, 0.1,
                            16, 16, 16, 16, nul) == gv.GV_ERR_ARG
     assert "mbar_prev" in gv.last_error()
+    # projections: K not a multiple of 8; a residual without GV_LINEAR_ADD
+    assert lib.gv_linear(16, 16, 60, 4100 + 2, 4096, 0, nul, 16, 16, 1 << 30, nul) == gv.GV_ERR_ARG
+    assert lib.gv_linear(16, 16, 60, 4096, 4096, 0, 16, 16, 16, 1 << 30, nul) == gv.GV_ERR_ARG
+    assert "residual" in gv.last_error()
+    assert lib.gv_rmsnorm(16, 16, 60, 4100, 1e-5, 16, nul) == gv.GV_ERR_ARG
+    assert gv.gv_linear_workspace(60, 4096, 1024, gv.GV_LINEAR_STORE) > 0
+    assert gv.gv_linear_workspace(60, 4096, 14336, gv.GV_LINEAR_SWIGLU) >= 60 * 28672 * 4
 
 
 def test_workspace_queries(lib):
