@@ -362,3 +362,50 @@ def make_tat_inputs(cfg, seed, device="cpu", p_plant=0.7, p_prev=0.7):
                      tokens=torch.from_numpy(tokens.astype(np.int32)).view(B, T).to(device),
                      feat_draft=fd.to(device), feat_target=ft.to(device),
                      mbar_prev=None if prev is None else prev.to(device))
+
+
+
+# --------------------------------------------------------------------------
+# Target decoder-layer weights for the whole verify forward (LLaMA-style:
+# RMSNorm, Q/K/V/O projections, SwiGLU MLP).  FFN widths are the public model
+# shapes; weights ~ N(0, 0.02), norm weights ~ 1 + N(0, 0.05), the draft
+# tokens' input embeddings ~ N(0, 1).
+# --------------------------------------------------------------------------
+
+FFN = {"llama2_7b": 11008, "llama3_8b": 14336, "llama2_13b_b4": 13824, "llama3_8b_chain_b16": 14336}
+
+
+@dataclass
+class ForwardWeights:
+    F: int
+    h0: torch.Tensor          # [B*N][H]  embeddings of the tree's tokens
+    attn_norm: torch.Tensor   # [L][H]
+    Wq: torch.Tensor          # [L][Hq*d][H]
+    Wk: torch.Tensor          # [L][Hkv*d][H]
+    Wv: torch.Tensor          # [L][Hkv*d][H]
+    Wo: torch.Tensor          # [L][H][Hq*d]
+    mlp_norm: torch.Tensor    # [L][H]
+    Wgu: torch.Tensor         # [L][2F][H]  gate rows, then up rows
+    Wd: torch.Tensor          # [L][H][F]
+    final_norm: torch.Tensor  # [H]
+
+
+def make_forward_weights(cfg, seed, device="cpu", layers=None, F=None):
+    L = cfg["L"] if layers is None else layers
+    F = FFN[cfg["name"]] if F is None else F
+    B, N, H, Hq, Hkv, d = cfg["B"], cfg["N"], cfg["H"], cfg["Hq"], cfg["Hkv"], cfg["d"]
+    dt = torch.bfloat16
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed) + 77)
+    std = cfg["std_w"]
+
+    def norm_w(*shape):
+        return (1.0 + 0.05 * torch.randn(shape, generator=gen, device=device, dtype=torch.float32)).to(dt)
+
+    return ForwardWeights(
+        F=F, h0=randn(gen, (B * N, H), 1.0, dt, device),
+        attn_norm=norm_w(L, H), Wq=randn(gen, (L, Hq * d, H), std, dt, device),
+        Wk=randn(gen, (L, Hkv * d, H), std, dt, device), Wv=randn(gen, (L, Hkv * d, H), std, dt, device),
+        Wo=randn(gen, (L, H, Hq * d), std, dt, device), mlp_norm=norm_w(L, H),
+        Wgu=randn(gen, (L, 2 * F, H), std, dt, device), Wd=randn(gen, (L, H, F), std, dt, device),
+        final_norm=norm_w(H))

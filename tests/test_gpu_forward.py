@@ -1,0 +1,77 @@
+"""The whole verify forward (decoder layers around the tree attention, final
+norm, LM head, acceptance) through the C ABI against the float64 oracle
+composed layer by layer.  Every stage rounds to bf16 on the GPU, so the
+hidden states are held to 3e-2 of their largest magnitude after the layers;
+the LM-head argmax is compared on the rows whose oracle margin is clear."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2502_11018_gb300 import inputs
+from paper_2502_11018_gb300.forward import VerifyForward
+from gpu_util import device, f64, rel_err
+
+pytestmark = pytest.mark.gpu
+
+TOL_H = 3e-2
+
+
+def _oracle_forward(cfg, inp, fw, L):
+    B, N, Hq, Hkv, d = cfg["B"], cfg["N"], cfg["Hq"], cfg["Hkv"], cfg["d"]
+    P = inp.prefix_len.cpu().numpy()
+    depth, pos, anc, st = oracle.tree_build(inp.parents.cpu().numpy(), P)
+    h = f64(fw.h0)
+    for l in range(L):
+        w = {"attn_norm": f64(fw.attn_norm[l]), "Wq": f64(fw.Wq[l]), "Wk": f64(fw.Wk[l]), "Wv": f64(fw.Wv[l]),
+             "Wo": f64(fw.Wo[l]), "mlp_norm": f64(fw.mlp_norm[l]), "Wg": f64(fw.Wgu[l][:fw.F]),
+             "Wu": f64(fw.Wgu[l][fw.F:]), "Wd": f64(fw.Wd[l])}
+        h, _, _ = oracle.decoder_layer(h, w, f64(inp.cacheK[l]), f64(inp.cacheV[l]), P, pos, anc, cfg["rope_base"],
+                                       B, N, Hq, Hkv, d)
+    return h
+
+
+@pytest.mark.parametrize("name,over,L,F", [
+    ("llama3_8b", dict(H=256, Hq=4, Hkv=2, V=1000, P=(100,)), 2, 512),
+    ("llama3_8b", dict(P=(512,)), 2, None),
+    ("llama2_13b_b4", dict(P=(64, 300, 17, 128)), 1, None),
+])
+def test_forward_parity(name, over, L, F):
+    dev = device()
+    cfg = inputs.config(name, **over)
+    inp = inputs.make_step_inputs(cfg, 21, device=dev, layers=L)
+    fw = inputs.make_forward_weights(cfg, 21, device=dev, layers=L, F=F)
+    fwd = VerifyForward(inp, fw)
+    fwd.run()
+    torch.cuda.synchronize()
+    ref_h = _oracle_forward(cfg, inp, fw, L)
+    got_h = f64(fwd.h)
+    assert np.isfinite(got_h).all()
+    assert rel_err(got_h, ref_h) <= TOL_H
+    # final norm and LM head: the argmax where the oracle's top-2 gap is clear
+    hf = oracle.rmsnorm(ref_h, f64(fw.final_norm))
+    logits = oracle.lmhead_logits(hf, f64(inp.W))
+    top2 = np.sort(logits, axis=1)[:, -2:]
+    clear = (top2[:, 1] - top2[:, 0]) > 0.05 * np.abs(logits).max()
+    ids = fwd.step.ids.cpu().numpy()
+    assert clear.sum() >= 1
+    np.testing.assert_array_equal(ids[clear], logits.argmax(axis=1)[clear])
+    assert (fwd.step.seq_status.cpu().numpy() == 0).all()
+
+
+def test_forward_graph_replay_matches_eager():
+    dev = device()
+    cfg = inputs.config("llama3_8b", H=256, Hq=4, Hkv=2, V=1000, P=(100,))
+    inp = inputs.make_step_inputs(cfg, 5, device=dev, layers=2)
+    fw = inputs.make_forward_weights(cfg, 5, device=dev, layers=2, F=512)
+    fwd = VerifyForward(inp, fw)
+    fwd.run()
+    torch.cuda.synchronize()
+    eager = (fwd.h.clone(), fwd.step.ids.clone(), fwd.step.path.clone())
+    fwd.capture()
+    for _ in range(2):
+        fwd.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(fwd.h, eager[0])
+    assert torch.equal(fwd.step.ids, eager[1]) and torch.equal(fwd.step.path, eager[2])
