@@ -88,11 +88,28 @@ def attention_bytes(cfg):
     return b
 
 
+def attention_splits(cfg):
+    """Key splits per attention unit, the rule the library applies: as many as
+    fit the SMs in one wave (at most 16, at least 4 when the cache holds 4096
+    keys or more, never more than a unit's blocks)."""
+    tiles = (cfg["G"] * cfg["N"] + 127) // 128 if "G" in cfg else (cfg["Hq"] // cfg["Hkv"] * cfg["N"] + 127) // 128
+    units = cfg["B"] * cfg["Hkv"] * tiles
+    c = torch.cuda.get_device_properties(0).multi_processor_count // units
+    if cfg["S_max"] >= 4096 and c < 4:
+        c = 4
+    c = min(c, (cfg["S_max"] + 127) // 128 + 1, 16)
+    return max(c, 1)
+
+
 def launches_per_step(cfg):
     """Kernels of this library one step launches: tree build, RoPE table, the
-    attention layers (split attention + merge on the bf16 tensor-core path, rotate +
-    split + combine on the fp32 path), LM head + merge, accept, compaction."""
-    per_layer = 2 if cfg["dtype"] == "bf16" else 3
+    attention layers (split attention + merge on the bf16 tensor-core path --
+    no merge when a unit has a single split --, rotate + split + combine on
+    the fp32 path), LM head + merge, accept, compaction."""
+    if cfg["dtype"] == "bf16":
+        per_layer = 1 if attention_splits(cfg) == 1 else 2
+    else:
+        per_layer = 3
     return 2 + per_layer * cfg["L"] + 2 + 1 + 1
 
 
@@ -322,11 +339,13 @@ def main():
     ap.add_argument("--seed", type=int, default=1000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention", "tat"],
+    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention", "tat", "forward"],
                     help="step: the benchmark; lmhead / attention: time that call alone "
                          "(a small, self-contained launch sequence for profiler captures); "
                          "tat: one token-alignable training pass (gv_tat_loss) on a "
-                         "4 x 2048-token batch, vocabulary 32000")
+                         "4 x 2048-token batch, vocabulary 32000; forward: the whole verify "
+                         "forward of the target (decoder layers around the path, random "
+                         "weights of the --config model's shape)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
 
@@ -352,6 +371,9 @@ def main():
     from paper_2502_11018_gb300.step import VerifyStep
     if args.kernel == "tat":
         run_tat(args, dev)
+        return
+    if args.kernel == "forward":
+        run_forward(args, dev)
         return
     cfg = inputs.config(args.config)
     if args.kernel != "step":
@@ -477,6 +499,46 @@ def run_kernel_only(args, cfg, dev):
                       "ms_per_call_graph": ms_graph, "algorithmic_bytes": nbytes,
                       "achieved_gbs_graph": gbs_graph,
                       "frac_of_measured_hbm_graph": gbs_graph / peaks["hbm_gbs"]}), flush=True)
+
+
+def forward_bytes(cfg, F, accept_len):
+    """Algorithmic bytes of the whole verify forward: every weight read once
+    (per layer Q/K/V/O, gate/up, down and the two norms; the final norm), the
+    verify path's own bytes (prefix K/V, LM head weight, compaction), and the
+    node activations each layer writes and reads back (x, q/k/v, attention
+    output, h twice, the MLP hidden)."""
+    es = 2
+    L, B, N, H, Hq, Hkv, d = cfg["L"], cfg["B"], cfg["N"], cfg["H"], cfg["Hq"], cfg["Hkv"], cfg["d"]
+    R = B * N
+    weights = L * es * (H * (Hq + 2 * Hkv) * d + Hq * d * H + 3 * H * F + 2 * H) + es * H
+    acts = L * R * es * (2 * H + (2 * Hq + 2 * Hkv) * d + 4 * H + 2 * F + 2 * H)
+    return weights + acts + step_bytes(cfg, accept_len)["total"]
+
+
+def run_forward(args, dev):
+    """The whole verify forward of the --config target, timed from a CUDA graph
+    with inputs (14 GB of LLaMA-3-8B-shaped weights) resident in HBM."""
+    from paper_2502_11018_gb300.forward import VerifyForward
+    cfg = inputs.config(args.config)
+    inp = inputs.make_step_inputs(cfg, args.seed, device=dev)
+    fw = inputs.make_forward_weights(cfg, args.seed, device=dev)
+    fwd = VerifyForward(inp, fw)
+    fwd.capture()
+    stream = torch.cuda.current_stream()
+    for _ in range(max(args.warmup, 3)):
+        fwd.replay()
+    torch.cuda.synchronize()
+    steps = max(3, min(args.steps, 100))
+    ms = event_time_ms(fwd.replay, steps, stream)
+    alen = fwd.step.accept_len.cpu().numpy()
+    nbytes = forward_bytes(cfg, fw.F, alen)
+    peaks = load_peaks()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    print(json.dumps({"kernel": "forward", "workload": cfg["name"], "ffn": fw.F, "layers": cfg["L"],
+                      "ms_per_step": ms, "verify_steps_per_s": 1e3 / ms,
+                      "accepted_tok_per_s": float(alen.sum()) * 1e3 / ms, "algorithmic_bytes": nbytes,
+                      "achieved_gbs": gbs, "frac_of_measured_hbm": gbs / peaks["hbm_gbs"],
+                      "data": "synthetic (seeded random weights, caches and draft trees)"}), flush=True)
 
 
 def tat_bytes(cfg):

@@ -20,6 +20,7 @@
  *
  *   gv_rmsnorm           RMSNorm of the node rows
  *   gv_linear            skinny projection x W^T with a fused epilogue
+ *   gv_linear_qkv        the Q, K and V projections as one weight stream
  *
  * and, for training the draft model (Section 4.1):
  *
@@ -336,6 +337,17 @@ int gv_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* o
 size_t gv_linear_workspace(int rows, int K, int n_out, int epilogue);
 int gv_linear(const void* x, const void* W, int rows, int K, int n_out, int epilogue,
               const void* residual, void* out, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * gv_linear_qkv -- the Q, K and V projections as one weight stream:
+ * Wqkv = [Wq ; Wk ; Wv] bf16 [n_q + 2 n_kv][K]; q [rows][n_q], k and v
+ * [rows][n_kv] (bf16, separate buffers, e.g. the gv_verify_attention inputs
+ * q [B][N][Hq][d], k_new / v_new [B][N][Hkv][d]).  Conditions and workspace
+ * as gv_linear's.
+ */
+size_t gv_linear_qkv_workspace(int rows, int K, int n_q, int n_kv);
+int gv_linear_qkv(const void* x, const void* Wqkv, int rows, int K, int n_q, int n_kv, void* q, void* k, void* v,
+                  void* workspace, size_t ws_bytes, void* stream);
 
 /* Static name of a status code. */
 const char* gv_status_string(int status);

@@ -65,7 +65,8 @@ int launch_tree_build(const int32_t*, const int32_t*, int, int, int32_t*, int32_
                       int32_t*, cudaStream_t);
 size_t linear_workspace_bytes(int rows, int K, int N);
 int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int epi, const void* residual,
-                  void* out, void* workspace, cudaStream_t st);
+                  void* out, void* workspace, cudaStream_t st, void* out1 = nullptr, void* out2 = nullptr,
+                  int n0 = 0, int n1 = 0);
 int launch_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, cudaStream_t st);
 int launch_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* fd,
                     const void* ft, int feat_dt, int B, int T, int V, int H, int k, int n,
@@ -491,6 +492,25 @@ int gv_linear(const void* x, const void* W, int rows, int K, int n_out, int epil
     GV_CHECK_ARG(ws_bytes >= gv_linear_workspace(rows, K, n_out, epilogue) && aligned16(workspace),
                  "gv_linear: workspace too small or misaligned");
     return launch_linear(x, W, rows, K, n_out, epilogue, residual, out, workspace, as_stream(stream));
+}
+
+size_t gv_linear_qkv_workspace(int rows, int K, int n_q, int n_kv) {
+    return gv_linear_workspace(rows, K, n_q + 2 * n_kv, GV_LINEAR_STORE);
+}
+
+int gv_linear_qkv(const void* x, const void* Wqkv, int rows, int K, int n_q, int n_kv, void* q, void* k, void* v,
+                  void* workspace, size_t ws_bytes, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(rows >= 1 && rows <= 256, "gv_linear_qkv: rows=%d outside 1..256", rows);
+    GV_CHECK_ARG(K >= 8 && K % 8 == 0 && n_q >= 8 && n_q % 8 == 0 && n_kv >= 8 && n_kv % 8 == 0,
+                 "gv_linear_qkv: K=%d, n_q=%d, n_kv=%d must be positive multiples of 8", K, n_q, n_kv);
+    GV_CHECK_ARG(x && Wqkv && q && k && v && workspace, "gv_linear_qkv: null pointer");
+    GV_CHECK_ARG(aligned16(x) && aligned16(Wqkv) && aligned16(q) && aligned16(k) && aligned16(v) &&
+                     aligned16(workspace),
+                 "gv_linear_qkv: pointers not 16-byte aligned");
+    GV_CHECK_ARG(ws_bytes >= gv_linear_qkv_workspace(rows, K, n_q, n_kv), "gv_linear_qkv: workspace too small");
+    return launch_linear(x, Wqkv, rows, K, n_q + 2 * n_kv, GV_LINEAR_STORE, nullptr, q, workspace,
+                         as_stream(stream), k, v, n_q, n_kv);
 }
 
 int gv_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, void* stream) {

@@ -239,9 +239,19 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
 // Adds the K splits of 8 consecutive output columns of one row and applies
 // the epilogue; one thread per (row, 8 columns), bf16 16-byte stores (NaN
 // partials of a GEMM that gave up propagate to the outputs).
+// Column split of the stored output: columns [0, n0) go to out0[rows][n0],
+// [n0, n0 + n1) to out1[rows][n1], the rest to out2 (the fused Q/K/V
+// projection); n1 == 0 stores everything to out0.
+struct OutSplit {
+    __nv_bfloat16* out0;
+    __nv_bfloat16* out1;
+    __nv_bfloat16* out2;
+    int n0, n1;
+};
+
 __global__ void __launch_bounds__(256)
 gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int n_out, int epi,
-                   const __nv_bfloat16* residual, __nv_bfloat16* out) {
+                   const __nv_bfloat16* residual, OutSplit os) {
     pdl_wait();
     pdl_trigger();
     const int per_row = n_out / 8;
@@ -286,7 +296,14 @@ gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int 
         __nv_bfloat162 h2 = __floats2bfloat162_rn(o[2 * e], o[2 * e + 1]);
         pk[e] = *reinterpret_cast<uint32_t*>(&h2);
     }
-    *reinterpret_cast<uint4*>(out + (size_t)r * n_out + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    __nv_bfloat16* dst;
+    if (os.n1 == 0 || c < os.n0)
+        dst = os.out0 + (size_t)r * (os.n1 == 0 ? n_out : os.n0) + c;
+    else if (c < os.n0 + os.n1)
+        dst = os.out1 + (size_t)r * os.n1 + (c - os.n0);
+    else
+        dst = os.out2 + (size_t)r * (n_out - os.n0 - os.n1) + (c - os.n0 - os.n1);
+    *reinterpret_cast<uint4*>(dst) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
 }
 
 // RMSNorm of one row per CTA: out = x / sqrt(mean(x^2) + eps) * w, fp32 math,
@@ -369,7 +386,8 @@ size_t linear_workspace_bytes(int rows, int K, int N) {
 }
 
 int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int epi, const void* residual,
-                  void* out, void* workspace, cudaStream_t st) {
+                  void* out, void* workspace, cudaStream_t st, void* out1 = nullptr, void* out2 = nullptr,
+                  int n0 = 0, int n1 = 0) {
     const int N = epi == GV_LINEAR_SWIGLU ? 2 * n_out : n_out;
     const GemmPlan p = gemm_plan(rows, N, K);
     GemmArgs a{};
@@ -400,8 +418,10 @@ int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int 
     rc = check_launch("gemm_tc_kernel");
     if (rc != GV_OK) return rc;
     const int items = rows * (n_out / 8);
+    OutSplit os{static_cast<__nv_bfloat16*>(out), static_cast<__nv_bfloat16*>(out1),
+                static_cast<__nv_bfloat16*>(out2), n0, n1};
     launch_pdl(gemm_reduce_kernel, dim3((items + 255) / 256), dim3(256), 0, st, (const float*)a.part, a.KS, rows,
-               N, n_out, epi, static_cast<const __nv_bfloat16*>(residual), static_cast<__nv_bfloat16*>(out));
+               N, n_out, epi, static_cast<const __nv_bfloat16*>(residual), os);
     return check_launch("gemm_reduce_kernel");
 }
 

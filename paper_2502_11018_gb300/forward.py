@@ -6,7 +6,7 @@ target forward verifies every draft token).
 Per layer, over the hidden states h [B*N][H] of the tree nodes:
 
     x = RMSNorm(h) * w_attn                      gv_rmsnorm
-    q, k, v = x Wq^T, x Wk^T, x Wv^T             gv_linear (store)
+    q, k, v = x Wq^T, x Wk^T, x Wv^T             gv_linear_qkv (one weight stream)
     o = TreeAttention(q, k, v)                   gv_verify_attention
     h = h + o Wo^T                               gv_linear (residual add, in place)
     x = RMSNorm(h) * w_mlp                       gv_rmsnorm
@@ -42,8 +42,9 @@ class VerifyForward:
         self.k = torch.zeros(B, N, Hkv, d, **bf)
         self.v = torch.zeros(B, N, Hkv, d, **bf)
         self.g = torch.zeros(R, fw.F, **bf)
-        shapes = [(H, Hq * d, 0), (H, Hkv * d, 0), (Hq * d, H, 1), (H, fw.F, 2), (fw.F, H, 1)]
-        ws = max(gv.gv_linear_workspace(R, K, n, e) for K, n, e in shapes)
+        shapes = [(Hq * d, H, 1), (H, fw.F, 2), (fw.F, H, 1)]
+        ws = max([gv.gv_linear_workspace(R, K, n, e) for K, n, e in shapes] +
+                 [gv.gv_linear_qkv_workspace(R, H, Hq * d, Hkv * d)])
         self.lin_ws = torch.empty(ws, dtype=torch.uint8, device=dev)
         # The verify step's own buffers (tree, attention outputs, LM head,
         # acceptance); its inputs' q / k_new / v_new / h are bound to ours.
@@ -58,9 +59,8 @@ class VerifyForward:
         R = self.h.shape[0]
         h_in = fw.h0 if l == 0 else self.h      # layer 0 reads the embeddings
         gv.gv_rmsnorm(h_in, fw.attn_norm[l], self.x, stream=stream)
-        self._lin(self.x, fw.Wq[l], self.q.view(R, -1), gv.GV_LINEAR_STORE, stream=stream)
-        self._lin(self.x, fw.Wk[l], self.k.view(R, -1), gv.GV_LINEAR_STORE, stream=stream)
-        self._lin(self.x, fw.Wv[l], self.v.view(R, -1), gv.GV_LINEAR_STORE, stream=stream)
+        gv.gv_linear_qkv(self.x, fw.Wqkv[l], self.q.view(R, -1), self.k.view(R, -1), self.v.view(R, -1),
+                         self.lin_ws, stream=stream)
         i = self.inp
         gv.gv_verify_attention(st.shape, self.q, self.k, self.v, i.cacheK[l], i.cacheV[l], i.prefix_len, st.rope,
                                st.anc, st.treeK[l], st.treeV[l], st.attn_out[l], st.attn_ws, stream)

@@ -35,7 +35,8 @@ GV_LINEAR_STORE, GV_LINEAR_ADD, GV_LINEAR_SWIGLU = 0, 1, 2
 EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "gv_verify_attention",
            "gv_lmhead_workspace", "gv_lmhead_select", "gv_lmhead_argmax_noalloc",
            "gv_accept_workspace", "gv_accept",
-           "gv_kv_compact", "gv_rmsnorm", "gv_linear_workspace", "gv_linear", "gv_tat_loss",
+           "gv_kv_compact", "gv_rmsnorm", "gv_linear_workspace", "gv_linear", "gv_linear_qkv_workspace",
+           "gv_linear_qkv", "gv_tat_loss",
            "gv_status_string", "gv_last_error", "gv_version")
 
 
@@ -82,6 +83,8 @@ def lib():
         "gv_rmsnorm": ([_vp, _vp, _i, _i, _f, _vp, _vp], _i),
         "gv_linear_workspace": ([_i, _i, _i, _i], _sz),
         "gv_linear": ([_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _sz, _vp], _i),
+        "gv_linear_qkv_workspace": ([_i, _i, _i, _i], _sz),
+        "gv_linear_qkv": ([_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp], _i),
         "gv_tat_loss": ([_vp, _i, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, _i, _vp, _f, _f,
                          _vp, _vp, _vp, _vp, _vp], _i),
         "gv_status_string": ([_i], ctypes.c_char_p),
@@ -259,4 +262,19 @@ def gv_linear(x, W, out, epilogue=0, residual=None, workspace=None, stream=None)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     return _check("gv_linear", lib().gv_linear(
         _ptr(x, "x"), _ptr(W, "W"), rows, K, n_out, int(epilogue), _ptr(residual, "residual"), _ptr(out, "out"),
+        _ptr(workspace, "workspace"), ws_bytes, _stream(stream)))
+
+
+def gv_linear_qkv_workspace(rows, K, n_q, n_kv):
+    return int(lib().gv_linear_qkv_workspace(rows, K, n_q, n_kv))
+
+
+def gv_linear_qkv(x, Wqkv, q, k, v, workspace, stream=None):
+    """q, k, v = x [Wq ; Wk ; Wv]^T, one weight stream (see include/gv.h)."""
+    rows, K = x.shape
+    n_q = q.numel() // rows
+    n_kv = k.numel() // rows
+    ws_bytes = workspace.numel() * workspace.element_size()
+    return _check("gv_linear_qkv", lib().gv_linear_qkv(
+        _ptr(x, "x"), _ptr(Wqkv, "Wqkv"), rows, K, n_q, n_kv, _ptr(q, "q"), _ptr(k, "k"), _ptr(v, "v"),
         _ptr(workspace, "workspace"), ws_bytes, _stream(stream)))

@@ -380,9 +380,7 @@ class ForwardWeights:
     F: int
     h0: torch.Tensor          # [B*N][H]  embeddings of the tree's tokens
     attn_norm: torch.Tensor   # [L][H]
-    Wq: torch.Tensor          # [L][Hq*d][H]
-    Wk: torch.Tensor          # [L][Hkv*d][H]
-    Wv: torch.Tensor          # [L][Hkv*d][H]
+    Wqkv: torch.Tensor        # [L][(Hq + 2 Hkv) * d][H]: Wq rows, then Wk, then Wv
     Wo: torch.Tensor          # [L][H][Hq*d]
     mlp_norm: torch.Tensor    # [L][H]
     Wgu: torch.Tensor         # [L][2F][H]  gate rows, then up rows
@@ -404,8 +402,7 @@ def make_forward_weights(cfg, seed, device="cpu", layers=None, F=None):
 
     return ForwardWeights(
         F=F, h0=randn(gen, (B * N, H), 1.0, dt, device),
-        attn_norm=norm_w(L, H), Wq=randn(gen, (L, Hq * d, H), std, dt, device),
-        Wk=randn(gen, (L, Hkv * d, H), std, dt, device), Wv=randn(gen, (L, Hkv * d, H), std, dt, device),
+        attn_norm=norm_w(L, H), Wqkv=randn(gen, (L, (Hq + 2 * Hkv) * d, H), std, dt, device),
         Wo=randn(gen, (L, H, Hq * d), std, dt, device), mlp_norm=norm_w(L, H),
         Wgu=randn(gen, (L, 2 * F, H), std, dt, device), Wd=randn(gen, (L, H, F), std, dt, device),
         final_norm=norm_w(H))

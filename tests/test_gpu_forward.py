@@ -24,7 +24,9 @@ def _oracle_forward(cfg, inp, fw, L):
     depth, pos, anc, st = oracle.tree_build(inp.parents.cpu().numpy(), P)
     h = f64(fw.h0)
     for l in range(L):
-        w = {"attn_norm": f64(fw.attn_norm[l]), "Wq": f64(fw.Wq[l]), "Wk": f64(fw.Wk[l]), "Wv": f64(fw.Wv[l]),
+        Wqkv = f64(fw.Wqkv[l])
+        nq, nkv = Hq * d, Hkv * d
+        w = {"attn_norm": f64(fw.attn_norm[l]), "Wq": Wqkv[:nq], "Wk": Wqkv[nq:nq + nkv], "Wv": Wqkv[nq + nkv:],
              "Wo": f64(fw.Wo[l]), "mlp_norm": f64(fw.mlp_norm[l]), "Wg": f64(fw.Wgu[l][:fw.F]),
              "Wu": f64(fw.Wgu[l][fw.F:]), "Wd": f64(fw.Wd[l])}
         h, _, _ = oracle.decoder_layer(h, w, f64(inp.cacheK[l]), f64(inp.cacheV[l]), P, pos, anc, cfg["rope_base"],

@@ -102,3 +102,21 @@ def test_linear_workspace_reuse_dirty():
         assert rel_err(f64(out), oracle.linear(f64(x), f64(W))) <= TOL
         outs.append(out.clone())
     assert torch.equal(outs[0], outs[2])
+
+
+@pytest.mark.parametrize("rows,K,nq,nkv", [(60, 4096, 4096, 1024), (240, 5120, 5120, 5120), (5, 256, 64, 32)])
+def test_linear_qkv_parity(rows, K, nq, nkv):
+    dev = device()
+    gen = torch.Generator().manual_seed(rows + nq + nkv)
+    x = _bf((rows, K), gen).to(dev)
+    W = _bf((nq + 2 * nkv, K), gen, 0.02).to(dev)
+    q = torch.empty(rows, nq, dtype=torch.bfloat16, device=dev)
+    k = torch.empty(rows, nkv, dtype=torch.bfloat16, device=dev)
+    v = torch.empty(rows, nkv, dtype=torch.bfloat16, device=dev)
+    ws = torch.empty(gv.gv_linear_qkv_workspace(rows, K, nq, nkv), dtype=torch.uint8, device=dev)
+    gv.gv_linear_qkv(x, W, q, k, v, ws)
+    torch.cuda.synchronize()
+    ref = oracle.linear(f64(x), f64(W))
+    assert rel_err(f64(q), ref[:, :nq]) <= TOL
+    assert rel_err(f64(k), ref[:, nq:nq + nkv]) <= TOL
+    assert rel_err(f64(v), ref[:, nq + nkv:]) <= TOL
