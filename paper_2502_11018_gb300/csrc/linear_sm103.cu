@@ -4,14 +4,15 @@
 //
 // The projections of a verify step are skinny: the R = B * N <= 256 tree
 // nodes times a weight W[N][K] that is read once from HBM (4096 x 4096 up to
-// 28672 x 4096 per matrix), so the kernel is a weight stream with the node
-// rows resident, like the LM head: TMA brings k-blocks of 64 of the node rows
-// (one or two M tiles of 128) and of BN weight rows into a ring of shared
-// memory stages, one lane issues tcgen05.mma into a double-buffered TMEM
-// accumulator, and four epilogue warps write the tile's fp32 sums.  A work
-// unit is (weight tile of BN rows, K split); the split count and BN are chosen
-// so that the units fill the SMs in as few waves as possible, and the fp32
-// partial sums of every split go to the workspace.  gemm_reduce_kernel then
+// 28672 x 4096 per matrix), so the kernel is a weight stream.  The weight
+// rows go on the MMA's M side (tiles of 128 or 256 rows) and the node rows on
+// its N side, so a k-block moves 16-32 KB of weights and only 8 KB of node
+// rows (64 rows).  TMA fills a ring of shared-memory stages, one lane issues
+// tcgen05.mma into a double-buffered TMEM accumulator, and four epilogue warps
+// write the tile's fp32 sums (TMEM lane = output column, column = node row).
+// A work unit is (weight tile, K split); the split count and tile height are
+// chosen so that the units fill the SMs in as few waves as possible, and the
+// fp32 partial sums of every split go to the workspace.  gemm_reduce_kernel then
 // adds the splits and applies the epilogue (store, residual add, or SwiGLU
 // over the gate and up halves), writing bf16.
 #include "gv_internal.cuh"
@@ -24,12 +25,17 @@ int make_map_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols
                 uint64_t row_stride_bytes);
 
 constexpr int GM_THREADS = 192;
-constexpr int GM_A_TILE = 128 * 128;    // 128 rows x 64 bf16
+constexpr int GM_W_TILE = 128 * 128;    // 128 weight rows x 64 bf16
 
+// The weight rows are the MMA's M side (tiles of BM = 128 * mm rows, mm MMAs
+// per k-step sharing one node-row operand) and the node rows its N side
+// (npad = rows rounded up to 32): the big dimension streams, the node rows
+// ride along (8 KB per k-block for 64 rows).
 struct GemmArgs {
-    int rows, mt;            // node rows (<= 256) and M tiles
-    int N, K;                // weight rows (GEMM output columns) and inner size
-    int BN, n_tiles, KS, kblocks, units;
+    int rows, npad;          // node rows, MMA N
+    int N, K;                // weight rows (GEMM output columns), inner size
+    int mm;                  // 128-row MMAs per weight tile
+    int n_tiles, KS, kblocks, units;
     int stages, stage_bytes;
     uint32_t tmem_cols;
     float* part;             // [KS][rows][N] fp32
@@ -71,7 +77,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
-    const int acc_cols = a.mt * a.BN;
+    const int BM = 128 * a.mm;
+    const int acc_cols = a.mm * a.npad;
+    const int x_off = a.mm * GM_W_TILE;       // node rows after the weight rows in a stage
     // k-block range of split ks (the splits differ by at most one block)
     auto kb_lo = [&](int ks) { return (int)(((long)a.kblocks * ks) / a.KS); };
 
@@ -80,7 +88,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         if (lane == 0) {
             const uint64_t pol_w = policy_evict_first();
             const uint64_t pol_x = policy_evict_last();
-            const uint32_t tx = (uint32_t)(a.mt * GM_A_TILE + a.BN * 128);
+            const uint32_t tx = (uint32_t)(BM * 128 + a.npad * 128);
             int s = 0;
             uint32_t ph = 0;
             int issued[8];
@@ -96,8 +104,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                 pre = min(a.stages, hi - lo);
                 for (int q = 0; q < pre; ++q) {
                     mbar_arrive_expect_tx(&full[q], tx);
-                    tma_load_2d(stage_base + (size_t)q * a.stage_bytes + a.mt * GM_A_TILE, &tmap_w, &full[q],
-                                (lo + q) * 64, nt * a.BN, pol_w);
+                    tma_load_2d(stage_base + (size_t)q * a.stage_bytes, &tmap_w, &full[q], (lo + q) * 64, nt * BM,
+                                pol_w);
                     issued[q] = 0;
                 }
             }
@@ -106,9 +114,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             if (u0 < a.units) {
                 const int lo = kb_lo(u0 % a.KS);
                 for (int q = 0; q < pre; ++q)
-                    for (int m = 0; m < a.mt; ++m)
-                        tma_load_2d(stage_base + (size_t)q * a.stage_bytes + m * GM_A_TILE, &tmap_x, &full[q],
-                                    (lo + q) * 64, m * 128, pol_x);
+                    tma_load_2d(stage_base + (size_t)q * a.stage_bytes + x_off, &tmap_x, &full[q], (lo + q) * 64, 0,
+                                pol_x);
             }
             s = pre % a.stages;
             ph = pre == a.stages ? 1u : 0u;
@@ -119,9 +126,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                     if (!mbar_wait(&empty[s], ph ^ 1u, abort)) goto producer_done;
                     mbar_arrive_expect_tx(&full[s], tx);
                     uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
-                    for (int m = 0; m < a.mt; ++m)
-                        tma_load_2d(st + m * GM_A_TILE, &tmap_x, &full[s], kb * 64, m * 128, pol_x);
-                    tma_load_2d(st + a.mt * GM_A_TILE, &tmap_w, &full[s], kb * 64, nt * a.BN, pol_w);
+                    tma_load_2d(st, &tmap_w, &full[s], kb * 64, nt * BM, pol_w);
+                    tma_load_2d(st + x_off, &tmap_x, &full[s], kb * 64, 0, pol_x);
                     issued[s] = (int)ph;
                     if (++s == a.stages) {
                         s = 0;
@@ -138,7 +144,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     } else if (warp == 1) {
         // -------------------------------------------------------- MMA issuer
         if (lane == 0) {
-            const uint32_t idesc = idesc_bf16(128, a.BN);
+            const uint32_t idesc = idesc_bf16(128, a.npad);
             int s = 0;
             uint32_t ph = 0;
             int i = 0;
@@ -157,12 +163,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                     }
                     tc_fence_after();
                     uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
-                    const uint64_t bdesc = sdesc_kmajor_sw128(smem_u32(st + a.mt * GM_A_TILE));
-                    for (int m = 0; m < a.mt; ++m) {
-                        const uint64_t adesc = sdesc_kmajor_sw128(smem_u32(st + m * GM_A_TILE));
+                    const uint64_t bdesc = sdesc_kmajor_sw128(smem_u32(st + x_off));
+                    for (int m = 0; m < a.mm; ++m) {
+                        const uint64_t adesc = sdesc_kmajor_sw128(smem_u32(st + m * GM_W_TILE));
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
-                            mma_bf16(d_base + (uint32_t)(m * a.BN), adesc + 2u * kk, bdesc + 2u * kk, idesc,
+                            mma_bf16(d_base + (uint32_t)(m * a.npad), adesc + 2u * kk, bdesc + 2u * kk, idesc,
                                      (kb != lo || kk != 0) ? 1u : 0u);
                     }
                     mma_commit(&empty[s]);
@@ -179,8 +185,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         }
     } else {
         // ----------------------------------------------------------- epilogue
+        // TMEM lane = weight row (output column n), TMEM column = node row r.
         const int sub = warp & 3;                 // TMEM lane quarter this warp may access
-        const int row_in_tile = sub * 32 + lane;
         pdl_wait();   // (before this role's global writes)
         // Once a wait gives up, this CTA's remaining tiles get NaN partials,
         // so that the reduction turns the affected outputs into NaN.
@@ -196,31 +202,23 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             }
             __syncwarp();
             tc_fence_after();
-            const int n0 = nt * a.BN;
-            for (int m = 0; m < a.mt; ++m) {
-                const int r = m * 128 + row_in_tile;
-                float* dst = a.part + ((size_t)ks * a.rows + r) * a.N;
-                for (int c0 = 0; c0 < a.BN; c0 += 32) {
+            for (int m = 0; m < a.mm; ++m) {
+                const int n = nt * BM + m * 128 + sub * 32 + lane;
+                float* dst = a.part + (size_t)ks * a.rows * a.N + n;
+                for (int c0 = 0; c0 < a.npad; c0 += 32) {
                     uint32_t v[32];
                     if (!failed) {
-                        tmem_ld32(tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * acc_cols + m * a.BN + c0),
+                        tmem_ld32(tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(acc * acc_cols + m * a.npad + c0),
                                   v);
                         tmem_wait_ld();
                     } else {
 #pragma unroll
                         for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(NAN);
                     }
-                    if (r < a.rows) {
-                        const int n = n0 + c0;
-                        if (n + 32 <= a.N && (a.N & 3) == 0) {
+                    if (n < a.N) {
 #pragma unroll
-                            for (int j = 0; j < 32; j += 4)
-                                *reinterpret_cast<float4*>(dst + n + j) =
-                                    make_float4(__uint_as_float(v[j]), __uint_as_float(v[j + 1]),
-                                                __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
-                        } else {
-                            for (int j = 0; j < 32 && n + j < a.N; ++j) dst[n + j] = __uint_as_float(v[j]);
-                        }
+                        for (int j = 0; j < 32; ++j)
+                            if (c0 + j < a.rows) dst[(size_t)(c0 + j) * a.N] = __uint_as_float(v[j]);
                     }
                 }
             }
@@ -236,9 +234,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     if (warp == 1) tmem_dealloc(tmem, a.tmem_cols);
 }
 
-// Adds the K splits of 8 consecutive output columns of one row and applies
-// the epilogue; one thread per (row, 8 columns), bf16 16-byte stores (NaN
-// partials of a GEMM that gave up propagate to the outputs).
 // Column split of the stored output: columns [0, n0) go to out0[rows][n0],
 // [n0, n0 + n1) to out1[rows][n1], the rest to out2 (the fused Q/K/V
 // projection); n1 == 0 stores everything to out0.
@@ -350,29 +345,30 @@ rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
 }
 
 // ----------------------------------------------------------------- host side
-// (BN, KS) minimising ceil(units / SMs) * per-unit cost, with a unit's cost
-// counted in weight rows streamed per k-block plus a fixed and an epilogue
-// share; larger BN on ties.
+// (mm, KS) minimising ceil(units / SMs) * per-unit cost, a unit's cost counted
+// in rows streamed per k-block (BM weight rows + npad node rows) plus an
+// epilogue share; larger tiles on ties.
 struct GemmPlan {
-    int BN, KS, n_tiles, kblocks, units, grid;
+    int mm, KS, n_tiles, kblocks, units, grid, npad;
 };
 
 static GemmPlan gemm_plan(int rows, int N, int K) {
-    const int mt = (rows + 127) / 128;
+    const int npad = (rows + 31) / 32 * 32;
     const int sms = sm_count();
     GemmPlan best{};
     long best_cost = -1;
     const int kblocks = (K + 63) / 64;
-    for (int bn = 64; bn <= 256 && 2 * mt * bn <= 512; bn += 32) {
-        const int tiles = (N + bn - 1) / bn;
+    for (int mm = 1; mm <= 2 && 2 * mm * npad <= 512; ++mm) {
+        const int bm = 128 * mm;
+        const int tiles = (N + bm - 1) / bm;
         for (int ks = 1; ks <= kblocks && ks <= 32; ++ks) {
             const long units = (long)tiles * ks;
             const long waves = (units + sms - 1) / sms;
             const long kb_per = (kblocks + ks - 1) / ks;
-            const long cost = waves * (kb_per * (bn + 8) + 3L * bn * mt);
-            if (best_cost < 0 || cost < best_cost || (cost == best_cost && bn > best.BN)) {
+            const long cost = waves * (kb_per * (bm + npad) + 2L * bm);
+            if (best_cost < 0 || cost < best_cost || (cost == best_cost && mm > best.mm)) {
                 best_cost = cost;
-                best = GemmPlan{bn, ks, tiles, kblocks, (int)units, 0};
+                best = GemmPlan{mm, ks, tiles, kblocks, (int)units, 0, npad};
             }
         }
     }
@@ -386,31 +382,30 @@ size_t linear_workspace_bytes(int rows, int K, int N) {
 }
 
 int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int epi, const void* residual,
-                  void* out, void* workspace, cudaStream_t st, void* out1 = nullptr, void* out2 = nullptr,
-                  int n0 = 0, int n1 = 0) {
+                  void* out, void* workspace, cudaStream_t st, void* out1, void* out2, int n0, int n1) {
     const int N = epi == GV_LINEAR_SWIGLU ? 2 * n_out : n_out;
     const GemmPlan p = gemm_plan(rows, N, K);
     GemmArgs a{};
     a.rows = rows;
-    a.mt = (rows + 127) / 128;
+    a.npad = p.npad;
     a.N = N;
     a.K = K;
-    a.BN = p.BN;
+    a.mm = p.mm;
     a.n_tiles = p.n_tiles;
     a.KS = p.KS;
     a.kblocks = p.kblocks;
     a.units = p.units;
-    a.stage_bytes = a.mt * GM_A_TILE + a.BN * 128;
+    a.stage_bytes = a.mm * GM_W_TILE + a.npad * 128;
     constexpr int SMEM_BUDGET = 220 * 1024;
     a.stages = (SMEM_BUDGET - 2048) / a.stage_bytes;
     if (a.stages > 8) a.stages = 8;
-    const int cols = 2 * a.mt * a.BN;
+    const int cols = 2 * a.mm * a.npad;
     a.tmem_cols = cols <= 32 ? 32 : cols <= 64 ? 64 : cols <= 128 ? 128 : cols <= 256 ? 256 : 512;
     a.part = static_cast<float*>(workspace);
     CUtensorMap mx, mw;
-    int rc = make_map_2d(&mx, x, (uint64_t)rows, (uint64_t)K, 128, (uint64_t)K * 2);
+    int rc = make_map_2d(&mx, x, (uint64_t)rows, (uint64_t)K, (uint32_t)a.npad, (uint64_t)K * 2);
     if (rc != GV_OK) return rc;
-    rc = make_map_2d(&mw, W, (uint64_t)N, (uint64_t)K, (uint32_t)a.BN, (uint64_t)K * 2);
+    rc = make_map_2d(&mw, W, (uint64_t)N, (uint64_t)K, (uint32_t)(128 * a.mm), (uint64_t)K * 2);
     if (rc != GV_OK) return rc;
     const size_t smem = (size_t)a.stages * a.stage_bytes + 8 * (2 * a.stages + 5) + 16;
     cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
