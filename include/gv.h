@@ -21,6 +21,7 @@
  *   gv_rmsnorm           RMSNorm of the node rows
  *   gv_linear            skinny projection x W^T with a fused epilogue
  *   gv_linear_qkv        the Q, K and V projections as one weight stream
+ *   gv_linear_add_rmsnorm  a residual projection fused with the next RMSNorm
  *
  * and, for training the draft model (Section 4.1):
  *
@@ -348,6 +349,17 @@ int gv_linear(const void* x, const void* W, int rows, int K, int n_out, int epil
 size_t gv_linear_qkv_workspace(int rows, int K, int n_q, int n_kv);
 int gv_linear_qkv(const void* x, const void* Wqkv, int rows, int K, int n_q, int n_kv, void* q, void* k, void* v,
                   void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * gv_linear_add_rmsnorm -- the residual projection fused with the RMSNorm
+ * that follows it in the layer: out = residual + x W^T (out may be residual)
+ * and norm_out = RMSNorm(out) * norm_w, computed from the stored bf16 out
+ * (eps as gv_rmsnorm's).  n_out <= 8192; other conditions and the workspace
+ * as gv_linear's with GV_LINEAR_ADD; norm_out is a separate buffer.
+ */
+int gv_linear_add_rmsnorm(const void* x, const void* W, int rows, int K, int n_out, const void* residual,
+                          void* out, const void* norm_w, float eps, void* norm_out, void* workspace, size_t ws_bytes,
+                          void* stream);
 
 /* Static name of a status code. */
 const char* gv_status_string(int status);

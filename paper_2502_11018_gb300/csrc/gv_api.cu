@@ -66,7 +66,8 @@ int launch_tree_build(const int32_t*, const int32_t*, int, int, int32_t*, int32_
 size_t linear_workspace_bytes(int rows, int K, int N);
 int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int epi, const void* residual,
                   void* out, void* workspace, cudaStream_t st, void* out1 = nullptr, void* out2 = nullptr,
-                  int n0 = 0, int n1 = 0);
+                  int n0 = 0, int n1 = 0, const void* norm_w = nullptr, float eps = 0.f,
+                  void* norm_out = nullptr);
 int launch_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, cudaStream_t st);
 int launch_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* fd,
                     const void* ft, int feat_dt, int B, int T, int V, int H, int k, int n,
@@ -511,6 +512,25 @@ int gv_linear_qkv(const void* x, const void* Wqkv, int rows, int K, int n_q, int
     GV_CHECK_ARG(ws_bytes >= gv_linear_qkv_workspace(rows, K, n_q, n_kv), "gv_linear_qkv: workspace too small");
     return launch_linear(x, Wqkv, rows, K, n_q + 2 * n_kv, GV_LINEAR_STORE, nullptr, q, workspace,
                          as_stream(stream), k, v, n_q, n_kv);
+}
+
+int gv_linear_add_rmsnorm(const void* x, const void* W, int rows, int K, int n_out, const void* residual,
+                          void* out, const void* norm_w, float eps, void* norm_out, void* workspace, size_t ws_bytes,
+                          void* stream) {
+    clear_error();
+    GV_CHECK_ARG(rows >= 1 && rows <= 256, "gv_linear_add_rmsnorm: rows=%d outside 1..256", rows);
+    GV_CHECK_ARG(K >= 8 && K % 8 == 0 && n_out >= 8 && n_out % 8 == 0 && n_out <= 8192,
+                 "gv_linear_add_rmsnorm: K=%d, n_out=%d (multiples of 8, n_out <= 8192)", K, n_out);
+    GV_CHECK_ARG(std::isfinite(eps) && eps >= 0.0f, "gv_linear_add_rmsnorm: eps %g", (double)eps);
+    GV_CHECK_ARG(x && W && residual && out && norm_w && norm_out && workspace, "gv_linear_add_rmsnorm: null pointer");
+    GV_CHECK_ARG(aligned16(x) && aligned16(W) && aligned16(residual) && aligned16(out) && aligned16(norm_w) &&
+                     aligned16(norm_out) && aligned16(workspace),
+                 "gv_linear_add_rmsnorm: pointers not 16-byte aligned");
+    GV_CHECK_ARG(norm_out != out && norm_out != residual, "gv_linear_add_rmsnorm: norm_out must be its own buffer");
+    GV_CHECK_ARG(ws_bytes >= gv_linear_workspace(rows, K, n_out, GV_LINEAR_ADD),
+                 "gv_linear_add_rmsnorm: workspace too small");
+    return launch_linear(x, W, rows, K, n_out, GV_LINEAR_ADD, residual, out, workspace, as_stream(stream), nullptr,
+                         nullptr, 0, 0, norm_w, eps, norm_out);
 }
 
 int gv_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, void* stream) {

@@ -301,6 +301,74 @@ gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int 
     *reinterpret_cast<uint4*>(dst) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
 }
 
+// The residual-add epilogue fused with the RMSNorm that follows it in the
+// layer: one CTA per row adds the K splits and the residual, writes the bf16
+// row h, and from the stored (rounded) values writes
+// norm_out = h / sqrt(mean(h^2) + eps) * w.  n_out % 8 == 0, n_out <= 8192.
+__global__ void __launch_bounds__(256)
+gemm_reduce_norm_kernel(const float* __restrict__ part, int KS, int rows, int n_out,
+                        const __nv_bfloat16* residual, __nv_bfloat16* out, const __nv_bfloat16* __restrict__ w,
+                        float eps, __nv_bfloat16* __restrict__ norm_out) {
+    __shared__ float red[8];
+    pdl_wait();
+    pdl_trigger();
+    const int r = blockIdx.x, tid = threadIdx.x;
+    constexpr int MAXC = 4;                       // 16-byte chunks per thread (n_out <= 8192)
+    float hv[MAXC][8];
+    float ss = 0.f;
+#pragma unroll
+    for (int q = 0; q < MAXC; ++q) {
+        const int c = (tid + q * 256) * 8;
+        if (c >= n_out) break;
+        float acc[8];
+        const uint4 rv = *reinterpret_cast<const uint4*>(residual + (size_t)r * n_out + c);
+        const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            acc[2 * e] = __uint_as_float(rw[e] << 16);
+            acc[2 * e + 1] = __uint_as_float(rw[e] & 0xffff0000u);
+        }
+        for (int ks = 0; ks < KS; ++ks) {
+            const float* p = part + ((size_t)ks * rows + r) * n_out + c;
+            const float4 a0 = *reinterpret_cast<const float4*>(p);
+            const float4 a1 = *reinterpret_cast<const float4*>(p + 4);
+            acc[0] += a0.x; acc[1] += a0.y; acc[2] += a0.z; acc[3] += a0.w;
+            acc[4] += a1.x; acc[5] += a1.y; acc[6] += a1.z; acc[7] += a1.w;
+        }
+        uint32_t pk[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(acc[2 * e], acc[2 * e + 1]);
+            pk[e] = *reinterpret_cast<uint32_t*>(&h2);
+            hv[q][2 * e] = __uint_as_float(pk[e] << 16);
+            hv[q][2 * e + 1] = __uint_as_float(pk[e] & 0xffff0000u);
+            ss += hv[q][2 * e] * hv[q][2 * e] + hv[q][2 * e + 1] * hv[q][2 * e + 1];
+        }
+        *reinterpret_cast<uint4*>(out + (size_t)r * n_out + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    }
+    ss = warp_sum(ss);
+    if ((tid & 31) == 0) red[tid >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+    for (int k = 0; k < 8; ++k) tot += red[k];
+    const float inv = rsqrtf(tot / (float)n_out + eps);
+#pragma unroll
+    for (int q = 0; q < MAXC; ++q) {
+        const int c = (tid + q * 256) * 8;
+        if (c >= n_out) break;
+        const uint4 g = *reinterpret_cast<const uint4*>(w + c);
+        const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
+        uint32_t pk[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(hv[q][2 * e] * inv * __uint_as_float(gw[e] << 16),
+                                                      hv[q][2 * e + 1] * inv * __uint_as_float(gw[e] & 0xffff0000u));
+            pk[e] = *reinterpret_cast<uint32_t*>(&h2);
+        }
+        *reinterpret_cast<uint4*>(norm_out + (size_t)r * n_out + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    }
+}
+
 // RMSNorm of one row per CTA: out = x / sqrt(mean(x^2) + eps) * w, fp32 math,
 // bf16 in and out (16-byte vectors; H % 8 == 0).
 __global__ void __launch_bounds__(256)
@@ -382,7 +450,8 @@ size_t linear_workspace_bytes(int rows, int K, int N) {
 }
 
 int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int epi, const void* residual,
-                  void* out, void* workspace, cudaStream_t st, void* out1, void* out2, int n0, int n1) {
+                  void* out, void* workspace, cudaStream_t st, void* out1, void* out2, int n0, int n1,
+                  const void* norm_w, float eps, void* norm_out) {
     const int N = epi == GV_LINEAR_SWIGLU ? 2 * n_out : n_out;
     const GemmPlan p = gemm_plan(rows, N, K);
     GemmArgs a{};
@@ -412,6 +481,12 @@ int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int 
     launch_pdl(gemm_tc_kernel, dim3(p.grid), dim3(GM_THREADS), smem, st, mx, mw, a);
     rc = check_launch("gemm_tc_kernel");
     if (rc != GV_OK) return rc;
+    if (norm_out) {
+        launch_pdl(gemm_reduce_norm_kernel, dim3(rows), dim3(256), 0, st, (const float*)a.part, a.KS, rows, n_out,
+                   static_cast<const __nv_bfloat16*>(residual), static_cast<__nv_bfloat16*>(out),
+                   static_cast<const __nv_bfloat16*>(norm_w), eps, static_cast<__nv_bfloat16*>(norm_out));
+        return check_launch("gemm_reduce_norm_kernel");
+    }
     const int items = rows * (n_out / 8);
     OutSplit os{static_cast<__nv_bfloat16*>(out), static_cast<__nv_bfloat16*>(out1),
                 static_cast<__nv_bfloat16*>(out2), n0, n1};

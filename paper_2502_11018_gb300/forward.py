@@ -5,15 +5,16 @@ target forward verifies every draft token).
 
 Per layer, over the hidden states h [B*N][H] of the tree nodes:
 
-    x = RMSNorm(h) * w_attn                      gv_rmsnorm
+    x = RMSNorm(h) * w_attn                      (fused into the previous call)
     q, k, v = x Wq^T, x Wk^T, x Wv^T             gv_linear_qkv (one weight stream)
     o = TreeAttention(q, k, v)                   gv_verify_attention
-    h = h + o Wo^T                               gv_linear (residual add, in place)
-    x = RMSNorm(h) * w_mlp                       gv_rmsnorm
+    h = h + o Wo^T; x = RMSNorm(h) * w_mlp       gv_linear_add_rmsnorm
     g = silu(x Wg^T) * (x Wu^T)                  gv_linear (SwiGLU)
-    h = h + g Wd^T                               gv_linear (residual add, in place)
+    h = h + g Wd^T; x = RMSNorm(h) * w_next      gv_linear_add_rmsnorm
 
-then RMSNorm(h) * w_final feeds gv_lmhead_select.  Nothing here computes: it
+where w_next is the next layer's w_attn, or after the last layer w_final,
+whose output feeds gv_lmhead_select; the first layer's input norm is
+gv_rmsnorm of the embeddings.  Nothing here computes: it
 owns buffers and issues the calls on one stream (graph-capturable).
 """
 
@@ -55,27 +56,29 @@ class VerifyForward:
         gv.gv_linear(x, W, out, epi, residual=residual, workspace=self.lin_ws, stream=stream)
 
     def layer(self, l, stream=None):
+        """Layer l; self.x holds RMSNorm(h) * w_attn[l] on entry."""
         fw, st = self.fw, self.step
         R = self.h.shape[0]
+        L = self.cfg["L"]
         h_in = fw.h0 if l == 0 else self.h      # layer 0 reads the embeddings
-        gv.gv_rmsnorm(h_in, fw.attn_norm[l], self.x, stream=stream)
         gv.gv_linear_qkv(self.x, fw.Wqkv[l], self.q.view(R, -1), self.k.view(R, -1), self.v.view(R, -1),
                          self.lin_ws, stream=stream)
         i = self.inp
         gv.gv_verify_attention(st.shape, self.q, self.k, self.v, i.cacheK[l], i.cacheV[l], i.prefix_len, st.rope,
                                st.anc, st.treeK[l], st.treeV[l], st.attn_out[l], st.attn_ws, stream)
-        self._lin(st.attn_out[l].view(R, -1), fw.Wo[l], self.h, gv.GV_LINEAR_ADD, residual=h_in, stream=stream)
-        gv.gv_rmsnorm(self.h, fw.mlp_norm[l], self.x, stream=stream)
+        gv.gv_linear_add_rmsnorm(st.attn_out[l].view(R, -1), fw.Wo[l], h_in, self.h, fw.mlp_norm[l], self.x,
+                                 self.lin_ws, stream=stream)
         self._lin(self.x, fw.Wgu[l], self.g, gv.GV_LINEAR_SWIGLU, stream=stream)
-        self._lin(self.g, fw.Wd[l], self.h, gv.GV_LINEAR_ADD, residual=self.h, stream=stream)
+        nxt_w, nxt_out = (fw.attn_norm[l + 1], self.x) if l + 1 < L else (fw.final_norm, self.inp.h)
+        gv.gv_linear_add_rmsnorm(self.g, fw.Wd[l], self.h, self.h, nxt_w, nxt_out, self.lin_ws, stream=stream)
 
     def run(self, stream=None):
         """Tree build, every layer, final norm, LM head, acceptance, compaction."""
         st = self.step
         st.tree(stream)
+        gv.gv_rmsnorm(self.fw.h0, self.fw.attn_norm[0], self.x, stream=stream)
         for l in range(self.cfg["L"]):
             self.layer(l, stream)
-        gv.gv_rmsnorm(self.h, self.fw.final_norm, self.inp.h, stream=stream)
         st.lmhead(stream)
         st.accept(stream)
         st.compact(stream)

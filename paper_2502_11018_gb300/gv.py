@@ -36,7 +36,7 @@ EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "g
            "gv_lmhead_workspace", "gv_lmhead_select", "gv_lmhead_argmax_noalloc",
            "gv_accept_workspace", "gv_accept",
            "gv_kv_compact", "gv_rmsnorm", "gv_linear_workspace", "gv_linear", "gv_linear_qkv_workspace",
-           "gv_linear_qkv", "gv_tat_loss",
+           "gv_linear_qkv", "gv_linear_add_rmsnorm", "gv_tat_loss",
            "gv_status_string", "gv_last_error", "gv_version")
 
 
@@ -85,6 +85,7 @@ def lib():
         "gv_linear": ([_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _sz, _vp], _i),
         "gv_linear_qkv_workspace": ([_i, _i, _i, _i], _sz),
         "gv_linear_qkv": ([_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp], _i),
+        "gv_linear_add_rmsnorm": ([_vp, _vp, _i, _i, _i, _vp, _vp, _vp, _f, _vp, _vp, _sz, _vp], _i),
         "gv_tat_loss": ([_vp, _i, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, _i, _vp, _f, _f,
                          _vp, _vp, _vp, _vp, _vp], _i),
         "gv_status_string": ([_i], ctypes.c_char_p),
@@ -278,3 +279,14 @@ def gv_linear_qkv(x, Wqkv, q, k, v, workspace, stream=None):
     return _check("gv_linear_qkv", lib().gv_linear_qkv(
         _ptr(x, "x"), _ptr(Wqkv, "Wqkv"), rows, K, n_q, n_kv, _ptr(q, "q"), _ptr(k, "k"), _ptr(v, "v"),
         _ptr(workspace, "workspace"), ws_bytes, _stream(stream)))
+
+
+def gv_linear_add_rmsnorm(x, W, residual, out, norm_w, norm_out, workspace, eps=1e-5, stream=None):
+    """out = residual + x W^T, norm_out = RMSNorm(out) * norm_w (see include/gv.h)."""
+    rows, K = x.shape
+    n_out = out.shape[1]
+    ws_bytes = workspace.numel() * workspace.element_size()
+    return _check("gv_linear_add_rmsnorm", lib().gv_linear_add_rmsnorm(
+        _ptr(x, "x"), _ptr(W, "W"), rows, K, n_out, _ptr(residual, "residual"), _ptr(out, "out"),
+        _ptr(norm_w, "norm_w"), float(eps), _ptr(norm_out, "norm_out"), _ptr(workspace, "workspace"), ws_bytes,
+        _stream(stream)))

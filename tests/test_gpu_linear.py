@@ -120,3 +120,22 @@ def test_linear_qkv_parity(rows, K, nq, nkv):
     assert rel_err(f64(q), ref[:, :nq]) <= TOL
     assert rel_err(f64(k), ref[:, nq:nq + nkv]) <= TOL
     assert rel_err(f64(v), ref[:, nq + nkv:]) <= TOL
+
+
+@pytest.mark.parametrize("rows,K,N", [(60, 4096, 4096), (240, 13824, 5120), (3, 64, 40)])
+def test_linear_add_rmsnorm_parity(rows, K, N):
+    dev = device()
+    gen = torch.Generator().manual_seed(rows + K)
+    x = _bf((rows, K), gen).to(dev)
+    W = _bf((N, K), gen, 0.02).to(dev)
+    h = _bf((rows, N), gen, 2.0).to(dev)
+    g = _bf((N,), gen).to(dev)
+    h0 = f64(h)
+    xn = torch.empty(rows, N, dtype=torch.bfloat16, device=dev)
+    ws = torch.empty(gv.gv_linear_workspace(rows, K, N, gv.GV_LINEAR_ADD), dtype=torch.uint8, device=dev)
+    gv.gv_linear_add_rmsnorm(x, W, h, h, g, xn, ws)      # in place on h
+    torch.cuda.synchronize()
+    ref_h = h0 + oracle.linear(f64(x), f64(W))
+    assert rel_err(f64(h), ref_h) <= TOL
+    # the norm is taken of the stored (rounded) h
+    assert rel_err(f64(xn), oracle.rmsnorm(f64(h), f64(g), 1e-5)) <= TOL
