@@ -24,7 +24,8 @@ What it computes (GRIFFIN, arXiv 2502.11018):
   predictable masks, chain alignment masks, masked per-sequence loss) in
   ``tat``;
 * the target model's decoder layers around the tree attention (RMSNorm,
-  projections, SwiGLU MLP, residuals) in ``layer``.
+  projections, SwiGLU MLP, residuals) in ``layer``;
+* the draft model's Token-Guided Fusion module (Eqs. 6-8) in ``tgf``.
 
 Every function works in float64 with plain loops or single library
 primitives (a matmul, a sort), in the order the definition states.
@@ -43,3 +44,4 @@ from .compact import kv_compact  # noqa: F401
 from .step import verify_step  # noqa: F401
 from .tat import predictable_mask, alignment_mask, token_loss, feature_loss, tat_pass  # noqa: F401
 from .layer import rmsnorm, linear, silu, swiglu, decoder_layer  # noqa: F401
+from .tgf import layernorm, tgf_forward  # noqa: F401
