@@ -339,13 +339,14 @@ def main():
     ap.add_argument("--seed", type=int, default=1000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention", "tat", "forward"],
+    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention", "tat", "forward", "tgf"],
                     help="step: the benchmark; lmhead / attention: time that call alone "
                          "(a small, self-contained launch sequence for profiler captures); "
                          "tat: one token-alignable training pass (gv_tat_loss) on a "
                          "4 x 2048-token batch, vocabulary 32000; forward: the whole verify "
                          "forward of the target (decoder layers around the path, random "
-                         "weights of the --config model's shape)")
+                         "weights of the --config model's shape); tgf: the draft model's "
+                         "token-guided fusion (gv_tgf) over 60 rows, d 4096, expansion 11008")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
 
@@ -374,6 +375,9 @@ def main():
         return
     if args.kernel == "forward":
         run_forward(args, dev)
+        return
+    if args.kernel == "tgf":
+        run_tgf(args, dev)
         return
     cfg = inputs.config(args.config)
     if args.kernel != "step":
@@ -598,6 +602,59 @@ def run_tat(args, dev):
                                 "kind": "oracle",
                                 "sample": f"float64 numpy oracle on {B} x {ts} of the {B} x {T} positions, "
                                           f"scaled linearly ({sec:.2f} s per pass)"}
+    print(json.dumps(line), flush=True)
+
+
+def tgf_bytes(cfg):
+    """Algorithmic bytes of one token-guided fusion call: the three weight
+    matrices and the seven vectors read once, F and x read, h and o written."""
+    rows, d, e = cfg["rows"], cfg["d"], cfg["e"]
+    return 2 * (2 * d * d + 2 * d * e + d * e + 6 * d + e) + 2 * rows * d * 4
+
+
+def run_tgf(args, dev):
+    """gv_tgf on the LLaMA-2-7B drafter's shape (60 rows, d 4096, expansion
+    11008), timed from a CUDA graph of back-to-back calls: the 337 MB of
+    weights are far above L2, so every call streams them from HBM."""
+    name = "tgf_llama2_7b"
+    cfg = inputs.TGF_CONFIGS[name]
+    ti = inputs.make_tgf_inputs(cfg, args.seed, device=dev)
+    rows, d, e = cfg["rows"], cfg["d"], cfg["e"]
+    h = torch.empty(rows, d, dtype=torch.bfloat16, device=dev)
+    o = torch.empty(rows, d, dtype=torch.bfloat16, device=dev)
+    ws = torch.empty(gv.gv_tgf_workspace(rows, d, e), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def call():
+        gv.gv_tgf(ti.F, ti.x, ti.w, h, o, ws, stream=torch.cuda.current_stream())
+
+    for _ in range(args.warmup):
+        call()
+    torch.cuda.synchronize()
+    reps = max(3, min(args.steps, 200))
+    g = graph_of(lambda: [call() for _ in range(4)])
+    g.replay()
+    torch.cuda.synchronize()
+    ms = event_time_ms(g.replay, reps, stream) / 4
+    nbytes = tgf_bytes(cfg)
+    peaks = load_peaks()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    line = {"kernel": "tgf", "workload": name, "config": cfg, "ms_per_call_graph": ms, "launches_per_call": 6,
+            "algorithmic_bytes": nbytes, "achieved_gbs_graph": gbs,
+            "frac_of_measured_hbm_graph": gbs / peaks["hbm_gbs"], "rows_per_s": rows / (ms * 1e-3)}
+    if not args.no_cpu_baseline:
+        # the float64 oracle on the host cores, on 8 of the 60 rows (its cost
+        # is the three float64 matrix products, linear in the rows), scaled
+        import oracle
+        rs = 8
+        w = {k: v.detach().cpu().double().numpy() for k, v in ti.w.items()}
+        t0 = time.perf_counter()
+        oracle.tgf_forward(ti.F[:rs].cpu().double().numpy(), ti.x[:rs].cpu().double().numpy(), w)
+        sec = (time.perf_counter() - t0) * (rows / rs)
+        line["cpu_baseline"] = {"value": rows / sec, "unit": "rows/s", "cores": torch.get_num_threads(),
+                                "kind": "oracle",
+                                "sample": f"float64 numpy oracle on {rs} of the {rows} rows, scaled linearly "
+                                          f"({sec:.2f} s per call)"}
     print(json.dumps(line), flush=True)
 
 

@@ -23,10 +23,11 @@
  *   gv_linear_qkv        the Q, K and V projections as one weight stream
  *   gv_linear_add_rmsnorm  a residual projection fused with the next RMSNorm
  *
- * and, for training the draft model (Section 4.1):
+ * and, for the draft model (Section 4):
  *
  *   gv_tat_loss          top-k predictable masks, chain alignment masks and
  *                        the masked loss of one token-alignable training pass
+ *   gv_tgf               the Token-Guided Fusion module (Eqs. 6-8)
  *
  * Conventions shared by every call:
  *  - Every pointer argument is DEVICE memory owned by the caller, unless the
@@ -85,7 +86,8 @@ typedef enum {
 typedef enum {
     GV_LINEAR_STORE = 0,   /* out = x W^T                                   */
     GV_LINEAR_ADD = 1,     /* out = residual + x W^T (out may be residual)  */
-    GV_LINEAR_SWIGLU = 2   /* out = silu(x Wg^T) * (x Wu^T), W = [Wg ; Wu]  */
+    GV_LINEAR_SWIGLU = 2,  /* out = silu(x Wg^T) * (x Wu^T), W = [Wg ; Wu]  */
+    GV_LINEAR_SILU = 3     /* out = silu(x W^T)                             */
 } gv_linear_epilogue;
 
 /* Shape of one attention layer of the verify pass. */
@@ -312,6 +314,37 @@ int gv_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const 
                 uint8_t* mask, float* ell, float* seq_loss, void* stream);
 
 /*
+ * gv_tgf -- the draft model's Token-Guided Fusion (Section 4.2, Eqs. 6-8) of
+ * rows of features F with the embeddings x of their tokens:
+ *
+ *   h = [F ; x] Wm^T + bm                     embedding fusion (Eq. 6)
+ *   z = [LN_h(h) ; LN_x(x)] Wu^T + bu         normalisation and expansion (Eq. 7)
+ *   o = silu(z) Wd^T + bd + h                 refinement (Eq. 8)
+ *
+ * LN_v(v) = (v - mean(v)) / sqrt(var(v) + eps) * g_v + b_v per row
+ * (population variance); [a ; b] is the concatenation along the row.
+ *
+ *   F, x      bf16 [rows][d]    1 <= rows <= 256; d a multiple of 64, <= 8192
+ *   Wm        bf16 [d][2d]      (output rows; columns: F's d, then x's d)
+ *   bm, g_h, b_h, g_x, b_x      bf16 [d]
+ *   Wu        bf16 [e][2d]      e the expansion width (a multiple of 8;
+ *                               4d in Section 4.2, 11008 for LLaMA-2-7B)
+ *   bu        bf16 [e]
+ *   Wd        bf16 [d][e];  bd bf16 [d]
+ *   h_out     bf16 [rows][d]    out: h (rounded to bf16; the residual of Eq. 8
+ *                               and the layer norm take this rounded h)
+ *   o_out     bf16 [rows][d]    out: o
+ *   workspace >= gv_tgf_workspace(rows, d, e) bytes
+ * fp32 accumulation and normalisation; z and silu(z) are rounded to bf16
+ * between the projections.  16-byte aligned pointers; outputs must not
+ * overlap the inputs or each other.  Six kernel launches, graph-capturable.
+ */
+size_t gv_tgf_workspace(int rows, int d, int e);
+int gv_tgf(const void* F, const void* x, int rows, int d, int e, const void* Wm, const void* bm, const void* g_h,
+           const void* b_h, const void* g_x, const void* b_x, const void* Wu, const void* bu, const void* Wd,
+           const void* bd, float eps, void* h_out, void* o_out, void* workspace, size_t ws_bytes, void* stream);
+
+/*
  * gv_rmsnorm -- out[r] = x[r] / sqrt(mean(x[r]^2) + eps) * w (the target
  * layer's input and post-attention norms, and the final norm before the LM
  * head).  bf16 x, w, out [rows][H] / [H]; fp32 arithmetic; H % 8 == 0,
@@ -330,7 +363,7 @@ int gv_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* o
  *                                      GV_LINEAR_SWIGLU (gate rows, then up rows)
  *   residual  bf16 [rows][n_out]       GV_LINEAR_ADD only (else NULL); out may be
  *                                      the same buffer
- *   out       bf16 [rows][n_out]
+ *   out       bf16 [rows][n_out]; GV_LINEAR_SILU gives silu(x W^T)
  *   workspace >= gv_linear_workspace(rows, K, n_out, epilogue) bytes
  * K % 8 == 0, n_out % 8 == 0, 16-byte aligned pointers.  A bounded wait that
  * gives up turns the affected outputs into NaN.

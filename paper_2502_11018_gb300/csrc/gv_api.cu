@@ -63,12 +63,11 @@ static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 // Kernel launchers defined in the other translation units.
 int launch_tree_build(const int32_t*, const int32_t*, int, int, int32_t*, int32_t*, uint64_t*,
                       int32_t*, cudaStream_t);
-size_t linear_workspace_bytes(int rows, int K, int N);
-int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int epi, const void* residual,
-                  void* out, void* workspace, cudaStream_t st, void* out1 = nullptr, void* out2 = nullptr,
-                  int n0 = 0, int n1 = 0, const void* norm_w = nullptr, float eps = 0.f,
-                  void* norm_out = nullptr);
 int launch_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, cudaStream_t st);
+size_t tgf_workspace_bytes(int rows, int d, int e);
+int launch_tgf(const void* F, const void* x, int rows, int d, int e, const void* Wm, const void* bm,
+               const void* g_h, const void* b_h, const void* g_x, const void* b_x, const void* Wu, const void* bu,
+               const void* Wd, const void* bd, float eps, void* h_out, void* o_out, void* ws, cudaStream_t st);
 int launch_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* fd,
                     const void* ft, int feat_dt, int B, int T, int V, int H, int k, int n,
                     const uint8_t* mbar_prev, float lam_tok, float lam_feat, uint8_t* mbar,
@@ -472,7 +471,7 @@ int gv_kv_compact(int L, int B, int N, int D, int Hkv, int d, int S_max, int dt,
 
 size_t gv_linear_workspace(int rows, int K, int n_out, int epilogue) {
     if (rows < 1 || rows > 256 || K < 8 || n_out < 8) return 0;
-    if (epilogue < GV_LINEAR_STORE || epilogue > GV_LINEAR_SWIGLU) return 0;
+    if (epilogue < GV_LINEAR_STORE || epilogue > GV_LINEAR_SILU) return 0;
     const int N = epilogue == GV_LINEAR_SWIGLU ? 2 * n_out : n_out;
     return align256(linear_workspace_bytes(rows, K, N));
 }
@@ -483,7 +482,7 @@ int gv_linear(const void* x, const void* W, int rows, int K, int n_out, int epil
     GV_CHECK_ARG(rows >= 1 && rows <= 256, "gv_linear: rows=%d outside 1..256", rows);
     GV_CHECK_ARG(K >= 8 && K % 8 == 0 && n_out >= 8 && n_out % 8 == 0,
                  "gv_linear: K=%d and n_out=%d must be positive multiples of 8", K, n_out);
-    GV_CHECK_ARG(epilogue >= GV_LINEAR_STORE && epilogue <= GV_LINEAR_SWIGLU, "gv_linear: epilogue %d",
+    GV_CHECK_ARG(epilogue >= GV_LINEAR_STORE && epilogue <= GV_LINEAR_SILU, "gv_linear: epilogue %d",
                  epilogue);
     GV_CHECK_ARG(x && W && out && workspace, "gv_linear: null pointer");
     GV_CHECK_ARG(aligned16(x) && aligned16(W) && aligned16(out), "gv_linear: pointers not 16-byte aligned");
@@ -492,7 +491,17 @@ int gv_linear(const void* x, const void* W, int rows, int K, int n_out, int epil
     GV_CHECK_ARG(!residual || aligned16(residual), "gv_linear: residual not 16-byte aligned");
     GV_CHECK_ARG(ws_bytes >= gv_linear_workspace(rows, K, n_out, epilogue) && aligned16(workspace),
                  "gv_linear: workspace too small or misaligned");
-    return launch_linear(x, W, rows, K, n_out, epilogue, residual, out, workspace, as_stream(stream));
+    LinearOp op;
+    op.x = x;
+    op.W = W;
+    op.rows = rows;
+    op.K = K;
+    op.n_out = n_out;
+    op.epi = epilogue;
+    op.residual = residual;
+    op.out = out;
+    op.ws = workspace;
+    return launch_linear(op, as_stream(stream));
 }
 
 size_t gv_linear_qkv_workspace(int rows, int K, int n_q, int n_kv) {
@@ -510,8 +519,19 @@ int gv_linear_qkv(const void* x, const void* Wqkv, int rows, int K, int n_q, int
                      aligned16(workspace),
                  "gv_linear_qkv: pointers not 16-byte aligned");
     GV_CHECK_ARG(ws_bytes >= gv_linear_qkv_workspace(rows, K, n_q, n_kv), "gv_linear_qkv: workspace too small");
-    return launch_linear(x, Wqkv, rows, K, n_q + 2 * n_kv, GV_LINEAR_STORE, nullptr, q, workspace,
-                         as_stream(stream), k, v, n_q, n_kv);
+    LinearOp op;
+    op.x = x;
+    op.W = Wqkv;
+    op.rows = rows;
+    op.K = K;
+    op.n_out = n_q + 2 * n_kv;
+    op.out = q;
+    op.out1 = k;
+    op.out2 = v;
+    op.n0 = n_q;
+    op.n1 = n_kv;
+    op.ws = workspace;
+    return launch_linear(op, as_stream(stream));
 }
 
 int gv_linear_add_rmsnorm(const void* x, const void* W, int rows, int K, int n_out, const void* residual,
@@ -529,8 +549,20 @@ int gv_linear_add_rmsnorm(const void* x, const void* W, int rows, int K, int n_o
     GV_CHECK_ARG(norm_out != out && norm_out != residual, "gv_linear_add_rmsnorm: norm_out must be its own buffer");
     GV_CHECK_ARG(ws_bytes >= gv_linear_workspace(rows, K, n_out, GV_LINEAR_ADD),
                  "gv_linear_add_rmsnorm: workspace too small");
-    return launch_linear(x, W, rows, K, n_out, GV_LINEAR_ADD, residual, out, workspace, as_stream(stream), nullptr,
-                         nullptr, 0, 0, norm_w, eps, norm_out);
+    LinearOp op;
+    op.x = x;
+    op.W = W;
+    op.rows = rows;
+    op.K = K;
+    op.n_out = n_out;
+    op.epi = GV_LINEAR_ADD;
+    op.residual = residual;
+    op.out = out;
+    op.norm_w = norm_w;
+    op.eps = eps;
+    op.norm_out = norm_out;
+    op.ws = workspace;
+    return launch_linear(op, as_stream(stream));
 }
 
 int gv_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, void* stream) {
@@ -540,6 +572,27 @@ int gv_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* o
     GV_CHECK_ARG(x && w && out, "gv_rmsnorm: null pointer");
     GV_CHECK_ARG(aligned16(x) && aligned16(w) && aligned16(out), "gv_rmsnorm: pointers not 16-byte aligned");
     return launch_rmsnorm(x, w, rows, H, eps, out, as_stream(stream));
+}
+
+size_t gv_tgf_workspace(int rows, int d, int e) {
+    if (rows < 1 || rows > 256 || d < 64 || d % 64 != 0 || d > 8192 || e < 8 || e % 8 != 0) return 0;
+    return align256(tgf_workspace_bytes(rows, d, e));
+}
+
+int gv_tgf(const void* F, const void* x, int rows, int d, int e, const void* Wm, const void* bm, const void* g_h,
+           const void* b_h, const void* g_x, const void* b_x, const void* Wu, const void* bu, const void* Wd,
+           const void* bd, float eps, void* h_out, void* o_out, void* workspace, size_t ws_bytes, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(rows >= 1 && rows <= 256, "gv_tgf: rows=%d outside 1..256", rows);
+    GV_CHECK_ARG(d >= 64 && d % 64 == 0 && d <= 8192, "gv_tgf: d=%d (a multiple of 64, at most 8192)", d);
+    GV_CHECK_ARG(e >= 8 && e % 8 == 0, "gv_tgf: e=%d (a positive multiple of 8)", e);
+    GV_CHECK_ARG(std::isfinite(eps) && eps >= 0.0f, "gv_tgf: eps %g", (double)eps);
+    const void* ptrs[] = {F, x, Wm, bm, g_h, b_h, g_x, b_x, Wu, bu, Wd, bd, h_out, o_out, workspace};
+    for (const void* p : ptrs) GV_CHECK_ARG(p && aligned16(p), "gv_tgf: tensor null or not 16-byte aligned");
+    GV_CHECK_ARG(h_out != o_out, "gv_tgf: h_out and o_out must be separate buffers");
+    GV_CHECK_ARG(ws_bytes >= gv_tgf_workspace(rows, d, e), "gv_tgf: workspace too small");
+    return launch_tgf(F, x, rows, d, e, Wm, bm, g_h, b_h, g_x, b_x, Wu, bu, Wd, bd, eps, h_out, o_out, workspace,
+                      as_stream(stream));
 }
 
 int gv_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* feat_draft,

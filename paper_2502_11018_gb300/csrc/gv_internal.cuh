@@ -92,6 +92,33 @@ __device__ __forceinline__ bool better(float va, int ia, float vb, int ib) {
     return (va > vb) || (va == vb && ia < ib) || (vb != vb && va == va);
 }
 
+// One skinny projection out = epilogue(x W^T + bias) on the tensor cores
+// (linear_sm103.cu).  The input may come in two column blocks: x holds
+// columns [0, k_split) and x2 columns [k_split, K) (k_split % 64 == 0), so
+// that a concatenation [a ; b] W^T is never materialised.
+struct LinearOp {
+    const void* x = nullptr;        // bf16 [rows][k_split], or [rows][K] when x2 is null
+    const void* x2 = nullptr;       // bf16 [rows][K - k_split] or null
+    int k_split = 0;
+    const void* W = nullptr;        // bf16 [N][K], N = n_out (2 * n_out for SwiGLU)
+    int rows = 0, K = 0, n_out = 0, epi = GV_LINEAR_STORE;
+    const void* bias = nullptr;     // bf16 [N], added to the sums before the epilogue, or null
+    const void* residual = nullptr; // bf16 [rows][n_out] (GV_LINEAR_ADD)
+    void* out = nullptr;            // bf16 [rows][n0 or n_out]
+    void* out1 = nullptr;           // column split of the stored output (n1 > 0)
+    void* out2 = nullptr;
+    int n0 = 0, n1 = 0;
+    const void* norm_w = nullptr;   // fused RMSNorm of the ADD result (norm_out non-null)
+    float eps = 0.f;
+    void* norm_out = nullptr;
+    void* ws = nullptr;             // fp32 partial sums, linear_workspace_bytes
+};
+size_t linear_workspace_bytes(int rows, int K, int N);
+// The GEMM alone: writes the fp32 partial sums part[KS][rows][N] to op.ws and
+// returns KS through *ks (the op's epilogue fields are ignored).
+int launch_gemm_partials(const LinearOp& op, cudaStream_t st, int* ks);
+int launch_linear(const LinearOp& op, cudaStream_t st);
+
 // Per-(slot, row) partial results of the LM-head selection, merged by
 // lmhead_merge_kernel.  Layout in the workspace (slots = producing tiles):
 //   float val[slots][rows][K]; int id[slots][rows][K];  (top-K, K = k or 1)

@@ -38,12 +38,13 @@ struct GemmArgs {
     int n_tiles, KS, kblocks, units;
     int stages, stage_bytes;
     uint32_t tmem_cols;
+    int kb_split;            // k-blocks [0, kb_split) from tmap_x, the rest from tmap_x2
     float* part;             // [KS][rows][N] fp32
 };
 
 __global__ void __launch_bounds__(GM_THREADS, 1)
-gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_w,
-               GemmArgs a) {
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_x2,
+               const __grid_constant__ CUtensorMap tmap_w, GemmArgs a) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* stage_base = smem_raw;
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw + (size_t)a.stages * a.stage_bytes);
@@ -70,6 +71,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         *abort = (smem_u32(smem_raw) & 1023u) != 0 ? 1 : 0;
         fence_mbar_init();
         prefetch_tmap(&tmap_x);
+        prefetch_tmap(&tmap_x2);
         prefetch_tmap(&tmap_w);
     }
     if (warp == 1) tmem_alloc(tmem_holder, a.tmem_cols);
@@ -89,6 +91,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             const uint64_t pol_w = policy_evict_first();
             const uint64_t pol_x = policy_evict_last();
             const uint32_t tx = (uint32_t)(BM * 128 + a.npad * 128);
+            // node rows of k-block kb, from whichever input block holds it
+            auto load_x = [&](uint8_t* dst, uint64_t* bar, int kb) {
+                if (kb < a.kb_split)
+                    tma_load_2d(dst, &tmap_x, bar, kb * 64, 0, pol_x);
+                else
+                    tma_load_2d(dst, &tmap_x2, bar, (kb - a.kb_split) * 64, 0, pol_x);
+            };
             int s = 0;
             uint32_t ph = 0;
             int issued[8];
@@ -113,9 +122,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             pdl_trigger();
             if (u0 < a.units) {
                 const int lo = kb_lo(u0 % a.KS);
-                for (int q = 0; q < pre; ++q)
-                    tma_load_2d(stage_base + (size_t)q * a.stage_bytes + x_off, &tmap_x, &full[q], (lo + q) * 64, 0,
-                                pol_x);
+                for (int q = 0; q < pre; ++q) load_x(stage_base + (size_t)q * a.stage_bytes + x_off, &full[q], lo + q);
             }
             s = pre % a.stages;
             ph = pre == a.stages ? 1u : 0u;
@@ -127,7 +134,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
                     mbar_arrive_expect_tx(&full[s], tx);
                     uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
                     tma_load_2d(st, &tmap_w, &full[s], kb * 64, nt * BM, pol_w);
-                    tma_load_2d(st + x_off, &tmap_x, &full[s], kb * 64, 0, pol_x);
+                    load_x(st + x_off, &full[s], kb);
                     issued[s] = (int)ph;
                     if (++s == a.stages) {
                         s = 0;
@@ -234,6 +241,17 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     if (warp == 1) tmem_dealloc(tmem, a.tmem_cols);
 }
 
+// acc[0..8) += the eight bf16 values at p (16-byte aligned).
+__device__ __forceinline__ void bf16x8_add(float* acc, const __nv_bfloat16* p) {
+    const uint4 v = *reinterpret_cast<const uint4*>(p);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        acc[2 * e] += __uint_as_float(w[e] << 16);
+        acc[2 * e + 1] += __uint_as_float(w[e] & 0xffff0000u);
+    }
+}
+
 // Column split of the stored output: columns [0, n0) go to out0[rows][n0],
 // [n0, n0 + n1) to out1[rows][n1], the rest to out2 (the fused Q/K/V
 // projection); n1 == 0 stores everything to out0.
@@ -246,7 +264,7 @@ struct OutSplit {
 
 __global__ void __launch_bounds__(256)
 gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int n_out, int epi,
-                   const __nv_bfloat16* residual, OutSplit os) {
+                   const __nv_bfloat16* __restrict__ bias, const __nv_bfloat16* residual, OutSplit os) {
     pdl_wait();
     pdl_trigger();
     const int per_row = n_out / 8;
@@ -256,6 +274,10 @@ gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int 
     float acc[8], up[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) acc[e] = up[e] = 0.f;
+    if (bias) {
+        bf16x8_add(acc, bias + c);
+        if (epi == GV_LINEAR_SWIGLU) bf16x8_add(up, bias + n_out + c);
+    }
     for (int ks = 0; ks < KS; ++ks) {
         const float* p = part + ((size_t)ks * rows + r) * N;
         const float4 a0 = *reinterpret_cast<const float4*>(p + c);
@@ -273,14 +295,13 @@ gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int 
     if (epi == GV_LINEAR_SWIGLU) {
 #pragma unroll
         for (int e = 0; e < 8; ++e) o[e] = acc[e] / (1.0f + __expf(-acc[e])) * up[e];
-    } else if (epi == GV_LINEAR_ADD) {
-        const uint4 rv = *reinterpret_cast<const uint4*>(residual + (size_t)r * n_out + c);
-        const uint32_t w[4] = {rv.x, rv.y, rv.z, rv.w};
+    } else if (epi == GV_LINEAR_SILU) {
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            o[2 * e] = acc[2 * e] + __uint_as_float(w[e] << 16);
-            o[2 * e + 1] = acc[2 * e + 1] + __uint_as_float(w[e] & 0xffff0000u);
-        }
+        for (int e = 0; e < 8; ++e) o[e] = acc[e] / (1.0f + __expf(-acc[e]));
+    } else if (epi == GV_LINEAR_ADD) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) o[e] = acc[e];
+        bf16x8_add(o, residual + (size_t)r * n_out + c);
     } else {
 #pragma unroll
         for (int e = 0; e < 8; ++e) o[e] = acc[e];
@@ -449,16 +470,14 @@ size_t linear_workspace_bytes(int rows, int K, int N) {
     return (size_t)p.KS * rows * N * sizeof(float);
 }
 
-int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int epi, const void* residual,
-                  void* out, void* workspace, cudaStream_t st, void* out1, void* out2, int n0, int n1,
-                  const void* norm_w, float eps, void* norm_out) {
-    const int N = epi == GV_LINEAR_SWIGLU ? 2 * n_out : n_out;
-    const GemmPlan p = gemm_plan(rows, N, K);
+int launch_gemm_partials(const LinearOp& op, cudaStream_t st, int* ks) {
+    const int N = op.epi == GV_LINEAR_SWIGLU ? 2 * op.n_out : op.n_out;
+    const GemmPlan p = gemm_plan(op.rows, N, op.K);
     GemmArgs a{};
-    a.rows = rows;
+    a.rows = op.rows;
     a.npad = p.npad;
     a.N = N;
-    a.K = K;
+    a.K = op.K;
     a.mm = p.mm;
     a.n_tiles = p.n_tiles;
     a.KS = p.KS;
@@ -470,28 +489,47 @@ int launch_linear(const void* x, const void* W, int rows, int K, int n_out, int 
     if (a.stages > 8) a.stages = 8;
     const int cols = 2 * a.mm * a.npad;
     a.tmem_cols = cols <= 32 ? 32 : cols <= 64 ? 64 : cols <= 128 ? 128 : cols <= 256 ? 256 : 512;
-    a.part = static_cast<float*>(workspace);
-    CUtensorMap mx, mw;
-    int rc = make_map_2d(&mx, x, (uint64_t)rows, (uint64_t)K, (uint32_t)a.npad, (uint64_t)K * 2);
+    a.part = static_cast<float*>(op.ws);
+    // one input block: x2's map is never read (kb_split = kblocks)
+    const int k1 = op.x2 ? op.k_split : op.K;
+    a.kb_split = op.x2 ? op.k_split / 64 : a.kblocks;
+    CUtensorMap mx, mx2, mw;
+    int rc = make_map_2d(&mx, op.x, (uint64_t)op.rows, (uint64_t)k1, (uint32_t)a.npad, (uint64_t)k1 * 2);
     if (rc != GV_OK) return rc;
-    rc = make_map_2d(&mw, W, (uint64_t)N, (uint64_t)K, (uint32_t)(128 * a.mm), (uint64_t)K * 2);
+    if (op.x2) {
+        const int k2 = op.K - op.k_split;
+        rc = make_map_2d(&mx2, op.x2, (uint64_t)op.rows, (uint64_t)k2, (uint32_t)a.npad, (uint64_t)k2 * 2);
+        if (rc != GV_OK) return rc;
+    } else {
+        mx2 = mx;
+    }
+    rc = make_map_2d(&mw, op.W, (uint64_t)N, (uint64_t)op.K, (uint32_t)(128 * a.mm), (uint64_t)op.K * 2);
     if (rc != GV_OK) return rc;
     const size_t smem = (size_t)a.stages * a.stage_bytes + 8 * (2 * a.stages + 5) + 16;
     cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    launch_pdl(gemm_tc_kernel, dim3(p.grid), dim3(GM_THREADS), smem, st, mx, mw, a);
-    rc = check_launch("gemm_tc_kernel");
+    launch_pdl(gemm_tc_kernel, dim3(p.grid), dim3(GM_THREADS), smem, st, mx, mx2, mw, a);
+    *ks = a.KS;
+    return check_launch("gemm_tc_kernel");
+}
+
+int launch_linear(const LinearOp& op, cudaStream_t st) {
+    int KS = 0;
+    int rc = launch_gemm_partials(op, st, &KS);
     if (rc != GV_OK) return rc;
-    if (norm_out) {
-        launch_pdl(gemm_reduce_norm_kernel, dim3(rows), dim3(256), 0, st, (const float*)a.part, a.KS, rows, n_out,
-                   static_cast<const __nv_bfloat16*>(residual), static_cast<__nv_bfloat16*>(out),
-                   static_cast<const __nv_bfloat16*>(norm_w), eps, static_cast<__nv_bfloat16*>(norm_out));
+    const float* part = static_cast<const float*>(op.ws);
+    const int N = op.epi == GV_LINEAR_SWIGLU ? 2 * op.n_out : op.n_out;
+    if (op.norm_out) {
+        launch_pdl(gemm_reduce_norm_kernel, dim3(op.rows), dim3(256), 0, st, part, KS, op.rows, op.n_out,
+                   static_cast<const __nv_bfloat16*>(op.residual), static_cast<__nv_bfloat16*>(op.out),
+                   static_cast<const __nv_bfloat16*>(op.norm_w), op.eps, static_cast<__nv_bfloat16*>(op.norm_out));
         return check_launch("gemm_reduce_norm_kernel");
     }
-    const int items = rows * (n_out / 8);
-    OutSplit os{static_cast<__nv_bfloat16*>(out), static_cast<__nv_bfloat16*>(out1),
-                static_cast<__nv_bfloat16*>(out2), n0, n1};
-    launch_pdl(gemm_reduce_kernel, dim3((items + 255) / 256), dim3(256), 0, st, (const float*)a.part, a.KS, rows,
-               N, n_out, epi, static_cast<const __nv_bfloat16*>(residual), os);
+    const int items = op.rows * (op.n_out / 8);
+    OutSplit os{static_cast<__nv_bfloat16*>(op.out), static_cast<__nv_bfloat16*>(op.out1),
+                static_cast<__nv_bfloat16*>(op.out2), op.n0, op.n1};
+    launch_pdl(gemm_reduce_kernel, dim3((items + 255) / 256), dim3(256), 0, st, part, KS, op.rows, N, op.n_out,
+               op.epi, static_cast<const __nv_bfloat16*>(op.bias), static_cast<const __nv_bfloat16*>(op.residual),
+               os);
     return check_launch("gemm_reduce_kernel");
 }
 

@@ -29,14 +29,14 @@ GV_F32 = 1
 GV_SELECT_ARGMAX = 0
 GV_SELECT_TOPK = 1
 GV_SELECT_LOGITS = 2
-GV_LINEAR_STORE, GV_LINEAR_ADD, GV_LINEAR_SWIGLU = 0, 1, 2
+GV_LINEAR_STORE, GV_LINEAR_ADD, GV_LINEAR_SWIGLU, GV_LINEAR_SILU = 0, 1, 2, 3
 
 # Every symbol include/gv.h declares.
 EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "gv_verify_attention",
            "gv_lmhead_workspace", "gv_lmhead_select", "gv_lmhead_argmax_noalloc",
            "gv_accept_workspace", "gv_accept",
            "gv_kv_compact", "gv_rmsnorm", "gv_linear_workspace", "gv_linear", "gv_linear_qkv_workspace",
-           "gv_linear_qkv", "gv_linear_add_rmsnorm", "gv_tat_loss",
+           "gv_linear_qkv", "gv_linear_add_rmsnorm", "gv_tat_loss", "gv_tgf_workspace", "gv_tgf",
            "gv_status_string", "gv_last_error", "gv_version")
 
 
@@ -88,6 +88,8 @@ def lib():
         "gv_linear_add_rmsnorm": ([_vp, _vp, _i, _i, _i, _vp, _vp, _vp, _f, _vp, _vp, _sz, _vp], _i),
         "gv_tat_loss": ([_vp, _i, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, _i, _vp, _f, _f,
                          _vp, _vp, _vp, _vp, _vp], _i),
+        "gv_tgf_workspace": ([_i, _i, _i], _sz),
+        "gv_tgf": ([_vp, _vp, _i, _i, _i] + [_vp] * 10 + [_f, _vp, _vp, _vp, _sz, _vp], _i),
         "gv_status_string": ([_i], ctypes.c_char_p),
         "gv_last_error": ([], ctypes.c_char_p),
         "gv_version": ([], _i),
@@ -243,6 +245,23 @@ def gv_tat_loss(logits, tokens, feat_draft, feat_target, k, n, mbar_prev, mbar, 
         _ptr(feat_target, "feat_target"), dtype_code(feat_draft), B, T, V, H, k, n,
         _ptr(mbar_prev, "mbar_prev"), float(lambda_tok), float(lambda_feat), _ptr(mbar, "mbar"),
         _ptr(mask, "mask"), _ptr(ell, "ell"), _ptr(seq_loss, "seq_loss"), _stream(stream)))
+
+
+def gv_tgf_workspace(rows, d, e):
+    return int(lib().gv_tgf_workspace(rows, d, e))
+
+
+def gv_tgf(F, x, w, h_out, o_out, workspace, eps=1e-5, stream=None):
+    """Token-Guided Fusion (see include/gv.h): F, x [rows][d]; ``w`` maps Wm,
+    bm, g_h, b_h, g_x, b_x, Wu, bu, Wd, bd to bf16 tensors; outputs h_out and
+    o_out [rows][d]."""
+    rows, d = F.shape
+    e = w["Wu"].shape[0]
+    ws_bytes = workspace.numel() * workspace.element_size()
+    names = ("Wm", "bm", "g_h", "b_h", "g_x", "b_x", "Wu", "bu", "Wd", "bd")
+    return _check("gv_tgf", lib().gv_tgf(
+        _ptr(F, "F"), _ptr(x, "x"), rows, d, e, *[_ptr(w[n], n) for n in names], float(eps),
+        _ptr(h_out, "h_out"), _ptr(o_out, "o_out"), _ptr(workspace, "workspace"), ws_bytes, _stream(stream)))
 
 
 def gv_rmsnorm(x, w, out, eps=1e-5, stream=None):

@@ -406,3 +406,48 @@ def make_forward_weights(cfg, seed, device="cpu", layers=None, F=None):
         Wo=randn(gen, (L, H, Hq * d), std, dt, device), mlp_norm=norm_w(L, H),
         Wgu=randn(gen, (L, 2 * F, H), std, dt, device), Wd=randn(gen, (L, H, F), std, dt, device),
         final_norm=norm_w(H))
+
+
+# --------------------------------------------------------------------------
+# Token-Guided Fusion (Section 4.2, Eqs. 6-8) of the draft model.  Rows are
+# the positions the draft model reads in one call (the 60 nodes of a
+# verified tree); d is the target's hidden size and e the expansion width
+# (11008 for the LLaMA-2-7B drafter of the Implementation Details appendix).
+# Features F ~ N(0, 1) (the target's hidden states), token embeddings
+# x ~ N(0, 0.02) (the scale of a LLaMA embedding table), projection weights
+# ~ N(0, 0.02), biases ~ N(0, 0.02), layer-norm gains ~ 1 + N(0, 0.05).
+# --------------------------------------------------------------------------
+
+TGF_CONFIGS = {
+    "tgf_small": dict(rows=7, d=128, e=520),           # ragged expansion (partial tiles)
+    "tgf_llama2_7b": dict(rows=60, d=4096, e=11008),
+    "tgf_llama2_7b_r256": dict(rows=256, d=4096, e=11008),
+}
+
+TGF_WEIGHTS = ("Wm", "bm", "g_h", "b_h", "g_x", "b_x", "Wu", "bu", "Wd", "bd")
+
+
+@dataclass
+class TgfInputs:
+    cfg: dict
+    F: torch.Tensor      # [rows][d]
+    x: torch.Tensor      # [rows][d]
+    w: dict              # TGF_WEIGHTS -> bf16 tensors (Wm [d][2d], Wu [e][2d], Wd [d][e], vectors)
+
+
+def make_tgf_inputs(cfg, seed, device="cpu"):
+    rows, d, e = cfg["rows"], cfg["d"], cfg["e"]
+    dt = torch.bfloat16
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed) + 313)
+
+    def gain(n):
+        return (1.0 + 0.05 * torch.randn((n,), generator=gen, device=device, dtype=torch.float32)).to(dt)
+
+    w = {"Wm": randn(gen, (d, 2 * d), 0.02, dt, device), "bm": randn(gen, (d,), 0.02, dt, device),
+         "g_h": gain(d), "b_h": randn(gen, (d,), 0.02, dt, device),
+         "g_x": gain(d), "b_x": randn(gen, (d,), 0.02, dt, device),
+         "Wu": randn(gen, (e, 2 * d), 0.02, dt, device), "bu": randn(gen, (e,), 0.02, dt, device),
+         "Wd": randn(gen, (d, e), 0.02, dt, device), "bd": randn(gen, (d,), 0.02, dt, device)}
+    return TgfInputs(cfg=dict(cfg), F=randn(gen, (rows, d), 1.0, dt, device),
+                     x=randn(gen, (rows, d), 0.02, dt, device), w=w)

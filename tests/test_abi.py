@@ -77,6 +77,18 @@ def test_host_side_validation(lib):
     assert lib.gv_rmsnorm(16, 16, 60, 4100, 1e-5, 16, nul) == gv.GV_ERR_ARG
     assert gv.gv_linear_workspace(60, 4096, 1024, gv.GV_LINEAR_STORE) > 0
     assert gv.gv_linear_workspace(60, 4096, 14336, gv.GV_LINEAR_SWIGLU) >= 60 * 28672 * 4
+    assert gv.gv_linear_workspace(60, 4096, 2048, gv.GV_LINEAR_SILU) > 0
+    assert gv.gv_linear_workspace(60, 4096, 2048, 4) == 0
+    # token-guided fusion: d not a multiple of 64, rows beyond 256, h_out == o_out
+    tgf_w = [16] * 10
+    assert lib.gv_tgf(16, 16, 60, 4100, 11008, *tgf_w, 1e-5, 16, 32, 16, 1 << 34, nul) == gv.GV_ERR_ARG
+    assert lib.gv_tgf(16, 16, 257, 4096, 11008, *tgf_w, 1e-5, 16, 32, 16, 1 << 34, nul) == gv.GV_ERR_ARG
+    assert lib.gv_tgf(16, 16, 60, 4096, 11008, *tgf_w, 1e-5, 16, 16, 16, 1 << 34, nul) == gv.GV_ERR_ARG
+    assert "separate" in gv.last_error()
+    assert lib.gv_tgf(16, 16, 60, 4096, 11008, *tgf_w, 1e-5, 16, 32, 16, 16, nul) == gv.GV_ERR_ARG
+    assert "workspace" in gv.last_error()
+    assert gv.gv_tgf_workspace(60, 4096, 11008) >= 60 * (2 * 4096 + 11008) * 2
+    assert gv.gv_tgf_workspace(60, 4100, 11008) == 0
 
 
 def test_workspace_queries(lib):
