@@ -25,7 +25,9 @@ What it computes (GRIFFIN, arXiv 2502.11018):
   ``tat``;
 * the target model's decoder layers around the tree attention (RMSNorm,
   projections, SwiGLU MLP, residuals) in ``layer``;
-* the draft model's Token-Guided Fusion module (Eqs. 6-8) in ``tgf``.
+* the draft model's Token-Guided Fusion module (Eqs. 6-8) in ``tgf``;
+* the dynamic draft tree built from top-k expansions and a rerank (the draft
+  side of a cycle) in ``draft_tree``.
 
 Every function works in float64 with plain loops or single library
 primitives (a matmul, a sort), in the order the definition states.
@@ -45,3 +47,4 @@ from .step import verify_step  # noqa: F401
 from .tat import predictable_mask, alignment_mask, token_loss, feature_loss, tat_pass  # noqa: F401
 from .layer import rmsnorm, linear, silu, swiglu, decoder_layer  # noqa: F401
 from .tgf import layernorm, tgf_forward  # noqa: F401
+from .draft_tree import draft_tree, pool_size  # noqa: F401
