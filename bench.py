@@ -339,14 +339,17 @@ def main():
     ap.add_argument("--seed", type=int, default=1000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention", "tat", "forward", "tgf"],
+    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention", "tat", "forward", "tgf",
+                                                           "draft_tree"],
                     help="step: the benchmark; lmhead / attention: time that call alone "
                          "(a small, self-contained launch sequence for profiler captures); "
                          "tat: one token-alignable training pass (gv_tat_loss) on a "
                          "4 x 2048-token batch, vocabulary 32000; forward: the whole verify "
                          "forward of the target (decoder layers around the path, random "
                          "weights of the --config model's shape); tgf: the draft model's "
-                         "token-guided fusion (gv_tgf) over 60 rows, d 4096, expansion 11008")
+                         "token-guided fusion (gv_tgf) over 60 rows, d 4096, expansion 11008; "
+                         "draft_tree: one cycle's dynamic draft tree (6 top-10 expansion steps "
+                         "over a 128256-token vocabulary, rerank to 60 nodes)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
 
@@ -378,6 +381,9 @@ def main():
         return
     if args.kernel == "tgf":
         run_tgf(args, dev)
+        return
+    if args.kernel == "draft_tree":
+        run_draft_tree(args, dev)
         return
     cfg = inputs.config(args.config)
     if args.kernel != "step":
@@ -655,6 +661,60 @@ def run_tgf(args, dev):
                                 "kind": "oracle",
                                 "sample": f"float64 numpy oracle on {rs} of the {rows} rows, scaled linearly "
                                           f"({sec:.2f} s per call)"}
+    print(json.dumps(line), flush=True)
+
+
+def draft_tree_bytes(cfg):
+    """Algorithmic bytes of one draft-tree construction: every step's logits
+    read once, the tree written."""
+    B, k, D, V, N = cfg["B"], cfg["k"], cfg["D"], cfg["V"], cfg["N"]
+    es = 2 if cfg["dtype"] == "bf16" else 4
+    return B * (1 + (D - 1) * k) * V * es + B * N * 8
+
+
+def run_draft_tree(args, dev):
+    """One cycle's draft tree on the LLaMA-3-8B drafter's shape (top-10 per
+    node, 6 steps, vocabulary 128256, 60 nodes), timed from a CUDA graph of
+    back-to-back constructions with the steps' logits resident in HBM."""
+    name = "draft_llama3_8b"
+    cfg = inputs.DRAFT_CONFIGS[name]
+    B, k, D, V, N = cfg["B"], cfg["k"], cfg["D"], cfg["V"], cfg["N"]
+    root, steps = inputs.make_draft_logits(cfg, args.seed, device=dev)
+    ws = torch.empty(gv.gv_draft_tree_workspace(B, k, D, V), dtype=torch.uint8, device=dev)
+    parents = torch.zeros((B, N), dtype=torch.int32, device=dev)
+    tokens = torch.zeros((B, N), dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def call():
+        st = torch.cuda.current_stream()
+        for j in range(D):
+            gv.gv_draft_tree_expand(j, k, D, steps[j], ws, root_token=root, stream=st)
+        gv.gv_draft_tree_finish(k, D, V, parents, tokens, ws, stream=st)
+
+    for _ in range(args.warmup):
+        call()
+    torch.cuda.synchronize()
+    reps = max(3, min(args.steps, 200))
+    g = graph_of(lambda: [call() for _ in range(4)])
+    g.replay()
+    torch.cuda.synchronize()
+    ms = event_time_ms(g.replay, reps, stream) / 4
+    nbytes = draft_tree_bytes(cfg)
+    peaks = load_peaks()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    line = {"kernel": "draft_tree", "workload": name, "config": cfg, "us_per_tree": ms * 1e3,
+            "launches_per_tree": 2 * D + 1, "algorithmic_bytes": nbytes, "achieved_gbs_graph": gbs,
+            "frac_of_measured_hbm_graph": gbs / peaks["hbm_gbs"], "trees_per_s": B / (ms * 1e-3)}
+    if not args.no_cpu_baseline:
+        import oracle
+        lg = [s.detach().cpu().float().numpy() for s in steps]
+        t0 = time.perf_counter()
+        for b in range(B):
+            oracle.draft_tree(int(root[b]), [x[b] for x in lg], k, D, N)
+        sec = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": B / sec, "unit": "trees/s", "cores": torch.get_num_threads(),
+                                "kind": "oracle", "sample": f"float64 numpy oracle on the whole workload "
+                                                            f"({B} tree, {sec:.2f} s)"}
     print(json.dumps(line), flush=True)
 
 

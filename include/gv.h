@@ -28,6 +28,9 @@
  *   gv_tat_loss          top-k predictable masks, chain alignment masks and
  *                        the masked loss of one token-alignable training pass
  *   gv_tgf               the Token-Guided Fusion module (Eqs. 6-8)
+ *   gv_draft_tree_expand / gv_draft_tree_finish
+ *                        the dynamic draft tree: top-k expansion steps and
+ *                        the rerank into the tree the verify pass takes
  *
  * Conventions shared by every call:
  *  - Every pointer argument is DEVICE memory owned by the caller, unless the
@@ -343,6 +346,47 @@ size_t gv_tgf_workspace(int rows, int d, int e);
 int gv_tgf(const void* F, const void* x, int rows, int d, int e, const void* Wm, const void* bm, const void* g_h,
            const void* b_h, const void* g_x, const void* b_x, const void* Wu, const void* bu, const void* Wd,
            const void* bd, float eps, void* h_out, void* o_out, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * gv_draft_tree_expand / gv_draft_tree_finish -- the dynamic draft tree of one
+ * cycle (60 nodes, depth 6 in the Implementation Details appendix; built the
+ * EAGLE-2 way from the top-k lists of Section 4.1's draft passes).  Per
+ * sequence b, a pool of nodes (token, parent, score) lives in the workspace:
+ *
+ *   step 0:       the pool is reset to the root (root_token[b], score 0); the
+ *                 root's k most probable tokens join it
+ *   step j >= 1:  each of the k nodes selected after step j-1 (slot s = the
+ *                 s-th best) proposes its k most probable tokens
+ *
+ * A candidate's score is its parent's score + log softmax(logits row)[token];
+ * the k best candidates of step j (larger score first, then the earlier
+ * pool position) are expanded at step j+1.  Within a row, tokens rank by
+ * larger logit, then lower id.  finish keeps the root and the N-1 best pool
+ * nodes (same order), numbered in pool order (parents before children).
+ *
+ *   logits      [B][rows][V]  draft logits (dt GV_F32 or GV_BF16); rows = 1
+ *                             at step 0, k after (row s = slot s); finite
+ *   root_token  int32 [B]     step 0 only (else may be NULL)
+ *   exp_token   int32 [B][k]  out, may be NULL: the tokens of the nodes to
+ *                             expand at the next step, best first (the
+ *                             drafter's next inputs; not written at step D-1)
+ *   exp_pool    int32 [B][k]  out, may be NULL: their pool positions (the
+ *                             root is 0; step j's candidates follow the
+ *                             earlier ones, slot-major)
+ *   parents     int32 [B][N]  out (finish): -1 for the root, else an index < i
+ *   tokens      int32 [B][N]  out (finish): token[0] = the root token
+ *   workspace   >= gv_draft_tree_workspace(B, k, D, V) bytes, the same buffer
+ *               for every step of a tree; steps run in order 0 .. D-1, then
+ *               finish.
+ * 1 <= k <= 16, 1 <= D <= 16, k <= V <= 262144, 1 + k + (D-1) k^2 <= 4096 pool nodes,
+ * 1 <= N <= min(64, pool nodes).  Scores are fp32.
+ */
+size_t gv_draft_tree_workspace(int B, int k, int D, int V);
+int gv_draft_tree_expand(int B, int k, int D, int V, int step, int dt, const int32_t* root_token,
+                         const void* logits, int32_t* exp_token, int32_t* exp_pool, void* workspace,
+                         size_t ws_bytes, void* stream);
+int gv_draft_tree_finish(int B, int k, int D, int V, int N, int32_t* parents, int32_t* tokens, void* workspace,
+                         size_t ws_bytes, void* stream);
 
 /*
  * gv_rmsnorm -- out[r] = x[r] / sqrt(mean(x[r]^2) + eps) * w (the target

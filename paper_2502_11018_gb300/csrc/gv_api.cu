@@ -65,6 +65,11 @@ int launch_tree_build(const int32_t*, const int32_t*, int, int, int32_t*, int32_
                       int32_t*, cudaStream_t);
 int launch_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, cudaStream_t st);
 size_t tgf_workspace_bytes(int rows, int d, int e);
+size_t draft_tree_workspace_bytes(int B, int k, int D, int V);
+int launch_draft_tree_expand(int B, int k, int D, int V, int step, int dt, const int32_t* root_token,
+                             const void* logits, int32_t* exp_token, int32_t* exp_pool, void* ws, cudaStream_t st);
+int launch_draft_tree_finish(int B, int k, int D, int N, int32_t* parents, int32_t* tokens, void* ws,
+                             cudaStream_t st);
 int launch_tgf(const void* F, const void* x, int rows, int d, int e, const void* Wm, const void* bm,
                const void* g_h, const void* b_h, const void* g_x, const void* b_x, const void* Wu, const void* bu,
                const void* Wd, const void* bd, float eps, void* h_out, void* o_out, void* ws, cudaStream_t st);
@@ -593,6 +598,44 @@ int gv_tgf(const void* F, const void* x, int rows, int d, int e, const void* Wm,
     GV_CHECK_ARG(ws_bytes >= gv_tgf_workspace(rows, d, e), "gv_tgf: workspace too small");
     return launch_tgf(F, x, rows, d, e, Wm, bm, g_h, b_h, g_x, b_x, Wu, bu, Wd, bd, eps, h_out, o_out, workspace,
                       as_stream(stream));
+}
+
+static bool draft_tree_shape_ok(int B, int k, int D, int V) {
+    if (B < 1 || k < 1 || k > 16 || D < 1 || D > 16 || V < k || V > 262144) return false;
+    return 1 + k + (long)(D - 1) * k * k <= 4096;
+}
+
+size_t gv_draft_tree_workspace(int B, int k, int D, int V) {
+    if (!draft_tree_shape_ok(B, k, D, V)) return 0;
+    return align256(draft_tree_workspace_bytes(B, k, D, V));
+}
+
+int gv_draft_tree_expand(int B, int k, int D, int V, int step, int dt, const int32_t* root_token,
+                         const void* logits, int32_t* exp_token, int32_t* exp_pool, void* workspace,
+                         size_t ws_bytes, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(draft_tree_shape_ok(B, k, D, V),
+                 "gv_draft_tree_expand: B=%d k=%d D=%d V=%d (1 <= k <= 16, 1 <= D <= 16, k <= V <= 262144, "
+                 "1 + k + (D-1) k^2 <= 4096)", B, k, D, V);
+    GV_CHECK_ARG(step >= 0 && step < D, "gv_draft_tree_expand: step %d outside 0..%d", step, D - 1);
+    GV_CHECK_ARG(dt == GV_F32 || dt == GV_BF16, "gv_draft_tree_expand: logits dtype %d", dt);
+    GV_CHECK_ARG(logits && workspace, "gv_draft_tree_expand: null pointer");
+    GV_CHECK_ARG(step > 0 || root_token, "gv_draft_tree_expand: step 0 needs root_token");
+    GV_CHECK_ARG(ws_bytes >= gv_draft_tree_workspace(B, k, D, V) && aligned16(workspace),
+                 "gv_draft_tree_expand: workspace too small or misaligned");
+    return launch_draft_tree_expand(B, k, D, V, step, dt, root_token, logits, exp_token, exp_pool, workspace,
+                                    as_stream(stream));
+}
+
+int gv_draft_tree_finish(int B, int k, int D, int V, int N, int32_t* parents, int32_t* tokens, void* workspace,
+                         size_t ws_bytes, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(draft_tree_shape_ok(B, k, D, V), "gv_draft_tree_finish: B=%d k=%d D=%d V=%d", B, k, D, V);
+    const int P = 1 + k + (D - 1) * k * k;
+    GV_CHECK_ARG(N >= 1 && N <= P && N <= 64, "gv_draft_tree_finish: N=%d outside 1..min(64, %d)", N, P);
+    GV_CHECK_ARG(parents && tokens && workspace, "gv_draft_tree_finish: null pointer");
+    GV_CHECK_ARG(ws_bytes >= gv_draft_tree_workspace(B, k, D, V), "gv_draft_tree_finish: workspace too small");
+    return launch_draft_tree_finish(B, k, D, N, parents, tokens, workspace, as_stream(stream));
 }
 
 int gv_tat_loss(const void* logits, int logits_dt, const int32_t* tokens, const void* feat_draft,

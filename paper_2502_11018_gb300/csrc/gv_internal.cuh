@@ -42,6 +42,15 @@ int device_cc();
 // visible.  pdl_trigger() lets the next kernel's CTAs launch; kernels that
 // trigger only after their own pdl_wait() keep the ordering transitive (the
 // next kernel starts after the previous one has completed).
+//
+// The split-K reduce kernels of the projections trigger before their wait, so
+// that the next projection's CTAs can take the SMs the current GEMM frees and
+// stream their first weight stages during its tail.  Their dependents (a
+// projection, the tree attention, the LM head) read nothing before their own
+// wait but constant weights and the KV cache of an earlier step; after it,
+// the reduce has completed, and with it the GEMM it waited for.  A dependent
+// grid launches only once every CTA of its primary has triggered, so no
+// grid's CTAs can be kept off the SMs by a later grid's.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");

@@ -265,8 +265,8 @@ struct OutSplit {
 __global__ void __launch_bounds__(256)
 gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int n_out, int epi,
                    const __nv_bfloat16* __restrict__ bias, const __nv_bfloat16* residual, OutSplit os) {
+    pdl_trigger();   // (early: see the split-K reduce note in gv_internal.cuh)
     pdl_wait();
-    pdl_trigger();
     const int per_row = n_out / 8;
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= rows * per_row) return;
@@ -278,6 +278,7 @@ gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int 
         bf16x8_add(acc, bias + c);
         if (epi == GV_LINEAR_SWIGLU) bf16x8_add(up, bias + n_out + c);
     }
+#pragma unroll 4
     for (int ks = 0; ks < KS; ++ks) {
         const float* p = part + ((size_t)ks * rows + r) * N;
         const float4 a0 = *reinterpret_cast<const float4*>(p + c);
@@ -326,44 +327,56 @@ gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int 
 // layer: one CTA per row adds the K splits and the residual, writes the bf16
 // row h, and from the stored (rounded) values writes
 // norm_out = h / sqrt(mean(h^2) + eps) * w.  n_out % 8 == 0, n_out <= 8192.
-__global__ void __launch_bounds__(256)
+// Each thread owns RN_MAXC 16-byte chunks of the row; the split loop runs
+// over all of them at once, so that a thread has up to 4 * RN_MAXC * 2 loads
+// of partial sums in flight (the partials sit in L2: the loop is latency-,
+// not bandwidth-bound).
+constexpr int RN_THREADS = 512;
+constexpr int RN_MAXC = 2;                         // n_out <= RN_THREADS * RN_MAXC * 8
+
+__global__ void __launch_bounds__(RN_THREADS)
 gemm_reduce_norm_kernel(const float* __restrict__ part, int KS, int rows, int n_out,
                         const __nv_bfloat16* residual, __nv_bfloat16* out, const __nv_bfloat16* __restrict__ w,
                         float eps, __nv_bfloat16* __restrict__ norm_out) {
-    __shared__ float red[8];
+    __shared__ float red[RN_THREADS / 32];
+    pdl_trigger();   // (early: see the split-K reduce note in gv_internal.cuh)
     pdl_wait();
-    pdl_trigger();
     const int r = blockIdx.x, tid = threadIdx.x;
-    constexpr int MAXC = 4;                       // 16-byte chunks per thread (n_out <= 8192)
-    float hv[MAXC][8];
+    float acc[RN_MAXC][8];
+#pragma unroll
+    for (int q = 0; q < RN_MAXC; ++q) {
+        const int c = (tid + q * RN_THREADS) * 8;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[q][e] = 0.f;
+        if (c < n_out) bf16x8_add(acc[q], residual + (size_t)r * n_out + c);
+    }
+#pragma unroll 4
+    for (int ks = 0; ks < KS; ++ks) {
+        const float* prow = part + ((size_t)ks * rows + r) * n_out;
+#pragma unroll
+        for (int q = 0; q < RN_MAXC; ++q) {
+            const int c = (tid + q * RN_THREADS) * 8;
+            if (c < n_out) {
+                const float4 a0 = *reinterpret_cast<const float4*>(prow + c);
+                const float4 a1 = *reinterpret_cast<const float4*>(prow + c + 4);
+                acc[q][0] += a0.x; acc[q][1] += a0.y; acc[q][2] += a0.z; acc[q][3] += a0.w;
+                acc[q][4] += a1.x; acc[q][5] += a1.y; acc[q][6] += a1.z; acc[q][7] += a1.w;
+            }
+        }
+    }
     float ss = 0.f;
 #pragma unroll
-    for (int q = 0; q < MAXC; ++q) {
-        const int c = (tid + q * 256) * 8;
+    for (int q = 0; q < RN_MAXC; ++q) {
+        const int c = (tid + q * RN_THREADS) * 8;
         if (c >= n_out) break;
-        float acc[8];
-        const uint4 rv = *reinterpret_cast<const uint4*>(residual + (size_t)r * n_out + c);
-        const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            acc[2 * e] = __uint_as_float(rw[e] << 16);
-            acc[2 * e + 1] = __uint_as_float(rw[e] & 0xffff0000u);
-        }
-        for (int ks = 0; ks < KS; ++ks) {
-            const float* p = part + ((size_t)ks * rows + r) * n_out + c;
-            const float4 a0 = *reinterpret_cast<const float4*>(p);
-            const float4 a1 = *reinterpret_cast<const float4*>(p + 4);
-            acc[0] += a0.x; acc[1] += a0.y; acc[2] += a0.z; acc[3] += a0.w;
-            acc[4] += a1.x; acc[5] += a1.y; acc[6] += a1.z; acc[7] += a1.w;
-        }
         uint32_t pk[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-            __nv_bfloat162 h2 = __floats2bfloat162_rn(acc[2 * e], acc[2 * e + 1]);
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(acc[q][2 * e], acc[q][2 * e + 1]);
             pk[e] = *reinterpret_cast<uint32_t*>(&h2);
-            hv[q][2 * e] = __uint_as_float(pk[e] << 16);
-            hv[q][2 * e + 1] = __uint_as_float(pk[e] & 0xffff0000u);
-            ss += hv[q][2 * e] * hv[q][2 * e] + hv[q][2 * e + 1] * hv[q][2 * e + 1];
+            acc[q][2 * e] = __uint_as_float(pk[e] << 16);          // the stored (rounded) h
+            acc[q][2 * e + 1] = __uint_as_float(pk[e] & 0xffff0000u);
+            ss += acc[q][2 * e] * acc[q][2 * e] + acc[q][2 * e + 1] * acc[q][2 * e + 1];
         }
         *reinterpret_cast<uint4*>(out + (size_t)r * n_out + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
     }
@@ -371,19 +384,20 @@ gemm_reduce_norm_kernel(const float* __restrict__ part, int KS, int rows, int n_
     if ((tid & 31) == 0) red[tid >> 5] = ss;
     __syncthreads();
     float tot = 0.f;
-    for (int k = 0; k < 8; ++k) tot += red[k];
+#pragma unroll
+    for (int k = 0; k < RN_THREADS / 32; ++k) tot += red[k];
     const float inv = rsqrtf(tot / (float)n_out + eps);
 #pragma unroll
-    for (int q = 0; q < MAXC; ++q) {
-        const int c = (tid + q * 256) * 8;
+    for (int q = 0; q < RN_MAXC; ++q) {
+        const int c = (tid + q * RN_THREADS) * 8;
         if (c >= n_out) break;
         const uint4 g = *reinterpret_cast<const uint4*>(w + c);
         const uint32_t gw[4] = {g.x, g.y, g.z, g.w};
         uint32_t pk[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-            __nv_bfloat162 h2 = __floats2bfloat162_rn(hv[q][2 * e] * inv * __uint_as_float(gw[e] << 16),
-                                                      hv[q][2 * e + 1] * inv * __uint_as_float(gw[e] & 0xffff0000u));
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(acc[q][2 * e] * inv * __uint_as_float(gw[e] << 16),
+                                                      acc[q][2 * e + 1] * inv * __uint_as_float(gw[e] & 0xffff0000u));
             pk[e] = *reinterpret_cast<uint32_t*>(&h2);
         }
         *reinterpret_cast<uint4*>(norm_out + (size_t)r * n_out + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
@@ -519,7 +533,7 @@ int launch_linear(const LinearOp& op, cudaStream_t st) {
     const float* part = static_cast<const float*>(op.ws);
     const int N = op.epi == GV_LINEAR_SWIGLU ? 2 * op.n_out : op.n_out;
     if (op.norm_out) {
-        launch_pdl(gemm_reduce_norm_kernel, dim3(op.rows), dim3(256), 0, st, part, KS, op.rows, op.n_out,
+        launch_pdl(gemm_reduce_norm_kernel, dim3(op.rows), dim3(RN_THREADS), 0, st, part, KS, op.rows, op.n_out,
                    static_cast<const __nv_bfloat16*>(op.residual), static_cast<__nv_bfloat16*>(op.out),
                    static_cast<const __nv_bfloat16*>(op.norm_w), op.eps, static_cast<__nv_bfloat16*>(op.norm_out));
         return check_launch("gemm_reduce_norm_kernel");

@@ -17,8 +17,8 @@
 
 namespace gv {
 
-constexpr int TGF_THREADS = 256;
-constexpr int TGF_MAXC = 4;              // 16-byte chunks per thread: d <= 8192
+constexpr int TGF_THREADS = 512;
+constexpr int TGF_MAXC = 2;              // 16-byte chunks per thread: d <= 8192
 
 __device__ __forceinline__ void unpack8(const uint4 v, float* f) {
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
@@ -39,22 +39,24 @@ __device__ __forceinline__ uint4 pack8(const float* f) {
     return make_uint4(pk[0], pk[1], pk[2], pk[3]);
 }
 
-// Sum of (a, b) over the CTA; red holds 2 * 8 floats and is reused after a barrier.
+// Sum of (a, b) over the CTA; red holds 2 * TGF_THREADS / 32 floats and is
+// reused after a barrier.
 __device__ __forceinline__ float2 block_sum2(float a, float b, float* red) {
     a = warp_sum(a);
     b = warp_sum(b);
     const int w = threadIdx.x >> 5;
     __syncthreads();                     // (red's previous use is over)
+    constexpr int NW = TGF_THREADS / 32;
     if ((threadIdx.x & 31) == 0) {
         red[w] = a;
-        red[8 + w] = b;
+        red[NW + w] = b;
     }
     __syncthreads();
     float2 t = make_float2(0.f, 0.f);
 #pragma unroll
-    for (int k = 0; k < TGF_THREADS / 32; ++k) {
+    for (int k = 0; k < NW; ++k) {
         t.x += red[k];
-        t.y += red[8 + k];
+        t.y += red[NW + k];
     }
     return t;
 }
@@ -69,29 +71,44 @@ tgf_norm_kernel(const float* __restrict__ part, int KS, int rows, int d, const _
                 const __nv_bfloat16* __restrict__ b_h, const __nv_bfloat16* __restrict__ g_x,
                 const __nv_bfloat16* __restrict__ b_x, float eps, __nv_bfloat16* __restrict__ h_out,
                 __nv_bfloat16* __restrict__ zin) {
-    __shared__ float red[16];
+    __shared__ float red[2 * TGF_THREADS / 32];
+    pdl_trigger();   // (early: see the split-K reduce note in gv_internal.cuh)
     pdl_wait();
-    pdl_trigger();
     const int r = blockIdx.x, tid = threadIdx.x;
     float hv[TGF_MAXC][8], xv[TGF_MAXC][8];
+#pragma unroll
+    for (int q = 0; q < TGF_MAXC; ++q) {
+        const int c = (tid + q * TGF_THREADS) * 8;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) hv[q][e] = xv[q][e] = 0.f;
+        if (c < d) {
+            unpack8(*reinterpret_cast<const uint4*>(bm + c), hv[q]);
+            unpack8(*reinterpret_cast<const uint4*>(x + (size_t)r * d + c), xv[q]);
+        }
+    }
+    // all the chunks' split sums at once (loads in flight; the partials sit in L2)
+#pragma unroll 4
+    for (int ks = 0; ks < KS; ++ks) {
+        const float* prow = part + ((size_t)ks * rows + r) * d;
+#pragma unroll
+        for (int q = 0; q < TGF_MAXC; ++q) {
+            const int c = (tid + q * TGF_THREADS) * 8;
+            if (c < d) {
+                const float4 a0 = *reinterpret_cast<const float4*>(prow + c);
+                const float4 a1 = *reinterpret_cast<const float4*>(prow + c + 4);
+                hv[q][0] += a0.x; hv[q][1] += a0.y; hv[q][2] += a0.z; hv[q][3] += a0.w;
+                hv[q][4] += a1.x; hv[q][5] += a1.y; hv[q][6] += a1.z; hv[q][7] += a1.w;
+            }
+        }
+    }
     float sh = 0.f, sx = 0.f;
 #pragma unroll
     for (int q = 0; q < TGF_MAXC; ++q) {
         const int c = (tid + q * TGF_THREADS) * 8;
         if (c >= d) break;
-        float acc[8];
-        unpack8(*reinterpret_cast<const uint4*>(bm + c), acc);
-        for (int ks = 0; ks < KS; ++ks) {
-            const float* p = part + ((size_t)ks * rows + r) * d + c;
-            const float4 a0 = *reinterpret_cast<const float4*>(p);
-            const float4 a1 = *reinterpret_cast<const float4*>(p + 4);
-            acc[0] += a0.x; acc[1] += a0.y; acc[2] += a0.z; acc[3] += a0.w;
-            acc[4] += a1.x; acc[5] += a1.y; acc[6] += a1.z; acc[7] += a1.w;
-        }
-        const uint4 hp = pack8(acc);
+        const uint4 hp = pack8(hv[q]);
         *reinterpret_cast<uint4*>(h_out + (size_t)r * d + c) = hp;
         unpack8(hp, hv[q]);                          // the stored (rounded) h
-        unpack8(*reinterpret_cast<const uint4*>(x + (size_t)r * d + c), xv[q]);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             sh += hv[q][e];

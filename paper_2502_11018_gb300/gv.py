@@ -37,6 +37,7 @@ EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "g
            "gv_accept_workspace", "gv_accept",
            "gv_kv_compact", "gv_rmsnorm", "gv_linear_workspace", "gv_linear", "gv_linear_qkv_workspace",
            "gv_linear_qkv", "gv_linear_add_rmsnorm", "gv_tat_loss", "gv_tgf_workspace", "gv_tgf",
+           "gv_draft_tree_workspace", "gv_draft_tree_expand", "gv_draft_tree_finish",
            "gv_status_string", "gv_last_error", "gv_version")
 
 
@@ -89,6 +90,9 @@ def lib():
         "gv_tat_loss": ([_vp, _i, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, _i, _vp, _f, _f,
                          _vp, _vp, _vp, _vp, _vp], _i),
         "gv_tgf_workspace": ([_i, _i, _i], _sz),
+        "gv_draft_tree_workspace": ([_i, _i, _i, _i], _sz),
+        "gv_draft_tree_expand": ([_i] * 6 + [_vp] * 5 + [_sz, _vp], _i),
+        "gv_draft_tree_finish": ([_i] * 5 + [_vp] * 3 + [_sz, _vp], _i),
         "gv_tgf": ([_vp, _vp, _i, _i, _i] + [_vp] * 10 + [_f, _vp, _vp, _vp, _sz, _vp], _i),
         "gv_status_string": ([_i], ctypes.c_char_p),
         "gv_last_error": ([], ctypes.c_char_p),
@@ -262,6 +266,31 @@ def gv_tgf(F, x, w, h_out, o_out, workspace, eps=1e-5, stream=None):
     return _check("gv_tgf", lib().gv_tgf(
         _ptr(F, "F"), _ptr(x, "x"), rows, d, e, *[_ptr(w[n], n) for n in names], float(eps),
         _ptr(h_out, "h_out"), _ptr(o_out, "o_out"), _ptr(workspace, "workspace"), ws_bytes, _stream(stream)))
+
+
+def gv_draft_tree_workspace(B, k, D, V):
+    return int(lib().gv_draft_tree_workspace(B, k, D, V))
+
+
+def gv_draft_tree_expand(step, k, D, logits, workspace, root_token=None, exp_token=None, exp_pool=None,
+                         stream=None):
+    """One expansion step of the draft tree (see include/gv.h): logits
+    [B][rows][V] (rows = 1 at step 0, else k), fp32 or bf16."""
+    B, _, V = logits.shape
+    ws_bytes = workspace.numel() * workspace.element_size()
+    return _check("gv_draft_tree_expand", lib().gv_draft_tree_expand(
+        B, k, D, V, step, dtype_code(logits), _ptr(root_token, "root_token"), _ptr(logits, "logits"),
+        _ptr(exp_token, "exp_token"), _ptr(exp_pool, "exp_pool"), _ptr(workspace, "workspace"), ws_bytes,
+        _stream(stream)))
+
+
+def gv_draft_tree_finish(k, D, V, parents, tokens, workspace, stream=None):
+    """The rerank: parents, tokens int32 [B][N] of the tree (see include/gv.h)."""
+    B, N = parents.shape
+    ws_bytes = workspace.numel() * workspace.element_size()
+    return _check("gv_draft_tree_finish", lib().gv_draft_tree_finish(
+        B, k, D, V, N, _ptr(parents, "parents"), _ptr(tokens, "tokens"), _ptr(workspace, "workspace"), ws_bytes,
+        _stream(stream)))
 
 
 def gv_rmsnorm(x, w, out, eps=1e-5, stream=None):

@@ -451,3 +451,40 @@ def make_tgf_inputs(cfg, seed, device="cpu"):
          "Wd": randn(gen, (d, e), 0.02, dt, device), "bd": randn(gen, (d,), 0.02, dt, device)}
     return TgfInputs(cfg=dict(cfg), F=randn(gen, (rows, d), 1.0, dt, device),
                      x=randn(gen, (rows, d), 0.02, dt, device), w=w)
+
+
+# --------------------------------------------------------------------------
+# Dynamic draft trees (top-k expansion steps + rerank).  One cycle of a
+# LLaMA-3-8B drafter: k = 10 tokens per expanded node, D = 6 steps, N = 60
+# tree nodes; the logits of each step are synthetic stand-ins for the draft
+# model's: N(0, 1) over the vocabulary plus eight planted tokens per row
+# raised by 14, 12, 11, 10, 9, 8, 7, 6 (a peaked distribution, top-1
+# probability about 0.7, like a trained drafter's).
+# --------------------------------------------------------------------------
+
+DRAFT_CONFIGS = {
+    "draft_small": dict(B=2, k=4, D=3, N=12, V=1000, dtype="f32"),
+    "draft_llama3_8b": dict(B=1, k=10, D=6, N=60, V=128256, dtype="f32"),
+    "draft_llama2_7b_b4": dict(B=4, k=10, D=6, N=60, V=32000, dtype="bf16"),
+}
+
+DRAFT_BOOSTS = (14.0, 12.0, 11.0, 10.0, 9.0, 8.0, 7.0, 6.0)
+
+
+def make_draft_logits(cfg, seed, device="cpu"):
+    """(root_token int32 [B], [step 0 logits [B][1][V], step j logits [B][k][V] ...])."""
+    B, k, D, V = cfg["B"], cfg["k"], cfg["D"], cfg["V"]
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed) + 919)
+    dt = torch.bfloat16 if cfg["dtype"] == "bf16" else torch.float32
+    steps = []
+    boosts = torch.tensor(DRAFT_BOOSTS, dtype=torch.float32, device=device)
+    for j in range(D):
+        rows = 1 if j == 0 else k
+        x = torch.randn((B, rows, V), generator=gen, dtype=torch.float32, device=device)
+        nb = min(len(DRAFT_BOOSTS), V)
+        pick = torch.rand((B, rows, V), generator=gen, device=device).argsort(dim=2)[:, :, :nb]
+        x.scatter_add_(2, pick, boosts[:nb].expand(B, rows, nb).contiguous())
+        steps.append(x.to(dt))
+    root = torch.randint(0, V, (B,), generator=gen, dtype=torch.int32, device=device)
+    return root, steps

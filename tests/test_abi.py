@@ -89,6 +89,15 @@ def test_host_side_validation(lib):
     assert "workspace" in gv.last_error()
     assert gv.gv_tgf_workspace(60, 4096, 11008) >= 60 * (2 * 4096 + 11008) * 2
     assert gv.gv_tgf_workspace(60, 4100, 11008) == 0
+    # draft tree: k beyond 16, a pool beyond 4096 nodes, step out of range, N beyond 64
+    assert gv.gv_draft_tree_workspace(1, 17, 6, 32000) == 0
+    assert gv.gv_draft_tree_workspace(1, 16, 17, 32000) == 0
+    assert gv.gv_draft_tree_workspace(1, 10, 6, 32000) > 0
+    assert lib.gv_draft_tree_expand(1, 10, 6, 32000, 6, gv.GV_F32, 16, 16, nul, nul, 16, 1 << 30, nul) == gv.GV_ERR_ARG
+    assert "step" in gv.last_error()
+    assert lib.gv_draft_tree_expand(1, 10, 6, 32000, 0, gv.GV_F32, nul, 16, nul, nul, 16, 1 << 30, nul) == gv.GV_ERR_ARG
+    assert "root_token" in gv.last_error()
+    assert lib.gv_draft_tree_finish(1, 10, 6, 32000, 65, 16, 16, 16, 1 << 30, nul) == gv.GV_ERR_ARG
 
 
 def test_workspace_queries(lib):
