@@ -15,6 +15,10 @@
 // fp32 partial sums of every split go to the workspace.  gemm_reduce_kernel then
 // adds the splits and applies the epilogue (store, residual add, or SwiGLU
 // over the gate and up halves), writing bf16.
+#include <map>
+#include <mutex>
+#include <utility>
+
 #include "gv_internal.cuh"
 #include "sm103.cuh"
 
@@ -26,6 +30,27 @@ int make_map_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols
 
 constexpr int GM_THREADS = 192;
 constexpr int GM_W_TILE = 128 * 128;    // 128 weight rows x 64 bf16
+
+// acc[0..8) += the eight bf16 values at p (16-byte aligned).
+__device__ __forceinline__ void bf16x8_add(float* acc, const __nv_bfloat16* p) {
+    const uint4 v = *reinterpret_cast<const uint4*>(p);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        acc[2 * e] += __uint_as_float(w[e] << 16);
+        acc[2 * e + 1] += __uint_as_float(w[e] & 0xffff0000u);
+    }
+}
+
+// Column split of the stored output: columns [0, n0) go to out0[rows][n0],
+// [n0, n0 + n1) to out1[rows][n1], the rest to out2 (the fused Q/K/V
+// projection); n1 == 0 stores everything to out0.
+struct OutSplit {
+    __nv_bfloat16* out0;
+    __nv_bfloat16* out1;
+    __nv_bfloat16* out2;
+    int n0, n1;
+};
 
 // The weight rows are the MMA's M side (tiles of BM = 128 * mm rows, mm MMAs
 // per k-step sharing one node-row operand) and the node rows its N side
@@ -39,9 +64,46 @@ struct GemmArgs {
     int stages, stage_bytes;
     uint32_t tmem_cols;
     int kb_split;            // k-blocks [0, kb_split) from tmap_x, the rest from tmap_x2
-    float* part;             // [KS][rows][N] fp32
+    float* part;             // [KS][rows][N] fp32 (split-K through global memory)
+    // cluster split-K: the KS CTAs of a tile form a cluster and reduce through
+    // distributed shared memory, applying the epilogue themselves
+    int n_out, epi;
+    const __nv_bfloat16* bias;
+    const __nv_bfloat16* residual;
+    OutSplit os;
 };
 
+// ---- thread-block cluster helpers (distributed shared memory) ----------------
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// the address of the same shared-memory location in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t dsmem_addr(uint32_t local, uint32_t rank) {
+    uint32_t d;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(local), "r"(rank));
+    return d;
+}
+__device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(addr)
+                 : "memory");
+    return v;
+}
+__device__ __forceinline__ int ld_dsmem_s32(uint32_t addr) {
+    int v;
+    asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+// every thread of every CTA of the cluster (called convergently by all threads)
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+template <bool CSK>
 __global__ void __launch_bounds__(GM_THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_x2,
                const __grid_constant__ CUtensorMap tmap_w, GemmArgs a) {
@@ -195,6 +257,29 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         // TMEM lane = weight row (output column n), TMEM column = node row r.
         const int sub = warp & 3;                 // TMEM lane quarter this warp may access
         pdl_wait();   // (before this role's global writes)
+        if constexpr (CSK) {
+            // The CTA's one unit: stage its fp32 sums as stage[node row][tile column]
+            // over the (now idle) stage ring, for the cluster's reduction.
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(&tfull[0], 0, abort);
+            ok = __shfl_sync(FULL, ok, 0);
+            __syncwarp();
+            tc_fence_after();
+            float* stg = reinterpret_cast<float*>(smem_raw);
+            if (ok) {
+                for (int m = 0; m < a.mm; ++m) {
+                    const int nl = m * 128 + sub * 32 + lane;
+                    for (int c0 = 0; c0 < a.npad; c0 += 32) {
+                        uint32_t v[32];
+                        tmem_ld32(tmem + ((uint32_t)(sub * 32) << 16) + (uint32_t)(m * a.npad + c0), v);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) stg[(size_t)(c0 + j) * BM + nl] = __uint_as_float(v[j]);
+                    }
+                }
+            }
+            tc_fence_before();
+        } else {
         // Once a wait gives up, this CTA's remaining tiles get NaN partials,
         // so that the reduction turns the affected outputs into NaN.
         bool failed = false;
@@ -233,6 +318,66 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
             __syncwarp();
             if (lane == 0 && !failed) mbar_arrive(&tempty[acc]);
         }
+        }
+    }
+
+    if constexpr (CSK) {
+        // All CTAs of the cluster have staged their split's sums; CTA `rank`
+        // reduces the tile columns [rank * BM / KS, (rank + 1) * BM / KS) over
+        // the splits in rank order (deterministic), applies the epilogue and
+        // writes bf16.  A split that gave up makes the outputs NaN.
+        pdl_wait();
+        __syncthreads();
+        cluster_sync_all();
+        const uint32_t rank = cluster_rank();
+        const int nt = blockIdx.x / a.KS;
+        const int width = BM / a.KS, chunks = width / 8;
+        const uint32_t stg0 = smem_u32(smem_raw), ab0 = smem_u32((const void*)abort);
+        bool bad = false;
+        for (int p = 0; p < a.KS; ++p) bad |= ld_dsmem_s32(dsmem_addr(ab0, (uint32_t)p)) != 0;
+        for (int it = threadIdx.x; it < a.rows * chunks; it += GM_THREADS) {
+            const int r = it / chunks, nl = (int)rank * width + (it - r * chunks) * 8;
+            const int n = nt * BM + nl;
+            if (n >= a.N) continue;
+            float acc[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+            if (a.bias) bf16x8_add(acc, a.bias + n);
+            const uint32_t off = (uint32_t)(((size_t)r * BM + nl) * 4);
+            for (int p = 0; p < a.KS; ++p) {
+                const uint32_t q = dsmem_addr(stg0 + off, (uint32_t)p);
+                const float4 v0 = ld_dsmem_f4(q), v1 = ld_dsmem_f4(q + 16);
+                acc[0] += v0.x; acc[1] += v0.y; acc[2] += v0.z; acc[3] += v0.w;
+                acc[4] += v1.x; acc[5] += v1.y; acc[6] += v1.z; acc[7] += v1.w;
+            }
+            if (a.epi == GV_LINEAR_SILU) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[e] = acc[e] / (1.0f + __expf(-acc[e]));
+            } else if (a.epi == GV_LINEAR_ADD) {
+                bf16x8_add(acc, a.residual + (size_t)r * a.n_out + n);
+            }
+            if (bad) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[e] = NAN;
+            }
+            uint32_t pk[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                __nv_bfloat162 h2 = __floats2bfloat162_rn(acc[2 * e], acc[2 * e + 1]);
+                pk[e] = *reinterpret_cast<uint32_t*>(&h2);
+            }
+            const OutSplit& os = a.os;
+            __nv_bfloat16* dst;
+            if (os.n1 == 0 || n < os.n0)
+                dst = os.out0 + (size_t)r * (os.n1 == 0 ? a.n_out : os.n0) + n;
+            else if (n < os.n0 + os.n1)
+                dst = os.out1 + (size_t)r * os.n1 + (n - os.n0);
+            else
+                dst = os.out2 + (size_t)r * (a.n_out - os.n0 - os.n1) + (n - os.n0 - os.n1);
+            *reinterpret_cast<uint4*>(dst) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        }
+        __syncwarp();
+        cluster_sync_all();        // (no CTA leaves while a peer may still read its shared memory)
     }
 
     tc_fence_before();
@@ -240,27 +385,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
     tc_fence_after();
     if (warp == 1) tmem_dealloc(tmem, a.tmem_cols);
 }
-
-// acc[0..8) += the eight bf16 values at p (16-byte aligned).
-__device__ __forceinline__ void bf16x8_add(float* acc, const __nv_bfloat16* p) {
-    const uint4 v = *reinterpret_cast<const uint4*>(p);
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-        acc[2 * e] += __uint_as_float(w[e] << 16);
-        acc[2 * e + 1] += __uint_as_float(w[e] & 0xffff0000u);
-    }
-}
-
-// Column split of the stored output: columns [0, n0) go to out0[rows][n0],
-// [n0, n0 + n1) to out1[rows][n1], the rest to out2 (the fused Q/K/V
-// projection); n1 == 0 stores everything to out0.
-struct OutSplit {
-    __nv_bfloat16* out0;
-    __nv_bfloat16* out1;
-    __nv_bfloat16* out2;
-    int n0, n1;
-};
 
 __global__ void __launch_bounds__(256)
 gemm_reduce_kernel(const float* __restrict__ part, int KS, int rows, int N, int n_out, int epi,
@@ -448,14 +572,65 @@ rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
 }
 
 // ----------------------------------------------------------------- host side
-// (mm, KS) minimising ceil(units / SMs) * per-unit cost, a unit's cost counted
-// in rows streamed per k-block (BM weight rows + npad node rows) plus an
-// epilogue share; larger tiles on ties.
+// Split-K through global memory: (mm, KS) minimising ceil(units / SMs) * per-unit
+// cost, a unit's cost counted in rows streamed per k-block (BM weight rows +
+// npad node rows) plus an epilogue share; larger tiles on ties.  Cluster
+// split-K (the KS CTAs of a tile in one cluster, KS in {2, 4}, one wave) costs
+// ceil(kblocks / KS) * (BM + npad) + BM, scaled by SMs / CTAs, and saves the
+// partial sums' round trip through L2 and the reduce launch (counted as
+// GM_REDUCE_COST).  With 60 node rows this picks the cluster form for the O
+// projection (4096 x 4096) and the drafter's fusion projections (4096 x 8192,
+// 4096 x 11008), where it measured 0.6-1.1 us faster, and the global form for
+// the Q/K/V (6144 x 4096) and down (4096 x 14336) projections, where the
+// cluster form measured 0.4-0.8 us slower.
 struct GemmPlan {
     int mm, KS, n_tiles, kblocks, units, grid, npad;
+    bool csk;
 };
 
-static GemmPlan gemm_plan(int rows, int N, int K) {
+int launch_rmsnorm(const void* x, const void* w, int rows, int H, float eps, void* out, cudaStream_t st);
+
+constexpr int GM_SMEM_BUDGET = 220 * 1024;
+constexpr long GM_REDUCE_COST = 3500;
+
+static int gemm_stage_bytes(int mm, int npad) { return mm * GM_W_TILE + npad * 128; }
+static int gemm_stages(int stage_bytes) {
+    const int n = (GM_SMEM_BUDGET - 2048) / stage_bytes;
+    return n > 8 ? 8 : n;
+}
+static size_t gemm_smem(int stages, int stage_bytes) { return (size_t)stages * stage_bytes + 8 * (2 * stages + 5) + 16; }
+
+// Clusters of c CTAs of the cluster split-K kernel resident at once (0 if
+// the device cannot say), per (c, shared memory size).
+static int gemm_max_clusters(int c, size_t smem) {
+    static std::map<std::pair<int, size_t>, int> cache;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    const auto key = std::make_pair(c, smem);
+    auto it = cache.find(key);
+    if (it != cache.end()) return it->second;
+    int n = 0;
+    if (cudaFuncSetAttribute(gemm_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
+        cudaSuccess) {
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = (unsigned)c;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3((unsigned)(c * 16));
+        cfg.blockDim = dim3(GM_THREADS);
+        cfg.dynamicSmemBytes = smem;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<true>, &cfg) != cudaSuccess) n = 0;
+    }
+    cudaGetLastError();
+    cache[key] = n;
+    return n;
+}
+
+static GemmPlan gemm_plan(int rows, int N, int K, bool allow_csk) {
     const int npad = (rows + 31) / 32 * 32;
     const int sms = sm_count();
     GemmPlan best{};
@@ -468,25 +643,41 @@ static GemmPlan gemm_plan(int rows, int N, int K) {
             const long units = (long)tiles * ks;
             const long waves = (units + sms - 1) / sms;
             const long kb_per = (kblocks + ks - 1) / ks;
-            const long cost = waves * (kb_per * (bm + npad) + 2L * bm);
+            const long cost = waves * (kb_per * (bm + npad) + 2L * bm) + GM_REDUCE_COST;
             if (best_cost < 0 || cost < best_cost || (cost == best_cost && mm > best.mm)) {
                 best_cost = cost;
-                best = GemmPlan{mm, ks, tiles, kblocks, (int)units, 0, npad};
+                best = GemmPlan{mm, ks, tiles, kblocks, (int)units, 0, npad, false};
             }
         }
     }
     best.grid = best.units < sms ? best.units : sms;
+    if (!allow_csk) return best;
+    for (int mm = 1; mm <= 2 && 2 * mm * npad <= 512; ++mm) {
+        const int bm = 128 * mm;
+        const int tiles = (N + bm - 1) / bm;
+        const int sb = gemm_stage_bytes(mm, npad), st = gemm_stages(sb);
+        if ((size_t)npad * bm * 4 > (size_t)st * sb) continue;        // the staged sums must fit the ring
+        for (int c = 2; c <= 4; c += 2) {
+            if (c > kblocks || tiles > gemm_max_clusters(c, gemm_smem(st, sb))) continue;
+            // (scaled by the SMs left idle: one SM streams only so fast, so fewer
+            // CTAs take proportionally longer)
+            const long ctas = (long)tiles * c;
+            const long cost = ((long)((kblocks + c - 1) / c) * (bm + npad) + bm) * sms / (ctas < sms ? ctas : sms);
+            if (cost < best_cost) {
+                best_cost = cost;
+                best = GemmPlan{mm, c, tiles, kblocks, tiles * c, tiles * c, npad, true};
+            }
+        }
+    }
     return best;
 }
 
 size_t linear_workspace_bytes(int rows, int K, int N) {
-    const GemmPlan p = gemm_plan(rows, N, K);
+    const GemmPlan p = gemm_plan(rows, N, K, false);     // (an upper bound of what any plan needs)
     return (size_t)p.KS * rows * N * sizeof(float);
 }
 
-int launch_gemm_partials(const LinearOp& op, cudaStream_t st, int* ks) {
-    const int N = op.epi == GV_LINEAR_SWIGLU ? 2 * op.n_out : op.n_out;
-    const GemmPlan p = gemm_plan(op.rows, N, op.K);
+static GemmArgs gemm_args(const LinearOp& op, const GemmPlan& p, int N) {
     GemmArgs a{};
     a.rows = op.rows;
     a.npad = p.npad;
@@ -497,41 +688,90 @@ int launch_gemm_partials(const LinearOp& op, cudaStream_t st, int* ks) {
     a.KS = p.KS;
     a.kblocks = p.kblocks;
     a.units = p.units;
-    a.stage_bytes = a.mm * GM_W_TILE + a.npad * 128;
-    constexpr int SMEM_BUDGET = 220 * 1024;
-    a.stages = (SMEM_BUDGET - 2048) / a.stage_bytes;
-    if (a.stages > 8) a.stages = 8;
+    a.stage_bytes = gemm_stage_bytes(a.mm, a.npad);
+    a.stages = gemm_stages(a.stage_bytes);
     const int cols = 2 * a.mm * a.npad;
     a.tmem_cols = cols <= 32 ? 32 : cols <= 64 ? 64 : cols <= 128 ? 128 : cols <= 256 ? 256 : 512;
     a.part = static_cast<float*>(op.ws);
+    a.kb_split = op.x2 ? op.k_split / 64 : a.kblocks;
+    a.n_out = op.n_out;
+    a.epi = op.epi;
+    a.bias = static_cast<const __nv_bfloat16*>(op.bias);
+    a.residual = static_cast<const __nv_bfloat16*>(op.residual);
+    a.os = OutSplit{static_cast<__nv_bfloat16*>(op.out), static_cast<__nv_bfloat16*>(op.out1),
+                    static_cast<__nv_bfloat16*>(op.out2), op.n0, op.n1};
+    return a;
+}
+
+static int gemm_maps(const LinearOp& op, const GemmArgs& a, CUtensorMap* mx, CUtensorMap* mx2, CUtensorMap* mw) {
     // one input block: x2's map is never read (kb_split = kblocks)
     const int k1 = op.x2 ? op.k_split : op.K;
-    a.kb_split = op.x2 ? op.k_split / 64 : a.kblocks;
-    CUtensorMap mx, mx2, mw;
-    int rc = make_map_2d(&mx, op.x, (uint64_t)op.rows, (uint64_t)k1, (uint32_t)a.npad, (uint64_t)k1 * 2);
+    int rc = make_map_2d(mx, op.x, (uint64_t)op.rows, (uint64_t)k1, (uint32_t)a.npad, (uint64_t)k1 * 2);
     if (rc != GV_OK) return rc;
     if (op.x2) {
         const int k2 = op.K - op.k_split;
-        rc = make_map_2d(&mx2, op.x2, (uint64_t)op.rows, (uint64_t)k2, (uint32_t)a.npad, (uint64_t)k2 * 2);
+        rc = make_map_2d(mx2, op.x2, (uint64_t)op.rows, (uint64_t)k2, (uint32_t)a.npad, (uint64_t)k2 * 2);
         if (rc != GV_OK) return rc;
     } else {
-        mx2 = mx;
+        *mx2 = *mx;
     }
-    rc = make_map_2d(&mw, op.W, (uint64_t)N, (uint64_t)op.K, (uint32_t)(128 * a.mm), (uint64_t)op.K * 2);
+    return make_map_2d(mw, op.W, (uint64_t)a.N, (uint64_t)op.K, (uint32_t)(128 * a.mm), (uint64_t)op.K * 2);
+}
+
+int launch_gemm_partials(const LinearOp& op, cudaStream_t st, int* ks) {
+    const int N = op.epi == GV_LINEAR_SWIGLU ? 2 * op.n_out : op.n_out;
+    const GemmPlan p = gemm_plan(op.rows, N, op.K, false);
+    GemmArgs a = gemm_args(op, p, N);
+    CUtensorMap mx, mx2, mw;
+    int rc = gemm_maps(op, a, &mx, &mx2, &mw);
     if (rc != GV_OK) return rc;
-    const size_t smem = (size_t)a.stages * a.stage_bytes + 8 * (2 * a.stages + 5) + 16;
-    cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    launch_pdl(gemm_tc_kernel, dim3(p.grid), dim3(GM_THREADS), smem, st, mx, mx2, mw, a);
+    const size_t smem = gemm_smem(a.stages, a.stage_bytes);
+    cudaFuncSetAttribute(gemm_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    launch_pdl(gemm_tc_kernel<false>, dim3(p.grid), dim3(GM_THREADS), smem, st, mx, mx2, mw, a);
     *ks = a.KS;
     return check_launch("gemm_tc_kernel");
 }
 
+// The cluster split-K form: one launch writes the epilogue's bf16 output.
+static int launch_gemm_csk(const LinearOp& op, const GemmPlan& p, cudaStream_t st) {
+    GemmArgs a = gemm_args(op, p, op.n_out);
+    CUtensorMap mx, mx2, mw;
+    int rc = gemm_maps(op, a, &mx, &mx2, &mw);
+    if (rc != GV_OK) return rc;
+    const size_t smem = gemm_smem(a.stages, a.stage_bytes);
+    cudaFuncSetAttribute(gemm_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = (unsigned)a.KS;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((unsigned)p.grid);
+    cfg.blockDim = dim3(GM_THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    cudaLaunchKernelEx(&cfg, gemm_tc_kernel<true>, mx, mx2, mw, a);
+    return check_launch("gemm_tc_kernel (cluster split-K)");
+}
+
 int launch_linear(const LinearOp& op, cudaStream_t st) {
+    const int N = op.epi == GV_LINEAR_SWIGLU ? 2 * op.n_out : op.n_out;
+    if (op.epi != GV_LINEAR_SWIGLU) {
+        const GemmPlan p = gemm_plan(op.rows, N, op.K, true);
+        if (p.csk) {
+            int rc = launch_gemm_csk(op, p, st);
+            if (rc != GV_OK || !op.norm_out) return rc;
+            return launch_rmsnorm(op.out, op.norm_w, op.rows, op.n_out, op.eps, op.norm_out, st);
+        }
+    }
     int KS = 0;
     int rc = launch_gemm_partials(op, st, &KS);
     if (rc != GV_OK) return rc;
     const float* part = static_cast<const float*>(op.ws);
-    const int N = op.epi == GV_LINEAR_SWIGLU ? 2 * op.n_out : op.n_out;
     if (op.norm_out) {
         launch_pdl(gemm_reduce_norm_kernel, dim3(op.rows), dim3(RN_THREADS), 0, st, part, KS, op.rows, op.n_out,
                    static_cast<const __nv_bfloat16*>(op.residual), static_cast<__nv_bfloat16*>(op.out),

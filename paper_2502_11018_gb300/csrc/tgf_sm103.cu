@@ -10,9 +10,10 @@
 // weight streams of gv_linear (tensor cores, split K, fp32 partial sums); the
 // concatenation [F ; x] is never built (the GEMM reads its K range from two
 // input blocks), and the bias, the two layer norms and the concatenation
-// [N_h(h) ; N_x(x)] all happen in one reduce kernel after the first GEMM.
-// Six launches: GEMM, tgf_norm_kernel, GEMM + SiLU reduce, GEMM + residual
-// reduce.  The weights (4d^2 + 4de bytes) are the traffic.
+// [N_h(h) ; N_x(x)] happen in one kernel after the first projection.  Each
+// projection is either a cluster split-K launch (the splits reduced through
+// distributed shared memory, the epilogue applied there) or a GEMM plus a
+// reduce kernel, as gv_linear's planner picks; four to six launches.  The weights (4d^2 + 4de bytes) are the traffic.
 #include "gv_internal.cuh"
 
 namespace gv {
@@ -61,7 +62,8 @@ __device__ __forceinline__ float2 block_sum2(float a, float b, float* red) {
     return t;
 }
 
-// One CTA per row r: h = sum of the K splits + bm, stored as bf16; then the two
+// One CTA per row r: h = sum of the K splits + bm, stored as bf16 (or, with
+// KS == 0, h as the projection stored it, bias included); then the two
 // layer norms (fp32, population variance, two passes over values held in
 // registers) of the stored h and of x, written side by side as zin[r] =
 // [N_h(h) ; N_x(x)] (2d wide), the next GEMM's input.
@@ -69,7 +71,7 @@ __global__ void __launch_bounds__(TGF_THREADS)
 tgf_norm_kernel(const float* __restrict__ part, int KS, int rows, int d, const __nv_bfloat16* __restrict__ bm,
                 const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ g_h,
                 const __nv_bfloat16* __restrict__ b_h, const __nv_bfloat16* __restrict__ g_x,
-                const __nv_bfloat16* __restrict__ b_x, float eps, __nv_bfloat16* __restrict__ h_out,
+                const __nv_bfloat16* __restrict__ b_x, float eps, __nv_bfloat16* h_out,
                 __nv_bfloat16* __restrict__ zin) {
     __shared__ float red[2 * TGF_THREADS / 32];
     pdl_trigger();   // (early: see the split-K reduce note in gv_internal.cuh)
@@ -82,7 +84,8 @@ tgf_norm_kernel(const float* __restrict__ part, int KS, int rows, int d, const _
 #pragma unroll
         for (int e = 0; e < 8; ++e) hv[q][e] = xv[q][e] = 0.f;
         if (c < d) {
-            unpack8(*reinterpret_cast<const uint4*>(bm + c), hv[q]);
+            // KS == 0: h (bias included) was stored by the projection itself
+            unpack8(*reinterpret_cast<const uint4*>((KS == 0 ? h_out + (size_t)r * d : bm) + c), hv[q]);
             unpack8(*reinterpret_cast<const uint4*>(x + (size_t)r * d + c), xv[q]);
         }
     }
@@ -106,9 +109,11 @@ tgf_norm_kernel(const float* __restrict__ part, int KS, int rows, int d, const _
     for (int q = 0; q < TGF_MAXC; ++q) {
         const int c = (tid + q * TGF_THREADS) * 8;
         if (c >= d) break;
-        const uint4 hp = pack8(hv[q]);
-        *reinterpret_cast<uint4*>(h_out + (size_t)r * d + c) = hp;
-        unpack8(hp, hv[q]);                          // the stored (rounded) h
+        if (KS > 0) {
+            const uint4 hp = pack8(hv[q]);
+            *reinterpret_cast<uint4*>(h_out + (size_t)r * d + c) = hp;
+            unpack8(hp, hv[q]);                      // the stored (rounded) h
+        }
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             sh += hv[q][e];
@@ -172,7 +177,7 @@ int launch_tgf(const void* F, const void* x, int rows, int d, int e, const void*
     __nv_bfloat16* zin = reinterpret_cast<__nv_bfloat16*>(base + al256(part));
     __nv_bfloat16* s = reinterpret_cast<__nv_bfloat16*>(base + al256(part) + al256((size_t)rows * 2 * d * 2));
 
-    // Eq. 6: partial sums of [F ; x] Wm^T, then bias and both layer norms (Eq. 7's input)
+    // Eq. 6: h = [F ; x] Wm^T + bm, then both layer norms (Eq. 7's input)
     LinearOp m;
     m.x = F;
     m.x2 = x;
@@ -181,11 +186,12 @@ int launch_tgf(const void* F, const void* x, int rows, int d, int e, const void*
     m.rows = rows;
     m.K = 2 * d;
     m.n_out = d;
+    m.bias = bm;
+    m.out = h_out;
     m.ws = ws;
-    int KS = 0;
-    int rc = launch_gemm_partials(m, st, &KS);
+    int rc = launch_linear(m, st);
     if (rc != GV_OK) return rc;
-    launch_pdl(tgf_norm_kernel, dim3(rows), dim3(TGF_THREADS), 0, st, static_cast<const float*>(ws), KS, rows, d,
+    launch_pdl(tgf_norm_kernel, dim3(rows), dim3(TGF_THREADS), 0, st, static_cast<const float*>(nullptr), 0, rows, d,
                static_cast<const __nv_bfloat16*>(bm), static_cast<const __nv_bfloat16*>(x),
                static_cast<const __nv_bfloat16*>(g_h), static_cast<const __nv_bfloat16*>(b_h),
                static_cast<const __nv_bfloat16*>(g_x), static_cast<const __nv_bfloat16*>(b_x), eps,
