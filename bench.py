@@ -416,12 +416,14 @@ def main():
 
     # The two kernels that dominate the step, each timed alone (replayed from
     # a CUDA graph on the stream it is launched on): the LM head, and the
-    # attention layers in order (the 32 layers' caches cycle through far more
-    # than L2 holds).
+    # attention layers in order as the step runs them (splits in layer order,
+    # each layer's merge beside the next splits; the 32 layers' caches cycle
+    # through far more than L2 holds).
     L = cfg["L"]
     g_lm = graph_of(lambda: step.lmhead(torch.cuda.current_stream()))
     lm_ms = event_time_ms(g_lm.replay, 20, stream)
-    g_attn = graph_of(lambda: [step.attention(l, torch.cuda.current_stream()) for l in range(L)])
+    g_attn = graph_of(lambda: (step.attention_layers(torch.cuda.current_stream()),
+                               step.join_merges(torch.cuda.current_stream())))
     attn_ms = event_time_ms(g_attn.replay, 10, stream) / L
     peaks = load_peaks()
     lm_gbs = lmhead_bytes(cfg) / (lm_ms * 1e-3) / 1e9

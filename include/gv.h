@@ -9,7 +9,8 @@
  *
  *   gv_tree_build        positions and ancestor bitmasks from a parent array
  *   gv_rope_table        RoPE cos/sin of every node (shared by all layers)
- *   gv_verify_attention  tree-masked attention of one layer (call per layer)
+ *   gv_verify_attention  tree-masked attention of one layer (call per layer;
+ *                        or its halves gv_verify_attention_split / _merge)
  *   gv_lmhead_select     LM-head projection fused with argmax / top-k / logits
  *   gv_accept            longest accepted root chain (T = 0) or recursive
  *                        rejection sampling (T > 0)
@@ -170,6 +171,26 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
                         const int32_t* prefix_len, const float* rope, const uint64_t* anc,
                         void* treeK, void* treeV, void* out,
                         void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * gv_verify_attention_split / gv_verify_attention_merge -- the two halves of
+ * gv_verify_attention, for callers that schedule them apart.  split takes
+ * gv_verify_attention's arguments and launches the key-split kernels: their
+ * partial rows go to the workspace, or, when the shape has a single split,
+ * the final rows to `out`.  merge combines the partial rows into `out` (a
+ * no-op for a single split); it reads only the workspace.  Run in that order
+ * (e.g. the merge on a second stream that waits for the split), the pair
+ * gives gv_verify_attention's results bit for bit; the workspace belongs to
+ * the pair until the merge has completed.  A verify step whose layers take
+ * their queries, keys and values as inputs needs no layer's merged output
+ * before the next layer's split: it can run the merges beside the splits,
+ * with a workspace per layer in flight.
+ */
+int gv_verify_attention_split(const gv_attn_shape* s, const void* q, const void* k_new, const void* v_new,
+                              const void* cacheK, const void* cacheV, const int32_t* prefix_len, const float* rope,
+                              const uint64_t* anc, void* treeK, void* treeV, void* out, void* workspace,
+                              size_t ws_bytes, void* stream);
+int gv_verify_attention_merge(const gv_attn_shape* s, void* out, void* workspace, size_t ws_bytes, void* stream);
 
 /*
  * gv_lmhead_select -- LM head fused with the per-node selection.

@@ -851,7 +851,19 @@ int attn_tc_splits(int units, int S_max) {
     return c;
 }
 
-int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
+int launch_attn_tc(const AttnArgs& a0, cudaStream_t st, int phase) {
+    const int units = a0.B * a0.Hkv * a0.tiles;
+    if (!(phase & 1)) {
+        if (a0.csize == 1) return GV_OK;   // the split kernel wrote the output
+        const int rmax = a0.G * a0.N < 128 ? a0.G * a0.N : 128;
+        cudaError_t e = launch_pdl(attn_merge_kernel, dim3((unsigned)(units * ((rmax + AM_ROWS - 1) / AM_ROWS))),
+                                   dim3(AM_ROWS * 16), 0, st, a0);
+        if (e != cudaSuccess) {
+            set_error("attn_merge_kernel launch: %s", cudaGetErrorString(e));
+            return GV_ERR_CUDA;
+        }
+        return GV_OK;
+    }
     CUtensorMap mk, mv, mq;
     const uint64_t rows = (uint64_t)a0.B * a0.Hkv * a0.S_max;
     int rc = make_map_2d(&mk, a0.cacheK, rows, 128, AT_BK, 256);
@@ -863,7 +875,6 @@ int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
     const size_t smem = attn_tc_smem();
     cudaFuncSetAttribute(attn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     cudaFuncSetAttribute(attn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    const int units = a0.B * a0.Hkv * a0.tiles;
     cudaError_t e = a0.csize == 1
                         ? launch_pdl(attn_tc_kernel<true>, dim3((unsigned)units), dim3(AT_NTH), smem, st, mk, mv,
                                      mq, a0)
@@ -873,7 +884,7 @@ int launch_attn_tc(const AttnArgs& a0, cudaStream_t st) {
         set_error("attn_tc_kernel launch: %s", cudaGetErrorString(e));
         return GV_ERR_CUDA;
     }
-    if (a0.csize == 1) return GV_OK;   // the split kernel wrote the output
+    if (a0.csize == 1 || !(phase & 2)) return GV_OK;   // (one split: the split kernel wrote the output)
     const int rmax = a0.G * a0.N < 128 ? a0.G * a0.N : 128;
     e = launch_pdl(attn_merge_kernel, dim3((unsigned)(units * ((rmax + AM_ROWS - 1) / AM_ROWS))),
                    dim3(AM_ROWS * 16), 0, st, a0);

@@ -271,29 +271,31 @@ size_t gv_verify_attention_workspace(const gv_attn_shape* s) {
     return attn_plan(s).total;
 }
 
-int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new,
-                        const void* v_new, const void* cacheK, const void* cacheV,
-                        const int32_t* prefix_len, const float* rope, const uint64_t* anc,
-                        void* treeK, void* treeV, void* out, void* workspace, size_t ws_bytes,
-                        void* stream) {
+// phase 1: the split kernels (partial rows, or the output when there is one
+// split); phase 2: the merge of the splits; 3: both.
+static int attention_call(const char* name, int phase, const gv_attn_shape* s, const void* q, const void* k_new,
+                          const void* v_new, const void* cacheK, const void* cacheV, const int32_t* prefix_len,
+                          const float* rope, const uint64_t* anc, void* treeK, void* treeV, void* out,
+                          void* workspace, size_t ws_bytes, void* stream) {
     clear_error();
     const int sst = attn_shape_status(s);
     if (sst == GV_ERR_UNSUPPORTED) {
-        set_error("gv_verify_attention: unsupported shape (N=%d d=%d G*N=%d dt=%d); fp32 needs "
+        set_error("%s: unsupported shape (N=%d d=%d G*N=%d dt=%d); fp32 needs "
                   "d in {64,128}, bf16 needs d=128 and G*N <= 256, N <= 64",
-                  s->N, s->d, (s->Hq / s->Hkv) * s->N, (int)s->dt);
+                  name, s->N, s->d, (s->Hq / s->Hkv) * s->N, (int)s->dt);
         return GV_ERR_UNSUPPORTED;
     }
-    GV_CHECK_ARG(sst == GV_OK, "gv_verify_attention: invalid shape");
-    const void* ptrs[] = {q, k_new, v_new, cacheK, cacheV, treeK, treeV, out, rope};
-    for (const void* p : ptrs)
-        GV_CHECK_ARG(p && aligned16(p), "gv_verify_attention: tensor null or not 16-byte aligned");
-    GV_CHECK_ARG(prefix_len && anc, "gv_verify_attention: null index pointer");
+    GV_CHECK_ARG(sst == GV_OK, "%s: invalid shape", name);
+    GV_CHECK_ARG(out && aligned16(out), "%s: out null or not 16-byte aligned", name);
+    if (phase & 1) {
+        const void* ptrs[] = {q, k_new, v_new, cacheK, cacheV, treeK, treeV, rope};
+        for (const void* p : ptrs) GV_CHECK_ARG(p && aligned16(p), "%s: tensor null or not 16-byte aligned", name);
+        GV_CHECK_ARG(prefix_len && anc, "%s: null index pointer", name);
+    }
     const AttnPlan plan = attn_plan(s);
-    GV_CHECK_ARG(workspace && ((uintptr_t)workspace & 255u) == 0,
-                 "gv_verify_attention: workspace null or not 256-byte aligned");
-    GV_CHECK_ARG(ws_bytes >= plan.total, "gv_verify_attention: workspace %zu < %zu bytes",
-                 ws_bytes, plan.total);
+    GV_CHECK_ARG(workspace && ((uintptr_t)workspace & 255u) == 0, "%s: workspace null or not 256-byte aligned",
+                 name);
+    GV_CHECK_ARG(ws_bytes >= plan.total, "%s: workspace %zu < %zu bytes", name, ws_bytes, plan.total);
     char* ws = static_cast<char*>(workspace);
     AttnArgs a{};
     a.B = s->B;
@@ -328,11 +330,35 @@ int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new
     cudaStream_t st = as_stream(stream);
     int rc;
     if (s->dt == GV_F32) {
-        if ((rc = launch_rope_tree_f32(a, st)) != GV_OK) return rc;
-        if ((rc = launch_attn_cc_f32(a, st)) != GV_OK) return rc;
-        return launch_attn_combine_f32(a, st);
+        if (phase & 1) {
+            if ((rc = launch_rope_tree_f32(a, st)) != GV_OK) return rc;
+            if ((rc = launch_attn_cc_f32(a, st)) != GV_OK) return rc;
+        }
+        return (phase & 2) ? launch_attn_combine_f32(a, st) : GV_OK;
     }
-    return launch_attn_tc(a, st);
+    return launch_attn_tc(a, st, phase);
+}
+
+int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new,
+                        const void* v_new, const void* cacheK, const void* cacheV,
+                        const int32_t* prefix_len, const float* rope, const uint64_t* anc,
+                        void* treeK, void* treeV, void* out, void* workspace, size_t ws_bytes,
+                        void* stream) {
+    return attention_call("gv_verify_attention", 3, s, q, k_new, v_new, cacheK, cacheV, prefix_len, rope, anc,
+                          treeK, treeV, out, workspace, ws_bytes, stream);
+}
+
+int gv_verify_attention_split(const gv_attn_shape* s, const void* q, const void* k_new, const void* v_new,
+                              const void* cacheK, const void* cacheV, const int32_t* prefix_len, const float* rope,
+                              const uint64_t* anc, void* treeK, void* treeV, void* out, void* workspace,
+                              size_t ws_bytes, void* stream) {
+    return attention_call("gv_verify_attention_split", 1, s, q, k_new, v_new, cacheK, cacheV, prefix_len, rope, anc,
+                          treeK, treeV, out, workspace, ws_bytes, stream);
+}
+
+int gv_verify_attention_merge(const gv_attn_shape* s, void* out, void* workspace, size_t ws_bytes, void* stream) {
+    return attention_call("gv_verify_attention_merge", 2, s, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
+                          nullptr, nullptr, nullptr, nullptr, out, workspace, ws_bytes, stream);
 }
 
 size_t gv_lmhead_workspace(int rows, int H, int V, int dt, int mode, int k) {

@@ -33,6 +33,7 @@ GV_LINEAR_STORE, GV_LINEAR_ADD, GV_LINEAR_SWIGLU, GV_LINEAR_SILU = 0, 1, 2, 3
 
 # Every symbol include/gv.h declares.
 EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "gv_verify_attention",
+           "gv_verify_attention_split", "gv_verify_attention_merge",
            "gv_lmhead_workspace", "gv_lmhead_select", "gv_lmhead_argmax_noalloc",
            "gv_accept_workspace", "gv_accept",
            "gv_kv_compact", "gv_rmsnorm", "gv_linear_workspace", "gv_linear", "gv_linear_qkv_workspace",
@@ -74,6 +75,8 @@ def lib():
         "gv_rope_table": ([_vp, _i, _i, _i, _f, _vp, _vp], _i),
         "gv_verify_attention_workspace": ([ctypes.POINTER(gv_attn_shape)], _sz),
         "gv_verify_attention": ([ctypes.POINTER(gv_attn_shape)] + [_vp] * 12 + [_sz, _vp], _i),
+        "gv_verify_attention_split": ([ctypes.POINTER(gv_attn_shape)] + [_vp] * 12 + [_sz, _vp], _i),
+        "gv_verify_attention_merge": ([ctypes.POINTER(gv_attn_shape), _vp, _vp, _sz, _vp], _i),
         "gv_lmhead_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
         "gv_lmhead_select": ([_vp, _vp, _i, _i, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp,
                               _sz, _vp], _i),
@@ -167,6 +170,24 @@ def attn_shape(B, N, Hq, Hkv, d, S_max, dt):
 
 def gv_verify_attention_workspace(shape):
     return int(lib().gv_verify_attention_workspace(ctypes.byref(shape)))
+
+
+def gv_verify_attention_split(shape, q, k_new, v_new, cacheK, cacheV, prefix_len, rope, anc, treeK,
+                              treeV, out, workspace, stream=None):
+    """The key-split half of gv_verify_attention (see include/gv.h)."""
+    return _check("gv_verify_attention_split", lib().gv_verify_attention_split(
+        ctypes.byref(shape), _ptr(q, "q"), _ptr(k_new, "k_new"), _ptr(v_new, "v_new"),
+        _ptr(cacheK, "cacheK"), _ptr(cacheV, "cacheV"), _ptr(prefix_len, "prefix_len"),
+        _ptr(rope, "rope"), _ptr(anc, "anc"), _ptr(treeK, "treeK"), _ptr(treeV, "treeV"),
+        _ptr(out, "out"), _ptr(workspace, "workspace"), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
+
+
+def gv_verify_attention_merge(shape, out, workspace, stream=None):
+    """The merge half of gv_verify_attention (see include/gv.h)."""
+    return _check("gv_verify_attention_merge", lib().gv_verify_attention_merge(
+        ctypes.byref(shape), _ptr(out, "out"), _ptr(workspace, "workspace"),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def gv_verify_attention(shape, q, k_new, v_new, cacheK, cacheV, prefix_len, rope, anc, treeK,

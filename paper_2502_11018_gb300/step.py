@@ -5,7 +5,11 @@ five calls of include/gv.h in order on one stream (GRIFFIN Section 3: draft,
 then one verify forward over every draft token, then accept):
 
 1. ``gv_tree_build`` and ``gv_rope_table`` (RoPE cos/sin shared by all layers);
-2. ``gv_verify_attention`` for every layer (per-layer tree K/V scratch);
+2. ``gv_verify_attention_split`` for every layer (per-layer tree K/V scratch), each
+   layer's ``gv_verify_attention_merge`` on a second stream: a layer's queries,
+   keys and values are inputs of the step, so no layer waits for an earlier
+   layer's merged output, and the merges run beside the next layers' splits
+   (a workspace per layer);
 3. ``gv_lmhead_select`` (argmax for T = 0, fp32 logits + LSE for T > 0);
 4. ``gv_accept``;
 5. ``gv_kv_compact`` into every layer's cache.
@@ -21,6 +25,13 @@ from .inputs import StepInputs
 
 
 class VerifyStep:
+    # Attention workspaces in rotation (a layer's merge may still read one):
+    # None gives every layer its own, so no split waits for an earlier merge.
+    # A wait on a merge in the split stream measured slower than the merges
+    # save (13.3 against 12.8 us a layer with 3 workspaces; 11.0 with one
+    # per layer, LLaMA-3-8B shape).
+    ATTN_SLOTS = None
+
     def __init__(self, inp: StepInputs):
         cfg = inp.cfg
         self.inp = inp
@@ -44,7 +55,12 @@ class VerifyStep:
         self.attn_out = torch.zeros(L, B, N, Hq, d, dtype=dt, device=dev)
         self.shape = gv.attn_shape(B, N, Hq, Hkv, d, S_max, self.dt_code)
         ws = gv.gv_verify_attention_workspace(self.shape)
-        self.attn_ws = torch.empty(max(ws, 256), dtype=torch.uint8, device=dev)
+        slots = L if self.ATTN_SLOTS is None else min(L, self.ATTN_SLOTS)
+        self.attn_ws_slots = [torch.empty(max(ws, 256), dtype=torch.uint8, device=dev) for _ in range(slots)]
+        self.attn_ws = self.attn_ws_slots[0]
+        self.merge_stream = torch.cuda.Stream(device=dev)
+        self._split_ev = [torch.cuda.Event() for _ in range(L)]
+        self._merge_ev = [torch.cuda.Event() for _ in range(L)]
         rows = B * N
         if self.T == 0.0:
             self.lm_mode = gv.GV_SELECT_ARGMAX
@@ -78,11 +94,41 @@ class VerifyStep:
         gv.gv_rope_table(self.pos, self.cfg["d"], self.cfg["rope_base"], self.rope, stream)
 
     def attention(self, layer, stream=None):
+        """One layer, both halves on ``stream`` (its merged output ready after it)."""
         i = self.inp
         gv.gv_verify_attention(self.shape, i.q[layer], i.k_new[layer], i.v_new[layer],
                                i.cacheK[layer], i.cacheV[layer], i.prefix_len, self.rope, self.anc,
                                self.treeK[layer], self.treeV[layer], self.attn_out[layer],
                                self.attn_ws, stream)
+
+    def attention_layers(self, stream=None, ready=None):
+        """Every layer: the splits on ``stream`` in layer order, each layer's
+        merge on ``merge_stream`` after its split.  ``ready`` maps a layer to
+        an event its split waits for (its inputs' copy).  The caller joins
+        the merges with ``join_merges`` before it needs the outputs (or ends
+        a graph capture)."""
+        i = self.inp
+        cur = stream if stream is not None else torch.cuda.current_stream()
+        side = self.merge_stream
+        side.wait_stream(cur)
+        n = len(self.attn_ws_slots)
+        for layer in range(self.cfg["L"]):
+            if ready is not None and layer in ready:
+                cur.wait_event(ready[layer])
+            if layer >= n:
+                cur.wait_event(self._merge_ev[layer - n])     # (its workspace is free again)
+            ws = self.attn_ws_slots[layer % n]
+            gv.gv_verify_attention_split(self.shape, i.q[layer], i.k_new[layer], i.v_new[layer],
+                                         i.cacheK[layer], i.cacheV[layer], i.prefix_len, self.rope, self.anc,
+                                         self.treeK[layer], self.treeV[layer], self.attn_out[layer], ws, cur)
+            self._split_ev[layer].record(cur)
+            side.wait_event(self._split_ev[layer])
+            gv.gv_verify_attention_merge(self.shape, self.attn_out[layer], ws, side)
+            self._merge_ev[layer].record(side)
+
+    def join_merges(self, stream=None):
+        cur = stream if stream is not None else torch.cuda.current_stream()
+        cur.wait_stream(self.merge_stream)
 
     def lmhead(self, stream=None):
         i = self.inp
@@ -110,11 +156,11 @@ class VerifyStep:
 
     def run(self, stream=None):
         self.tree(stream)
-        for layer in range(self.cfg["L"]):
-            self.attention(layer, stream)
+        self.attention_layers(stream)
         self.lmhead(stream)
         self.accept(stream)
         self.compact(stream)
+        self.join_merges(stream)
 
     # -------------------------------------------------------------- graphs --
     def capture(self):
@@ -211,16 +257,14 @@ class VerifyStep:
             late.record(copy_stream)
         self.tree(stream)
         first = {a: ev for (a, _), ev in zip(groups, ready)}
-        for layer in range(L):
-            if layer in first:
-                stream.wait_event(first[layer])
-            self.attention(layer, stream)
+        self.attention_layers(stream, ready=first)
         stream.wait_event(late)
         self.lmhead(stream)
         self.accept(stream)
         self.compact(stream)
         with torch.cuda.stream(stream):
             host_out.copy_(self.result, non_blocking=True)
+        self.join_merges(stream)
 
     def capture_from_host(self, host, host_out):
         """Capture ``run_from_host`` into a CUDA graph (after one eager run)

@@ -133,3 +133,40 @@ def test_step_from_host_matches_device(name, layers):
     assert torch.equal(res[:B], ref.accept_len.cpu())
     assert torch.equal(res[B:B + B * (D + 1)].view(B, D + 1), ref.out_tokens.cpu())
     assert torch.equal(res[B + B * (D + 1):].view(B, D + 1), ref.path.cpu())
+
+
+@pytest.mark.parametrize("name,layers", [("llama3_8b", 7), ("tiny_f32", 4), ("llama3_8b_chain_b16", 4)])
+def test_side_merges_match_sequential_layers(name, layers):
+    # The step's schedule (splits in layer order, each merge on a second
+    # stream, workspaces in rotation) gives the outputs of calling
+    # gv_verify_attention layer by layer, bit for bit, eagerly and replayed.
+    dev = device()
+    cfg = inputs.config(name)
+    inp = inputs.make_step_inputs(cfg, 13, device="cpu", layers=layers)
+    step = VerifyStep(to_device(inp, dev))
+    step.tree()
+    for layer in range(layers):
+        step.attention(layer)
+    torch.cuda.synchronize()
+    seq = (step.attn_out.clone(), step.treeK.clone(), step.treeV.clone())
+    step.attn_out.zero_()
+    for ws in step.attn_ws_slots:
+        ws.fill_(0xFF)
+    step.attention_layers()
+    step.join_merges()
+    torch.cuda.synchronize()
+    assert torch.equal(step.attn_out, seq[0])
+    assert torch.equal(step.treeK, seq[1]) and torch.equal(step.treeV, seq[2])
+    step.attn_out.zero_()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        cur = torch.cuda.current_stream()
+        step.attention_layers(cur)
+        step.join_merges(cur)
+    g.replay()
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(step.attn_out, seq[0])
