@@ -103,14 +103,17 @@ def attention_splits(cfg):
 
 def launches_per_step(cfg):
     """Kernels of this library one step launches: tree build, RoPE table, the
-    attention layers (split attention + merge on the bf16 tensor-core path --
-    no merge when a unit has a single split --, rotate + split + combine on
-    the fp32 path), LM head + merge, accept, compaction."""
+    attention layers (on the bf16 tensor-core path one rotation of every
+    layer's queries and tree keys -- two launches -- then split attention +
+    merge per layer, no merge when a unit has a single split; rotate + split +
+    combine per layer on the fp32 path), LM head + merge, accept, compaction."""
     if cfg["dtype"] == "bf16":
         per_layer = 1 if attention_splits(cfg) == 1 else 2
+        rotate = 2 if cfg["d"] == 128 else 0
     else:
         per_layer = 3
-    return 2 + per_layer * cfg["L"] + 2 + 1 + 1
+        rotate = 0
+    return 2 + rotate + per_layer * cfg["L"] + 2 + 1 + 1
 
 
 def lmhead_bytes(cfg):

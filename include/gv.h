@@ -9,6 +9,8 @@
  *
  *   gv_tree_build        positions and ancestor bitmasks from a parent array
  *   gv_rope_table        RoPE cos/sin of every node (shared by all layers)
+ *   gv_rope_apply        (optional) the rotation of every layer's tree
+ *                        queries and keys, ahead of the attention calls
  *   gv_verify_attention  tree-masked attention of one layer (call per layer;
  *                        or its halves gv_verify_attention_split / _merge)
  *   gv_lmhead_select     LM-head projection fused with argmax / top-k / logits
@@ -155,7 +157,10 @@ int gv_rope_table(const int32_t* pos, int B, int N, int d, float rope_base, floa
  *   cacheK/V   [B][Hkv][S_max][d] cache of this layer; rows < P_b are
  *                                 read (keys stored already rotated)  (dt)
  *   prefix_len int32 [B]          P_b <= S_max
- *   rope       fp32 [B][N][d/2][2] from gv_rope_table
+ *   rope       fp32 [B][N][d/2][2] from gv_rope_table; or NULL (bf16 only)
+ *                                 when q and k_new arrive already rotated
+ *                                 (gv_rope_apply: the same arithmetic, so the
+ *                                 results are bit-identical)
  *   anc        uint64 [B][N]       from gv_tree_build
  *   treeK/V    [B][Hkv][N][d]     out: rotated tree keys / the values, the
  *                                 scratch gv_kv_compact reads        (dt)
@@ -166,6 +171,19 @@ int gv_rope_table(const int32_t* pos, int B, int N, int d, float rope_base, floa
  * ordered on the device (same stream or an event between them).
  */
 size_t gv_verify_attention_workspace(const gv_attn_shape* s);
+/*
+ * gv_rope_apply -- the RoPE rotation gv_verify_attention applies to its tree
+ * queries and keys, done ahead of time for L layers at once (bf16, d = 128):
+ * q_out[l] = RoPE(q[l]), k_out[l] = RoPE(k_new[l]) with the cos/sin of
+ * rope[b][i] (gv_rope_table).  Layer l of the inputs starts at
+ * q + l * q_layer_stride (and k_new + l * k_layer_stride) elements; the
+ * outputs are packed [L][B][N][Hq][d] and [L][B][N][Hkv][d].  Feeding them to
+ * gv_verify_attention with rope = NULL gives the same results as the
+ * unrotated inputs with the table.
+ */
+int gv_rope_apply(const gv_attn_shape* s, int L, const void* q, size_t q_layer_stride, const void* k_new,
+                  size_t k_layer_stride, const float* rope, void* q_out, void* k_out, void* stream);
+
 int gv_verify_attention(const gv_attn_shape* s, const void* q, const void* k_new,
                         const void* v_new, const void* cacheK, const void* cacheV,
                         const int32_t* prefix_len, const float* rope, const uint64_t* anc,

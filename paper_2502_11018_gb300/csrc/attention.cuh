@@ -40,7 +40,9 @@ int launch_rope_table(const int32_t* pos, int B, int N, int d, float base, float
 int launch_rope_tree_f32(const AttnArgs& a, cudaStream_t st);
 int launch_attn_combine_f32(const AttnArgs& a, cudaStream_t st);
 int launch_attn_cc_f32(const AttnArgs& a, cudaStream_t st);
-int launch_attn_tc(const AttnArgs& a, cudaStream_t st, int phase);   // phase: 1 split kernel, 2 merge, 3 both
+int launch_attn_tc(const AttnArgs& a, cudaStream_t st, int phase);
+int launch_rope_apply(const void* x, size_t layer_stride, int L, int B, int N, int H, const float* rope, void* out,
+                      cudaStream_t st);   // phase: 1 split kernel, 2 merge, 3 both
 int attn_tc_splits(int units, int S_max);
 
 }  // namespace gv

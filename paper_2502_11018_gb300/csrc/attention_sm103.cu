@@ -230,6 +230,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
     // (cos, sin) of pairs 8c + 2q, 8c + 2q + 1 of node n of sequence b, read
     // from the per-step RoPE table (L2-resident: every CTA of the sequence
     // reads the same N x 512 B).
+    // (no table: the queries and tree keys arrive rotated, gv_rope_apply)
+    const bool rotate = a.rope != nullptr;
     const float4* rope_b = reinterpret_cast<const float4*>(a.rope) + (size_t)b * a.N * 32;
     auto rope_cs = [&](int n, int c, int q) -> float4 { return __ldg(rope_b + n * 32 + c * 4 + q); };
     volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
@@ -420,7 +422,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             for (int c = 0; c < 4; ++c)
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
-                    rcs[4 * c + q] = row_ok ? rope_cs(node, 4 * kh + c, q) : make_float4(0.f, 0.f, 0.f, 0.f);
+                    rcs[4 * c + q] = (rotate && row_ok) ? rope_cs(node, 4 * kh + c, q) : make_float4(0.f, 0.f, 0.f, 0.f);
             if (has_tree) {
                 // Rotated tree keys and the values into stage 0 (and into the
                 // tree K/V scratch in global memory for gv_kv_compact).
@@ -436,10 +438,15 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
                         const uint4 k0 = __ldg(kr + c), k1 = __ldg(kr + 8 + c);
                         vlo = __ldg(vr + c);
                         vhi = __ldg(vr + 8 + c);
-                        float4 cs[4];
+                        if (rotate) {
+                            float4 cs[4];
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) cs[q] = rope_cs(j, c, q);
-                        rope8(k0, k1, cs, klo, khi);
+                            for (int q = 0; q < 4; ++q) cs[q] = rope_cs(j, c, q);
+                            rope8(k0, k1, cs, klo, khi);
+                        } else {
+                            klo = k0;
+                            khi = k1;
+                        }
                         uint4* tk = reinterpret_cast<uint4*>(a.treeK) + ((size_t)bg * a.N + j) * 16;
                         uint4* tv = reinterpret_cast<uint4*>(a.treeV) + ((size_t)bg * a.N + j) * 16;
                         if (tile0 == 0) {
@@ -466,7 +473,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             // landed: loads first, the rotation in registers, then the stores.
             {
                 const int w = mbar_wait(q_raw, 0, abort) ? 1 : 0;   // every lane observes the copy
-                if (__all_sync(FULL, w) && ok) {
+                if (__all_sync(FULL, w) && ok && rotate) {
                     uint4 lo[4], hi[4];
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
@@ -797,6 +804,44 @@ attn_merge_kernel(AttnArgs a) {
     reinterpret_cast<uint4*>(o)[ch] =
         make_uint4(pack_bf16(acc[0] * inv, acc[1] * inv), pack_bf16(acc[2] * inv, acc[3] * inv),
                    pack_bf16(acc[4] * inv, acc[5] * inv), pack_bf16(acc[6] * inv, acc[7] * inv));
+}
+
+// gv_rope_apply: the rotation the split kernel applies to its queries and tree
+// keys (rope8, the same arithmetic), ahead of time for L layers.  One thread
+// per (row, 16-byte chunk of the low half): rows are [L][B][N][H] of d = 128.
+__global__ void __launch_bounds__(256)
+rope_apply_kernel(const __nv_bfloat16* __restrict__ x, size_t layer_stride, int L, int B, int N, int H,
+                  const float* __restrict__ rope, __nv_bfloat16* __restrict__ out) {
+    pdl_wait();
+    pdl_trigger();
+    const size_t t = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const size_t rows = (size_t)L * B * N * H;
+    if (t >= rows * 8) return;
+    const size_t row = t >> 3;
+    const int c = (int)(t & 7);
+    const int l = (int)(row / ((size_t)B * N * H));
+    const size_t r = row - (size_t)l * B * N * H;          // (b, n, h) within the layer
+    const size_t bn = r / H;                               // b * N + n
+    const uint4* src = reinterpret_cast<const uint4*>(x + (size_t)l * layer_stride + r * 128);
+    const uint4 lo = __ldg(src + c), hi = __ldg(src + 8 + c);
+    const float4* cs = reinterpret_cast<const float4*>(rope) + bn * 32 + c * 4;
+    float4 c4[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) c4[q] = __ldg(cs + q);
+    uint4 olo, ohi;
+    rope8(lo, hi, c4, olo, ohi);
+    uint4* dst = reinterpret_cast<uint4*>(out) + row * 16;
+    dst[c] = olo;
+    dst[8 + c] = ohi;
+}
+
+int launch_rope_apply(const void* x, size_t layer_stride, int L, int B, int N, int H, const float* rope, void* out,
+                      cudaStream_t st) {
+    const size_t threads = (size_t)L * B * N * H * 8;
+    if (threads == 0) return GV_OK;
+    launch_pdl(rope_apply_kernel, dim3((unsigned)((threads + 255) / 256)), dim3(256), 0, st,
+               static_cast<const __nv_bfloat16*>(x), layer_stride, L, B, N, H, rope, static_cast<__nv_bfloat16*>(out));
+    return check_launch("rope_apply_kernel");
 }
 
 // ----------------------------------------------------------------- host side

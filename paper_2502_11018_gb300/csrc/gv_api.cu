@@ -288,9 +288,12 @@ static int attention_call(const char* name, int phase, const gv_attn_shape* s, c
     GV_CHECK_ARG(sst == GV_OK, "%s: invalid shape", name);
     GV_CHECK_ARG(out && aligned16(out), "%s: out null or not 16-byte aligned", name);
     if (phase & 1) {
-        const void* ptrs[] = {q, k_new, v_new, cacheK, cacheV, treeK, treeV, rope};
+        const void* ptrs[] = {q, k_new, v_new, cacheK, cacheV, treeK, treeV};
         for (const void* p : ptrs) GV_CHECK_ARG(p && aligned16(p), "%s: tensor null or not 16-byte aligned", name);
         GV_CHECK_ARG(prefix_len && anc, "%s: null index pointer", name);
+        // no table: q and k_new arrive rotated (bf16 path only)
+        GV_CHECK_ARG(rope ? aligned16(rope) : s->dt == GV_BF16,
+                     "%s: rope not 16-byte aligned, or NULL on the fp32 path", name);
     }
     const AttnPlan plan = attn_plan(s);
     GV_CHECK_ARG(workspace && ((uintptr_t)workspace & 255u) == 0, "%s: workspace null or not 256-byte aligned",
@@ -359,6 +362,25 @@ int gv_verify_attention_split(const gv_attn_shape* s, const void* q, const void*
 int gv_verify_attention_merge(const gv_attn_shape* s, void* out, void* workspace, size_t ws_bytes, void* stream) {
     return attention_call("gv_verify_attention_merge", 2, s, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
                           nullptr, nullptr, nullptr, nullptr, out, workspace, ws_bytes, stream);
+}
+
+int gv_rope_apply(const gv_attn_shape* s, int L, const void* q, size_t q_layer_stride, const void* k_new,
+                  size_t k_layer_stride, const float* rope, void* q_out, void* k_out, void* stream) {
+    clear_error();
+    GV_CHECK_ARG(s && s->dt == GV_BF16 && s->d == 128 && s->B >= 1 && s->N >= 1 && s->Hq >= 1 && s->Hkv >= 1,
+                 "gv_rope_apply: bf16 with d = 128 only");
+    GV_CHECK_ARG(L >= 1, "gv_rope_apply: L=%d", L);
+    const size_t nq = (size_t)s->B * s->N * s->Hq * 128, nk = (size_t)s->B * s->N * s->Hkv * 128;
+    GV_CHECK_ARG((L == 1 || (q_layer_stride >= nq && k_layer_stride >= nk)) && q_layer_stride % 8 == 0 &&
+                     k_layer_stride % 8 == 0,
+                 "gv_rope_apply: layer strides %zu, %zu (elements; >= one layer, multiples of 8)", q_layer_stride,
+                 k_layer_stride);
+    const void* ptrs[] = {q, k_new, rope, q_out, k_out};
+    for (const void* p : ptrs) GV_CHECK_ARG(p && aligned16(p), "gv_rope_apply: tensor null or not 16-byte aligned");
+    cudaStream_t st = as_stream(stream);
+    int rc = launch_rope_apply(q, q_layer_stride, L, s->B, s->N, s->Hq, rope, q_out, st);
+    if (rc != GV_OK) return rc;
+    return launch_rope_apply(k_new, k_layer_stride, L, s->B, s->N, s->Hkv, rope, k_out, st);
 }
 
 size_t gv_lmhead_workspace(int rows, int H, int V, int dt, int mode, int k) {

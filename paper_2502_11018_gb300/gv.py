@@ -33,7 +33,7 @@ GV_LINEAR_STORE, GV_LINEAR_ADD, GV_LINEAR_SWIGLU, GV_LINEAR_SILU = 0, 1, 2, 3
 
 # Every symbol include/gv.h declares.
 EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "gv_verify_attention",
-           "gv_verify_attention_split", "gv_verify_attention_merge",
+           "gv_verify_attention_split", "gv_verify_attention_merge", "gv_rope_apply",
            "gv_lmhead_workspace", "gv_lmhead_select", "gv_lmhead_argmax_noalloc",
            "gv_accept_workspace", "gv_accept",
            "gv_kv_compact", "gv_rmsnorm", "gv_linear_workspace", "gv_linear", "gv_linear_qkv_workspace",
@@ -77,6 +77,7 @@ def lib():
         "gv_verify_attention": ([ctypes.POINTER(gv_attn_shape)] + [_vp] * 12 + [_sz, _vp], _i),
         "gv_verify_attention_split": ([ctypes.POINTER(gv_attn_shape)] + [_vp] * 12 + [_sz, _vp], _i),
         "gv_verify_attention_merge": ([ctypes.POINTER(gv_attn_shape), _vp, _vp, _sz, _vp], _i),
+        "gv_rope_apply": ([ctypes.POINTER(gv_attn_shape), _i, _vp, _sz, _vp, _sz, _vp, _vp, _vp, _vp], _i),
         "gv_lmhead_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
         "gv_lmhead_select": ([_vp, _vp, _i, _i, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp,
                               _sz, _vp], _i),
@@ -180,6 +181,24 @@ def gv_verify_attention_split(shape, q, k_new, v_new, cacheK, cacheV, prefix_len
         _ptr(cacheK, "cacheK"), _ptr(cacheV, "cacheV"), _ptr(prefix_len, "prefix_len"),
         _ptr(rope, "rope"), _ptr(anc, "anc"), _ptr(treeK, "treeK"), _ptr(treeV, "treeV"),
         _ptr(out, "out"), _ptr(workspace, "workspace"), workspace.numel() * workspace.element_size(),
+        _stream(stream)))
+
+
+def gv_rope_apply(shape, q, k_new, rope, q_out, k_out, stream=None):
+    """Rotate L layers' tree queries and keys (see include/gv.h): q [L][B][N][Hq][d]
+    and k_new [L][B][N][Hkv][d], each layer contiguous (any layer stride, e.g.
+    views of a packed per-layer buffer); outputs packed."""
+    L = q.shape[0]
+
+    def layered(t, name):
+        if not (isinstance(t, torch.Tensor) and t.is_cuda and t[0].is_contiguous()):
+            raise ValueError(f"{name}: CUDA tensor whose layers are contiguous expected")
+        return ctypes.c_void_p(t.data_ptr()), (t.stride(0) if L > 1 else t[0].numel())
+
+    qp, qs = layered(q, "q")
+    kp, ks = layered(k_new, "k_new")
+    return _check("gv_rope_apply", lib().gv_rope_apply(
+        ctypes.byref(shape), L, qp, qs, kp, ks, _ptr(rope, "rope"), _ptr(q_out, "q_out"), _ptr(k_out, "k_out"),
         _stream(stream)))
 
 

@@ -9,7 +9,8 @@ then one verify forward over every draft token, then accept):
    layer's ``gv_verify_attention_merge`` on a second stream: a layer's queries,
    keys and values are inputs of the step, so no layer waits for an earlier
    layer's merged output, and the merges run beside the next layers' splits
-   (a workspace per layer);
+   (a workspace per layer); on the bf16 path one ``gv_rope_apply`` rotates
+   every layer's queries and tree keys ahead of the splits;
 3. ``gv_lmhead_select`` (argmax for T = 0, fp32 logits + LSE for T > 0);
 4. ``gv_accept``;
 5. ``gv_kv_compact`` into every layer's cache.
@@ -59,6 +60,12 @@ class VerifyStep:
         self.attn_ws_slots = [torch.empty(max(ws, 256), dtype=torch.uint8, device=dev) for _ in range(slots)]
         self.attn_ws = self.attn_ws_slots[0]
         self.merge_stream = torch.cuda.Stream(device=dev)
+        # bf16 (d = 128): every layer's queries and tree keys are rotated by
+        # one gv_rope_apply ahead of the splits, which then take rope = NULL
+        self.prerotate = self.dt_code == gv.GV_BF16 and d == 128
+        if self.prerotate:
+            self.q_rot = torch.empty(L, B, N, Hq, d, dtype=dt, device=dev)
+            self.k_rot = torch.empty(L, B, N, Hkv, d, dtype=dt, device=dev)
         self._split_ev = [torch.cuda.Event() for _ in range(L)]
         self._merge_ev = [torch.cuda.Event() for _ in range(L)]
         rows = B * N
@@ -108,19 +115,28 @@ class VerifyStep:
         the merges with ``join_merges`` before it needs the outputs (or ends
         a graph capture)."""
         i = self.inp
+        L = self.cfg["L"]
         cur = stream if stream is not None else torch.cuda.current_stream()
         side = self.merge_stream
         side.wait_stream(cur)
         n = len(self.attn_ws_slots)
-        for layer in range(self.cfg["L"]):
+        starts = sorted(ready) if ready is not None else [0]
+        ends = {a: b for a, b in zip(starts, starts[1:] + [L])}
+        for layer in range(L):
             if ready is not None and layer in ready:
                 cur.wait_event(ready[layer])
+            if self.prerotate and layer in ends:
+                e = ends[layer]
+                gv.gv_rope_apply(self.shape, i.q[layer:e], i.k_new[layer:e], self.rope, self.q_rot[layer:e],
+                                 self.k_rot[layer:e], cur)
             if layer >= n:
                 cur.wait_event(self._merge_ev[layer - n])     # (its workspace is free again)
             ws = self.attn_ws_slots[layer % n]
-            gv.gv_verify_attention_split(self.shape, i.q[layer], i.k_new[layer], i.v_new[layer],
-                                         i.cacheK[layer], i.cacheV[layer], i.prefix_len, self.rope, self.anc,
-                                         self.treeK[layer], self.treeV[layer], self.attn_out[layer], ws, cur)
+            q, k, rope = ((self.q_rot[layer], self.k_rot[layer], None) if self.prerotate
+                          else (i.q[layer], i.k_new[layer], self.rope))
+            gv.gv_verify_attention_split(self.shape, q, k, i.v_new[layer], i.cacheK[layer], i.cacheV[layer],
+                                         i.prefix_len, rope, self.anc, self.treeK[layer], self.treeV[layer],
+                                         self.attn_out[layer], ws, cur)
             self._split_ev[layer].record(cur)
             side.wait_event(self._split_ev[layer])
             gv.gv_verify_attention_merge(self.shape, self.attn_out[layer], ws, side)
