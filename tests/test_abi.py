@@ -89,6 +89,12 @@ def test_host_side_validation(lib):
     assert "workspace" in gv.last_error()
     assert gv.gv_tgf_workspace(60, 4096, 11008) >= 60 * (2 * 4096 + 11008) * 2
     assert gv.gv_tgf_workspace(60, 4100, 11008) == 0
+    # rotation ahead of the attention: bf16 with d = 128 only; a layer stride below one layer
+    f32 = gv.attn_shape(1, 60, 32, 8, 128, 4224, gv.GV_F32)
+    assert lib.gv_rope_apply(ctypes.byref(f32), 2, 16, 1 << 20, 16, 1 << 20, 16, 16, 16, nul) == gv.GV_ERR_ARG
+    bf = gv.attn_shape(1, 60, 32, 8, 128, 4224, gv.GV_BF16)
+    assert lib.gv_rope_apply(ctypes.byref(bf), 2, 16, 64, 16, 1 << 20, 16, 16, 16, nul) == gv.GV_ERR_ARG
+    assert "stride" in gv.last_error()
     # draft tree: k beyond 16, a pool beyond 4096 nodes, step out of range, N beyond 64
     assert gv.gv_draft_tree_workspace(1, 17, 6, 32000) == 0
     assert gv.gv_draft_tree_workspace(1, 16, 17, 32000) == 0
