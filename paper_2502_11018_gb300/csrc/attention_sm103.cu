@@ -337,7 +337,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant_
             if (lane == 0) {
                 const uint32_t idesc_s = idesc_bf16(128, AT_BK);
                 const uint32_t idesc_o = idesc_bf16(128, 128, /*b_mn_major=*/true);
-                bool mok = mbar_wait(q_full, 0, abort);
+                // (queries that arrive rotated are used as the copy lands them)
+                bool mok = mbar_wait(rotate ? q_full : q_raw, 0, abort);
                 tc_fence_after();
                 // S_j = Q K_j^T into S buffer j % 3, as soon as block j's K
                 // has landed and PV_{j-3} has consumed that buffer.
