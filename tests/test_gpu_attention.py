@@ -107,3 +107,40 @@ def test_attention_repeatable_on_reused_workspace():
     ro, _, _ = oracle.tree_attention(f64(q), f64(k), f64(v), f64(cK), f64(cV), P,
                                      oracle.tree_build(parents, P)[1], oracle.tree_build(parents, P)[2], 5e5)
     assert rel_err(f64(outs[2]), ro) <= TOL_ATTN["bf16"]
+
+
+@pytest.mark.parametrize("case", [4, 6, 9])
+def test_rope_apply_matches_the_oracle_and_the_kernel(case):
+    # gv_rope_apply over two layers against the oracle's float64 rotation
+    # (one bf16 rounding), and the attention with rope = NULL on the rotated
+    # inputs against the attention that rotates them itself, bit for bit.
+    dtype, B, N, Hq, Hkv, d, P, base, std = CASES[case]
+    dev = device()
+    parents, P, S_max, q, k, v, cK, cV = _case(dtype, B, N, Hq, Hkv, d, P, base, std, 40 + case)
+    out, tK, tV, pos, anc = run_gpu_attention(dev, parents, P, S_max, q, k, v, cK, cV, base)
+    rope = torch.zeros(B, N, d // 2, 2, dtype=torch.float32, device=dev)
+    gv.gv_rope_table(pos, d, base, rope)
+    shape = gv.attn_shape(B, N, Hq, Hkv, d, S_max, gv.GV_BF16)
+    q2 = torch.stack([q, q.flip(0) if B > 1 else q]).to(dev)      # two layers
+    k2 = torch.stack([k, k]).to(dev)
+    q_rot = torch.empty_like(q2)
+    k_rot = torch.empty_like(k2)
+    gv.gv_rope_apply(shape, q2, k2, rope, q_rot, k_rot)
+    torch.cuda.synchronize()
+    posn = pos.cpu().numpy()
+    for b in range(B):
+        ref_q = oracle.rope_rotate(f64(q2[0, b]), posn[b], base)
+        ref_k = oracle.rope_rotate(f64(k2[1, b]), posn[b], base)
+        assert rel_err(f64(q_rot[0, b]), ref_q) <= TOL_ROT["bf16"]
+        assert rel_err(f64(k_rot[1, b]), ref_k) <= TOL_ROT["bf16"]
+    # the kernel's own rotation of the tree keys (treeK is [B][Hkv][N][d])
+    assert torch.equal(k_rot[0].permute(0, 2, 1, 3), tK)
+    tK2 = torch.zeros_like(tK)
+    tV2 = torch.zeros_like(tV)
+    out2 = torch.zeros_like(out)
+    ws = torch.full((gv.gv_verify_attention_workspace(shape),), 0xFF, dtype=torch.uint8, device=dev)
+    t32 = torch.as_tensor(P, dtype=torch.int32, device=dev)
+    gv.gv_verify_attention(shape, q_rot[0], k_rot[0], v.to(dev), cK.to(dev), cV.to(dev), t32, None, anc, tK2,
+                           tV2, out2, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(out2, out) and torch.equal(tK2, tK) and torch.equal(tV2, tV)
