@@ -323,20 +323,23 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
 
     if constexpr (CSK) {
         // All CTAs of the cluster have staged their split's sums; CTA `rank`
-        // reduces the tile columns [rank * BM / KS, (rank + 1) * BM / KS) over
-        // the splits in rank order (deterministic), applies the epilogue and
-        // writes bf16.  A split that gave up makes the outputs NaN.
+        // reduces its share of the tile's columns (8-column chunks
+        // [rank * BM/8 / KS, (rank + 1) * BM/8 / KS)) over the splits in rank
+        // order (deterministic), applies the epilogue and writes bf16.  A
+        // split that gave up makes the outputs NaN.
         pdl_wait();
         __syncthreads();
         cluster_sync_all();
         const uint32_t rank = cluster_rank();
         const int nt = blockIdx.x / a.KS;
-        const int width = BM / a.KS, chunks = width / 8;
+        // this rank's 8-column chunks of the tile (the ranks split BM / 8 chunks as evenly as they go)
+        const int nch = BM / 8;
+        const int c_lo = (int)rank * nch / a.KS, chunks = ((int)rank + 1) * nch / a.KS - c_lo;
         const uint32_t stg0 = smem_u32(smem_raw), ab0 = smem_u32((const void*)abort);
         bool bad = false;
         for (int p = 0; p < a.KS; ++p) bad |= ld_dsmem_s32(dsmem_addr(ab0, (uint32_t)p)) != 0;
         for (int it = threadIdx.x; it < a.rows * chunks; it += GM_THREADS) {
-            const int r = it / chunks, nl = (int)rank * width + (it - r * chunks) * 8;
+            const int r = it / chunks, nl = (c_lo + (it - r * chunks)) * 8;
             const int n = nt * BM + nl;
             if (n >= a.N) continue;
             float acc[8];
@@ -582,7 +585,11 @@ rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
 // projection (4096 x 4096) and the drafter's fusion projections (4096 x 8192,
 // 4096 x 11008), where it measured 0.6-1.1 us faster, and the global form for
 // the Q/K/V (6144 x 4096) and down (4096 x 14336) projections, where the
-// cluster form measured 0.4-0.8 us slower.
+// cluster form measured 0.4-0.8 us slower.  (Other cluster sizes -- the
+// kernel splits a tile's columns unevenly when KS does not divide BM / 8 --
+// measured no better: Q/K/V in clusters of 5 took 17.7 us against 17.1, the
+// 11008 x 8192 fusion projection in clusters of 3 took 39.0 us against the
+// global form's ~35.)
 struct GemmPlan {
     int mm, KS, n_tiles, kblocks, units, grid, npad;
     bool csk;
