@@ -102,12 +102,22 @@ def attention_splits(cfg):
     return max(c, 1)
 
 
+def layers_call(cfg):
+    """Whether the step runs every layer's attention in one
+    gv_verify_attention_layers call (bf16, d = 128, G * N <= 256, B <= 64)."""
+    G = cfg["Hq"] // cfg["Hkv"]
+    return cfg["dtype"] == "bf16" and cfg["d"] == 128 and G * cfg["N"] <= 256 and cfg["B"] <= 64
+
+
 def launches_per_step(cfg):
     """Kernels of this library one step launches: tree build, RoPE table, the
-    attention layers (on the bf16 tensor-core path one rotation of every
-    layer's queries and tree keys -- two launches -- then split attention +
-    merge per layer, no merge when a unit has a single split; rotate + split +
-    combine per layer on the fp32 path), LM head + merge, accept, compaction."""
+    attention (one multi-layer call -- its rotation pass and the persistent
+    kernel -- on the bf16 path; otherwise one rotation of every layer's
+    queries and tree keys -- two launches -- then split attention + merge per
+    layer, no merge when a unit has a single split; rotate + split + combine
+    per layer on the fp32 path), LM head + merge, accept, compaction."""
+    if layers_call(cfg):
+        return 2 + 2 + 2 + 1 + 1
     if cfg["dtype"] == "bf16":
         per_layer = 1 if attention_splits(cfg) == 1 else 2
         rotate = 2 if cfg["d"] == 128 else 0
@@ -343,10 +353,13 @@ def main():
     ap.add_argument("--seed", type=int, default=1000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention", "tat", "forward", "tgf",
-                                                           "draft_tree"],
+    ap.add_argument("--layers", type=int, default=0,
+                    help="--kernel attention_layers: layers of the call (default: the workload's)")
+    ap.add_argument("--kernel", default="step", choices=["step", "lmhead", "attention", "attention_layers", "tat",
+                                                           "forward", "tgf", "draft_tree"],
                     help="step: the benchmark; lmhead / attention: time that call alone "
                          "(a small, self-contained launch sequence for profiler captures); "
+                         "attention_layers: one gv_verify_attention_layers call over --layers layers; "
                          "tat: one token-alignable training pass (gv_tat_loss) on a "
                          "4 x 2048-token batch, vocabulary 32000; forward: the whole verify "
                          "forward of the target (decoder layers around the path, random "
@@ -390,6 +403,9 @@ def main():
         run_draft_tree(args, dev)
         return
     cfg = inputs.config(args.config)
+    if args.kernel == "attention_layers":
+        run_attention_layers(args, cfg, dev)
+        return
     if args.kernel != "step":
         run_kernel_only(args, cfg, dev)
         return
@@ -515,6 +531,36 @@ def run_kernel_only(args, cfg, dev):
                       "ms_per_call_graph": ms_graph, "algorithmic_bytes": nbytes,
                       "achieved_gbs_graph": gbs_graph,
                       "frac_of_measured_hbm_graph": gbs_graph / peaks["hbm_gbs"]}), flush=True)
+
+
+def run_attention_layers(args, cfg, dev):
+    """One gv_verify_attention_layers call over the first --layers layers of
+    the workload (its rotation pass and the persistent attention kernel),
+    replayed from a CUDA graph; calls cycle over two copies of the caches
+    when one copy fits in L2."""
+    from paper_2502_11018_gb300.step import VerifyStep
+    layers = args.layers if args.layers > 0 else cfg["L"]
+    inp = inputs.make_step_inputs(cfg, args.seed, device=dev, layers=layers)
+    step = VerifyStep(inp)
+    if not step.layers_call:
+        raise SystemExit(f"{cfg['name']}: no multi-layer attention for this shape")
+    step.tree()
+    stream = torch.cuda.current_stream()
+    fn = lambda: step.attention_layers(torch.cuda.current_stream())  # noqa: E731
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    g = graph_of(fn)
+    g.replay()
+    torch.cuda.synchronize()
+    reps = max(3, min(args.steps, 200))
+    ms = event_time_ms(g.replay, reps, stream)
+    nbytes = attention_bytes(cfg) * layers
+    peaks = load_peaks()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    print(json.dumps({"kernel": "attention_layers", "workload": cfg["name"], "layers": layers,
+                      "ms_per_call_graph": ms, "us_per_layer": ms * 1e3 / layers, "algorithmic_bytes": nbytes,
+                      "achieved_gbs_graph": gbs, "frac_of_measured_hbm_graph": gbs / peaks["hbm_gbs"]}), flush=True)
 
 
 def forward_bytes(cfg, F, accept_len):

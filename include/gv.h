@@ -211,6 +211,43 @@ int gv_verify_attention_split(const gv_attn_shape* s, const void* q, const void*
 int gv_verify_attention_merge(const gv_attn_shape* s, void* out, void* workspace, size_t ws_bytes, void* stream);
 
 /*
+ * gv_verify_attention_layers -- the tree attention of L layers in one call.
+ * Section 3: one target forward pass verifies every draft token; when the
+ * caller holds the tree queries, keys and values of several layers at once
+ * (a verify step whose layers' inputs are given), their attentions are
+ * independent problems and run as one persistent launch.  The results equal
+ * L calls of gv_verify_attention (same rotation, mask and softmax; the
+ * combination of partial results may round differently in the last bf16
+ * bit).  Layer l of an input starts l * (its layer stride) elements after its
+ * pointer; the outputs are packed by layer.
+ *
+ *   q          [L][B][N][Hq][d]      tree queries, unrotated, stride q_layer_stride
+ *   k_new      [L][B][N][Hkv][d]     tree keys, unrotated, stride k_layer_stride
+ *   v_new      [L][B][N][Hkv][d]     tree values, stride v_layer_stride
+ *   cacheK/V   [L][B][Hkv][S_max][d] caches, stride cache_layer_stride; rows
+ *                                    < P_b are read (keys stored rotated)
+ *   prefix_len int32 [B], rope fp32 [B][N][d/2][2] (gv_rope_table), anc
+ *                                    uint64 [B][N] (gv_tree_build)
+ *   treeK/V    [L][B][Hkv][N][d]     out: rotated tree keys / the values
+ *                                    (what gv_kv_compact reads)
+ *   out        [L][B][N][Hq][d]      out: attention outputs
+ *   workspace  >= gv_verify_attention_layers_workspace(s, L) bytes, 256-byte
+ *              aligned; contents need no initialisation and are clobbered.
+ * bf16 only, d = 128, 1 <= B <= 64, N <= 64, (Hq/Hkv) * N <= 256 (else
+ * GV_ERR_UNSUPPORTED); strides are element counts, multiples of 8, each at
+ * least one layer (ignored for L = 1).  All tensors 16-byte aligned.  Two
+ * calls that share a workspace must be ordered on the device.  A bounded
+ * device-side wait that gives up turns the affected output rows into NaN.
+ */
+size_t gv_verify_attention_layers_workspace(const gv_attn_shape* s, int L);
+int gv_verify_attention_layers(const gv_attn_shape* s, int L, const void* q, int64_t q_layer_stride,
+                               const void* k_new, int64_t k_layer_stride, const void* v_new,
+                               int64_t v_layer_stride, const void* cacheK, const void* cacheV,
+                               int64_t cache_layer_stride, const int32_t* prefix_len, const float* rope,
+                               const uint64_t* anc, void* treeK, void* treeV, void* out, void* workspace,
+                               size_t ws_bytes, void* stream);
+
+/*
  * gv_lmhead_select -- LM head fused with the per-node selection.
  * Section 3 / Eq. 1: the LM head maps a final hidden feature to a token;
  * Section 4.1 ranks candidates by their top-k; Section 5 decodes at T in {0,1}.

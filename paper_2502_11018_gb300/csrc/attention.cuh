@@ -35,6 +35,35 @@ struct AttnArgs {
     int tiles;        // M tiles of 128 query rows per (sequence, KV head); unit = (b, g, tile)
 };
 
+// gv_verify_attention_layers: workspace plan and call (attention_layers_sm103.cu).
+struct AttnLayersPlan {
+    int T;            // 128-row M tiles per (sequence, KV head): 1 or 2
+    int ctas;         // CTAs of the persistent kernel (one per SM)
+    int ncnt;         // arrival counters, L * B * Hkv
+    size_t q_rot, cnt, part, part_lse, total;   // byte offsets into the workspace
+};
+struct AttnLayersCall {
+    int L, B, N, Hq, Hkv, S_max;
+    const void* q;
+    long long q_ls;   // layer strides in elements
+    const void* k_new;
+    long long k_ls;
+    const void* v_new;
+    long long v_ls;
+    const void* cacheK;
+    const void* cacheV;
+    long long cache_ls;
+    const int32_t* prefix_len;
+    const float* rope;
+    const uint64_t* anc;
+    void* treeK;
+    void* treeV;
+    void* out;
+    void* workspace;
+};
+AttnLayersPlan attn_layers_plan(int L, int B, int N, int Hq, int Hkv);
+int launch_attn_layers(const AttnLayersCall& c, cudaStream_t st);
+
 int launch_rope_table(const int32_t* pos, int B, int N, int d, float base, float* rope,
                       cudaStream_t st);
 int launch_rope_tree_f32(const AttnArgs& a, cudaStream_t st);

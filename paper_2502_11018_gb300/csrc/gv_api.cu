@@ -383,6 +383,71 @@ int gv_rope_apply(const gv_attn_shape* s, int L, const void* q, size_t q_layer_s
     return launch_rope_apply(k_new, k_layer_stride, L, s->B, s->N, s->Hkv, rope, k_out, st);
 }
 
+static int attn_layers_shape_ok(const gv_attn_shape* s, int L) {
+    return s && s->dt == GV_BF16 && s->d == 128 && L >= 1 && s->B >= 1 && s->B <= 64 && s->N >= 1 &&
+           s->N <= 64 && s->Hkv >= 1 && s->Hq >= s->Hkv && s->Hq % s->Hkv == 0 &&
+           (s->Hq / s->Hkv) * s->N <= 256 && s->S_max >= 1;
+}
+
+size_t gv_verify_attention_layers_workspace(const gv_attn_shape* s, int L) {
+    if (!attn_layers_shape_ok(s, L)) return 0;
+    return attn_layers_plan(L, s->B, s->N, s->Hq, s->Hkv).total;
+}
+
+int gv_verify_attention_layers(const gv_attn_shape* s, int L, const void* q, int64_t q_layer_stride,
+                               const void* k_new, int64_t k_layer_stride, const void* v_new, int64_t v_layer_stride,
+                               const void* cacheK, const void* cacheV, int64_t cache_layer_stride,
+                               const int32_t* prefix_len, const float* rope, const uint64_t* anc, void* treeK,
+                               void* treeV, void* out, void* workspace, size_t ws_bytes, void* stream) {
+    clear_error();
+    if (!attn_layers_shape_ok(s, L)) {
+        set_error("gv_verify_attention_layers: unsupported shape (bf16, d = 128, L >= 1, 1 <= B <= 64, "
+                  "1 <= N <= 64, G * N <= 256 needed)");
+        return s ? GV_ERR_UNSUPPORTED : GV_ERR_ARG;
+    }
+    const long long nq = (long long)s->B * s->N * s->Hq * 128, nk = (long long)s->B * s->N * s->Hkv * 128;
+    const long long nc = (long long)s->B * s->Hkv * s->S_max * 128;
+    GV_CHECK_ARG((L == 1 || (q_layer_stride >= nq && k_layer_stride >= nk && v_layer_stride >= nk &&
+                             cache_layer_stride >= nc)) &&
+                     q_layer_stride % 8 == 0 && k_layer_stride % 8 == 0 && v_layer_stride % 8 == 0 &&
+                     cache_layer_stride % 8 == 0 && q_layer_stride >= 0 && k_layer_stride >= 0 &&
+                     v_layer_stride >= 0 && cache_layer_stride >= 0,
+                 "gv_verify_attention_layers: layer strides (elements) must cover a layer and be multiples of 8");
+    const void* ptrs[] = {q, k_new, v_new, cacheK, cacheV, rope, treeK, treeV, out};
+    for (const void* p : ptrs)
+        GV_CHECK_ARG(p && aligned16(p), "gv_verify_attention_layers: tensor null or not 16-byte aligned");
+    GV_CHECK_ARG(prefix_len && anc && ((uintptr_t)anc & 7u) == 0, "gv_verify_attention_layers: null index pointer");
+    const AttnLayersPlan plan = attn_layers_plan(L, s->B, s->N, s->Hq, s->Hkv);
+    GV_CHECK_ARG(workspace && ((uintptr_t)workspace & 255u) == 0,
+                 "gv_verify_attention_layers: workspace null or not 256-byte aligned");
+    GV_CHECK_ARG(ws_bytes >= plan.total, "gv_verify_attention_layers: workspace %zu < %zu bytes", ws_bytes,
+                 plan.total);
+    AttnLayersCall c{};
+    c.L = L;
+    c.B = s->B;
+    c.N = s->N;
+    c.Hq = s->Hq;
+    c.Hkv = s->Hkv;
+    c.S_max = s->S_max;
+    c.q = q;
+    c.q_ls = L == 1 ? nq : q_layer_stride;
+    c.k_new = k_new;
+    c.k_ls = L == 1 ? nk : k_layer_stride;
+    c.v_new = v_new;
+    c.v_ls = L == 1 ? nk : v_layer_stride;
+    c.cacheK = cacheK;
+    c.cacheV = cacheV;
+    c.cache_ls = L == 1 ? nc : cache_layer_stride;
+    c.prefix_len = prefix_len;
+    c.rope = rope;
+    c.anc = anc;
+    c.treeK = treeK;
+    c.treeV = treeV;
+    c.out = out;
+    c.workspace = workspace;
+    return launch_attn_layers(c, as_stream(stream));
+}
+
 size_t gv_lmhead_workspace(int rows, int H, int V, int dt, int mode, int k) {
     if (rows < 1 || H < 1 || V < 1 || mode < 0 || mode > 2) return 0;
     if (mode == GV_SELECT_TOPK && (k < 1 || k > 16)) return 0;

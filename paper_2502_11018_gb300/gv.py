@@ -34,6 +34,7 @@ GV_LINEAR_STORE, GV_LINEAR_ADD, GV_LINEAR_SWIGLU, GV_LINEAR_SILU = 0, 1, 2, 3
 # Every symbol include/gv.h declares.
 EXPORTS = ("gv_tree_build", "gv_rope_table", "gv_verify_attention_workspace", "gv_verify_attention",
            "gv_verify_attention_split", "gv_verify_attention_merge", "gv_rope_apply",
+           "gv_verify_attention_layers_workspace", "gv_verify_attention_layers",
            "gv_lmhead_workspace", "gv_lmhead_select", "gv_lmhead_argmax_noalloc",
            "gv_accept_workspace", "gv_accept",
            "gv_kv_compact", "gv_rmsnorm", "gv_linear_workspace", "gv_linear", "gv_linear_qkv_workspace",
@@ -59,6 +60,7 @@ _vp = ctypes.c_void_p
 _i = ctypes.c_int
 _f = ctypes.c_float
 _sz = ctypes.c_size_t
+_i64 = ctypes.c_int64
 
 
 def lib():
@@ -78,6 +80,9 @@ def lib():
         "gv_verify_attention_split": ([ctypes.POINTER(gv_attn_shape)] + [_vp] * 12 + [_sz, _vp], _i),
         "gv_verify_attention_merge": ([ctypes.POINTER(gv_attn_shape), _vp, _vp, _sz, _vp], _i),
         "gv_rope_apply": ([ctypes.POINTER(gv_attn_shape), _i, _vp, _sz, _vp, _sz, _vp, _vp, _vp, _vp], _i),
+        "gv_verify_attention_layers_workspace": ([ctypes.POINTER(gv_attn_shape), _i], _sz),
+        "gv_verify_attention_layers": ([ctypes.POINTER(gv_attn_shape), _i, _vp, _i64, _vp, _i64, _vp, _i64,
+                                        _vp, _vp, _i64] + [_vp] * 7 + [_sz, _vp], _i),
         "gv_lmhead_workspace": ([_i, _i, _i, _i, _i, _i], _sz),
         "gv_lmhead_select": ([_vp, _vp, _i, _i, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp,
                               _sz, _vp], _i),
@@ -217,6 +222,38 @@ def gv_verify_attention(shape, q, k_new, v_new, cacheK, cacheV, prefix_len, rope
         _ptr(rope, "rope"), _ptr(anc, "anc"), _ptr(treeK, "treeK"), _ptr(treeV, "treeV"),
         _ptr(out, "out"), _ptr(workspace, "workspace"), workspace.numel() * workspace.element_size(),
         _stream(stream)))
+
+
+def gv_verify_attention_layers_workspace(shape, L):
+    return int(lib().gv_verify_attention_layers_workspace(ctypes.byref(shape), int(L)))
+
+
+def _layered(t, name, L):
+    """(pointer, layer stride in elements) of a [L][...] CUDA tensor whose
+    layers are each contiguous (any layer stride, e.g. views of a packed
+    per-layer buffer)."""
+    if not (isinstance(t, torch.Tensor) and t.is_cuda and t[0].is_contiguous()):
+        raise ValueError(f"{name}: CUDA tensor whose layers are contiguous expected")
+    return ctypes.c_void_p(t.data_ptr()), (t.stride(0) if L > 1 else t[0].numel())
+
+
+def gv_verify_attention_layers(shape, q, k_new, v_new, cacheK, cacheV, prefix_len, rope, anc, treeK, treeV,
+                               out, workspace, stream=None):
+    """The attention of L layers in one call (see include/gv.h): q, k_new,
+    v_new, cacheK, cacheV are [L][...] with contiguous layers; treeK, treeV
+    and out packed [L][...]."""
+    L = q.shape[0]
+    qp, qs = _layered(q, "q", L)
+    kp, ks = _layered(k_new, "k_new", L)
+    vp, vs = _layered(v_new, "v_new", L)
+    ckp, cs = _layered(cacheK, "cacheK", L)
+    cvp, cs2 = _layered(cacheV, "cacheV", L)
+    if cs != cs2:
+        raise ValueError("cacheK and cacheV need the same layer stride")
+    return _check("gv_verify_attention_layers", lib().gv_verify_attention_layers(
+        ctypes.byref(shape), L, qp, qs, kp, ks, vp, vs, ckp, cvp, cs, _ptr(prefix_len, "prefix_len"),
+        _ptr(rope, "rope"), _ptr(anc, "anc"), _ptr(treeK, "treeK"), _ptr(treeV, "treeV"), _ptr(out, "out"),
+        _ptr(workspace, "workspace"), workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def gv_lmhead_workspace(rows, H, V, dt, mode, k=1):

@@ -5,12 +5,13 @@ five calls of include/gv.h in order on one stream (GRIFFIN Section 3: draft,
 then one verify forward over every draft token, then accept):
 
 1. ``gv_tree_build`` and ``gv_rope_table`` (RoPE cos/sin shared by all layers);
-2. ``gv_verify_attention_split`` for every layer (per-layer tree K/V scratch), each
-   layer's ``gv_verify_attention_merge`` on a second stream: a layer's queries,
-   keys and values are inputs of the step, so no layer waits for an earlier
-   layer's merged output, and the merges run beside the next layers' splits
-   (a workspace per layer); on the bf16 path one ``gv_rope_apply`` rotates
-   every layer's queries and tree keys ahead of the splits;
+2. the attention of every layer.  A layer's queries, keys and values are
+   inputs of the step, so the layers are independent problems: on the bf16
+   path (G * N <= 256) one ``gv_verify_attention_layers`` call runs all of
+   them in one persistent launch; otherwise ``gv_verify_attention_split`` for
+   every layer (per-layer tree K/V scratch), each layer's
+   ``gv_verify_attention_merge`` on a second stream beside the next layers'
+   splits (a workspace per layer);
 3. ``gv_lmhead_select`` (argmax for T = 0, fp32 logits + LSE for T > 0);
 4. ``gv_accept``;
 5. ``gv_kv_compact`` into every layer's cache.
@@ -33,7 +34,10 @@ class VerifyStep:
     # per layer, LLaMA-3-8B shape).
     ATTN_SLOTS = None
 
-    def __init__(self, inp: StepInputs):
+    def __init__(self, inp: StepInputs, layers_call=None):
+        """``layers_call``: run every layer's attention in one
+        gv_verify_attention_layers call (None: whenever the shape allows it;
+        False: the per-layer split/merge calls)."""
         cfg = inp.cfg
         self.inp = inp
         self.cfg = cfg
@@ -60,9 +64,14 @@ class VerifyStep:
         self.attn_ws_slots = [torch.empty(max(ws, 256), dtype=torch.uint8, device=dev) for _ in range(slots)]
         self.attn_ws = self.attn_ws_slots[0]
         self.merge_stream = torch.cuda.Stream(device=dev)
+        # bf16 with G * N <= 256: every layer's attention in one call
+        self.layers_call = gv.gv_verify_attention_layers_workspace(self.shape, L) > 0 and layers_call is not False
+        if self.layers_call:
+            self.attn_ws_layers = torch.empty(gv.gv_verify_attention_layers_workspace(self.shape, L),
+                                              dtype=torch.uint8, device=dev)
         # bf16 (d = 128): every layer's queries and tree keys are rotated by
         # one gv_rope_apply ahead of the splits, which then take rope = NULL
-        self.prerotate = self.dt_code == gv.GV_BF16 and d == 128
+        self.prerotate = not self.layers_call and self.dt_code == gv.GV_BF16 and d == 128
         if self.prerotate:
             self.q_rot = torch.empty(L, B, N, Hq, d, dtype=dt, device=dev)
             self.k_rot = torch.empty(L, B, N, Hkv, d, dtype=dt, device=dev)
@@ -109,14 +118,26 @@ class VerifyStep:
                                self.attn_ws, stream)
 
     def attention_layers(self, stream=None, ready=None):
-        """Every layer: the splits on ``stream`` in layer order, each layer's
-        merge on ``merge_stream`` after its split.  ``ready`` maps a layer to
-        an event its split waits for (its inputs' copy).  The caller joins
-        the merges with ``join_merges`` before it needs the outputs (or ends
-        a graph capture)."""
+        """Every layer's attention: one ``gv_verify_attention_layers`` call
+        (one per group of layers when ``ready`` is given); else the splits on
+        ``stream`` in layer order, each layer's merge on ``merge_stream`` after
+        its split.  ``ready`` maps a layer to an event that the layers from it
+        on wait for (their inputs' copy).  The caller joins the merges with
+        ``join_merges`` before it needs the outputs (or ends a graph
+        capture)."""
         i = self.inp
         L = self.cfg["L"]
         cur = stream if stream is not None else torch.cuda.current_stream()
+        if self.layers_call:
+            # one call per group of layers whose inputs arrive together
+            starts = sorted(ready) if ready is not None else [0]
+            for a, b in zip(starts, starts[1:] + [L]):
+                if ready is not None:
+                    cur.wait_event(ready[a])
+                gv.gv_verify_attention_layers(self.shape, i.q[a:b], i.k_new[a:b], i.v_new[a:b], i.cacheK[a:b],
+                                              i.cacheV[a:b], i.prefix_len, self.rope, self.anc, self.treeK[a:b],
+                                              self.treeV[a:b], self.attn_out[a:b], self.attn_ws_layers, cur)
+            return
         side = self.merge_stream
         side.wait_stream(cur)
         n = len(self.attn_ws_slots)
@@ -143,6 +164,8 @@ class VerifyStep:
             self._merge_ev[layer].record(side)
 
     def join_merges(self, stream=None):
+        if self.layers_call:
+            return    # (no merges on a second stream)
         cur = stream if stream is not None else torch.cuda.current_stream()
         cur.wait_stream(self.merge_stream)
 

@@ -112,7 +112,18 @@ def test_step_from_host_matches_device(name, layers):
     cfg = inputs.config(name)
     inp = inputs.make_step_inputs(cfg, 11, device="cpu", layers=layers)
     ref = VerifyStep(to_device(inp, dev))
-    ref.run()
+    # the reference issues the attention in the host-fed step's layer groups
+    # (one multi-layer call per group cuts the work the same way)
+    ready = {}
+    for a, _ in VerifyStep._copy_groups(layers):
+        ready[a] = torch.cuda.Event()
+        ready[a].record()
+    ref.tree()
+    ref.attention_layers(ready=ready)
+    ref.lmhead()
+    ref.accept()
+    ref.compact()
+    ref.join_merges()
     torch.cuda.synchronize()
     step = VerifyStep(to_device(inp, dev))
     host, res = step.host_buffers()
@@ -137,13 +148,13 @@ def test_step_from_host_matches_device(name, layers):
 
 @pytest.mark.parametrize("name,layers", [("llama3_8b", 7), ("tiny_f32", 4), ("llama3_8b_chain_b16", 4)])
 def test_side_merges_match_sequential_layers(name, layers):
-    # The step's schedule (splits in layer order, each merge on a second
+    # The per-layer schedule (splits in layer order, each merge on a second
     # stream, workspaces in rotation) gives the outputs of calling
     # gv_verify_attention layer by layer, bit for bit, eagerly and replayed.
     dev = device()
     cfg = inputs.config(name)
     inp = inputs.make_step_inputs(cfg, 13, device="cpu", layers=layers)
-    step = VerifyStep(to_device(inp, dev))
+    step = VerifyStep(to_device(inp, dev), layers_call=False)
     step.tree()
     for layer in range(layers):
         step.attention(layer)
@@ -170,3 +181,38 @@ def test_side_merges_match_sequential_layers(name, layers):
     g.replay()
     torch.cuda.synchronize()
     assert torch.equal(step.attn_out, seq[0])
+
+
+@pytest.mark.parametrize("name,layers", [("llama3_8b", 6), ("llama3_8b_chain_b16", 3), ("llama2_7b", 2)])
+def test_layers_call_matches_per_layer_schedule(name, layers):
+    # One gv_verify_attention_layers call for every layer against the
+    # per-layer schedule: the tree K/V scratch bit for bit, the outputs within
+    # the attention tolerance (the two cut the keys differently), eagerly and
+    # replayed from a CUDA graph (the replays repeat the eager bits).
+    dev = device()
+    cfg = inputs.config(name)
+    inp = inputs.make_step_inputs(cfg, 17, device="cpu", layers=layers)
+    d_inp = to_device(inp, dev)
+    per = VerifyStep(d_inp, layers_call=False)
+    per.tree()
+    per.attention_layers()
+    per.join_merges()
+    step = VerifyStep(d_inp)
+    assert step.layers_call
+    step.tree()
+    step.attention_layers()
+    torch.cuda.synchronize()
+    assert torch.equal(step.treeK, per.treeK) and torch.equal(step.treeV, per.treeV)
+    for layer in range(layers):
+        assert rel_err(f64(step.attn_out[layer]), f64(per.attn_out[layer])) <= TOL_ATTN["bf16"]
+    eager = step.attn_out.clone()
+    step.attn_out.zero_()
+    step.attn_ws_layers.fill_(0xFF)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step.attention_layers(torch.cuda.current_stream())
+    g.replay()
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(step.attn_out, eager)
