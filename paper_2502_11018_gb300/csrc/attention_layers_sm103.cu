@@ -775,6 +775,33 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
                 pdl_wait();
                 waited = true;
             }
+            // A piece of a unit cut between CTAs: the unit's pieces are one in
+            // every CTA of [cf, cl] whose range is not empty (ranges are empty
+            // when there are fewer blocks than CTAs).  When the unit has two
+            // pieces and the other one has already arrived (an acquiring read
+            // of the unit's counter), this piece combines the two straight
+            // from its accumulators and the other's partial rows; otherwise it
+            // writes its own partial rows and counts itself (below).
+            const long long U0 = pc.u0;
+            int cf = 0, cl = -1, npieces = 0, other_slot = -1;
+            bool combine = false;
+            if (!pc.direct) {
+                cf = cta_of(U0, W, C);
+                cl = cta_of(U0 + pc.nb - 1, W, C);
+                for (int cc = cf; cc <= cl; ++cc) {
+                    const long long sc = (long long)cc * W / C;
+                    if (sc == (long long)(cc + 1) * W / C) continue;
+                    ++npieces;
+                    if (cc != c) other_slot = 2 * cc + (U0 <= sc ? 0 : 1);
+                }
+                if (t_id == 0) {
+                    const bool ready = npieces == 2 && atomicAdd(a.cnt + pc.unit, 0) == 1;
+                    __threadfence();
+                    *last_flag = ready ? 2 : 0;
+                }
+                named_bar_sync(1, AL_NSM);
+                combine = *last_flag == 2;
+            }
             // Rows of this piece: with two tiles each stream writes its tile's
             // rows; with one tile the two accumulators (disjoint key sets of
             // the same rows) combine, and stream s writes d columns 64 s ..
@@ -798,7 +825,7 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
             const int c_lo = T == 2 ? 0 : 64 * s, c_n = T == 2 ? 128 : 64;   // d columns this thread writes
             __nv_bfloat16* dst = nullptr;
             if (rv) {
-                if (pc.direct) {
+                if (pc.direct || combine) {
                     const int i = qr / G, h = pc.g * G + qr % G;
                     dst = a.out + ((((size_t)pc.l * a.B + pc.b) * N + i) * a.Hq + h) * 128;
                 } else {
@@ -806,11 +833,31 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
                 }
             }
             const uint32_t o_other = lane_base + AL_OCOL + 128u * (uint32_t)(1 - s);
+            // (combining: the other piece's log2-sum-exp and partial columns,
+            // all loads issued at once)
+            uint4 pr[16];
+            float a_self = 1.f, a_part = 0.f;
+            if (combine && rv) {
+                const size_t prow = ((size_t)other_slot * T + tile) * 128 + row;
+                const float lse_o = __ldcg(a.part_lse + prow);
+                const uint4* src = reinterpret_cast<const uint4*>(a.part + prow * 128 + c_lo);
+#pragma unroll
+                for (int q = 0; q < 16; ++q)
+                    if (q < c_n / 8) pr[q] = __ldcg(src + q);
+                const float lse_s = ltot > 0.f ? M + log2f(ltot) : -INFINITY;
+                const float Mc = fmaxf(lse_s, lse_o);
+                const float es = lse_s == -INFINITY ? 0.f : fast_exp2(lse_s - Mc);
+                const float eo = lse_o == -INFINITY ? 0.f : fast_exp2(lse_o - Mc);
+                a_self = es / (es + eo);
+                a_part = eo / (es + eo);                     // (NaN when the other gave up)
+            }
             if (ok) {
                 tc_fence_after();
                 const float inv = ltot > 0.f ? 1.0f / ltot : 0.f;
-                const float fs = w_self * inv, fo = w_other * inv;
-                for (int c0 = 0; c0 < c_n; c0 += 16) {
+                const float fs = w_self * inv * a_self, fo = w_other * inv * a_self;
+#pragma unroll
+                for (int c0 = 0; c0 < 128; c0 += 16) {
+                    if (c0 >= c_n) break;
                     // (the columns of O this thread writes: c_lo + c0 ..)
                     uint32_t os[16], oo[16];
                     if (has_self) tmem_ld16(ocol + (uint32_t)(c_lo + c0), os);
@@ -829,38 +876,40 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
                                 v0 = fmaf(__uint_as_float(oo[2 * u]), fo, v0);
                                 v1 = fmaf(__uint_as_float(oo[2 * u + 1]), fo, v1);
                             }
+                            if (combine) {
+                                const uint4 q4 = pr[c0 / 8 + (u >> 2)];
+                                const uint32_t pw = (u & 3) == 0 ? q4.x : (u & 3) == 1 ? q4.y : (u & 3) == 2 ? q4.z : q4.w;
+                                const float2 f = unpack_bf16(pw);
+                                v0 = fmaf(f.x, a_part, v0);
+                                v1 = fmaf(f.y, a_part, v1);
+                            }
                             pv[u] = pack_bf16(v0, v1);
                         }
                         st_global_v8(dst + c_lo + c0, pv);
                     }
                 }
             } else if (dst) {
-                // Gave up: NaN rows (whole piece) or an invalid partial.
-                const uint32_t fill = pc.direct ? pack_bf16(NAN, NAN) : 0u;
+                // Gave up: NaN rows (whole piece, or combined) or an invalid partial.
+                const uint32_t fill = (pc.direct || combine) ? pack_bf16(NAN, NAN) : 0u;
                 const uint32_t pv[8] = {fill, fill, fill, fill, fill, fill, fill, fill};
                 for (int e = 0; e < c_n; e += 16) st_global_v8(dst + c_lo + e, pv);
             }
-            if (!pc.direct && rv && (T == 2 || s == 0))
+            if (!pc.direct && !combine && rv && (T == 2 || s == 0))
                 a.part_lse[((size_t)pc.slot * T + tile) * 128 + row] =
                     ok ? (ltot > 0.f ? M + log2f(ltot) : -INFINITY) : NAN;
             // O has been read: the next piece's PV may overwrite it.
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(o_free);
-            if (!pc.direct) {
+            if (combine) {
+                // (the other piece had arrived: the unit is done)
+                if (t_id == 0) a.cnt[pc.unit] = 0;   // ready for the next call
+            } else if (!pc.direct) {
                 // Count this piece in the unit's arrivals; the last piece to
-                // arrive combines the unit's pieces into the output.  The
-                // unit's pieces: one in every CTA of [cf, cl] whose range is
-                // not empty (ranges are empty when there are fewer blocks than
-                // CTAs).
+                // arrive combines the unit's pieces into the output.
                 __threadfence();
                 named_bar_sync(1, AL_NSM);
-                const long long U0 = pc.u0, U1 = pc.u0 + pc.nb;
-                const int cf = cta_of(U0, W, C), cl = cta_of(U1 - 1, W, C);
                 if (t_id == 0) {
-                    int npieces = 0;
-                    for (int cc = cf; cc <= cl; ++cc)
-                        npieces += (long long)cc * W / C < (long long)(cc + 1) * W / C ? 1 : 0;
                     const int old = atomicAdd(a.cnt + pc.unit, 1);
                     __threadfence();
                     *last_flag = old == npieces - 1 ? 1 : 0;
