@@ -133,7 +133,9 @@ int gv_tree_build(const int32_t* parents, const int32_t* prefix_len, int B, int 
  * Every layer of the verify forward pass (Section 3) rotates the draft
  * tokens' queries and keys at the same positions, so the angles are formed
  * once: rope[b][i][j] = {cos(a), sin(a)} with a = pos[b][i] * rope_base^(-2j/d)
- * computed in double and rounded to fp32, for j < d/2 (rotate-half RoPE).
+ * for j < d/2 (rotate-half RoPE).  The angle is formed and reduced modulo
+ * 2 pi in double; cos and sin of the remainder are within 3e-7 of the exact
+ * values, stored as fp32.
  *
  *   pos   int32 [B][N]          from gv_tree_build
  *   rope  fp32  [B][N][d/2][2]  out

@@ -15,35 +15,54 @@
 // output; attn_combine_kernel rescales and sums the splits.  Query rows of one
 // KV head are its G query heads x N nodes (row = head_in_group * N + node), so
 // every K/V tile is read once for all heads that share it.
+#include <cmath>
+
 #include "gv_internal.cuh"
 #include "attention.cuh"
 
 namespace gv {
 
 // -------------------------------------------------------------- rope table --
-// One thread per (sequence, node, frequency j < d/2): the angle
-// pos * base^(-2j/d) is formed in double once per verify step and stored as
-// fp32 (cos, sin); every layer's RoPE reads this table.
+// One thread per (sequence, node, frequency j < d/2).  The frequencies
+// base^(-2j/d) arrive from the host in double (one pow per frequency and
+// call); the angle a = pos * base^(-2j/d) is formed in double and reduced
+// modulo 2 pi there (2 pi as the sum of two doubles, each product taken in a
+// fused multiply-add, so a - k 2pi_hi is rounded once), so r = a - 2 pi k in
+// [-pi, pi] keeps double accuracy.  r = r_hi + r_lo in two
+// floats; cos and sin of r_hi in fp32 and one first-order step in r_lo give
+// cos(r), sin(r) to a few fp32 ulps, stored as fp32 (cos, sin).  (Double
+// sin/cos would cost a hundred fp64 operations per thread.)
+struct RopeFreqs {
+    double theta[128];
+};
+
 __global__ void __launch_bounds__(64)
-rope_table_kernel(const int32_t* __restrict__ pos, int B, int N, int d, double base,
+rope_table_kernel(const int32_t* __restrict__ pos, int B, int N, int half, RopeFreqs f,
                   float2* __restrict__ rope) {
-    const int half = d >> 1;
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
     const int j = idx % half;
-    const double theta = pow(base, -2.0 * (double)j / (double)d);   // (before the wait)
+    const double theta = f.theta[j];
     pdl_wait();
     pdl_trigger();
     if (idx >= B * N * half) return;
-    const int bi = idx / half;
-    double sn, cs;
-    sincos((double)pos[bi] * theta, &sn, &cs);
-    rope[idx] = make_float2((float)cs, (float)sn);
+    const double a = (double)pos[idx / half] * theta;
+    constexpr double kTwoPiHi = 6.283185307179586;            // 2 pi rounded to double
+    constexpr double kTwoPiLo = 2.4492935982947064e-16;       // 2 pi - kTwoPiHi
+    constexpr double kInvTwoPi = 0.15915494309189535;
+    const double k = rint(a * kInvTwoPi);
+    const double r = fma(-k, kTwoPiLo, fma(-k, kTwoPiHi, a));
+    const float rh = (float)r, rl = (float)(r - (double)rh);
+    float sh, ch;
+    sincosf(rh, &sh, &ch);
+    rope[idx] = make_float2(fmaf(-sh, rl, ch), fmaf(ch, rl, sh));
 }
 
 int launch_rope_table(const int32_t* pos, int B, int N, int d, float base, float* rope,
                       cudaStream_t st) {
-    const int total = B * N * (d / 2);
-    launch_pdl(rope_table_kernel, dim3((total + 63) / 64), dim3(64), 0, st, pos, B, N, d, (double)base,
+    const int half = d / 2, total = B * N * half;
+    RopeFreqs f{};
+    for (int j = 0; j < half; ++j) f.theta[j] = std::pow((double)base, -2.0 * (double)j / (double)d);
+    launch_pdl(rope_table_kernel, dim3((total + 63) / 64), dim3(64), 0, st, pos, B, N, half, f,
                reinterpret_cast<float2*>(rope));
     return check_launch("rope_table_kernel");
 }
