@@ -17,11 +17,16 @@ ranks divided by the slowest rank's time.
 """
 
 import argparse
+import contextlib
+import ctypes
+import hashlib
 import json
 import os
+import platform
 import statistics
 import subprocess
 import sys
+import threading
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -35,13 +40,41 @@ from paper_2502_11018_gb300 import gv, inputs  # noqa: E402
 METRIC = "verify steps/s and accepted tok/s (LLaMA-3-8B shape, 60-node tree); % HBM roofline"
 UNIT = "verify_steps/s"
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one
-# ncu capture of the kernel as it is now, keyed by (kernel, workload); a kernel
-# changed since its capture has no entry.
+# ncu capture, keyed by (kernel, workload), with the SHA-256 of the kernel's
+# source files at capture time: when the sources have changed since, the
+# figure no longer describes the kernel and the line reports null.
 TRAFFIC = {
-    # attn_tc_kernel with queries and tree keys that arrive rotated (the merge
-    # kernel reads the partials from L2): profiles/attn_tc_llama3_8b_layer.md
-    ("verify_attention", "llama3_8b"): 17567403,
+    # tree_prep_kernel + attn_layers_kernel of one gv_verify_attention_layers
+    # call over the 32 layers (23.6 MB + 580.1 MB), per layer
+    ("verify_attention", "llama3_8b"): {
+        "bytes": 18865552,
+        "sources": ["paper_2502_11018_gb300/csrc/attention_layers_sm103.cu",
+                    "paper_2502_11018_gb300/csrc/attn_common.cuh", "paper_2502_11018_gb300/csrc/sm103.cuh"],
+        "sha256": "6b94506fc05301b2ffff00016fe1538d230ce20e113b580443b8e7892c6caf64"},
+    ("lmhead_select", "llama3_8b"): {
+        "bytes": 1058406656,
+        "sources": ["paper_2502_11018_gb300/csrc/lmhead_sm103.cu", "paper_2502_11018_gb300/csrc/sm103.cuh"],
+        "sha256": "9afeefd6a0f9ac9e367be9926dfb83772ce5117a48e99bd611f581fab3c5bdd6"},
 }
+OTHER_CONFIGS = ("llama2_7b", "llama2_13b_b4", "mixtral_attn", "tiny_f32")
+
+
+def sources_sha256(files):
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def traffic_of(kernel, workload):
+    e = TRAFFIC.get((kernel, workload))
+    if e is None:
+        return None
+    try:
+        return e["bytes"] if sources_sha256(e["sources"]) == e["sha256"] else None
+    except OSError:
+        return None
 
 
 def load_peaks():
@@ -136,8 +169,82 @@ def lmhead_bytes(cfg):
     return b
 
 
+class NvmlClocks:
+    """SM clock and clock-event reasons of the benchmark's GPU, read through
+    NVML (read-only queries, through ctypes) by a background thread about
+    every half millisecond; samples taken between start() and stop() count."""
+
+    REASONS = {0x8: "hw_slowdown", 0x40: "hw_thermal_slowdown", 0x20: "sw_thermal_slowdown",
+               0x4: "sw_power_cap"}
+    NVML_CLOCK_SM = 1
+
+    def __init__(self, device_index):
+        self.lib = self.h = None
+        self.samples = []
+        self.window = None
+        self._stop = threading.Event()
+        self._thread = None
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            uuid = getattr(torch.cuda.get_device_properties(device_index), "uuid", None)
+            ok = False
+            if uuid is not None:
+                u = str(uuid)
+                u = u if u.startswith("GPU-") else "GPU-" + u
+                ok = lib.nvmlDeviceGetHandleByUUID(u.encode(), ctypes.byref(h)) == 0
+            if not ok and lib.nvmlDeviceGetHandleByIndex_v2(device_index, ctypes.byref(h)) != 0:
+                return
+            self.reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                lib.nvmlDeviceGetCurrentClocksThrottleReasons
+            self.lib, self.h = lib, h
+        except (OSError, AttributeError):
+            self.lib = None
+
+    def _run(self):
+        clk, rs = ctypes.c_uint(), ctypes.c_ulonglong()
+        while not self._stop.is_set():
+            if self.lib.nvmlDeviceGetClockInfo(self.h, self.NVML_CLOCK_SM, ctypes.byref(clk)) == 0 and \
+                    self.reasons_fn(self.h, ctypes.byref(rs)) == 0:
+                self.samples.append((time.perf_counter(), clk.value, rs.value))
+            time.sleep(0.0005)
+
+    def begin(self):
+        """Start sampling (before the region, so the thread is running)."""
+        if self.lib is None:
+            return
+        self._thread = threading.Thread(target=self._run, daemon=True)
+        self._thread.start()
+        time.sleep(0.005)
+
+    def start(self):
+        self.window = [time.perf_counter(), None]
+
+    def stop(self):
+        if self.window is not None:
+            self.window[1] = time.perf_counter()
+
+    def end(self):
+        if self._thread is None or self.window is None:
+            return None
+        self._stop.set()
+        self._thread.join(timeout=5)
+        t0, t1 = self.window
+        inside = [x for x in self.samples if t0 <= x[0] <= t1]
+        if not inside:
+            return None
+        mx = ctypes.c_uint()
+        self.lib.nvmlDeviceGetMaxClockInfo(self.h, self.NVML_CLOCK_SM, ctypes.byref(mx))
+        reasons = sorted({n for _, _, r in inside for bit, n in self.REASONS.items() if r & bit})
+        return {"sm_mhz": statistics.median(c for _, c, _ in inside), "sm_max_mhz": float(mx.value),
+                "reasons": reasons, "samples": len(inside), "source": "nvml"}
+
+
 class ClockSampler:
-    """nvidia-smi clocks / throttle reasons sampled during the timed region."""
+    """nvidia-smi clocks / throttle reasons sampled during the timed region
+    (used where NVML cannot be loaded)."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -211,52 +318,128 @@ def event_time_ms(fn, iters, stream):
     return start.elapsed_time(end) / iters
 
 
-def oracle_step_sample(inp, cfg, ls, vs):
-    """Time the float64 oracle on a bounded sample of one step.
+def replay_times_ms(fn, iters, stream, flush=None):
+    """Time `iters` calls with one event pair each (events on the launching
+    stream): the mean and each call's time.  Back to back, the mean is over
+    the whole region; with `flush` (run between calls, outside the pairs: an
+    L2 flush for a working set that fits in L2) it is the mean of the calls."""
+    if flush is None:
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(iters + 1)]
+        ev[0].record(stream)
+        for i in range(iters):
+            fn()
+            ev[i + 1].record(stream)
+        ev[-1].synchronize()
+        per = [ev[i].elapsed_time(ev[i + 1]) for i in range(iters)]
+        return ev[0].elapsed_time(ev[-1]) / iters, per
+    pairs = []
+    for _ in range(iters):
+        flush()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        pairs.append((a, b))
+    pairs[-1][1].synchronize()
+    per = [a.elapsed_time(b) for a, b in pairs]
+    return sum(per) / iters, per
 
-    The sample is the whole step with attention on the first ``ls`` layers and
-    the LM head on the first ``vs`` vocabulary rows (acceptance then runs on
-    that slice).  Returns the full-step time extrapolated linearly in layers
-    and vocabulary rows, and the time the sample took.
-    """
+
+def percentiles(per):
+    q = sorted(per)
+
+    def at(f):
+        return q[min(len(q) - 1, max(0, int(round(f * (len(q) - 1)))))]
+    return {"ms_p10": at(0.10), "ms_p50": at(0.50), "ms_p90": at(0.90)}
+
+
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the machine)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.machine()
+
+
+def _openblas_thread_apis():
+    """(set, get) thread-count functions of every OpenBLAS library loaded in
+    this process (numpy's BLAS), for hosts without threadpoolctl."""
+    names = [("openblas_set_num_threads", "openblas_get_num_threads"),
+             ("scipy_openblas_set_num_threads64_", "scipy_openblas_get_num_threads64_"),
+             ("openblas_set_num_threads64_", "openblas_get_num_threads64_"),
+             ("scipy_openblas_set_num_threads", "scipy_openblas_get_num_threads")]
+    apis = []
+    try:
+        paths = set()
+        with open("/proc/self/maps") as f:
+            for line in f:
+                parts = line.split()
+                if len(parts) >= 6 and "openblas" in parts[-1].lower():
+                    paths.add(parts[-1])
+        for path in sorted(paths):
+            lib = ctypes.CDLL(path)
+            for sn, gn in names:
+                if hasattr(lib, sn) and hasattr(lib, gn):
+                    apis.append((getattr(lib, sn), getattr(lib, gn)))
+                    break
+    except OSError:
+        pass
+    return apis
+
+
+@contextlib.contextmanager
+def blas_threads(n):
+    """Run the block with numpy's BLAS and torch's CPU ops on n threads."""
+    import numpy  # noqa: F401  (loads the BLAS library)
+    prev_torch = torch.get_num_threads()
+    torch.set_num_threads(n)
+    try:
+        try:
+            from threadpoolctl import threadpool_limits
+        except ImportError:
+            threadpool_limits = None
+        if threadpool_limits is not None:
+            with threadpool_limits(n):
+                yield
+        else:
+            apis = _openblas_thread_apis()
+            prev = [g() for _, g in apis]
+            for sfn, _ in apis:
+                sfn(n)
+            try:
+                yield
+            finally:
+                for (sfn, _), v in zip(apis, prev):
+                    sfn(v)
+    finally:
+        torch.set_num_threads(prev_torch)
+
+
+def oracle_full_step(host_inp):
+    """Seconds the float64 oracle takes for one whole verify step: tree build,
+    every layer's tree attention, the whole LM head, acceptance and the
+    compaction of every layer's cache."""
     import oracle
-    from oracle.step import as_f64
-    T = cfg.get("temperature", 0.0)
-    P = as_f64(inp.prefix_len)
-    parents, tokens = as_f64(inp.parents), as_f64(inp.tokens)
     t0 = time.perf_counter()
-    depth, pos, anc, st = oracle.tree_build(parents, P)
-    tk, tv = [], []
-    for layer in range(ls):
-        _, k_, v_ = oracle.tree_attention(as_f64(inp.q[layer]), as_f64(inp.k_new[layer]),
-                                          as_f64(inp.v_new[layer]), as_f64(inp.cacheK[layer]),
-                                          as_f64(inp.cacheV[layer]), P, pos, anc, cfg["rope_base"])
-        tk.append(k_)
-        tv.append(v_)
-    t1 = time.perf_counter()
-    logits = oracle.lmhead_logits(as_f64(inp.h), as_f64(inp.W[:vs]))
-    t2 = time.perf_counter()
-    D = cfg["D"]
-    if T == 0.0:
-        choice, _ = oracle.select_argmax(logits)
-        path, alen, _, st = oracle.accept_greedy(parents, tokens, choice, D, st)
-    else:
-        B, N = parents.shape
-        path, alen, _, st, _ = oracle.accept_sampling(
-            parents, tokens % vs, logits.reshape(B, N, vs), as_f64(inp.draft_logits[..., :vs]),
-            as_f64(inp.u_acc), as_f64(inp.u_res), D, T, st)
-    import numpy as np
-    oracle.kv_compact(np.stack(tk), np.stack(tv), as_f64(inp.cacheK[:ls]), as_f64(inp.cacheV[:ls]),
-                      path, alen, P, st)
-    t3 = time.perf_counter()
-    est = (t1 - t0) * cfg["L"] / ls + (t2 - t1) * cfg["V"] / vs + (t3 - t2)
-    return est, t3 - t0
+    oracle.verify_step(host_inp)
+    return time.perf_counter() - t0
 
 
-def sample_desc(cfg, ls, vs, est, took):
-    return (f"float64 numpy oracle: whole step with attention on {ls} of {cfg['L']} layers and the "
-            f"LM head on {vs} of {cfg['V']} vocabulary rows; full-step time extrapolated linearly "
-            f"in layers and rows ({est:.2f} s/step; the sample took {took:.1f} s)")
+def full_step_desc(cfg):
+    return (f"one whole step of the float64 numpy oracle: tree build, all {cfg['L']} layers' tree attention, "
+            f"the LM head over all {cfg['V']} vocabulary rows, acceptance and the compaction of every layer's "
+            f"cache (inputs converted from the device copies inside the timing)")
 
 
 def host_inputs(cfg, seed, layers, dev_inp=None):
@@ -275,27 +458,18 @@ def host_inputs(cfg, seed, layers, dev_inp=None):
     return type(dev_inp)(**kw)
 
 
-def cpu_baseline(cfg, seed, dev_inp=None, budget_s=15.0):
-    """The oracle as it stands, timed on the host cores on a bounded sample
-    sized to roughly `budget_s` seconds."""
-    ls = min(cfg["L"], 4)
-    inp = host_inputs(cfg, seed, ls, dev_inp)
-    # Calibrate on one layer and an eighth of the vocabulary, then size the sample.
-    v8 = max(1, cfg["V"] // 8)
-    est1, took1 = oracle_step_sample(inp, cfg, 1, v8)
-    ls, vs = sample_size(cfg, est1, budget_s)
-    est, took = oracle_step_sample(inp, cfg, ls, vs)
-    return {"value": 1.0 / est, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": sample_desc(cfg, ls, vs, est, took), "seconds_per_step": est,
-            "layers": ls, "vocab_rows": vs}
-
-
-def sample_size(cfg, est_full, budget_s):
-    """Layers (<= 4) and vocabulary rows whose oracle time is about budget_s."""
-    frac = min(1.0, budget_s / max(est_full, 1e-6))
-    ls = max(1, min(4, int(round(cfg["L"] * frac))))
-    vs = max(256, min(cfg["V"], int(cfg["V"] * frac)))
-    return ls, vs
+def cpu_baseline(cfg, seed, dev_inp=None):
+    """The oracle as it stands, timed on the host cores: one whole step with
+    every core, and one on a single thread."""
+    inp = host_inputs(cfg, seed, cfg["L"], dev_inp)
+    cores = len(os.sched_getaffinity(0))
+    with blas_threads(cores):
+        t_all = oracle_full_step(inp)
+    with blas_threads(1):
+        t_one = oracle_full_step(inp)
+    return {"value": 1.0 / t_all, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": full_step_desc(cfg) + f"; {t_all:.2f} s on {cores} threads, {t_one:.2f} s on 1 thread",
+            "seconds_per_step": t_all, "seconds_per_step_1thread": t_one, "cpu_model": cpu_model()}
 
 
 def bench_config(cfg, world):
@@ -309,35 +483,38 @@ def bench_config(cfg, world):
 
 
 def run_reference(args):
-    """The reference arm: the float64 oracle on the host cores, each step a
-    bounded sample of the workload sized so the whole run takes a few minutes."""
+    """The reference arm: the float64 oracle on the host cores, every step one
+    whole verify step of the workload.  Steps run until --steps or until about
+    two minutes of steps have run; `steps` is the number that ran."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     cfg = inputs.config(args.config)
-    inp = host_inputs(cfg, args.seed, min(cfg["L"], 4))
-    budget = max(0.5, min(20.0, 150.0 / max(1, args.steps + args.warmup)))
-    est1, _ = oracle_step_sample(inp, cfg, 1, max(1, cfg["V"] // 8))
-    ls, vs = sample_size(cfg, est1, budget)
-    for _ in range(args.warmup):
-        oracle_step_sample(inp, cfg, ls, vs)
-    vals = []
-    t0 = time.perf_counter()
-    took = 0.0
-    for _ in range(args.steps):
-        est, tk = oracle_step_sample(inp, cfg, ls, vs)
-        vals.append(est)
-        took += tk
-    wall = time.perf_counter() - t0
-    v = 1.0 / statistics.mean(vals)
-    desc = sample_desc(cfg, ls, vs, statistics.mean(vals), took / max(1, args.steps))
-    line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": 1000.0 * statistics.mean(vals),
+    inp = host_inputs(cfg, args.seed, cfg["L"])
+    cores = len(os.sched_getaffinity(0))
+    budget_s = 120.0
+    wall0 = time.perf_counter()
+    with blas_threads(cores):
+        warm = min(args.warmup, 1)
+        for _ in range(warm):
+            oracle_full_step(inp)
+        times = []
+        t0 = time.perf_counter()
+        while len(times) < max(1, args.steps):
+            times.append(oracle_full_step(inp))
+            if time.perf_counter() - t0 + statistics.mean(times) > budget_s:
+                break
+    wall = time.perf_counter() - wall0
+    mean = statistics.mean(times)
+    v = 1.0 / mean
+    desc = full_step_desc(cfg) + f"; {len(times)} steps of {args.steps} requested (about {budget_s:.0f} s of steps)"
+    line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": len(times),
+            "steps_requested": args.steps, "warmup": warm, "ms_per_step": 1000.0 * mean,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded random weights, caches and draft trees)", "impl": "reference",
-            "config": bench_config(cfg, args.gpus),
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-                             "sample": desc},
+            "config": bench_config(cfg, args.gpus), **percentiles([1000.0 * t for t in times]),
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
+                             "cpu_model": cpu_model()},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "wall_s": wall}
     print(json.dumps(line), flush=True)
@@ -352,6 +529,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--seed", type=int, default=1000)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-other-configs", action="store_true",
+                    help="measure only --config (not also the other workloads under `configs`)")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--layers", type=int, default=0,
                     help="--kernel attention_layers: layers of the call (default: the workload's)")
@@ -417,16 +596,23 @@ def main():
         step.replay()
     torch.cuda.synchronize()
 
-    clocks = ClockSampler(local)
+    clocks = NvmlClocks(local)
+    smi = None
+    if clocks.lib is None:
+        smi = ClockSampler(local)
+    clocks.begin()
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize()
+    if smi is not None:
+        smi.start()
     clocks.start()
-    ms = event_time_ms(step.replay, args.steps, stream)
+    ms, per = replay_times_ms(step.replay, args.steps, stream)
     torch.cuda.synchronize()
+    clocks.stop()
     if dist is not None:
         dist.barrier()
-    clk = clocks.stop()
+    clk = smi.stop() if smi is not None else clocks.end()
     accept_len = step.accept_len.cpu().tolist()
     t_max = ms
     if dist is not None:
@@ -434,26 +620,8 @@ def main():
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         t_max = float(t.item())
 
-    # The two kernels that dominate the step, each timed alone (replayed from
-    # a CUDA graph on the stream it is launched on): the LM head, and the
-    # attention layers in order as the step runs them (splits in layer order,
-    # each layer's merge beside the next splits; the 32 layers' caches cycle
-    # through far more than L2 holds).
-    L = cfg["L"]
-    g_lm = graph_of(lambda: step.lmhead(torch.cuda.current_stream()))
-    lm_ms = event_time_ms(g_lm.replay, 20, stream)
-    g_attn = graph_of(lambda: (step.attention_layers(torch.cuda.current_stream()),
-                               step.join_merges(torch.cuda.current_stream())))
-    attn_ms = event_time_ms(g_attn.replay, 10, stream) / L
+    kernels = kernel_times(step, cfg, stream)
     peaks = load_peaks()
-    lm_gbs = lmhead_bytes(cfg) / (lm_ms * 1e-3) / 1e9
-    attn_gbs = attention_bytes(cfg) / (attn_ms * 1e-3) / 1e9
-    kernels = {
-        "lmhead_select": {"ms_per_launch": lm_ms, "launches_per_step": 1,
-                          "algorithmic_bytes": lmhead_bytes(cfg), "achieved_gbs": lm_gbs},
-        "verify_attention": {"ms_per_launch": attn_ms, "launches_per_step": L,
-                             "algorithmic_bytes": attention_bytes(cfg), "achieved_gbs": attn_gbs},
-    }
     dom = max(kernels, key=lambda k: kernels[k]["ms_per_launch"] * kernels[k]["launches_per_step"])
     dk = kernels[dom]
     sb = step_bytes(cfg, accept_len)
@@ -465,7 +633,7 @@ def main():
 
     line = {
         "metric": METRIC, "value": world * 1000.0 / t_max, "unit": UNIT, "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max, **percentiles(per),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg["dtype"],
         "data": "synthetic (seeded random weights, caches and draft trees)",
         "config": bench_config(cfg, world),
@@ -476,20 +644,86 @@ def main():
                          "peak_source": peaks["source"]},
         "roofline": {"kernel": dom, "bound": "hbm", "achieved": dk["achieved_gbs"],
                      "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                     "frac": dk["achieved_gbs"] / peaks["hbm_gbs"], "traffic": TRAFFIC.get((dom, cfg["name"])),
+                     "frac": dk["achieved_gbs"] / peaks["hbm_gbs"], "traffic": traffic_of(dom, cfg["name"]),
                      "ms_per_launch": dk["ms_per_launch"], "peak_source": peaks["source"]},
         "kernels": kernels,
         "gpu_launches": launches_per_step(cfg) * args.steps,
         "e2e": e2e,
         "clocks": clk,
     }
+    del step, inp
+    torch.cuda.empty_cache()
+    if not args.no_other_configs:
+        # The other workloads, each measured the same way in this process
+        # (per-replay events over max(--steps, 20) graph replays).
+        line["configs"] = {name: measure_config(name, args.seed + rank, max(args.steps, 20), args.warmup, dev,
+                                                stream, peaks)
+                           for name in OTHER_CONFIGS}
     if rank == 0 and not args.no_cpu_baseline:
-        cb = cpu_baseline(cfg, args.seed, dev_inp=inp)
-        line["cpu_baseline"] = {k: cb[k] for k in ("value", "unit", "cores", "kind", "sample")}
+        cb = cpu_baseline(cfg, args.seed)
+        line["cpu_baseline"] = {k: cb[k] for k in ("value", "unit", "cores", "kind", "sample",
+                                                   "seconds_per_step_1thread", "cpu_model")}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.destroy_process_group()
+
+
+def kernel_times(step, cfg, stream):
+    """The two kernels that dominate a step, each timed alone (replayed from a
+    CUDA graph on the stream it is launched on): the LM head, and the
+    attention layers in order as the step runs them (the layers' caches cycle
+    through far more than L2 holds)."""
+    L = cfg["L"]
+    g_lm = graph_of(lambda: step.lmhead(torch.cuda.current_stream()))
+    lm_ms = event_time_ms(g_lm.replay, 20, stream)
+    g_attn = graph_of(lambda: (step.attention_layers(torch.cuda.current_stream()),
+                               step.join_merges(torch.cuda.current_stream())))
+    attn_ms = event_time_ms(g_attn.replay, 10, stream) / L
+    peaks = load_peaks()
+    lm_gbs = lmhead_bytes(cfg) / (lm_ms * 1e-3) / 1e9
+    attn_gbs = attention_bytes(cfg) / (attn_ms * 1e-3) / 1e9
+    return {
+        "lmhead_select": {"ms_per_launch": lm_ms, "launches_per_step": 1, "algorithmic_bytes": lmhead_bytes(cfg),
+                          "achieved_gbs": lm_gbs, "frac": lm_gbs / peaks["hbm_gbs"]},
+        "verify_attention": {"ms_per_launch": attn_ms, "launches_per_step": L,
+                             "algorithmic_bytes": attention_bytes(cfg), "achieved_gbs": attn_gbs,
+                             "frac": attn_gbs / peaks["hbm_gbs"]},
+    }
+
+
+def measure_config(name, seed, steps, warmup, dev, stream, peaks):
+    """One workload's step: per-replay times of its CUDA graph, throughput,
+    HBM roofline fraction of the step and of its two dominant kernels."""
+    from paper_2502_11018_gb300.step import VerifyStep
+    cfg = inputs.config(name)
+    inp = inputs.make_step_inputs(cfg, seed, device=dev)
+    step = VerifyStep(inp)
+    step.capture()
+    for _ in range(max(warmup, 3)):
+        step.replay()
+    torch.cuda.synchronize()
+    # A working set that fits in the 129 MB L2 (the tiny workload) is flushed
+    # between replays by writing a 512 MB buffer.
+    flush = None
+    config = bench_config(cfg, 1)
+    if step_bytes(cfg, [cfg["D"]] * cfg["B"])["total"] < 256 * 2**20:
+        junk = torch.empty(512 * 2**20, dtype=torch.uint8, device=dev)
+        flush = lambda: junk.fill_(1)  # noqa: E731
+        config["l2"] = "flushed between replays (512 MB write, outside the timed pairs)"
+    ms, per = replay_times_ms(step.replay, steps, stream, flush)
+    accept_len = step.accept_len.cpu().tolist()
+    sb = step_bytes(cfg, accept_len)
+    gbs = sb["total"] / (ms * 1e-3) / 1e9
+    out = {"ms_per_step": ms, **percentiles(per), "steps": steps, "verify_steps_per_s": 1000.0 / ms,
+           "accepted_tok_per_s": sum(accept_len) * 1000.0 / ms, "accept_len": accept_len, "dtype": cfg["dtype"],
+           "config": config, "gpu_launches_per_step": launches_per_step(cfg),
+           "hbm_roofline": {"step_bytes": sb["total"], "achieved_gbs": gbs, "frac": gbs / peaks["hbm_gbs"],
+                            "peak_gbs": peaks["hbm_gbs"], "peak_source": peaks["source"]},
+           "kernels": kernel_times(step, cfg, stream)}
+    del step, inp
+    torch.cuda.empty_cache()
+    return out
 
 
 def run_kernel_only(args, cfg, dev):
