@@ -68,45 +68,50 @@ int launch_rope_table(const int32_t* pos, int B, int N, int d, float base, float
 }
 
 // ---------------------------------------------------------------- prologue --
-// fp32 path: one thread per (sequence, node, frequency) rotates that
-// frequency's pair of every query head (into the q_rot workspace, grouped by
-// KV head) and of every key head (into the tree K scratch), and copies v.
+// fp32 path: one thread per (sequence, node, frequency, head) rotates that
+// frequency's pair of one query head (into the q_rot workspace, grouped by
+// KV head) or of one key head (into the tree K scratch, copying v with it).
 __global__ void __launch_bounds__(128)
 rope_tree_f32_kernel(const float* __restrict__ q, const float* __restrict__ k_new,
                      const float* __restrict__ v_new, const float2* __restrict__ rope, int B, int N,
                      int Hq, int Hkv, int d, float* __restrict__ q_rot, float* __restrict__ treeK,
                      float* __restrict__ treeV, int q_rows_pad) {
     const int half = d >> 1;
-    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= B * N * half) return;
-    const int j = idx % half;
-    const int i = (idx / half) % N;
-    const int b = idx / (half * N);
-    const float2 r = rope[idx];
+    const int H = Hq + Hkv;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)B * N * half * H) return;
+    const int hh = (int)(idx % H);
+    const long long pidx = idx / H;                 // (b, i, j)
+    const int j = (int)(pidx % half);
+    const int i = (int)((pidx / half) % N);
+    const int b = (int)(pidx / ((long long)half * N));
+    const float2 r = rope[pidx];
     const float c = r.x, s = r.y;
     const int G = Hq / Hkv;
-    for (int h = 0; h < Hq; ++h) {
+    if (hh < Hq) {
+        const int h = hh;
         const size_t src = (((size_t)b * N + i) * Hq + h) * d;
         const float x0 = q[src + j], x1 = q[src + j + half];
         const int g = h / G, hl = h % G;
         const size_t dst = (((size_t)b * Hkv + g) * q_rows_pad + (size_t)hl * N + i) * d;
         q_rot[dst + j] = x0 * c - x1 * s;
         q_rot[dst + j + half] = x1 * c + x0 * s;
-    }
-    for (int g = 0; g < Hkv; ++g) {
+    } else {
+        const int g = hh - Hq;
         const size_t src = (((size_t)b * N + i) * Hkv + g) * d;
         const size_t dst = (((size_t)b * Hkv + g) * N + i) * d;
         const float x0 = k_new[src + j], x1 = k_new[src + j + half];
+        const float v0 = v_new[src + j], v1 = v_new[src + j + half];
         treeK[dst + j] = x0 * c - x1 * s;
         treeK[dst + j + half] = x1 * c + x0 * s;
-        treeV[dst + j] = v_new[src + j];
-        treeV[dst + j + half] = v_new[src + j + half];
+        treeV[dst + j] = v0;
+        treeV[dst + j + half] = v1;
     }
 }
 
 int launch_rope_tree_f32(const AttnArgs& a, cudaStream_t st) {
-    const int total = a.B * a.N * (a.d / 2);
-    rope_tree_f32_kernel<<<(total + 127) / 128, 128, 0, st>>>(
+    const long long total = (long long)a.B * a.N * (a.d / 2) * (a.Hq + a.Hkv);
+    rope_tree_f32_kernel<<<(unsigned)((total + 127) / 128), 128, 0, st>>>(
         static_cast<const float*>(a.q), static_cast<const float*>(a.k_new),
         static_cast<const float*>(a.v_new), reinterpret_cast<const float2*>(a.rope), a.B, a.N, a.Hq,
         a.Hkv, a.d, static_cast<float*>(a.q_rot), static_cast<float*>(a.treeK),
@@ -116,6 +121,8 @@ int launch_rope_tree_f32(const AttnArgs& a, cudaStream_t st) {
 
 // ----------------------------------------------------------------- combine --
 // One warp per output row (b, node, head): out = sum_s e^{m_s - M} o_s / sum_s e^{m_s - M} l_s.
+// Lane s reads split s's (m, l) (32 splits per pass), so the splits' loads are
+// in flight together; the partial rows follow four splits at a time.
 template <typename T, int D>
 __global__ void __launch_bounds__(256)
 attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ part_ml, int B,
@@ -128,18 +135,33 @@ attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ 
     const int r = hl * N + i;
     const size_t bg = (size_t)b * Hkv + g;
     float M = -INFINITY;
-    for (int s = 0; s < nsplit; ++s) M = fmaxf(M, part_ml[((bg * nsplit + s) * R + r) * 2]);
+    for (int s0 = 0; s0 < nsplit; s0 += 32)
+        if (s0 + lane < nsplit) M = fmaxf(M, part_ml[((bg * nsplit + s0 + lane) * R + r) * 2]);
+    M = warp_max(M);
     float L = 0.f;
     float acc[D / 32] = {};
-    for (int s = 0; s < nsplit; ++s) {
-        const size_t pr = (bg * nsplit + s) * R + r;
-        const float m = part_ml[pr * 2];
-        if (m == -INFINITY) continue;
-        const float wgt = __expf(m - M);
-        L += wgt * part_ml[pr * 2 + 1];
+    for (int s0 = 0; s0 < nsplit; s0 += 32) {
+        const int sl = s0 + lane;
+        float wgt = 0.f;
+        if (sl < nsplit) {
+            const size_t pr = (bg * nsplit + sl) * R + r;
+            const float m = part_ml[pr * 2];
+            if (m != -INFINITY) {
+                wgt = __expf(m - M);
+                L += wgt * part_ml[pr * 2 + 1];
+            }
+        }
+        const int cnt = min(32, nsplit - s0);
+#pragma unroll 4
+        for (int t = 0; t < cnt; ++t) {
+            const float wt = __shfl_sync(FULL, wgt, t);
+            if (wt == 0.f) continue;
+            const float* po = part_o + ((bg * nsplit + s0 + t) * R + r) * D;
 #pragma unroll
-        for (int j = 0; j < D / 32; ++j) acc[j] += wgt * part_o[pr * D + lane + 32 * j];
+            for (int j = 0; j < D / 32; ++j) acc[j] = fmaf(wt, po[lane + 32 * j], acc[j]);
+        }
     }
+    L = warp_sum(L);
     const float inv = 1.0f / L;
     T* o = out + (((size_t)b * N + i) * Hq + h) * D;
 #pragma unroll
@@ -160,21 +182,25 @@ int launch_attn_combine_f32(const AttnArgs& a, cudaStream_t st) {
 }
 
 // -------------------------------------------------------- CUDA-core splits --
-// Block = (sequence, KV head, 64-row chunk of the query rows) x split.
-// 4 threads per query row: each scores 8 of a 32-key tile and owns d/4 output
-// columns (c = lane_in_row + 4 j, so the 4 threads hit different banks).
-constexpr int CC_ROWS = 64;
-constexpr int CC_KEYS = 32;
+// Block = (sequence, KV head, chunk of ROWS query rows) x split, 256 threads:
+// TPR = 256 / ROWS threads per query row, each scoring KPT = 64 / TPR keys of
+// a 64-key tile (a whole split: one round of loads per block) and owning
+// D / TPR output columns (c = lane_in_row + TPR j, so a row's threads hit
+// different banks).  ROWS = 16 when the unit has at most 16 query rows (small
+// workloads: every thread has a row), else 64.
+constexpr int CC_KEYS = 64;
 
-template <typename T, int D>
+template <typename T, int D, int ROWS>
 __global__ void __launch_bounds__(256)
 attn_cc_kernel(AttnArgs a) {
+    static_assert(sizeof(T) == 4, "the CUDA-core attention stages fp32 rows");
+    constexpr int TPR = 256 / ROWS, KPT = CC_KEYS / TPR, CPT = D / TPR;
     extern __shared__ float smem[];
-    float* sQ = smem;                          // [64][D+1]
-    float* sK = sQ + CC_ROWS * (D + 1);        // [32][D+1]
-    float* sV = sK + CC_KEYS * (D + 1);        // [32][D+1]
-    float* sS = sV + CC_KEYS * (D + 1);        // [64][33]
-    const int nrc = (a.R + CC_ROWS - 1) / CC_ROWS;
+    float* sQ = smem;                          // [ROWS][D+1]
+    float* sK = sQ + ROWS * (D + 1);           // [CC_KEYS][D+1]
+    float* sV = sK + CC_KEYS * (D + 1);        // [CC_KEYS][D+1]
+    float* sS = sV + CC_KEYS * (D + 1);        // [ROWS][CC_KEYS + 1]
+    const int nrc = (a.R + ROWS - 1) / ROWS;
     const int bg = blockIdx.x / nrc, rc = blockIdx.x % nrc;
     const int b = bg / a.Hkv;
     const int split = blockIdx.y;
@@ -182,13 +208,13 @@ attn_cc_kernel(AttnArgs a) {
     const bool tree = split == a.nsplit - 1;
     const int k_lo = tree ? 0 : split * a.kps;
     const int k_hi = tree ? a.N : min(P, k_lo + a.kps);
-    const int tid = threadIdx.x, row = tid >> 2, kg = tid & 3;
-    const int r = rc * CC_ROWS + row;
+    const int tid = threadIdx.x, row = tid / TPR, kg = tid % TPR;
+    const int r = rc * ROWS + row;
     float* po = a.part_o + ((size_t)bg * a.nsplit + split) * a.R * D;
     float* pml = a.part_ml + ((size_t)bg * a.nsplit + split) * a.R * 2;
     if (k_lo >= k_hi) {
         if (r < a.R) {
-            for (int j = 0; j < D / 4; ++j) po[(size_t)r * D + kg + 4 * j] = 0.f;
+            for (int j = 0; j < CPT; ++j) po[(size_t)r * D + kg + TPR * j] = 0.f;
             if (kg == 0) {
                 pml[r * 2] = -INFINITY;
                 pml[r * 2 + 1] = 0.f;
@@ -199,73 +225,114 @@ attn_cc_kernel(AttnArgs a) {
     const unsigned long long anc =
         (tree && r < a.R) ? a.anc[(size_t)b * a.N + (r % a.N)] : 0ull;
     const float* qsrc = static_cast<const float*>(a.q_rot) + (size_t)bg * a.q_rows_pad * D;
-    for (int e = tid; e < CC_ROWS * D; e += 256) {
-        const int rr = e / D, c = e % D;
-        const int gr = rc * CC_ROWS + rr;
-        sQ[rr * (D + 1) + c] = gr < a.R ? qsrc[(size_t)gr * D + c] : 0.f;
+    {
+        // (each thread's loads issued together before its stores)
+        constexpr int NQ = ROWS * D / 4 / 256;
+        float4 x[NQ];
+#pragma unroll
+        for (int i = 0; i < NQ; ++i) {
+            const int e = tid + 256 * i, rr = e / (D / 4), c = 4 * (e % (D / 4));
+            const int gr = rc * ROWS + rr;
+            x[i] = gr < a.R ? *reinterpret_cast<const float4*>(qsrc + (size_t)gr * D + c)
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int i = 0; i < NQ; ++i) {
+            const int e = tid + 256 * i, rr = e / (D / 4), c = 4 * (e % (D / 4));
+            float* q = sQ + rr * (D + 1) + c;
+            q[0] = x[i].x;
+            q[1] = x[i].y;
+            q[2] = x[i].z;
+            q[3] = x[i].w;
+        }
     }
     const T* Kb = tree ? static_cast<const T*>(a.treeK) + (size_t)bg * a.N * D
                        : static_cast<const T*>(a.cacheK) + (size_t)bg * a.S_max * D;
     const T* Vb = tree ? static_cast<const T*>(a.treeV) + (size_t)bg * a.N * D
                        : static_cast<const T*>(a.cacheV) + (size_t)bg * a.S_max * D;
     float m = -INFINITY, l = 0.f;
-    float o[D / 4];
+    float o[CPT];
 #pragma unroll
-    for (int j = 0; j < D / 4; ++j) o[j] = 0.f;
+    for (int j = 0; j < CPT; ++j) o[j] = 0.f;
     for (int kt = k_lo; kt < k_hi; kt += CC_KEYS) {
         __syncthreads();
-        for (int e = tid; e < CC_KEYS * D; e += 256) {
-            const int kk = e / D, c = e % D;
-            const int key = kt + kk;
-            float kv = 0.f, vv = 0.f;
-            if (key < k_hi) {
-                kv = to_f32(Kb[(size_t)key * D + c]);
-                vv = to_f32(Vb[(size_t)key * D + c]);
+        {
+            // K and V rows of the tile, zeros past k_hi (each thread's loads
+            // issued together before its stores)
+            constexpr int NK = CC_KEYS * D / 4 / 256;
+            float4 xk[NK], xv[NK];
+#pragma unroll
+            for (int i = 0; i < NK; ++i) {
+                const int e = tid + 256 * i, kk = e / (D / 4), c = 4 * (e % (D / 4));
+                const int key = kt + kk;
+                xk[i] = xv[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (key < k_hi) {
+                    xk[i] = *reinterpret_cast<const float4*>(Kb + (size_t)key * D + c);
+                    xv[i] = *reinterpret_cast<const float4*>(Vb + (size_t)key * D + c);
+                }
             }
-            sK[kk * (D + 1) + c] = kv;
-            sV[kk * (D + 1) + c] = vv;
+#pragma unroll
+            for (int i = 0; i < NK; ++i) {
+                const int e = tid + 256 * i, kk = e / (D / 4), c = 4 * (e % (D / 4));
+                float* k = sK + kk * (D + 1) + c;
+                float* v = sV + kk * (D + 1) + c;
+                k[0] = xk[i].x;
+                k[1] = xk[i].y;
+                k[2] = xk[i].z;
+                k[3] = xk[i].w;
+                v[0] = xv[i].x;
+                v[1] = xv[i].y;
+                v[2] = xv[i].z;
+                v[3] = xv[i].w;
+            }
         }
         __syncthreads();
-        float s[8];
+        // Scores of this thread's KPT keys: each query value read once.
+        float acc[KPT];
+#pragma unroll
+        for (int jj = 0; jj < KPT; ++jj) acc[jj] = 0.f;
+#pragma unroll 8
+        for (int c = 0; c < D; ++c) {
+            const float qv = sQ[row * (D + 1) + c];
+#pragma unroll
+            for (int jj = 0; jj < KPT; ++jj) acc[jj] = fmaf(qv, sK[(kg * KPT + jj) * (D + 1) + c], acc[jj]);
+        }
+        float s[KPT];
         float tmax = -INFINITY;
 #pragma unroll
-        for (int jj = 0; jj < 8; ++jj) {
-            const int kk = kg * 8 + jj;
-            float acc = 0.f;
-#pragma unroll 16
-            for (int c = 0; c < D; ++c) acc = fmaf(sQ[row * (D + 1) + c], sK[kk * (D + 1) + c], acc);
-            const int key = kt + kk;
+        for (int jj = 0; jj < KPT; ++jj) {
+            const int key = kt + kg * KPT + jj;
             const bool ok = key < k_hi && (!tree || ((anc >> key) & 1ull));
-            s[jj] = ok ? acc * a.scale : -INFINITY;
+            s[jj] = ok ? acc[jj] * a.scale : -INFINITY;
             tmax = fmaxf(tmax, s[jj]);
         }
-        tmax = fmaxf(tmax, __shfl_xor_sync(FULL, tmax, 1));
-        tmax = fmaxf(tmax, __shfl_xor_sync(FULL, tmax, 2));
+#pragma unroll
+        for (int o2 = 1; o2 < TPR; o2 <<= 1) tmax = fmaxf(tmax, __shfl_xor_sync(FULL, tmax, o2));
         const float mnew = fmaxf(m, tmax);
         const float alpha = (mnew == -INFINITY) ? 1.f : __expf(m - mnew);
         float psum = 0.f;
 #pragma unroll
-        for (int jj = 0; jj < 8; ++jj) {
+        for (int jj = 0; jj < KPT; ++jj) {
             const float p = (s[jj] == -INFINITY) ? 0.f : __expf(s[jj] - mnew);
-            sS[row * 33 + kg * 8 + jj] = p;
+            sS[row * (CC_KEYS + 1) + kg * KPT + jj] = p;
             psum += p;
         }
-        psum += __shfl_xor_sync(FULL, psum, 1);
-        psum += __shfl_xor_sync(FULL, psum, 2);
+#pragma unroll
+        for (int o2 = 1; o2 < TPR; o2 <<= 1) psum += __shfl_xor_sync(FULL, psum, o2);
         l = l * alpha + psum;
         m = mnew;
         __syncwarp();
 #pragma unroll
-        for (int j = 0; j < D / 4; ++j) o[j] *= alpha;
+        for (int j = 0; j < CPT; ++j) o[j] *= alpha;
         for (int kk = 0; kk < CC_KEYS; ++kk) {
-            const float p = sS[row * 33 + kk];
+            const float p = sS[row * (CC_KEYS + 1) + kk];
 #pragma unroll
-            for (int j = 0; j < D / 4; ++j) o[j] = fmaf(p, sV[kk * (D + 1) + kg + 4 * j], o[j]);
+            for (int j = 0; j < CPT; ++j) o[j] = fmaf(p, sV[kk * (D + 1) + kg + TPR * j], o[j]);
         }
     }
     if (r < a.R) {
 #pragma unroll
-        for (int j = 0; j < D / 4; ++j) po[(size_t)r * D + kg + 4 * j] = o[j];
+        for (int j = 0; j < CPT; ++j) po[(size_t)r * D + kg + TPR * j] = o[j];
         if (kg == 0) {
             pml[r * 2] = m;
             pml[r * 2 + 1] = l;
@@ -273,25 +340,26 @@ attn_cc_kernel(AttnArgs a) {
     }
 }
 
-template <typename T, int D>
+template <typename T, int D, int ROWS>
 static int launch_cc(const AttnArgs& a, cudaStream_t st) {
-    const size_t smem = sizeof(float) * (CC_ROWS * (D + 1) + 2 * CC_KEYS * (D + 1) + CC_ROWS * 33);
+    const size_t smem = sizeof(float) * (ROWS * (D + 1) + 2 * CC_KEYS * (D + 1) + ROWS * (CC_KEYS + 1));
     static thread_local int attr_dev = -1;
     int dev = 0;
     cudaGetDevice(&dev);
     if (attr_dev != dev) {
-        cudaFuncSetAttribute(attn_cc_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaFuncSetAttribute(attn_cc_kernel<T, D, ROWS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
         attr_dev = dev;
     }
-    const int nrc = (a.R + CC_ROWS - 1) / CC_ROWS;
+    const int nrc = (a.R + ROWS - 1) / ROWS;
     dim3 grid(a.B * a.Hkv * nrc, a.nsplit);
-    attn_cc_kernel<T, D><<<grid, 256, smem, st>>>(a);
+    attn_cc_kernel<T, D, ROWS><<<grid, 256, smem, st>>>(a);
     return check_launch("attn_cc_kernel");
 }
 
 int launch_attn_cc_f32(const AttnArgs& a, cudaStream_t st) {
-    return a.d == 128 ? launch_cc<float, 128>(a, st) : launch_cc<float, 64>(a, st);
+    if (a.R <= 16) return a.d == 128 ? launch_cc<float, 128, 16>(a, st) : launch_cc<float, 64, 16>(a, st);
+    return a.d == 128 ? launch_cc<float, 128, 64>(a, st) : launch_cc<float, 64, 64>(a, st);
 }
 
 }  // namespace gv

@@ -92,7 +92,7 @@ int launch_lmhead_merge(SelectPartials, int, int, int32_t*, float*, float*, floa
 int lmhead_tc_grid(int slots_capacity);
 
 // ---------------------------------------------------------- attention plan --
-constexpr int KPS_F32 = 256;   // prefix keys per split, CUDA-core path
+constexpr int KPS_F32 = 64;    // prefix keys per split, CUDA-core path
 
 struct AttnPlan {
     size_t q_rot, part_o, part_ml, total;
@@ -147,7 +147,7 @@ static AttnPlan attn_plan(const gv_attn_shape* s) {
 }
 
 // ------------------------------------------------------------ lmhead plan --
-constexpr int CC_TV = 64;        // vocabulary tile of the CUDA-core (fp32) kernel
+constexpr int CC_TV = 32;        // vocabulary tile of the CUDA-core (fp32) kernel
 constexpr int TC_SLOTS = 256;    // partial slots of the tensor-core kernel (one per CTA)
 
 struct LmPlan {

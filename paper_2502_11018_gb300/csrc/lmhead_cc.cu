@@ -6,18 +6,28 @@
 // tensor cores' tf32 mode would round the operands to 10-bit mantissas, well
 // outside the 1e-4 relative tolerance fp32 results are held to.
 //
-// Tile: 64 vocabulary rows x 32 hidden-state rows per 256-thread block, the
-// hidden dimension streamed through shared memory 32 at a time; each thread
-// owns a 4 (vocab) x 2 (rows) patch of scores.  The selection then runs on
-// the tile in shared memory and leaves one partial result per (tile, row) in
-// the workspace; lmhead_merge_kernel reduces the partials of every row.
+// Tile: 32 vocabulary rows x 16 hidden-state rows per 256-thread block
+// (grid: vocabulary tiles x row tiles, so even a 4096-row vocabulary spreads
+// over most SMs).  The block stages its W rows and hidden-state rows for 512
+// of the hidden dimension at a time in shared memory, every thread's loads in
+// flight at once; lane l of each warp scores vocabulary row l against all 16
+// hidden-state rows (16 accumulators, the hidden-state values read as
+// warp-wide broadcasts), and the 8 warps take interleaved 4-wide slices of
+// the hidden dimension, summed across warps at the end.  The selection then
+// runs on the tile in shared memory and leaves one partial result per (tile,
+// row) in the workspace; lmhead_merge_kernel reduces the partials of every
+// row.
 #include "gv_internal.cuh"
 
 namespace gv {
 
-constexpr int CC_TV = 64;   // vocab rows per tile
-constexpr int CC_TR = 32;   // hidden-state rows per tile
-constexpr int CC_TK = 32;   // hidden dim per stage
+constexpr int CC_TV = 32;            // vocab rows per tile (a warp's lanes)
+constexpr int CC_TR = 16;            // hidden-state rows per tile
+constexpr int CC_KC = 512;           // hidden dim staged per pass
+constexpr int CC_KS = CC_KC + 4;     // staged row stride: 16-byte rows, the 8 lanes of a
+                                     // quarter-warp's 16-byte loads on distinct banks
+constexpr size_t CC_SMEM = sizeof(float) * ((size_t)(CC_TV + CC_TR) * CC_KS + 8 * CC_TR * (CC_TV + 1) +
+                                            CC_TR * (CC_TV + 1));
 
 // Top-K (value desc, id asc) of `cnt` candidates held two per lane, by K
 // rounds of warp argmax.  Lane 0 returns the lists.
@@ -57,72 +67,108 @@ template <typename T>
 __global__ void __launch_bounds__(256)
 lmhead_cc_kernel(const T* __restrict__ h, const T* __restrict__ W, int rows, int H, int V,
                  int mode, int K, float* __restrict__ logits, SelectPartials part) {
-    __shared__ float sW[CC_TK][CC_TV + 1];
-    __shared__ float sH[CC_TK][CC_TR + 1];
-    __shared__ float sS[CC_TR][CC_TV + 1];
-    const int tid = threadIdx.x;
+    static_assert(sizeof(T) == 4, "the CUDA-core LM head stages fp32 operands");
+    extern __shared__ float cc_smem[];
+    float* sW = cc_smem;                              // [CC_TV][CC_KS]
+    float* sH = sW + CC_TV * CC_KS;                   // [CC_TR][CC_KS]
+    float* sRed = sH + CC_TR * CC_KS;                 // [8 warps][CC_TR][CC_TV + 1]
+    float(*sS)[CC_TV + 1] = reinterpret_cast<float(*)[CC_TV + 1]>(sRed + 8 * CC_TR * (CC_TV + 1));
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int v0 = blockIdx.x * CC_TV;
     const int r0 = blockIdx.y * CC_TR;
-    const int tv = tid & 15, tr = tid >> 4;
-    float acc[4][2] = {};
-    for (int k0 = 0; k0 < H; k0 += CC_TK) {
-        for (int e = tid; e < CC_TV * CC_TK; e += 256) {
-            const int vv = e / CC_TK, kk = e % CC_TK;
-            const int v = v0 + vv, k = k0 + kk;
-            sW[kk][vv] = (v < V && k < H) ? to_f32(W[(size_t)v * H + k]) : 0.f;
-        }
-        for (int e = tid; e < CC_TR * CC_TK; e += 256) {
-            const int rr = e / CC_TK, kk = e % CC_TK;
-            const int r = r0 + rr, k = k0 + kk;
-            sH[kk][rr] = (r < rows && k < H) ? to_f32(h[(size_t)r * H + k]) : 0.f;
+    float acc[CC_TR];
+#pragma unroll
+    for (int r = 0; r < CC_TR; ++r) acc[r] = 0.f;
+    for (int k0 = 0; k0 < H; k0 += CC_KC) {
+        const int kc = min(CC_KC, H - k0), kc4 = (kc + 3) & ~3;
+        __syncthreads();
+        // Stage W rows v0.. and hidden rows r0.. for k0 .. k0 + kc (zeros past
+        // the vocabulary, the rows and kc, up to kc4).
+        if ((H & 3) == 0) {
+            // 16-byte rows: float4 loads (kc is then a multiple of 4), each
+            // thread's loads issued together before its stores.
+            const int q4 = kc >> 2;
+            constexpr int NW = CC_TV * (CC_KC / 4) / 256, NH = CC_TR * (CC_KC / 4) / 256;
+            float4 xw[NW], xh[NH];
+#pragma unroll
+            for (int i = 0; i < NW; ++i) {
+                const int e = tid + 256 * i, vv = e / q4, kk = 4 * (e - vv * q4), v = v0 + vv;
+                xw[i] = (vv < CC_TV && v < V) ? *reinterpret_cast<const float4*>(W + (size_t)v * H + k0 + kk)
+                                              : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int i = 0; i < NH; ++i) {
+                const int e = tid + 256 * i, rr = e / q4, kk = 4 * (e - rr * q4), r = r0 + rr;
+                xh[i] = (rr < CC_TR && r < rows) ? *reinterpret_cast<const float4*>(h + (size_t)r * H + k0 + kk)
+                                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int i = 0; i < NW; ++i) {
+                const int e = tid + 256 * i, vv = e / q4, kk = 4 * (e - vv * q4);
+                if (vv < CC_TV) *reinterpret_cast<float4*>(sW + vv * CC_KS + kk) = xw[i];
+            }
+#pragma unroll
+            for (int i = 0; i < NH; ++i) {
+                const int e = tid + 256 * i, rr = e / q4, kk = 4 * (e - rr * q4);
+                if (rr < CC_TR) *reinterpret_cast<float4*>(sH + rr * CC_KS + kk) = xh[i];
+            }
+        } else {
+            for (int e = tid; e < CC_TV * kc4; e += 256) {
+                const int vv = e / kc4, kk = e - vv * kc4;
+                const int v = v0 + vv;
+                sW[vv * CC_KS + kk] = (v < V && kk < kc) ? to_f32(W[(size_t)v * H + k0 + kk]) : 0.f;
+            }
+            for (int e = tid; e < CC_TR * kc4; e += 256) {
+                const int rr = e / kc4, kk = e - rr * kc4;
+                const int r = r0 + rr;
+                sH[rr * CC_KS + kk] = (r < rows && kk < kc) ? to_f32(h[(size_t)r * H + k0 + kk]) : 0.f;
+            }
         }
         __syncthreads();
-#pragma unroll 8
-        for (int kk = 0; kk < CC_TK; ++kk) {
-            float wv[4], hv[2];
+        const float* wrow = sW + lane * CC_KS;
+        for (int kk = 4 * warp; kk < kc4; kk += 32) {
+            const float4 w4 = *reinterpret_cast<const float4*>(wrow + kk);
 #pragma unroll
-            for (int a = 0; a < 4; ++a) wv[a] = sW[kk][tv + 16 * a];
-#pragma unroll
-            for (int c = 0; c < 2; ++c) hv[c] = sH[kk][tr + 16 * c];
-#pragma unroll
-            for (int a = 0; a < 4; ++a)
-#pragma unroll
-                for (int c = 0; c < 2; ++c) acc[a][c] = fmaf(wv[a], hv[c], acc[a][c]);
+            for (int r = 0; r < CC_TR; ++r) {
+                const float4 h4 = *reinterpret_cast<const float4*>(sH + r * CC_KS + kk);
+                acc[r] = fmaf(w4.x, h4.x, fmaf(w4.y, h4.y, fmaf(w4.z, h4.z, fmaf(w4.w, h4.w, acc[r]))));
+            }
         }
-        __syncthreads();
     }
+    // Sum the warps' slices of the hidden dimension.
 #pragma unroll
-    for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int c = 0; c < 2; ++c) {
-            const int vv = tv + 16 * a, rr = tr + 16 * c;
-            const bool valid = (v0 + vv < V) && (r0 + rr < rows);
-            sS[rr][vv] = valid ? acc[a][c] : -INFINITY;
-            if (mode == GV_SELECT_LOGITS && valid) logits[(size_t)(r0 + rr) * V + v0 + vv] = acc[a][c];
-        }
+    for (int r = 0; r < CC_TR; ++r) sRed[(warp * CC_TR + r) * (CC_TV + 1) + lane] = acc[r];
     __syncthreads();
-    // Selection: warp w handles rows w, w+8, w+16, w+24 of the tile.
-    const int warp = tid >> 5, lane = tid & 31;
+    for (int e = tid; e < CC_TR * CC_TV; e += 256) {
+        const int rr = e / CC_TV, vv = e % CC_TV;
+        float x = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) x += sRed[(w * CC_TR + rr) * (CC_TV + 1) + vv];
+        const bool valid = (v0 + vv < V) && (r0 + rr < rows);
+        sS[rr][vv] = valid ? x : -INFINITY;
+        if (mode == GV_SELECT_LOGITS && valid) logits[(size_t)(r0 + rr) * V + v0 + vv] = x;
+    }
+    __syncthreads();
+    // Selection: warp w handles rows w and w + 8 of the tile, lane l the
+    // tile's vocabulary row l.
     const int slot = blockIdx.x;
     for (int rr = warp; rr < CC_TR; rr += 8) {
         const int r = r0 + rr;
         if (r >= rows) break;
-        const float x0 = sS[rr][lane], x1 = sS[rr][lane + 32];
+        const float x0 = sS[rr][lane];
         if (mode == GV_SELECT_LOGITS) {
-            const float m = warp_max(fmaxf(x0, x1));
+            const float m = warp_max(x0);
             float s = 0.f;
             if (x0 != -INFINITY) s += __expf(x0 - m);
-            if (x1 != -INFINITY) s += __expf(x1 - m);
             s = warp_sum(s);
             if (lane == 0) {
                 part.m[(size_t)slot * rows + r] = m;
                 part.s[(size_t)slot * rows + r] = (m == -INFINITY) ? 0.f : s;
             }
         } else {
-            const int i0 = v0 + lane, i1 = v0 + lane + 32;
+            const int i0 = v0 + lane;
             const size_t o = ((size_t)slot * rows + r) * K;
-            warp_topk(x0, i0 < V ? i0 : INT32_MAX, x1, i1 < V ? i1 : INT32_MAX, K,
-                      part.val + o, part.id + o);
+            warp_topk(x0, i0 < V ? i0 : INT32_MAX, -INFINITY, INT32_MAX, K, part.val + o, part.id + o);
         }
     }
 }
@@ -245,8 +291,15 @@ int launch_lmhead_merge(SelectPartials part, int mode, int K, int32_t* ids, floa
 int launch_lmhead_cc(const float* h, const float* W, int rows, int H, int V, int mode, int K,
                      float* logits, SelectPartials part, int32_t* ids, float* vals, float* row_max,
                      float* row_lse, cudaStream_t st) {
+    static thread_local int attr_dev = -1;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (attr_dev != dev) {
+        cudaFuncSetAttribute(lmhead_cc_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)CC_SMEM);
+        attr_dev = dev;
+    }
     dim3 grid((V + CC_TV - 1) / CC_TV, (rows + CC_TR - 1) / CC_TR);
-    lmhead_cc_kernel<float><<<grid, 256, 0, st>>>(h, W, rows, H, V, mode, K, logits, part);
+    lmhead_cc_kernel<float><<<grid, 256, CC_SMEM, st>>>(h, W, rows, H, V, mode, K, logits, part);
     const int rc = check_launch("lmhead_cc_kernel");
     if (rc != GV_OK) return rc;
     return launch_lmhead_merge(part, mode, K, ids, vals, row_max, row_lse, nullptr, st);
