@@ -606,8 +606,9 @@ def main():
     torch.cuda.synchronize()
     if smi is not None:
         smi.start()
+    flush, l2_note = l2_flush_for(cfg, dev)
     clocks.start()
-    ms, per = replay_times_ms(step.replay, args.steps, stream)
+    ms, per = replay_times_ms(step.replay, args.steps, stream, flush)
     torch.cuda.synchronize()
     clocks.stop()
     if dist is not None:
@@ -636,7 +637,7 @@ def main():
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_max, **percentiles(per),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg["dtype"],
         "data": "synthetic (seeded random weights, caches and draft trees)",
-        "config": bench_config(cfg, world),
+        "config": {**bench_config(cfg, world), "l2": l2_note},
         "accepted_tok_per_s": world * sum(accept_len) * 1000.0 / t_max,
         "accept_len": accept_len,
         "hbm_roofline": {"step_bytes": sb["total"], "achieved_gbs": step_gbs,
@@ -692,6 +693,15 @@ def kernel_times(step, cfg, stream):
     }
 
 
+def l2_flush_for(cfg, dev):
+    """(flush, note): a working set that fits in the 129 MB L2 (the tiny
+    workload) is flushed between replays by writing a 512 MB buffer."""
+    if step_bytes(cfg, [cfg["D"]] * cfg["B"])["total"] >= 256 * 2**20:
+        return None, "working set above L2 (no flush needed)"
+    junk = torch.empty(512 * 2**20, dtype=torch.uint8, device=dev)
+    return (lambda: junk.fill_(1)), "flushed between replays (512 MB write, outside the timed pairs)"
+
+
 def measure_config(name, seed, steps, warmup, dev, stream, peaks):
     """One workload's step: per-replay times of its CUDA graph, throughput,
     HBM roofline fraction of the step and of its two dominant kernels."""
@@ -703,14 +713,9 @@ def measure_config(name, seed, steps, warmup, dev, stream, peaks):
     for _ in range(max(warmup, 3)):
         step.replay()
     torch.cuda.synchronize()
-    # A working set that fits in the 129 MB L2 (the tiny workload) is flushed
-    # between replays by writing a 512 MB buffer.
-    flush = None
+    flush, note = l2_flush_for(cfg, dev)
     config = bench_config(cfg, 1)
-    if step_bytes(cfg, [cfg["D"]] * cfg["B"])["total"] < 256 * 2**20:
-        junk = torch.empty(512 * 2**20, dtype=torch.uint8, device=dev)
-        flush = lambda: junk.fill_(1)  # noqa: E731
-        config["l2"] = "flushed between replays (512 MB write, outside the timed pairs)"
+    config["l2"] = note
     ms, per = replay_times_ms(step.replay, steps, stream, flush)
     accept_len = step.accept_len.cpu().tolist()
     sb = step_bytes(cfg, accept_len)
