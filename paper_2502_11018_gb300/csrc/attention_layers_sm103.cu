@@ -86,7 +86,7 @@ constexpr int AL_OFF_V = AL_OFF_K + AL_KST * AL_TILE;
 constexpr int AL_OFF_BAR = AL_OFF_V + AL_VST * AL_TILE;
 constexpr int AL_NBAR = 3 * AL_KST + 3 * AL_VST + 12 + 5;
 constexpr int AL_OFF_MISC = AL_OFF_BAR + 8 * AL_NBAR;
-constexpr int AL_OFF_ML = AL_OFF_MISC + 16;            // float2 (m, l) [2 streams][128 rows]
+constexpr int AL_OFF_ML = AL_OFF_MISC + 32;            // float2 (m, l) [2 streams][128 rows]
 constexpr int AL_OFF_NB = AL_OFF_ML + 2 * 128 * 8;     // int [AL_MAXB]
 constexpr int AL_OFF_P = AL_OFF_NB + 4 * AL_MAXB;      // int [AL_MAXB] prefix lengths
 constexpr int AL_SMEM = AL_OFF_P + 4 * AL_MAXB;
@@ -319,6 +319,10 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
     uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(smem + AL_OFF_MISC);
     volatile int* abort = reinterpret_cast<volatile int*>(smem + AL_OFF_MISC + 4);
     volatile int* last_flag = reinterpret_cast<volatile int*>(smem + AL_OFF_MISC + 8);
+    // [2] a split piece's decision to combine, published by thread 0 with the
+    // piece-end vote (two words, alternating by piece: a word is rewritten
+    // only after every thread has passed the next piece's vote)
+    volatile int* cmb_flag = reinterpret_cast<volatile int*>(smem + AL_OFF_MISC + 12);
     int* snb = reinterpret_cast<int*>(smem + AL_OFF_NB);
     int* sP = reinterpret_cast<int*>(smem + AL_OFF_P);
 
@@ -638,6 +642,7 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
         bool waited = false;
         Walk wk = walk0;
         Piece pc;
+        int npc = 0;           // pieces so far
         int m0 = 0;            // this stream's jobs before the piece
         while (wk.next(pc)) {
             const int P = min(max(a.prefix_len[pc.b], 0), a.S_max);
@@ -760,17 +765,9 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
                 }
             }
             // ------------------------------------------------- the piece's rows
-            // This stream's last PV has landed; every softmax thread agrees on
-            // whether the piece completed.
-            int w = ok ? 1 : 0;
-            if (w && nmine > 0 && lane == 0) {
-                const int ml = m - 1;   // this stream's last job
-                w = mbar_wait(&pv_done[2 * s + (ml & 1)], (uint32_t)(ml >> 1) & 1u, abort);
-            }
-            w = __shfl_sync(FULL, w, 0);
-            ok = bar_and(1, AL_NSM, w);
             // The output and the workspace may still be read by the grid this
-            // one follows (an earlier call's): wait for it before writing.
+            // one follows (an earlier call's), and the arrival counters are
+            // zeroed by the one right before: wait for it first.
             if (!waited) {
                 pdl_wait();
                 waited = true;
@@ -779,12 +776,13 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
             // every CTA of [cf, cl] whose range is not empty (ranges are empty
             // when there are fewer blocks than CTAs).  When the unit has two
             // pieces and the other one has already arrived (an acquiring read
-            // of the unit's counter), this piece combines the two straight
-            // from its accumulators and the other's partial rows; otherwise it
-            // writes its own partial rows and counts itself (below).
+            // of the unit's counter, taken by thread 0 while the last PV lands
+            // and published with the vote), this piece combines the two
+            // straight from its accumulators and the other's partial rows;
+            // otherwise it writes its own partial rows and counts itself
+            // (below).
             const long long U0 = pc.u0;
             int cf = 0, cl = -1, npieces = 0, other_slot = -1;
-            bool combine = false;
             if (!pc.direct) {
                 cf = cta_of(U0, W, C);
                 cl = cta_of(U0 + pc.nb - 1, W, C);
@@ -797,11 +795,20 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
                 if (t_id == 0) {
                     const bool ready = npieces == 2 && atomicAdd(a.cnt + pc.unit, 0) == 1;
                     __threadfence();
-                    *last_flag = ready ? 2 : 0;
+                    cmb_flag[npc & 1] = ready ? 1 : 0;
                 }
-                named_bar_sync(1, AL_NSM);
-                combine = *last_flag == 2;
             }
+            // This stream's last PV has landed; every softmax thread agrees on
+            // whether the piece completed.
+            int w = ok ? 1 : 0;
+            if (w && nmine > 0 && lane == 0) {
+                const int ml = m - 1;   // this stream's last job
+                w = mbar_wait(&pv_done[2 * s + (ml & 1)], (uint32_t)(ml >> 1) & 1u, abort);
+            }
+            w = __shfl_sync(FULL, w, 0);
+            ok = bar_and(1, AL_NSM, w);
+            const bool combine = !pc.direct && cmb_flag[npc & 1] != 0;
+            ++npc;
             // Rows of this piece: with two tiles each stream writes its tile's
             // rows; with one tile the two accumulators (disjoint key sets of
             // the same rows) combine, and stream s writes d columns 64 s ..
@@ -834,16 +841,17 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
             }
             const uint32_t o_other = lane_base + AL_OCOL + 128u * (uint32_t)(1 - s);
             // (combining: the other piece's log2-sum-exp and partial columns,
-            // all loads issued at once)
-            uint4 pr[16];
+            // 32 columns at a time, each quarter's loads issued one quarter
+            // ahead)
+            uint4 pr[2][4];
+            const uint4* psrc = nullptr;
             float a_self = 1.f, a_part = 0.f;
             if (combine && rv) {
                 const size_t prow = ((size_t)other_slot * T + tile) * 128 + row;
                 const float lse_o = __ldcg(a.part_lse + prow);
-                const uint4* src = reinterpret_cast<const uint4*>(a.part + prow * 128 + c_lo);
+                psrc = reinterpret_cast<const uint4*>(a.part + prow * 128 + c_lo);
 #pragma unroll
-                for (int q = 0; q < 16; ++q)
-                    if (q < c_n / 8) pr[q] = __ldcg(src + q);
+                for (int q = 0; q < 4; ++q) pr[0][q] = __ldcg(psrc + q);
                 const float lse_s = ltot > 0.f ? M + log2f(ltot) : -INFINITY;
                 const float Mc = fmaxf(lse_s, lse_o);
                 const float es = lse_s == -INFINITY ? 0.f : fast_exp2(lse_s - Mc);
@@ -855,37 +863,53 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
                 tc_fence_after();
                 const float inv = ltot > 0.f ? 1.0f / ltot : 0.f;
                 const float fs = w_self * inv * a_self, fo = w_other * inv * a_self;
+                // 32 columns at a time: their TMEM loads issued together, one wait
 #pragma unroll
-                for (int c0 = 0; c0 < 128; c0 += 16) {
-                    if (c0 >= c_n) break;
-                    // (the columns of O this thread writes: c_lo + c0 ..)
-                    uint32_t os[16], oo[16];
-                    if (has_self) tmem_ld16(ocol + (uint32_t)(c_lo + c0), os);
-                    if (has_other) tmem_ld16(o_other + (uint32_t)(c_lo + c0), oo);
+                for (int qt = 0; qt < 4; ++qt) {
+                    if (32 * qt >= c_n) break;
+                    const int cq = c_lo + 32 * qt;       // (the columns of O this thread writes)
+                    uint32_t os[32], oo[32];
+                    if (has_self) {
+                        tmem_ld16(ocol + (uint32_t)cq, *reinterpret_cast<uint32_t(*)[16]>(&os[0]));
+                        tmem_ld16(ocol + (uint32_t)(cq + 16), *reinterpret_cast<uint32_t(*)[16]>(&os[16]));
+                    }
+                    if (has_other) {
+                        tmem_ld16(o_other + (uint32_t)cq, *reinterpret_cast<uint32_t(*)[16]>(&oo[0]));
+                        tmem_ld16(o_other + (uint32_t)(cq + 16), *reinterpret_cast<uint32_t(*)[16]>(&oo[16]));
+                    }
+                    if (psrc && 32 * (qt + 1) < c_n) {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) pr[(qt + 1) & 1][q] = __ldcg(psrc + 4 * (qt + 1) + q);
+                    }
                     tmem_wait_ld();
                     if (dst) {
-                        uint32_t pv[8];
 #pragma unroll
-                        for (int u = 0; u < 8; ++u) {
-                            float v0 = 0.f, v1 = 0.f;
-                            if (has_self) {
-                                v0 = __uint_as_float(os[2 * u]) * fs;
-                                v1 = __uint_as_float(os[2 * u + 1]) * fs;
+                        for (int g16 = 0; g16 < 2; ++g16) {
+                            uint32_t pv[8];
+#pragma unroll
+                            for (int u = 0; u < 8; ++u) {
+                                const int e = 16 * g16 + 2 * u;     // column pair within the quarter
+                                float v0 = 0.f, v1 = 0.f;
+                                if (has_self) {
+                                    v0 = __uint_as_float(os[e]) * fs;
+                                    v1 = __uint_as_float(os[e + 1]) * fs;
+                                }
+                                if (has_other) {
+                                    v0 = fmaf(__uint_as_float(oo[e]), fo, v0);
+                                    v1 = fmaf(__uint_as_float(oo[e + 1]), fo, v1);
+                                }
+                                if (combine) {
+                                    const uint4 q4 = pr[qt & 1][e >> 3];
+                                    const int wd = (e >> 1) & 3;
+                                    const uint32_t pw = wd == 0 ? q4.x : wd == 1 ? q4.y : wd == 2 ? q4.z : q4.w;
+                                    const float2 f = unpack_bf16(pw);
+                                    v0 = fmaf(f.x, a_part, v0);
+                                    v1 = fmaf(f.y, a_part, v1);
+                                }
+                                pv[u] = pack_bf16(v0, v1);
                             }
-                            if (has_other) {
-                                v0 = fmaf(__uint_as_float(oo[2 * u]), fo, v0);
-                                v1 = fmaf(__uint_as_float(oo[2 * u + 1]), fo, v1);
-                            }
-                            if (combine) {
-                                const uint4 q4 = pr[c0 / 8 + (u >> 2)];
-                                const uint32_t pw = (u & 3) == 0 ? q4.x : (u & 3) == 1 ? q4.y : (u & 3) == 2 ? q4.z : q4.w;
-                                const float2 f = unpack_bf16(pw);
-                                v0 = fmaf(f.x, a_part, v0);
-                                v1 = fmaf(f.y, a_part, v1);
-                            }
-                            pv[u] = pack_bf16(v0, v1);
+                            st_global_v8(dst + cq + 16 * g16, pv);
                         }
-                        st_global_v8(dst + c_lo + c0, pv);
                     }
                 }
             } else if (dst) {
