@@ -77,3 +77,58 @@ def test_forward_graph_replay_matches_eager():
     torch.cuda.synchronize()
     assert torch.equal(fwd.h, eager[0])
     assert torch.equal(fwd.step.ids, eager[1]) and torch.equal(fwd.step.path, eager[2])
+
+
+def test_forward_full_depth_llama3_8b_per_layer():
+    """The whole 32-layer LLaMA-3-8B verify forward (prefix 4096, 60-node
+    tree, FFN 14336, random weights), run layer by layer on the GPU.  Sampled
+    layers are checked against the float64 oracle layer fed with the GPU's own
+    input to that layer (so bf16 error does not compound across layers) at the
+    2e-2 hidden-state tolerance; the LM-head argmax against the oracle on the
+    GPU's final hidden states, on rows whose oracle margin is clear."""
+    from paper_2502_11018_gb300 import gv
+    dev = device()
+    cfg = inputs.config("llama3_8b")
+    L = cfg["L"]
+    inp = inputs.make_step_inputs(cfg, 23, device=dev)
+    fw = inputs.make_forward_weights(cfg, 23, device=dev)
+    fwd = VerifyForward(inp, fw)
+    st = fwd.step
+    st.tree()
+    gv.gv_rmsnorm(fw.h0, fw.attn_norm[0], fwd.x)
+    sample = (0, 1, 15, 30, L - 1)
+    kept = {}
+    for l in range(L):
+        if l in sample:
+            kept[l] = (fw.h0 if l == 0 else fwd.h).clone()
+        fwd.layer(l)
+        if l in sample:
+            torch.cuda.synchronize()
+            kept[l] = (kept[l], fwd.h.clone())
+    st.lmhead()
+    st.accept()
+    st.compact()
+    torch.cuda.synchronize()
+    B, N, Hq, Hkv, d = cfg["B"], cfg["N"], cfg["Hq"], cfg["Hkv"], cfg["d"]
+    P = inp.prefix_len.cpu().numpy()
+    depth, pos, anc, _ = oracle.tree_build(inp.parents.cpu().numpy(), P)
+    nq, nkv = Hq * d, Hkv * d
+    for l in sample:
+        h_in, h_out = kept[l]
+        Wqkv = f64(fw.Wqkv[l])
+        w = {"attn_norm": f64(fw.attn_norm[l]), "Wq": Wqkv[:nq], "Wk": Wqkv[nq:nq + nkv], "Wv": Wqkv[nq + nkv:],
+             "Wo": f64(fw.Wo[l]), "mlp_norm": f64(fw.mlp_norm[l]), "Wg": f64(fw.Wgu[l][:fw.F]),
+             "Wu": f64(fw.Wgu[l][fw.F:]), "Wd": f64(fw.Wd[l])}
+        ref, _, _ = oracle.decoder_layer(f64(h_in), w, f64(inp.cacheK[l]), f64(inp.cacheV[l]), P, pos, anc,
+                                         cfg["rope_base"], B, N, Hq, Hkv, d)
+        got = f64(h_out)
+        assert np.isfinite(got).all(), l
+        assert rel_err(got, ref) <= 2e-2, (l, rel_err(got, ref))
+    hf = oracle.rmsnorm(f64(fwd.h), f64(fw.final_norm))
+    logits = oracle.lmhead_logits(hf, f64(inp.W))
+    top2 = np.sort(logits, axis=1)[:, -2:]
+    clear = (top2[:, 1] - top2[:, 0]) > 0.02 * np.abs(logits).max()
+    ids = st.ids.cpu().numpy().reshape(-1)
+    assert clear.sum() >= 1
+    np.testing.assert_array_equal(ids[clear], logits.argmax(axis=1)[clear])
+    assert (st.seq_status.cpu().numpy() == 0).all()
