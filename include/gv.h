@@ -267,6 +267,12 @@ int gv_verify_attention_layers(const gv_attn_shape* s, int L, const void* q, int
  *   Unused outputs may be NULL.
  *   workspace >= gv_lmhead_workspace(rows, H, V, dt, mode, k) bytes.
  * H must be a multiple of 8 (bf16) or 4 (fp32); rows >= 1.
+ * Device-side timeout (bf16 path): every wait inside the kernel is bounded
+ * (about a second); a kernel that gives up does not fault, and the call still
+ * returns GV_OK (it was enqueued), but its results mark the failure once the
+ * stream has run: ids = -1 and vals = NaN (argmax, top-k), row_max = row_lse
+ * = NaN (logits).  A caller that cannot rule this out checks for ids < 0 (or
+ * NaN) before passing the ids on, e.g. to gv_accept.
  */
 size_t gv_lmhead_workspace(int rows, int H, int V, int dt, int mode, int k);
 int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int dt, int mode,
@@ -288,13 +294,15 @@ int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int d
  * (a file-scope __device__ array, one per device, reserved when the library
  * is loaded): per-CTA argmax partials of up to GV_NOALLOC_MAX_ROWS rows and
  * an error word, which each call zeroes on the stream before its kernels.
- * The first call on a device looks the array's address up
- * (cudaGetSymbolAddress) and caches it; make that first call before any
- * stream capture.  Nothing is allocated by any call.
+ * Every call looks the array's address up (cudaGetSymbolAddress, which
+ * allocates nothing), so a reset or replaced context is handled; make the
+ * first call on a device before any stream capture (the lookup itself is not
+ * captured).  Nothing is allocated by any call.
  * rows > GV_NOALLOC_MAX_ROWS returns GV_ERR_UNSUPPORTED (message in
  * gv_last_error()), before anything is enqueued.
  * Calls that overlap in time on one device (different streams, or host
  * threads without ordering) share the scratch and race: serialise them.
+ * Device-side timeout: as for gv_lmhead_select, ids = -1 and vals = NaN.
  */
 #define GV_NOALLOC_MAX_ROWS 256
 int gv_lmhead_argmax_noalloc(const void* h, const void* W, int rows, int H, int V,

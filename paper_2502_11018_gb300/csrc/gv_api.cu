@@ -185,34 +185,17 @@ constexpr size_t NOALLOC_ERR_OFF = NOALLOC_ID_OFF + NOALLOC_ENTRIES * sizeof(int
 constexpr size_t NOALLOC_BYTES = NOALLOC_ERR_OFF + 256;
 __device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_BYTES];
 
-constexpr int NOALLOC_MAX_DEVICES = 64;
-static std::mutex g_noalloc_mu;
-static void* g_noalloc_addr[NOALLOC_MAX_DEVICES];
-
-// Address of the scratch on the current device, looked up once per device.
+// Address of the scratch in the current device's context.  Looked up on
+// every call (cudaGetSymbolAddress allocates nothing), so a context that was
+// reset or replaced since an earlier call gets its own array's address.
 static int noalloc_scratch(char** out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) {
-        set_error("gv_lmhead_argmax_noalloc: cudaGetDevice: %s", cudaGetErrorString(e));
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || !p) {
+        set_error("gv_lmhead_argmax_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
         return GV_ERR_CUDA;
     }
-    if (dev < 0 || dev >= NOALLOC_MAX_DEVICES) {
-        set_error("gv_lmhead_argmax_noalloc: device %d beyond the %d supported", dev,
-                  NOALLOC_MAX_DEVICES);
-        return GV_ERR_UNSUPPORTED;
-    }
-    std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    if (!g_noalloc_addr[dev]) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess || !p) {
-            set_error("gv_lmhead_argmax_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
-            return GV_ERR_CUDA;
-        }
-        g_noalloc_addr[dev] = p;
-    }
-    *out = static_cast<char*>(g_noalloc_addr[dev]);
+    *out = static_cast<char*>(p);
     return GV_OK;
 }
 

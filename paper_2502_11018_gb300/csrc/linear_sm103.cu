@@ -332,7 +332,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant
         cluster_sync_all();
         const uint32_t rank = cluster_rank();
         const int nt = blockIdx.x / a.KS;
-        // this rank's 8-column chunks of the tile (the ranks split BM / 8 chunks as evenly as they go)
+        // this rank's 8-column chunks of the tile (the ranks split BM / 8 chunks
+        // as evenly as they go; the planner forms clusters of 2 and 4 only,
+        // which divide BM / 8, so an uneven split is not reached from the API)
         const int nch = BM / 8;
         const int c_lo = (int)rank * nch / a.KS, chunks = ((int)rank + 1) * nch / a.KS - c_lo;
         const uint32_t stg0 = smem_u32(smem_raw), ab0 = smem_u32((const void*)abort);
