@@ -115,7 +115,7 @@ def test_step_from_host_matches_device(name, layers):
     # the reference issues the attention in the host-fed step's layer groups
     # (one multi-layer call per group cuts the work the same way)
     ready = {}
-    for a, _ in VerifyStep._copy_groups(layers):
+    for a, _ in ref._copy_groups(layers):
         ready[a] = torch.cuda.Event()
         ready[a].record()
     ref.tree()
