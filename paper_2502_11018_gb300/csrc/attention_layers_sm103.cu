@@ -12,16 +12,18 @@
 // or two 128-row M tiles, T) against its keys, cut into 128-key blocks.
 // Block 0 of a unit holds the N tree keys (masked per query row by its
 // ancestor bitmask), blocks 1 .. ceil(P_b / 128) the cached prefix.  The
-// blocks of all units, in (l, b, g, block) order, form one sequence of W
-// blocks that is cut into gridDim.x contiguous ranges of equal length
-// (stream-K): CTA c takes blocks [c W / C, (c + 1) W / C).  A unit inside one
-// range is a whole piece, whose rows go straight to the output.  A unit cut
-// by range ends has pieces in consecutive CTAs; each piece writes its
-// normalised partial rows and their log2-sum-exp to a slot of the workspace
-// (slot 2c for the first piece of CTA c, 2c + 1 for its last) and counts
-// itself in the unit's arrival counter; the piece that arrives last combines
-// all pieces into the output and zeroes the counter.  No CTA waits for
-// another.
+// blocks of all units, in (l, b, g, block) order, each unit followed by
+// AL_DELTA positions without a block (the weight of a unit's end: an epilogue
+// and a pipeline restart for the CTA that holds it), form one sequence of W
+// positions that is cut into gridDim.x contiguous ranges of equal length
+// (stream-K): CTA c takes the blocks at positions [c W / C, (c + 1) W / C).
+// A unit inside one range is a whole piece, whose rows go straight to the
+// output.  A unit cut by range ends has pieces in consecutive CTAs; a piece
+// either combines with the unit's other piece if that one has arrived, or
+// writes its normalised partial rows and their log2-sum-exp to a slot of the
+// workspace (slot 2c for the first piece of CTA c, 2c + 1 for its last) and
+// counts itself in the unit's arrival counter; the last of three or more
+// pieces combines them all into the output.  No CTA waits for another.
 //
 // Both tiles of a unit share each staged K/V block (GQA: the G heads of a KV
 // head read one K/V stream): per block, S_t = Q_t K^T and O_t += P_t V for
@@ -77,6 +79,7 @@ static_assert(128 * AL_REG_LOW + 256 * AL_REG_HIGH <= 384 * 168, "register split
 constexpr uint32_t AL_OCOL = 256;          // O of tile t at columns 256 + 128 t
 constexpr uint32_t AL_TMEM_COLS = 512;
 constexpr int AL_MAXB = 64;                // sequences per call
+constexpr int AL_DELTA = 2;                // positions without a block after each unit (see Walk)
 
 // Shared memory: Q tiles | K ring | V ring | barriers | misc | the two
 // streams' row maxima and sums | blocks per unit and prefix length of each
@@ -111,41 +114,52 @@ namespace {
 // One piece: blocks [j0, j1) of unit (l, b, g), in the CTA's range.
 struct Piece {
     int l, b, g, j0, j1, nb, unit;
-    long long u0;    // the unit's first block in the block sequence
+    long long u0;    // the unit's first position in the (weighted) sequence
     bool direct;     // the whole unit
     int slot;        // partial slot (split pieces)
 };
 
-// Walks the pieces of the block range [w, w_end) of CTA c.
+// Walks the pieces of the range [w, w_end) of CTA c.  Positions: a unit of
+// sequence b spans nb[b] + AL_DELTA positions, its blocks and then AL_DELTA
+// without a block (a unit's end costs the CTA that holds it an epilogue and
+// a pipeline restart; weighting the ends evens the CTAs' times).
 struct Walk {
     long long w, w_end, w_begin, Wl;
     int B, Hkv, c;
     const int* nb;   // blocks per unit of sequence b
     __device__ __forceinline__ bool next(Piece& p) {
-        if (w >= w_end) return false;
-        const long long l = w / Wl;
-        long long r = w - l * Wl;
-        int b = 0;
-        while (b < B - 1 && r >= (long long)Hkv * nb[b]) {
-            r -= (long long)Hkv * nb[b];
-            ++b;
+        while (w < w_end) {
+            const long long l = w / Wl;
+            long long r = w - l * Wl;
+            int b = 0;
+            while (b < B - 1 && r >= (long long)Hkv * (nb[b] + AL_DELTA)) {
+                r -= (long long)Hkv * (nb[b] + AL_DELTA);
+                ++b;
+            }
+            const int n = nb[b], vn = n + AL_DELTA;
+            const int g = (int)(r / vn);
+            const int j0 = (int)(r - (long long)g * vn);
+            if (j0 >= n) {                 // (past the unit's blocks)
+                w += vn - j0;
+                continue;
+            }
+            const long long len = min((long long)(n - j0), w_end - w);
+            p.l = (int)l;
+            p.b = b;
+            p.g = g;
+            p.j0 = j0;
+            p.j1 = j0 + (int)len;
+            p.nb = n;
+            p.unit = ((int)l * B + b) * Hkv + g;
+            p.u0 = w - j0;
+            p.direct = j0 == 0 && len == n;
+            // (the CTA's first piece when its unit starts at or before the
+            // range, the rule the combining CTA applies to find the slot)
+            p.slot = 2 * c + (p.u0 <= w_begin ? 0 : 1);
+            w += len;
+            return true;
         }
-        const int n = nb[b];
-        const int g = (int)(r / n);
-        const int j0 = (int)(r - (long long)g * n);
-        const long long len = min((long long)(n - j0), w_end - w);
-        p.l = (int)l;
-        p.b = b;
-        p.g = g;
-        p.j0 = j0;
-        p.j1 = j0 + (int)len;
-        p.nb = n;
-        p.unit = ((int)l * B + b) * Hkv + g;
-        p.u0 = w - j0;
-        p.direct = j0 == 0 && len == n;
-        p.slot = 2 * c + (w == w_begin ? 0 : 1);
-        w += len;
-        return true;
+        return false;
     }
 };
 
@@ -376,7 +390,7 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
 
     // This CTA's block range.
     long long Wl = 0;
-    for (int b = 0; b < a.B; ++b) Wl += snb[b];
+    for (int b = 0; b < a.B; ++b) Wl += snb[b] + AL_DELTA;
     Wl *= a.Hkv;
     const long long W = Wl * a.L;
     const int C = gridDim.x, c = blockIdx.x;
