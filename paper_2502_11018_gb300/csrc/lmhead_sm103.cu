@@ -39,6 +39,7 @@ struct LmTcArgs {
     int rows;          // rows of this launch (<= 256)
     int row0;          // first global row of this launch (partials are indexed globally)
     int V, BN, mt, n_tiles, kblocks, stages, stage_bytes;
+    int a_bytes;       // hidden-row bytes per stage (see launch_lmhead_tc)
     uint32_t tmem_cols;
     int mode, K;
     float* logits;     // [rows_total][V] (mode LOGITS)
@@ -91,7 +92,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
         if (lane == 0) {
             const uint64_t pol_w = policy_evict_first();
             const uint64_t pol_h = policy_evict_last();
-            const uint32_t tx = (uint32_t)(a.mt * LM_A_TILE_BYTES + a.BN * 128);
+            const uint32_t tx = (uint32_t)(a.a_bytes + a.BN * 128);
             int s = 0;
             uint32_t ph = 0;
             int issued[8];   // parity of the last load issued into each stage, or -1
@@ -103,8 +104,8 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
             const int pre = t0 < a.n_tiles ? (a.stages < a.kblocks ? a.stages : a.kblocks) : 0;
             for (int q = 0; q < pre; ++q) {
                 mbar_arrive_expect_tx(&full[q], tx);
-                tma_load_2d(stage_base + (size_t)q * a.stage_bytes + a.mt * LM_A_TILE_BYTES, &tmap_w, &full[q],
-                            q * 64, t0 * a.BN, pol_w);
+                tma_load_2d(stage_base + (size_t)q * a.stage_bytes + a.a_bytes, &tmap_w, &full[q], q * 64,
+                            t0 * a.BN, pol_w);
                 issued[q] = 0;
             }
             pdl_wait();
@@ -122,7 +123,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
                     uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
                     for (int m = 0; m < a.mt; ++m)
                         tma_load_2d(st + m * LM_A_TILE_BYTES, &tmap_h, &full[s], kb * 64, m * 128, pol_h);
-                    tma_load_2d(st + a.mt * LM_A_TILE_BYTES, &tmap_w, &full[s], kb * 64, t * a.BN, pol_w);
+                    tma_load_2d(st + a.a_bytes, &tmap_w, &full[s], kb * 64, t * a.BN, pol_w);
                     issued[s] = (int)ph;
                     if (++s == a.stages) {
                         s = 0;
@@ -158,7 +159,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
                     }
                     tc_fence_after();
                     uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
-                    const uint64_t bdesc = sdesc_kmajor_sw128(smem_u32(st + a.mt * LM_A_TILE_BYTES));
+                    const uint64_t bdesc = sdesc_kmajor_sw128(smem_u32(st + a.a_bytes));
                     for (int m = 0; m < a.mt; ++m) {
                         const uint64_t adesc = sdesc_kmajor_sw128(smem_u32(st + m * LM_A_TILE_BYTES));
 #pragma unroll
@@ -381,7 +382,14 @@ int launch_lmhead_tc(const void* h, const void* W, int rows, int H, int V, int m
         a.BN = lmhead_pick_bn(V, a.mt, grid);
         a.n_tiles = (V + a.BN - 1) / a.BN;
         a.kblocks = (H + 63) / 64;
-        a.stage_bytes = a.mt * LM_A_TILE_BYTES + a.BN * 128;
+        // With at most 64 rows the hidden-row box is 64 rows (8 KB a k-block)
+        // and the stage holds only those: the M = 128 MMA's A rows 64..127
+        // then read the first 8 KB of the same stage's W tile (landed shared
+        // memory), which only feeds TMEM lanes of rows >= rows, never read
+        // back.  The freed 8 KB a stage buys a deeper ring.
+        const int h_box = r <= 64 ? 64 : 128;
+        a.a_bytes = r <= 64 ? h_box * 128 : a.mt * LM_A_TILE_BYTES;
+        a.stage_bytes = a.a_bytes + a.BN * 128;
         a.stages = (SMEM_BUDGET - 2048) / a.stage_bytes;
         if (a.stages > 8) a.stages = 8;
         const int cols = 2 * a.mt * a.BN;
@@ -393,7 +401,7 @@ int launch_lmhead_tc(const void* h, const void* W, int rows, int H, int V, int m
         a.err = err;
         CUtensorMap mh, mw;
         const char* hb = static_cast<const char*>(h) + (size_t)row0 * H * 2;
-        int rc = make_map_2d(&mh, hb, (uint64_t)r, (uint64_t)H, 128, (uint64_t)H * 2);
+        int rc = make_map_2d(&mh, hb, (uint64_t)r, (uint64_t)H, (uint32_t)h_box, (uint64_t)H * 2);
         if (rc != GV_OK) return rc;
         rc = make_map_2d(&mw, W, (uint64_t)V, (uint64_t)H, (uint32_t)a.BN, (uint64_t)H * 2);
         if (rc != GV_OK) return rc;
