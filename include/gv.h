@@ -236,7 +236,7 @@ int gv_verify_attention_merge(const gv_attn_shape* s, void* out, void* workspace
  *   workspace  >= gv_verify_attention_layers_workspace(s, L) bytes, 256-byte
  *              aligned; contents need no initialisation and are clobbered.
  * bf16 only, d = 128, 1 <= B <= 64, N <= 64, (Hq/Hkv) * N <= 256 and
- * 8 L B N (Hq + 2 Hkv) < 2^31 (else GV_ERR_UNSUPPORTED); strides are element
+ * 8 L B N (Hq + 2 Hkv) <= 2^30 (else GV_ERR_UNSUPPORTED); strides are element
  * counts, multiples of 8, each at least one layer (ignored for L = 1).  All tensors 16-byte aligned.  Two
  * calls that share a workspace must be ordered on the device.  A bounded
  * device-side wait that gives up turns the affected output rows into NaN.

@@ -981,16 +981,17 @@ tree_prep_kernel(const __nv_bfloat16* __restrict__ q, long long q_ls, const __nv
                  int ncnt) {
     pdl_wait();
     pdl_trigger();
-    const long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    // (32-bit index arithmetic: the host bounds 8 L B N (Hq + 2 Hkv) by 2^30)
+    const int t = blockIdx.x * blockDim.x + threadIdx.x;
     if (t < ncnt) cnt[t] = 0;
-    const long long nq = (long long)L * B * N * Hq, nk = (long long)L * B * N * Hkv;
-    const int c = (int)(t & 7);
+    const int nqr = B * N * Hq, nkr = B * N * Hkv;
+    const int nq = L * nqr, nk = L * nkr;
+    const int c = t & 7;
     if (t < 8 * nq) {
-        const long long row = t >> 3;
-        const long long per = (long long)B * N * Hq;
-        const long long l = row / per, r = row - l * per;
-        const long long bn = r / Hq;
-        const uint4* src = reinterpret_cast<const uint4*>(q + l * q_ls + r * 128);
+        const int row = t >> 3;
+        const int l = row / nqr, r = row - l * nqr;
+        const int bn = r / Hq;
+        const uint4* src = reinterpret_cast<const uint4*>(q + l * q_ls + (long long)r * 128);
         const uint4 lo = __ldg(src + c), hi = __ldg(src + 8 + c);
         const float4* cs = reinterpret_cast<const float4*>(rope) + bn * 32 + c * 4;
         float4 c4[4];
@@ -998,23 +999,22 @@ tree_prep_kernel(const __nv_bfloat16* __restrict__ q, long long q_ls, const __nv
         for (int e = 0; e < 4; ++e) c4[e] = __ldg(cs + e);
         uint4 olo, ohi;
         rope8(lo, hi, c4, olo, ohi);
-        uint4* dst = reinterpret_cast<uint4*>(q_rot) + row * 16;
+        uint4* dst = reinterpret_cast<uint4*>(q_rot) + (long long)row * 16;
         dst[c] = olo;
         dst[8 + c] = ohi;
         return;
     }
-    const long long u = t - 8 * nq;
+    const int u = t - 8 * nq;
     if (u >= 16 * nk) return;
     const bool isk = u < 8 * nk;
-    const long long row = (isk ? u : u - 8 * nk) >> 3;
-    const long long per = (long long)B * N * Hkv;
-    const long long l = row / per, r = row - l * per;          // r = (b * N + n) * Hkv + h
-    const long long bn = r / Hkv;
-    const int h = (int)(r - bn * Hkv);
-    const int b = (int)(bn / N), n = (int)(bn - (long long)b * N);
-    const long long drow = ((l * B + b) * Hkv + h) * N + n;    // [L][B][Hkv][N]
+    const int row = (isk ? u : u - 8 * nk) >> 3;
+    const int l = row / nkr, r = row - l * nkr;               // r = (b * N + n) * Hkv + h
+    const int bn = r / Hkv;
+    const int h = r - bn * Hkv;
+    const int b = bn / N, n = bn - b * N;
+    const long long drow = ((long long)(l * B + b) * Hkv + h) * N + n;   // [L][B][Hkv][N]
     if (isk) {
-        const uint4* src = reinterpret_cast<const uint4*>(k + l * k_ls + r * 128);
+        const uint4* src = reinterpret_cast<const uint4*>(k + l * k_ls + (long long)r * 128);
         const uint4 lo = __ldg(src + c), hi = __ldg(src + 8 + c);
         const float4* cs = reinterpret_cast<const float4*>(rope) + bn * 32 + c * 4;
         float4 c4[4];
@@ -1026,7 +1026,7 @@ tree_prep_kernel(const __nv_bfloat16* __restrict__ q, long long q_ls, const __nv
         dst[c] = olo;
         dst[8 + c] = ohi;
     } else {
-        const uint4* src = reinterpret_cast<const uint4*>(v + l * v_ls + r * 128);
+        const uint4* src = reinterpret_cast<const uint4*>(v + l * v_ls + (long long)r * 128);
         uint4* dst = reinterpret_cast<uint4*>(treeV) + drow * 16;
         dst[c] = __ldg(src + c);
         dst[8 + c] = __ldg(src + 8 + c);

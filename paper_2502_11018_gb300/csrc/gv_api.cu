@@ -370,7 +370,7 @@ static int attn_layers_shape_ok(const gv_attn_shape* s, int L) {
     return s && s->dt == GV_BF16 && s->d == 128 && L >= 1 && s->B >= 1 && s->B <= 64 && s->N >= 1 &&
            s->N <= 64 && s->Hkv >= 1 && s->Hq >= s->Hkv && s->Hq % s->Hkv == 0 &&
            (s->Hq / s->Hkv) * s->N <= 256 && s->S_max >= 1 &&
-           8LL * L * s->B * s->N * (s->Hq + 2LL * s->Hkv) < (1LL << 31);
+           8LL * L * s->B * s->N * (s->Hq + 2LL * s->Hkv) <= (1LL << 30);
 }
 
 size_t gv_verify_attention_layers_workspace(const gv_attn_shape* s, int L) {
@@ -386,7 +386,7 @@ int gv_verify_attention_layers(const gv_attn_shape* s, int L, const void* q, int
     clear_error();
     if (!attn_layers_shape_ok(s, L)) {
         set_error("gv_verify_attention_layers: unsupported shape (bf16, d = 128, L >= 1, 1 <= B <= 64, "
-                  "1 <= N <= 64, G * N <= 256, 8 L B N (Hq + 2 Hkv) < 2^31 needed)");
+                  "1 <= N <= 64, G * N <= 256, 8 L B N (Hq + 2 Hkv) <= 2^30 needed)");
         return s ? GV_ERR_UNSUPPORTED : GV_ERR_ARG;
     }
     const long long nq = (long long)s->B * s->N * s->Hq * 128, nk = (long long)s->B * s->N * s->Hkv * 128;
