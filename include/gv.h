@@ -290,10 +290,11 @@ int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int d
  *   h [rows][H] bf16, W [V][H] bf16, ids int32[rows], vals fp32[rows] (may
  *   be NULL); 1 <= rows <= GV_NOALLOC_MAX_ROWS, H a multiple of 8.
  *
- * Scratch: a fixed 512 KB + 256 B array in the library's own device memory
+ * Scratch: a fixed 512 KB + 1 KB array in the library's own device memory
  * (a file-scope __device__ array, one per device, reserved when the library
  * is loaded): per-CTA argmax partials of up to GV_NOALLOC_MAX_ROWS rows and
- * an error word, which each call zeroes on the stream before its kernels.
+ * per-CTA status words, which each call's projection kernel rewrites (no
+ * memset precedes its kernels).
  * Every call looks the array's address up (cudaGetSymbolAddress, which
  * allocates nothing), so a reset or replaced context is handled; make the
  * first call on a device before any stream capture (the lookup itself is not

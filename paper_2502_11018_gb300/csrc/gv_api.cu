@@ -170,7 +170,7 @@ static LmPlan lm_plan(int rows, int V, int dt, int mode, int k) {
     p.s = off;
     off += align256(n * sizeof(float));
     p.err = off;
-    off += 256;
+    off += align256((size_t)TC_SLOTS * sizeof(int));
     p.total = off;
     return p;
 }
@@ -178,11 +178,11 @@ static LmPlan lm_plan(int rows, int V, int dt, int mode, int k) {
 // ------------------------------------------- allocation-free LM head scratch --
 // gv_lmhead_argmax_noalloc keeps its scratch in the library's own device
 // memory: the argmax partials (value, id) of up to GV_NOALLOC_MAX_ROWS rows
-// for up to TC_SLOTS CTAs, then the error word of the bounded waits.
+// for up to TC_SLOTS CTAs, then the per-CTA status words of the bounded waits.
 constexpr size_t NOALLOC_ENTRIES = (size_t)TC_SLOTS * GV_NOALLOC_MAX_ROWS;
 constexpr size_t NOALLOC_ID_OFF = NOALLOC_ENTRIES * sizeof(float);
 constexpr size_t NOALLOC_ERR_OFF = NOALLOC_ID_OFF + NOALLOC_ENTRIES * sizeof(int);
-constexpr size_t NOALLOC_BYTES = NOALLOC_ERR_OFF + 256;
+constexpr size_t NOALLOC_BYTES = NOALLOC_ERR_OFF + (size_t)TC_SLOTS * sizeof(int);
 __device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_BYTES];
 
 // Address of the scratch in the current device's context.  Looked up on
@@ -475,7 +475,6 @@ int gv_lmhead_select(const void* h, const void* W, int rows, int H, int V, int d
         return launch_lmhead_cc(static_cast<const float*>(h), static_cast<const float*>(W), rows, H,
                                 V, mode, plan.K, logits, part, ids, vals, row_max, row_lse, st);
     int* err = reinterpret_cast<int*>(ws + plan.err);
-    if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return check_launch("memset");
     part.slots = lmhead_tc_grid(TC_SLOTS);
     int rc = launch_lmhead_tc(h, W, rows, H, V, mode, plan.K, logits, part, err, st);
     if (rc != GV_OK) return rc;
@@ -509,7 +508,6 @@ int gv_lmhead_argmax_noalloc(const void* h, const void* W, int rows, int H, int 
     part.K = 1;
     int* err = reinterpret_cast<int*>(ws + NOALLOC_ERR_OFF);
     cudaStream_t st = as_stream(stream);
-    if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return check_launch("memset");
     rc = launch_lmhead_tc(h, W, rows, H, V, GV_SELECT_ARGMAX, 1, nullptr, part, err, st);
     if (rc != GV_OK) return rc;
     return launch_lmhead_merge(part, GV_SELECT_ARGMAX, 1, ids, vals, nullptr, nullptr, err, st);

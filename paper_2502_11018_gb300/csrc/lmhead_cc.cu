@@ -186,7 +186,8 @@ lmhead_merge_kernel(SelectPartials part, int mode, int K, int32_t* __restrict__ 
     const int r = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int rows = part.rows;
-    if (err != nullptr && *err != 0) {
+    // err: the projection kernel's per-CTA status words (one per slot)
+    if (err != nullptr && __syncthreads_or(tid < part.slots && err[tid] != 0)) {
         // A bounded wait in the projection kernel gave up: no valid result.
         if (mode == GV_SELECT_LOGITS) {
             if (tid == 0 && row_max) row_max[r] = NAN;

@@ -6,10 +6,13 @@
 // written (the paper's closing remark on fusing kernels to cut memory
 // traffic).  The weight W[V][H] is read from HBM exactly once.
 //
-// One persistent CTA per SM walks vocabulary tiles of BN rows (round robin).
-// Per tile:  S[r][v] = sum_k h[r][k] W[v][k]  with the hidden rows on the MMA
-// M side (128 rows per M tile, rows beyond `rows` are zero-filled by TMA) and
-// BN vocabulary rows on the N side, both operands K-major with the 128-byte
+// One persistent CTA per SM takes a contiguous range of the vocabulary: the
+// V rows, in groups of 16, are cut into as many equal ranges as CTAs (they
+// differ by at most one group), and a CTA's range into `tpc` tiles of k or
+// k + 1 groups.  Per tile:  S[r][v] = sum_k h[r][k] W[v][k]  with the hidden
+// rows on the MMA M side (128 rows per M tile, rows beyond `rows` are
+// zero-filled by TMA) and the tile's vocabulary rows on the N side (one
+// tensor map per tile height), both operands K-major with the 128-byte
 // swizzle, fp32 accumulators in tensor memory, double-buffered so the MMA of
 // tile i+1 overlaps the epilogue of tile i.
 //
@@ -34,23 +37,41 @@ using namespace sm103;
 
 constexpr int LM_THREADS = 192;
 constexpr int LM_A_TILE_BYTES = 128 * 128;   // 128 rows x 64 bf16
+constexpr int LM_PRE_STAGES = 2;             // W stages issued before the dependency wait
 
 struct LmTcArgs {
     int rows;          // rows of this launch (<= 256)
     int row0;          // first global row of this launch (partials are indexed globally)
-    int V, BN, mt, n_tiles, kblocks, stages, stage_bytes;
+    int V, mt, kblocks, stages, stage_bytes;
+    int groups;        // 16-row vocabulary groups, ceil(V / 16)
+    int tpc;           // tiles per CTA
+    int bn_small;      // rows of the smaller tile height (tmap_ws), 0 if there is none
+    int bn_max;        // rows of the larger tile height (tmap_wb): TMEM columns per M tile
     int a_bytes;       // hidden-row bytes per stage (see launch_lmhead_tc)
     uint32_t tmem_cols;
     int mode, K;
     float* logits;     // [rows_total][V] (mode LOGITS)
     SelectPartials part;
-    int* err;
+    int* err;          // [grid] per-CTA status: 0, or GV_ERR_TIMEOUT after a bounded wait gave up
 };
+
+// Tile i of this CTA: vocabulary rows [v0, v0 + n); n = 0 means no tile.
+struct LmTile {
+    int v0, n;
+};
+__device__ __forceinline__ LmTile lm_tile(const LmTcArgs& a, int i) {
+    const int C = gridDim.x, c = blockIdx.x;
+    const int gc0 = (int)((long long)c * a.groups / C);
+    const int gcn = (int)((long long)(c + 1) * a.groups / C) - gc0;
+    const int g0 = gc0 + (int)((long long)gcn * i / a.tpc);
+    const int g1 = gc0 + (int)((long long)gcn * (i + 1) / a.tpc);
+    return {g0 * 16, (g1 - g0) * 16};
+}
 
 template <int KM>
 __global__ void __launch_bounds__(LM_THREADS, 1)
-lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_constant__ CUtensorMap tmap_w,
-                 LmTcArgs a) {
+lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_constant__ CUtensorMap tmap_ws,
+                 const __grid_constant__ CUtensorMap tmap_wb, LmTcArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
@@ -78,34 +99,40 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
         *abort = 0;
         fence_mbar_init();
         prefetch_tmap(&tmap_h);
-        prefetch_tmap(&tmap_w);
+        prefetch_tmap(&tmap_ws);
+        prefetch_tmap(&tmap_wb);
     }
     if (warp == 1) tmem_alloc(tmem_holder, a.tmem_cols);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
-    const int acc_cols = a.mt * a.BN;
+    const int acc_cols = a.mt * a.bn_max;
+    // (the map of a tile's height)
+    auto wmap = [&](int n) { return n == a.bn_small ? &tmap_ws : &tmap_wb; };
 
     if (warp == 0) {
         // ------------------------------------------------------ TMA producer
         if (lane == 0) {
             const uint64_t pol_w = policy_evict_first();
             const uint64_t pol_h = policy_evict_last();
-            const uint32_t tx = (uint32_t)(a.a_bytes + a.BN * 128);
             int s = 0;
             uint32_t ph = 0;
             int issued[8];   // parity of the last load issued into each stage, or -1
             for (int q = 0; q < 8; ++q) issued[q] = -1;
-            // The first ring fill of W (a weight: no kernel of the stream
-            // writes it) streams before the dependency wait; the hidden rows,
-            // written upstream, are loaded after it.
-            const int t0 = blockIdx.x;
-            const int pre = t0 < a.n_tiles ? (a.stages < a.kblocks ? a.stages : a.kblocks) : 0;
+            // The first W stages (a weight: no kernel of the stream writes it)
+            // stream before the dependency wait; the hidden rows, written
+            // upstream, are loaded after it.  Two stages: a deeper early fill
+            // measured about 1 us slower (its burst meets the preceding
+            // kernel's last CTAs).
+            int i0 = 0;
+            LmTile t0 = lm_tile(a, 0);
+            while (t0.n == 0 && ++i0 < a.tpc) t0 = lm_tile(a, i0);
+            const int pre = t0.n > 0 ? min(LM_PRE_STAGES, a.stages < a.kblocks ? a.stages : a.kblocks) : 0;
             for (int q = 0; q < pre; ++q) {
-                mbar_arrive_expect_tx(&full[q], tx);
-                tma_load_2d(stage_base + (size_t)q * a.stage_bytes + a.a_bytes, &tmap_w, &full[q], q * 64,
-                            t0 * a.BN, pol_w);
+                mbar_arrive_expect_tx(&full[q], (uint32_t)(a.a_bytes + t0.n * 128));
+                tma_load_2d(stage_base + (size_t)q * a.stage_bytes + a.a_bytes, wmap(t0.n), &full[q], q * 64,
+                            t0.v0, pol_w);
                 issued[q] = 0;
             }
             pdl_wait();
@@ -116,14 +143,17 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
                                 &full[q], q * 64, m * 128, pol_h);
             s = pre % a.stages;
             ph = pre == a.stages ? 1u : 0u;
-            for (int t = blockIdx.x; t < a.n_tiles; t += gridDim.x) {
-                for (int kb = t == t0 ? pre : 0; kb < a.kblocks; ++kb) {
+            for (int ti = i0; ti < a.tpc; ++ti) {
+                const LmTile tl = lm_tile(a, ti);
+                if (tl.n == 0) continue;
+                const uint32_t tx = (uint32_t)(a.a_bytes + tl.n * 128);
+                for (int kb = ti == i0 ? pre : 0; kb < a.kblocks; ++kb) {
                     if (!mbar_wait(&empty[s], ph ^ 1u, abort)) goto producer_done;
                     mbar_arrive_expect_tx(&full[s], tx);
                     uint8_t* st = stage_base + (size_t)s * a.stage_bytes;
                     for (int m = 0; m < a.mt; ++m)
                         tma_load_2d(st + m * LM_A_TILE_BYTES, &tmap_h, &full[s], kb * 64, m * 128, pol_h);
-                    tma_load_2d(st + a.a_bytes, &tmap_w, &full[s], kb * 64, t * a.BN, pol_w);
+                    tma_load_2d(st + a.a_bytes, wmap(tl.n), &full[s], kb * 64, tl.v0, pol_w);
                     issued[s] = (int)ph;
                     if (++s == a.stages) {
                         s = 0;
@@ -142,11 +172,13 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
     } else if (warp == 1) {
         // -------------------------------------------------------- MMA issuer
         if (lane == 0) {
-            const uint32_t idesc = idesc_bf16(128, a.BN);
             int s = 0;
             uint32_t ph = 0;
-            int i = 0;
-            for (int t = blockIdx.x; t < a.n_tiles; t += gridDim.x, ++i) {
+            int i = 0;      // tiles with rows so far
+            for (int ti = 0; ti < a.tpc; ++ti) {
+                const LmTile tl = lm_tile(a, ti);
+                if (tl.n == 0) continue;
+                const uint32_t idesc = idesc_bf16(128, tl.n);
                 const int acc = i & 1;
                 if (!mbar_wait(&tempty[acc], ((uint32_t)(i >> 1) & 1u) ^ 1u, abort)) break;
                 tc_fence_after();
@@ -164,7 +196,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
                         const uint64_t adesc = sdesc_kmajor_sw128(smem_u32(st + m * LM_A_TILE_BYTES));
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
-                            mma_bf16(d_base + (uint32_t)(m * a.BN), adesc + 2u * kk, bdesc + 2u * kk,
+                            mma_bf16(d_base + (uint32_t)(m * a.bn_max), adesc + 2u * kk, bdesc + 2u * kk,
                                      idesc, (kb | kk) != 0);
                     }
                     mma_commit(&empty[s]);
@@ -175,6 +207,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
                 }
                 if (!ok) break;
                 mma_commit(&tfull[acc]);
+                ++i;
             }
             // Every MMA this thread issued has completed once `drain` flips.
             mma_commit(drain);
@@ -198,8 +231,10 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
                 li[m][q] = INT32_MAX;
             }
         }
-        int i = 0;
-        for (int t = blockIdx.x; t < a.n_tiles; t += gridDim.x, ++i) {
+        int i = 0;      // tiles with rows so far
+        for (int ti = 0; ti < a.tpc; ++ti) {
+            const LmTile tl = lm_tile(a, ti);
+            if (tl.n == 0) continue;
             const int acc = i & 1;
             int ok = 1;
             if (lane == 0) ok = mbar_wait(&tfull[acc], (uint32_t)(i >> 1) & 1u, abort);
@@ -207,40 +242,53 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
             if (!ok) break;
             __syncwarp();
             tc_fence_after();
-            const int v_tile = t * a.BN;
+            const int v_tile = tl.v0;
+            const int vlim = min(a.V, tl.v0 + tl.n);   // ids at or past it are not this tile's
 #pragma unroll
             for (int m = 0; m < 2; ++m) {
                 if (m >= a.mt) break;
                 const int r = a.row0 + m * 128 + row_in_tile;
                 const bool row_ok = m * 128 + row_in_tile < a.rows;
-                for (int c0 = 0; c0 < a.BN; c0 += 32) {
+                for (int c0 = 0; c0 < tl.n; c0 += 32) {
                     uint32_t v[32];
-                    tmem_ld32(tmem + ((uint32_t)(sub * 32) << 16) +
-                                  (uint32_t)(acc * acc_cols + m * a.BN + c0), v);
+                    const uint32_t taddr = tmem + ((uint32_t)(sub * 32) << 16) +
+                                           (uint32_t)(acc * acc_cols + m * a.bn_max + c0);
+                    if (c0 + 32 <= tl.n) {
+                        tmem_ld32(taddr, v);
+                    } else {
+                        // a 16-column tail (tile heights are multiples of 16)
+                        uint32_t v16[16];
+                        tmem_ld16(taddr, v16);
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            v[j] = v16[j];
+                            v[16 + j] = 0u;
+                        }
+                    }
                     tmem_wait_ld();
                     const int id0 = v_tile + c0;
                     if (a.mode == GV_SELECT_LOGITS) {
                         float cmax = -INFINITY;
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
-                            if (id0 + j < a.V) cmax = fmaxf(cmax, __uint_as_float(v[j]));
+                            if (id0 + j < vlim) cmax = fmaxf(cmax, __uint_as_float(v[j]));
                         const float mnew = fmaxf(rm[m], cmax);
                         float sum = 0.f;
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
-                            if (id0 + j < a.V) sum += __expf(__uint_as_float(v[j]) - mnew);
+                            if (id0 + j < vlim) sum += __expf(__uint_as_float(v[j]) - mnew);
                         rs[m] = rs[m] * __expf(rm[m] - mnew) + sum;
                         rm[m] = mnew;
                         if (row_ok) {
                             float* dst = a.logits + (size_t)r * a.V + id0;
-                            if (id0 + 32 <= a.V && (a.V & 3) == 0) {
+                            if (id0 + 32 <= vlim && (a.V & 3) == 0) {
 #pragma unroll
                                 for (int j = 0; j < 32; j += 4)
                                     *reinterpret_cast<float4*>(dst + j) = make_float4(
                                         __uint_as_float(v[j]), __uint_as_float(v[j + 1]),
                                         __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
                             } else {
-                                for (int j = 0; j < 32 && id0 + j < a.V; ++j) dst[j] = __uint_as_float(v[j]);
+                                for (int j = 0; j < 32 && id0 + j < vlim; ++j) dst[j] = __uint_as_float(v[j]);
                             }
                         }
                     } else {
@@ -249,7 +297,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
                             float cv = __uint_as_float(v[j]);
                             int ci = id0 + j;
                             // ids only grow, so a strict '>' keeps the lower id on ties
-                            if (ci < a.V && cv > lv[m][KM - 1]) {
+                            if (ci < vlim && cv > lv[m][KM - 1]) {
 #pragma unroll
                                 for (int q = 0; q < KM; ++q) {
                                     if (cv > lv[m][q]) {
@@ -269,6 +317,7 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[acc]);
+            ++i;
         }
         // Per-CTA partial of every row this thread owns.
         const int slot = blockIdx.x;
@@ -297,7 +346,14 @@ lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmap_h, const __grid_consta
     __syncthreads();
     tc_fence_after();
     if (warp == 1) tmem_dealloc(tmem, a.tmem_cols);
-    if (threadIdx.x == 0 && *abort) atomicExch(a.err, GV_ERR_TIMEOUT);
+    // Every CTA rewrites its status word each call (the first row chunk
+    // clears it, any chunk may raise it), so no memset precedes the launch.
+    if (threadIdx.x == 0) {
+        if (*abort)
+            a.err[blockIdx.x] = GV_ERR_TIMEOUT;
+        else if (a.row0 == 0)
+            a.err[blockIdx.x] = 0;
+    }
 }
 
 // ----------------------------------------------------------------- host side
@@ -342,23 +398,6 @@ int make_map_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols
     return GV_OK;
 }
 
-// Vocabulary tile width: the multiple of 32 (<= 256 / mt) that minimises the
-// estimated time ceil(tiles / ctas) * (BN + per-tile overhead).
-int lmhead_pick_bn(int V, int mt, int ctas) {
-    int best = 64;
-    long best_cost = -1;
-    for (int bn = 64; bn * mt <= 256; bn += 32) {
-        const long tiles = (V + bn - 1) / bn;
-        const long waves = (tiles + ctas - 1) / ctas;
-        const long cost = waves * (bn + 16);
-        if (best_cost < 0 || cost < best_cost) {
-            best_cost = cost;
-            best = bn;
-        }
-    }
-    return best;
-}
-
 // Number of CTAs (= partial slots) the tensor-core LM head launches with.
 int lmhead_tc_grid(int slots_capacity) {
     const int c = sm_count();
@@ -379,41 +418,57 @@ int launch_lmhead_tc(const void* h, const void* W, int rows, int H, int V, int m
         a.row0 = row0;
         a.V = V;
         a.mt = (r + 127) / 128;
-        a.BN = lmhead_pick_bn(V, a.mt, grid);
-        a.n_tiles = (V + a.BN - 1) / a.BN;
+        // Balanced vocabulary ranges: ceil(V / 16) groups of 16 rows cut into
+        // `grid` ranges, each into tpc tiles of at most 16 / mt groups (TMEM:
+        // two accumulators of mt x tile columns in 512); the tiles then have
+        // kmin or kmin + 1 groups.
+        a.groups = (V + 15) / 16;
+        const int gmax_tile = 16 / a.mt;
+        const int gcmax = (a.groups + grid - 1) / grid;
+        a.tpc = std::max(1, (gcmax + gmax_tile - 1) / gmax_tile);
+        const int kmin = (a.groups / grid) / a.tpc, kmax = (gcmax + a.tpc - 1) / a.tpc;
+        a.bn_max = 16 * kmax;
+        a.bn_small = kmin >= 1 && kmin < kmax ? 16 * kmin : 0;
         a.kblocks = (H + 63) / 64;
-        // With at most 64 rows the hidden-row box is 64 rows (8 KB a k-block)
-        // and the stage holds only those: the M = 128 MMA's A rows 64..127
-        // then read the first 8 KB of the same stage's W tile (landed shared
-        // memory), which only feeds TMEM lanes of rows >= rows, never read
-        // back.  The freed 8 KB a stage buys a deeper ring.
-        const int h_box = r <= 64 ? 64 : 128;
-        a.a_bytes = r <= 64 ? h_box * 128 : a.mt * LM_A_TILE_BYTES;
-        a.stage_bytes = a.a_bytes + a.BN * 128;
+        // With at most 64 rows and W tiles of at least 64 rows (8 KB a
+        // k-block) the hidden-row box is 64 rows and the stage holds only
+        // those: the M = 128 MMA's A rows 64..127 then read the first 8 KB of
+        // the same stage's W tile (landed shared memory), which only feeds
+        // TMEM lanes of rows >= rows, never read back.  The freed 8 KB a stage
+        // buys a deeper ring.  A smaller W tile would leave those 8 KB short
+        // of the stage (past the ring's end in the last one), so the A tile
+        // then keeps its full 16 KB.
+        const bool alias = r <= 64 && a.bn_max >= 64;
+        const int h_box = alias ? 64 : 128;
+        a.a_bytes = alias ? h_box * 128 : a.mt * LM_A_TILE_BYTES;
+        a.stage_bytes = a.a_bytes + a.bn_max * 128;
         a.stages = (SMEM_BUDGET - 2048) / a.stage_bytes;
         if (a.stages > 8) a.stages = 8;
-        const int cols = 2 * a.mt * a.BN;
+        const int cols = 2 * a.mt * a.bn_max;
         a.tmem_cols = cols <= 32 ? 32 : cols <= 64 ? 64 : cols <= 128 ? 128 : cols <= 256 ? 256 : 512;
         a.mode = mode;
         a.K = K;
         a.logits = logits;
         a.part = part;
         a.err = err;
-        CUtensorMap mh, mw;
+        CUtensorMap mh, mws, mwb;
         const char* hb = static_cast<const char*>(h) + (size_t)row0 * H * 2;
         int rc = make_map_2d(&mh, hb, (uint64_t)r, (uint64_t)H, (uint32_t)h_box, (uint64_t)H * 2);
         if (rc != GV_OK) return rc;
-        rc = make_map_2d(&mw, W, (uint64_t)V, (uint64_t)H, (uint32_t)a.BN, (uint64_t)H * 2);
+        rc = make_map_2d(&mwb, W, (uint64_t)V, (uint64_t)H, (uint32_t)a.bn_max, (uint64_t)H * 2);
+        if (rc != GV_OK) return rc;
+        rc = make_map_2d(&mws, W, (uint64_t)V, (uint64_t)H, (uint32_t)(a.bn_small ? a.bn_small : a.bn_max),
+                         (uint64_t)H * 2);
         if (rc != GV_OK) return rc;
         const size_t smem = 1024 + (size_t)a.stages * a.stage_bytes + 8 * (2 * a.stages + 5) + 16;
         if (mode == GV_SELECT_TOPK) {
             cudaFuncSetAttribute(lmhead_tc_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)smem);
-            launch_pdl(lmhead_tc_kernel<16>, dim3(grid), dim3(LM_THREADS), smem, st, mh, mw, a);
+            launch_pdl(lmhead_tc_kernel<16>, dim3(grid), dim3(LM_THREADS), smem, st, mh, mws, mwb, a);
         } else {
             cudaFuncSetAttribute(lmhead_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)smem);
-            launch_pdl(lmhead_tc_kernel<1>, dim3(grid), dim3(LM_THREADS), smem, st, mh, mw, a);
+            launch_pdl(lmhead_tc_kernel<1>, dim3(grid), dim3(LM_THREADS), smem, st, mh, mws, mwb, a);
         }
         rc = check_launch("lmhead_tc_kernel");
         if (rc != GV_OK) return rc;

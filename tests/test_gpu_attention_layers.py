@@ -124,8 +124,21 @@ def test_attention_layers_matches_per_layer_calls():
         assert rel_err(f64(out[l]), f64(o1)) <= TOL_ATTN["bf16"]
 
 
+def _within_ulp(x, y):
+    """x and y (bf16) differ by at most one bf16 ulp of y, element by element."""
+    xf, yf = x.float().cpu(), y.float().cpu()
+    assert torch.equal(torch.isnan(xf), torch.isnan(yf))
+    ulp = torch.where(yf == 0, torch.full_like(yf, 2.0 ** -133),
+                      torch.ldexp(torch.ones_like(yf), torch.frexp(yf.abs()).exponent - 8))
+    assert bool(((xf - yf).abs().nan_to_num(0.0) <= ulp).all())
+
+
 def test_attention_layers_reused_workspace_and_strided_layers():
-    """Three calls on one dirty workspace agree bit for bit, and inputs given
+    """Eight calls on one dirty workspace agree -- the tree K/V scratch bit for
+    bit, the outputs to one bf16 ulp: a unit cut between two CTAs is combined
+    by whichever of its pieces arrives second, from that piece's fp32
+    accumulators and the other's bf16 partial rows, so the last rounding
+    depends on which piece it is -- and inputs given
     as views of a packed per-layer buffer (q | k_new | v_new per layer) give
     the same bits as contiguous ones."""
     dev = device()
@@ -133,9 +146,10 @@ def test_attention_layers_reused_workspace_and_strided_layers():
     parents, P, S_max, q, k, v, cK, cV = _case(L, B, N, Hq, Hkv, P, 22)
     shape = gv.attn_shape(B, N, Hq, Hkv, 128, S_max, gv.GV_BF16)
     ws = torch.full((gv.gv_verify_attention_layers_workspace(shape, L),), 0xFF, dtype=torch.uint8, device=dev)
-    outs = [run_layers(dev, parents, P, S_max, q, k, v, cK, cV, base, ws) for _ in range(3)]
+    outs = [run_layers(dev, parents, P, S_max, q, k, v, cK, cV, base, ws) for _ in range(8)]
     for o in outs[1:]:
-        assert all(torch.equal(a, b) for a, b in zip(o, outs[0]))
+        assert torch.equal(o[1], outs[0][1]) and torch.equal(o[2], outs[0][2])
+        _within_ulp(o[0], outs[0][0])
     nq, nk = q[0].numel(), k[0].numel()
     packed = torch.empty(L, nq + 2 * nk, dtype=torch.bfloat16, device=dev)
     packed[:, :nq] = q.reshape(L, nq).to(dev)
@@ -150,5 +164,6 @@ def test_attention_layers_reused_workspace_and_strided_layers():
     out = torch.zeros(L, B, N, Hq, 128, dtype=torch.bfloat16, device=dev)
     gv.gv_verify_attention_layers(shape, qv, kv, vv, cK.to(dev), cV.to(dev), Pd, rope, anc, tK, tV, out, ws)
     torch.cuda.synchronize()
-    assert torch.equal(out, outs[0][0]) and torch.equal(tK, outs[0][1]) and torch.equal(tV, outs[0][2])
+    assert torch.equal(tK, outs[0][1]) and torch.equal(tV, outs[0][2])
+    _within_ulp(out, outs[0][0])
     check_layers(outs[0][0], outs[0][1], outs[0][2], parents, P, q, k, v, cK, cV, base)
