@@ -12,9 +12,10 @@
 // or two 128-row M tiles, T) against its keys, cut into 128-key blocks.
 // Block 0 of a unit holds the N tree keys (masked per query row by its
 // ancestor bitmask), blocks 1 .. ceil(P_b / 128) the cached prefix.  The
-// blocks of all units, in (l, b, g, block) order, each unit followed by
-// AL_DELTA positions without a block (the weight of a unit's end: an epilogue
-// and a pipeline restart for the CTA that holds it), form one sequence of W
+// blocks of all units, in (l, b, g, block) order, each unit's blocks between
+// AL_DSTART and AL_DEND positions without a block (the weights of a unit's
+// start and end: pipeline restarts and epilogues for the CTAs that hold
+// them), form one sequence of W
 // positions that is cut into gridDim.x contiguous ranges of equal length
 // (stream-K): CTA c takes the blocks at positions [c W / C, (c + 1) W / C).
 // A unit inside one range is a whole piece, whose rows go straight to the
@@ -79,7 +80,8 @@ static_assert(128 * AL_REG_LOW + 256 * AL_REG_HIGH <= 384 * 168, "register split
 constexpr uint32_t AL_OCOL = 256;          // O of tile t at columns 256 + 128 t
 constexpr uint32_t AL_TMEM_COLS = 512;
 constexpr int AL_MAXB = 64;                // sequences per call
-constexpr int AL_DELTA = 2;                // positions without a block after each unit (see Walk)
+constexpr int AL_DSTART = 2;               // positions without a block before each unit's blocks (see Walk)
+constexpr int AL_DEND = 0;                 // ... and after them
 
 // Shared memory: Q tiles | K ring | V ring | barriers | misc | the two
 // streams' row maxima and sums | blocks per unit and prefix length of each
@@ -120,9 +122,10 @@ struct Piece {
 };
 
 // Walks the pieces of the range [w, w_end) of CTA c.  Positions: a unit of
-// sequence b spans nb[b] + AL_DELTA positions, its blocks and then AL_DELTA
-// without a block (a unit's end costs the CTA that holds it an epilogue and
-// a pipeline restart; weighting the ends evens the CTAs' times).
+// sequence b spans AL_DSTART + nb[b] + AL_DEND positions: AL_DSTART without a
+// block, its blocks, AL_DEND without a block (a unit's start and end cost
+// the CTAs that hold them a pipeline restart and an epilogue; weighting them
+// evens the CTAs' times).
 struct Walk {
     long long w, w_end, w_begin, Wl;
     int B, Hkv, c;
@@ -132,15 +135,19 @@ struct Walk {
             const long long l = w / Wl;
             long long r = w - l * Wl;
             int b = 0;
-            while (b < B - 1 && r >= (long long)Hkv * (nb[b] + AL_DELTA)) {
-                r -= (long long)Hkv * (nb[b] + AL_DELTA);
+            while (b < B - 1 && r >= (long long)Hkv * (nb[b] + AL_DSTART + AL_DEND)) {
+                r -= (long long)Hkv * (nb[b] + AL_DSTART + AL_DEND);
                 ++b;
             }
-            const int n = nb[b], vn = n + AL_DELTA;
+            const int n = nb[b], vn = AL_DSTART + n + AL_DEND;
             const int g = (int)(r / vn);
-            const int j0 = (int)(r - (long long)g * vn);
+            const int j0 = (int)(r - (long long)g * vn) - AL_DSTART;
+            if (j0 < 0) {                  // (before the unit's blocks)
+                w -= j0;
+                continue;
+            }
             if (j0 >= n) {                 // (past the unit's blocks)
-                w += vn - j0;
+                w += n + AL_DEND - j0;
                 continue;
             }
             const long long len = min((long long)(n - j0), w_end - w);
@@ -390,7 +397,7 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
 
     // This CTA's block range.
     long long Wl = 0;
-    for (int b = 0; b < a.B; ++b) Wl += snb[b] + AL_DELTA;
+    for (int b = 0; b < a.B; ++b) Wl += snb[b] + AL_DSTART + AL_DEND;
     Wl *= a.Hkv;
     const long long W = Wl * a.L;
     const int C = gridDim.x, c = blockIdx.x;

@@ -81,11 +81,17 @@ def run_layers(dev, parents, P, S_max, q, k, v, cK, cV, base, ws=None):
     return out, tK, tV
 
 
-def check_layers(out, tK, tV, parents, P, q, k, v, cK, cV, base):
+def oracle_layers(parents, P, q, k, v, cK, cV, base):
+    """The float64 oracle's (out, tree K, tree V) of every layer."""
     depth, pos, anc, _ = oracle.tree_build(parents, P)
+    return [oracle.tree_attention(f64(q[l]), f64(k[l]), f64(v[l]), f64(cK[l]), f64(cV[l]), P, pos, anc, base)
+            for l in range(q.shape[0])]
+
+
+def check_layers(out, tK, tV, parents, P, q, k, v, cK, cV, base, refs=None):
+    refs = refs if refs is not None else oracle_layers(parents, P, q, k, v, cK, cV, base)
     for l in range(q.shape[0]):
-        ro, rK, rV = oracle.tree_attention(f64(q[l]), f64(k[l]), f64(v[l]), f64(cK[l]), f64(cV[l]), P, pos, anc,
-                                           base)
+        ro, rK, rV = refs[l]
         o = f64(out[l])
         assert np.isfinite(o).all(), l
         assert rel_err(o, ro) <= TOL_ATTN["bf16"], (l, rel_err(o, ro))
@@ -124,23 +130,15 @@ def test_attention_layers_matches_per_layer_calls():
         assert rel_err(f64(out[l]), f64(o1)) <= TOL_ATTN["bf16"]
 
 
-def _within_ulp(x, y):
-    """x and y (bf16) differ by at most one bf16 ulp of y, element by element."""
-    xf, yf = x.float().cpu(), y.float().cpu()
-    assert torch.equal(torch.isnan(xf), torch.isnan(yf))
-    ulp = torch.where(yf == 0, torch.full_like(yf, 2.0 ** -133),
-                      torch.ldexp(torch.ones_like(yf), torch.frexp(yf.abs()).exponent - 8))
-    assert bool(((xf - yf).abs().nan_to_num(0.0) <= ulp).all())
-
-
 def test_attention_layers_reused_workspace_and_strided_layers():
-    """Eight calls on one dirty workspace agree -- the tree K/V scratch bit for
-    bit, the outputs to one bf16 ulp: a unit cut between two CTAs is combined
-    by whichever of its pieces arrives second, from that piece's fp32
-    accumulators and the other's bf16 partial rows, so the last rounding
-    depends on which piece it is -- and inputs given
-    as views of a packed per-layer buffer (q | k_new | v_new per layer) give
-    the same bits as contiguous ones."""
+    """Eight calls on one dirty workspace: the tree K/V scratch agrees bit for
+    bit, and every call's outputs pass the float64 oracle's bound and agree
+    with the first call's to 2^-6 of their scale.  (A unit cut between two
+    CTAs is combined by whichever of its pieces arrives second, from its fp32
+    accumulators and the other's bf16 partial rows, or merged from both
+    partials when they arrive together: equally valid roundings, so calls
+    need not agree bit for bit.)  Inputs given as views of a packed per-layer
+    buffer (q | k_new | v_new per layer) give the same tree K/V bits."""
     dev = device()
     L, B, N, Hq, Hkv, P, base = 4, 2, 60, 32, 8, [1000, 3000], 5e5
     parents, P, S_max, q, k, v, cK, cV = _case(L, B, N, Hq, Hkv, P, 22)
@@ -149,7 +147,10 @@ def test_attention_layers_reused_workspace_and_strided_layers():
     outs = [run_layers(dev, parents, P, S_max, q, k, v, cK, cV, base, ws) for _ in range(8)]
     for o in outs[1:]:
         assert torch.equal(o[1], outs[0][1]) and torch.equal(o[2], outs[0][2])
-        _within_ulp(o[0], outs[0][0])
+        assert rel_err(f64(o[0]), f64(outs[0][0])) <= 2.0 ** -6
+    refs = oracle_layers(parents, P, q, k, v, cK, cV, base)
+    for o in outs:
+        check_layers(o[0], o[1], o[2], parents, P, q, k, v, cK, cV, base, refs)
     nq, nk = q[0].numel(), k[0].numel()
     packed = torch.empty(L, nq + 2 * nk, dtype=torch.bfloat16, device=dev)
     packed[:, :nq] = q.reshape(L, nq).to(dev)
@@ -165,5 +166,4 @@ def test_attention_layers_reused_workspace_and_strided_layers():
     gv.gv_verify_attention_layers(shape, qv, kv, vv, cK.to(dev), cV.to(dev), Pd, rope, anc, tK, tV, out, ws)
     torch.cuda.synchronize()
     assert torch.equal(tK, outs[0][1]) and torch.equal(tV, outs[0][2])
-    _within_ulp(out, outs[0][0])
-    check_layers(outs[0][0], outs[0][1], outs[0][2], parents, P, q, k, v, cK, cV, base)
+    assert rel_err(f64(out), f64(outs[0][0])) <= 2.0 ** -6
