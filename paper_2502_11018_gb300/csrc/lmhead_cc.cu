@@ -10,10 +10,10 @@
 // (grid: vocabulary tiles x row tiles, so even a 4096-row vocabulary spreads
 // over most SMs).  The block stages its W rows and hidden-state rows for 512
 // of the hidden dimension at a time in shared memory, every thread's loads in
-// flight at once; lane l of each warp scores vocabulary row l against all 16
-// hidden-state rows (16 accumulators, the hidden-state values read as
-// warp-wide broadcasts), and the 8 warps take interleaved 4-wide slices of
-// the hidden dimension, summed across warps at the end.  The selection then
+// flight at once; each thread scores a 4 x 4 sub-tile (vocabulary rows
+// vq + 8 i against hidden-state rows rq + 4 j: 16 accumulators, 8 16-byte
+// shared-memory loads per 64 FMAs), and the 8 warps take interleaved 4-wide
+// slices of the hidden dimension, summed across warps at the end.  The selection then
 // runs on the tile in shared memory and leaves one partial result per (tile,
 // row) in the workspace; lmhead_merge_kernel reduces the partials of every
 // row.
@@ -76,9 +76,14 @@ lmhead_cc_kernel(const T* __restrict__ h, const T* __restrict__ W, int rows, int
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int v0 = blockIdx.x * CC_TV;
     const int r0 = blockIdx.y * CC_TR;
-    float acc[CC_TR];
+    // Thread (warp w, lane): vocabulary rows vq + 8 i and hidden rows
+    // rq + 4 j (i, j < 4) of the tile, hidden dimension 4 w, 4 w + 32, ...
+    const int vq = lane & 7, rq = lane >> 3;
+    float acc[4][4];
 #pragma unroll
-    for (int r = 0; r < CC_TR; ++r) acc[r] = 0.f;
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
     for (int k0 = 0; k0 < H; k0 += CC_KC) {
         const int kc = min(CC_KC, H - k0), kc4 = (kc + 3) & ~3;
         __syncthreads();
@@ -125,19 +130,27 @@ lmhead_cc_kernel(const T* __restrict__ h, const T* __restrict__ W, int rows, int
             }
         }
         __syncthreads();
-        const float* wrow = sW + lane * CC_KS;
+        // (a warp's 16-byte loads hit 8 consecutive W rows and 4 consecutive
+        // hidden rows, each shared by 4 or 8 lanes: distinct bank groups)
         for (int kk = 4 * warp; kk < kc4; kk += 32) {
-            const float4 w4 = *reinterpret_cast<const float4*>(wrow + kk);
+            float4 w4[4], h4[4];
 #pragma unroll
-            for (int r = 0; r < CC_TR; ++r) {
-                const float4 h4 = *reinterpret_cast<const float4*>(sH + r * CC_KS + kk);
-                acc[r] = fmaf(w4.x, h4.x, fmaf(w4.y, h4.y, fmaf(w4.z, h4.z, fmaf(w4.w, h4.w, acc[r]))));
-            }
+            for (int i = 0; i < 4; ++i) w4[i] = *reinterpret_cast<const float4*>(sW + (vq + 8 * i) * CC_KS + kk);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) h4[j] = *reinterpret_cast<const float4*>(sH + (rq + 4 * j) * CC_KS + kk);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    acc[i][j] = fmaf(w4[i].x, h4[j].x,
+                                     fmaf(w4[i].y, h4[j].y, fmaf(w4[i].z, h4[j].z, fmaf(w4[i].w, h4[j].w, acc[i][j]))));
         }
     }
     // Sum the warps' slices of the hidden dimension.
 #pragma unroll
-    for (int r = 0; r < CC_TR; ++r) sRed[(warp * CC_TR + r) * (CC_TV + 1) + lane] = acc[r];
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) sRed[(warp * CC_TR + rq + 4 * j) * (CC_TV + 1) + vq + 8 * i] = acc[i][j];
     __syncthreads();
     for (int e = tid; e < CC_TR * CC_TV; e += 256) {
         const int rr = e / CC_TV, vv = e % CC_TV;
