@@ -76,6 +76,8 @@ rope_tree_f32_kernel(const float* __restrict__ q, const float* __restrict__ k_ne
                      const float* __restrict__ v_new, const float2* __restrict__ rope, int B, int N,
                      int Hq, int Hkv, int d, float* __restrict__ q_rot, float* __restrict__ treeK,
                      float* __restrict__ treeV, int q_rows_pad) {
+    pdl_wait();
+    pdl_trigger();
     const int half = d >> 1;
     const int H = Hq + Hkv;
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -111,7 +113,7 @@ rope_tree_f32_kernel(const float* __restrict__ q, const float* __restrict__ k_ne
 
 int launch_rope_tree_f32(const AttnArgs& a, cudaStream_t st) {
     const long long total = (long long)a.B * a.N * (a.d / 2) * (a.Hq + a.Hkv);
-    rope_tree_f32_kernel<<<(unsigned)((total + 127) / 128), 128, 0, st>>>(
+    launch_pdl(rope_tree_f32_kernel, dim3((unsigned)((total + 127) / 128)), dim3(128), 0, st,
         static_cast<const float*>(a.q), static_cast<const float*>(a.k_new),
         static_cast<const float*>(a.v_new), reinterpret_cast<const float2*>(a.rope), a.B, a.N, a.Hq,
         a.Hkv, a.d, static_cast<float*>(a.q_rot), static_cast<float*>(a.treeK),
@@ -127,6 +129,8 @@ template <typename T, int D>
 __global__ void __launch_bounds__(256)
 attn_combine_kernel(const float* __restrict__ part_o, const float* __restrict__ part_ml, int B,
                     int N, int Hq, int Hkv, int nsplit, int R, T* __restrict__ out) {
+    pdl_wait();
+    pdl_trigger();
     const int w = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (w >= B * N * Hq) return;
@@ -173,11 +177,11 @@ int launch_attn_combine_f32(const AttnArgs& a, cudaStream_t st) {
     const int blocks = (warps * 32 + 255) / 256;
     float* out = static_cast<float*>(a.out);
     if (a.d == 128)
-        attn_combine_kernel<float, 128><<<blocks, 256, 0, st>>>(a.part_o, a.part_ml, a.B, a.N, a.Hq,
-                                                                a.Hkv, a.nsplit, a.R, out);
+        launch_pdl(attn_combine_kernel<float, 128>, dim3(blocks), dim3(256), 0, st, a.part_o, a.part_ml, a.B, a.N,
+                   a.Hq, a.Hkv, a.nsplit, a.R, out);
     else
-        attn_combine_kernel<float, 64><<<blocks, 256, 0, st>>>(a.part_o, a.part_ml, a.B, a.N, a.Hq,
-                                                               a.Hkv, a.nsplit, a.R, out);
+        launch_pdl(attn_combine_kernel<float, 64>, dim3(blocks), dim3(256), 0, st, a.part_o, a.part_ml, a.B, a.N,
+                   a.Hq, a.Hkv, a.nsplit, a.R, out);
     return check_launch("attn_combine_kernel");
 }
 
@@ -200,6 +204,8 @@ attn_cc_kernel(AttnArgs a) {
     float* sK = sQ + ROWS * (D + 1);           // [CC_KEYS][D+1]
     float* sV = sK + CC_KEYS * (D + 1);        // [CC_KEYS][D+1]
     float* sS = sV + CC_KEYS * (D + 1);        // [ROWS][CC_KEYS + 1]
+    pdl_wait();
+    pdl_trigger();
     const int nrc = (a.R + ROWS - 1) / ROWS;
     const int bg = blockIdx.x / nrc, rc = blockIdx.x % nrc;
     const int b = bg / a.Hkv;
@@ -353,7 +359,7 @@ static int launch_cc(const AttnArgs& a, cudaStream_t st) {
     }
     const int nrc = (a.R + ROWS - 1) / ROWS;
     dim3 grid(a.B * a.Hkv * nrc, a.nsplit);
-    attn_cc_kernel<T, D, ROWS><<<grid, 256, smem, st>>>(a);
+    launch_pdl(attn_cc_kernel<T, D, ROWS>, grid, dim3(256), smem, st, a);
     return check_launch("attn_cc_kernel");
 }
 

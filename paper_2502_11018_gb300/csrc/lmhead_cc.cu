@@ -73,6 +73,8 @@ lmhead_cc_kernel(const T* __restrict__ h, const T* __restrict__ W, int rows, int
     float* sH = sW + CC_TV * CC_KS;                   // [CC_TR][CC_KS]
     float* sRed = sH + CC_TR * CC_KS;                 // [8 warps][CC_TR][CC_TV + 1]
     float(*sS)[CC_TV + 1] = reinterpret_cast<float(*)[CC_TV + 1]>(sRed + 8 * CC_TR * (CC_TV + 1));
+    pdl_wait();
+    pdl_trigger();
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int v0 = blockIdx.x * CC_TV;
     const int r0 = blockIdx.y * CC_TR;
@@ -313,7 +315,7 @@ int launch_lmhead_cc(const float* h, const float* W, int rows, int H, int V, int
         attr_dev = dev;
     }
     dim3 grid((V + CC_TV - 1) / CC_TV, (rows + CC_TR - 1) / CC_TR);
-    lmhead_cc_kernel<float><<<grid, 256, CC_SMEM, st>>>(h, W, rows, H, V, mode, K, logits, part);
+    launch_pdl(lmhead_cc_kernel<float>, grid, dim3(256), CC_SMEM, st, h, W, rows, H, V, mode, K, logits, part);
     const int rc = check_launch("lmhead_cc_kernel");
     if (rc != GV_OK) return rc;
     return launch_lmhead_merge(part, mode, K, ids, vals, row_max, row_lse, nullptr, st);
