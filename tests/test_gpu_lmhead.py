@@ -25,6 +25,13 @@ CASES = [
     ("bf16", 1, 128, 4097),        # ragged vocab tail
     ("bf16", 240, 5120, 32000),    # 4 sequences x 60 nodes, LLaMA-2-13B hidden
     ("bf16", 61, 1024, 50000),
+    # vocabulary splits of the tensor-core kernel: five tiles of 13 / 14 row
+    # groups per CTA at the 64-row limit of the stage layout that lets the
+    # MMA read past the hidden rows; fewer 16-row groups than CTAs; one
+    # partial group
+    ("bf16", 64, 256, 160000),
+    ("bf16", 3, 64, 100),
+    ("bf16", 2, 64, 15),
 ]
 
 
@@ -59,7 +66,7 @@ def test_argmax_parity(case):
     assert rel_err(vals.cpu().numpy(), rval) <= TOL_LOGITS[dtype]
 
 
-@pytest.mark.parametrize("case", [0, 2, 3, 4])
+@pytest.mark.parametrize("case", [0, 2, 3, 4, 6, 7])
 @pytest.mark.parametrize("k", [1, 3, 10, 16])
 def test_topk_parity(case, k):
     dev = device()
@@ -87,7 +94,7 @@ def test_topk_parity(case, k):
             assert abs(ref[r, gi[r, j]] - gval[r, j]) <= tol
 
 
-@pytest.mark.parametrize("case", [0, 2, 3])
+@pytest.mark.parametrize("case", [0, 2, 3, 6, 7, 8])
 def test_logits_lse_parity(case):
     dev = device()
     dtype, rows, H, V = CASES[case]
