@@ -32,6 +32,8 @@ CASES = [
     (2, 1, 61, 16, 4, [777], 5e5),                   # 244 rows per KV head
     (2, 16, 3, 32, 8, [512, 768, 1024, 1536] * 4, 5e5),   # batched chains
     (2, 4, 60, 40, 40, [64, 65, 255, 256], 1e4),     # ragged batch, MHA
+    (1, 64, 4, 8, 8, [(37 * i) % 600 for i in range(64)], 1e4),   # 64 sequences, the most a call takes
+    (2, 2, 40, 12, 4, [333, 0], 5e5),                # G = 3: 42 nodes per 128-row tile, 120 rows
 ]
 
 
