@@ -147,7 +147,7 @@ static AttnPlan attn_plan(const gv_attn_shape* s) {
 }
 
 // ------------------------------------------------------------ lmhead plan --
-constexpr int CC_TV = 32;        // vocabulary tile of the CUDA-core (fp32) kernel
+constexpr int CC_TV = 16;        // vocabulary tile of the CUDA-core (fp32) kernel
 constexpr int TC_SLOTS = 256;    // partial slots of the tensor-core kernel (one per CTA)
 
 struct LmPlan {

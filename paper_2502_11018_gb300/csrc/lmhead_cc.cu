@@ -6,13 +6,13 @@
 // tensor cores' tf32 mode would round the operands to 10-bit mantissas, well
 // outside the 1e-4 relative tolerance fp32 results are held to.
 //
-// Tile: 32 vocabulary rows x 16 hidden-state rows per 256-thread block
-// (grid: vocabulary tiles x row tiles, so even a 4096-row vocabulary spreads
-// over most SMs).  The block stages its W rows and hidden-state rows for 512
+// Tile: 16 vocabulary rows x 16 hidden-state rows per 256-thread block
+// (grid: vocabulary tiles x row tiles, so a 4096-row vocabulary spreads over
+// every SM).  The block stages its W rows and hidden-state rows for 512
 // of the hidden dimension at a time in shared memory, every thread's loads in
-// flight at once; each thread scores a 4 x 4 sub-tile (vocabulary rows
-// vq + 8 i against hidden-state rows rq + 4 j: 16 accumulators, 8 16-byte
-// shared-memory loads per 64 FMAs), and the 8 warps take interleaved 4-wide
+// flight at once; each thread scores a 2 x 4 sub-tile (vocabulary rows
+// vq + 8 i against hidden-state rows rq + 4 j: 8 accumulators, 6 16-byte
+// shared-memory loads per 32 FMAs), and the 8 warps take interleaved 4-wide
 // slices of the hidden dimension, summed across warps at the end.  The selection then
 // runs on the tile in shared memory and leaves one partial result per (tile,
 // row) in the workspace; lmhead_merge_kernel reduces the partials of every
@@ -21,7 +21,8 @@
 
 namespace gv {
 
-constexpr int CC_TV = 32;            // vocab rows per tile (a warp's lanes)
+constexpr int CC_TV = 16;            // vocab rows per tile (a multiple of 8, at most a warp's lanes)
+constexpr int CC_VI = CC_TV / 8;      // vocabulary rows per thread
 constexpr int CC_TR = 16;            // hidden-state rows per tile
 constexpr int CC_KC = 512;           // hidden dim staged per pass
 constexpr int CC_KS = CC_KC + 4;     // staged row stride: 16-byte rows, the 8 lanes of a
@@ -81,9 +82,9 @@ lmhead_cc_kernel(const T* __restrict__ h, const T* __restrict__ W, int rows, int
     // Thread (warp w, lane): vocabulary rows vq + 8 i and hidden rows
     // rq + 4 j (i, j < 4) of the tile, hidden dimension 4 w, 4 w + 32, ...
     const int vq = lane & 7, rq = lane >> 3;
-    float acc[4][4];
+    float acc[CC_VI][4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < CC_VI; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
     for (int k0 = 0; k0 < H; k0 += CC_KC) {
@@ -135,13 +136,13 @@ lmhead_cc_kernel(const T* __restrict__ h, const T* __restrict__ W, int rows, int
         // (a warp's 16-byte loads hit 8 consecutive W rows and 4 consecutive
         // hidden rows, each shared by 4 or 8 lanes: distinct bank groups)
         for (int kk = 4 * warp; kk < kc4; kk += 32) {
-            float4 w4[4], h4[4];
+            float4 w4[CC_VI], h4[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) w4[i] = *reinterpret_cast<const float4*>(sW + (vq + 8 * i) * CC_KS + kk);
+            for (int i = 0; i < CC_VI; ++i) w4[i] = *reinterpret_cast<const float4*>(sW + (vq + 8 * i) * CC_KS + kk);
 #pragma unroll
             for (int j = 0; j < 4; ++j) h4[j] = *reinterpret_cast<const float4*>(sH + (rq + 4 * j) * CC_KS + kk);
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
+            for (int i = 0; i < CC_VI; ++i)
 #pragma unroll
                 for (int j = 0; j < 4; ++j)
                     acc[i][j] = fmaf(w4[i].x, h4[j].x,
@@ -150,7 +151,7 @@ lmhead_cc_kernel(const T* __restrict__ h, const T* __restrict__ W, int rows, int
     }
     // Sum the warps' slices of the hidden dimension.
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < CC_VI; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) sRed[(warp * CC_TR + rq + 4 * j) * (CC_TV + 1) + vq + 8 * i] = acc[i][j];
     __syncthreads();
@@ -170,7 +171,7 @@ lmhead_cc_kernel(const T* __restrict__ h, const T* __restrict__ W, int rows, int
     for (int rr = warp; rr < CC_TR; rr += 8) {
         const int r = r0 + rr;
         if (r >= rows) break;
-        const float x0 = sS[rr][lane];
+        const float x0 = lane < CC_TV ? sS[rr][lane] : -INFINITY;
         if (mode == GV_SELECT_LOGITS) {
             const float m = warp_max(x0);
             float s = 0.f;
