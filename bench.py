@@ -52,9 +52,9 @@ TRAFFIC = {
                     "paper_2502_11018_gb300/csrc/attn_common.cuh", "paper_2502_11018_gb300/csrc/sm103.cuh"],
         "sha256": "ed051a9e55204bba2de96fc3292927c0749f0ba16c78da30052f52a639472368"},
     ("lmhead_select", "llama3_8b"): {
-        "bytes": 1058259712,
+        "bytes": 1058401280,
         "sources": ["paper_2502_11018_gb300/csrc/lmhead_sm103.cu", "paper_2502_11018_gb300/csrc/sm103.cuh"],
-        "sha256": "6ff8a310867b9bcb936de895d36b7fbfe5d69d4196a9f7615f4a9884d90f66c7"},
+        "sha256": "67e6139a14cf3f2221a497fbc99ff4c54a1f111451c6cea1c8969d9b5fd805d7"},
 }
 OTHER_CONFIGS = ("llama2_7b", "llama2_13b_b4", "mixtral_attn", "tiny_f32")
 
