@@ -232,6 +232,12 @@ __device__ __forceinline__ int cta_of(long long w, long long W, int C) {
     return (int)(((w + 1) * C - 1) / W);
 }
 
+// The tile count of a unit as a type (the piece epilogue is compiled per count).
+template <int V>
+struct AlTiles {
+    static constexpr int value = V;
+};
+
 // 32-byte store of 8 words (sm_100+).
 __device__ __forceinline__ void st_global_v8(void* p, const uint32_t (&r)[8]) {
     asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(r[0]), "r"(r[1]),
@@ -850,77 +856,71 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
                 ltot = w_self * l_run + w_other * o2.y;
                 named_bar_sync(1, AL_NSM);
             }
-            const int c_lo = T == 2 ? 0 : 64 * s, c_n = T == 2 ? 128 : 64;   // d columns this thread writes
-            __nv_bfloat16* dst = nullptr;
-            if (rv) {
-                if (pc.direct || combine) {
-                    const int i = qr / G, h = pc.g * G + qr % G;
-                    dst = a.out + ((((size_t)pc.l * a.B + pc.b) * N + i) * a.Hq + h) * 128;
-                } else {
-                    dst = a.part + (((size_t)pc.slot * T + tile) * 128 + row) * 128;
+            // The rows out, compiled once per tile count: with two tiles a
+            // thread writes all 128 d columns of its tile's row from one
+            // accumulator, with one tile 64 columns (64 s ..) from two.
+            auto rows_out = [&](auto tiles) {
+                constexpr int TT = decltype(tiles)::value;
+                constexpr int CN = TT == 2 ? 128 : 64;       // d columns this thread writes
+                const int c_lo = TT == 2 ? 0 : 64 * s;
+                __nv_bfloat16* dst = nullptr;
+                if (rv) {
+                    if (pc.direct || combine) {
+                        const int i = qr / G, h = pc.g * G + qr % G;
+                        dst = a.out + ((((size_t)pc.l * a.B + pc.b) * N + i) * a.Hq + h) * 128;
+                    } else {
+                        dst = a.part + (((size_t)pc.slot * TT + tile) * 128 + row) * 128;
+                    }
                 }
-            }
-            const uint32_t o_other = lane_base + AL_OCOL + 128u * (uint32_t)(1 - s);
-            // (combining: the other piece's log2-sum-exp and partial columns,
-            // 32 columns at a time, each quarter's loads issued one quarter
-            // ahead)
-            uint4 pr[2][4];
-            const uint4* psrc = nullptr;
-            float a_self = 1.f, a_part = 0.f;
-            if (combine && rv) {
-                const size_t prow = ((size_t)other_slot * T + tile) * 128 + row;
-                const float lse_o = __ldcg(a.part_lse + prow);
-                psrc = reinterpret_cast<const uint4*>(a.part + prow * 128 + c_lo);
+                const uint32_t o_other = lane_base + AL_OCOL + 128u * (uint32_t)(1 - s);
+                // (combining: the other piece's log2-sum-exp and partial
+                // columns, loaded 64 columns ahead of their use into a ring of
+                // eight 16-byte chunks)
+                uint4 pr[8];
+                const uint4* psrc = nullptr;
+                float a_self = 1.f, a_part = 0.f;
+                if (combine && rv) {
+                    const size_t prow = ((size_t)other_slot * TT + tile) * 128 + row;
+                    const float lse_o = __ldcg(a.part_lse + prow);
+                    psrc = reinterpret_cast<const uint4*>(a.part + prow * 128 + c_lo);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) pr[0][q] = __ldcg(psrc + q);
-                const float lse_s = ltot > 0.f ? M + log2f(ltot) : -INFINITY;
-                const float Mc = fmaxf(lse_s, lse_o);
-                const float es = lse_s == -INFINITY ? 0.f : fast_exp2(lse_s - Mc);
-                const float eo = lse_o == -INFINITY ? 0.f : fast_exp2(lse_o - Mc);
-                a_self = es / (es + eo);
-                a_part = eo / (es + eo);                     // (NaN when the other gave up)
-            }
-            if (ok) {
-                tc_fence_after();
-                const float inv = ltot > 0.f ? 1.0f / ltot : 0.f;
-                const float fs = w_self * inv * a_self, fo = w_other * inv * a_self;
-                // 32 columns at a time: their TMEM loads issued together, one wait
+                    for (int q = 0; q < 8; ++q) pr[q] = __ldcg(psrc + q);
+                    const float lse_s = ltot > 0.f ? M + log2f(ltot) : -INFINITY;
+                    const float Mc = fmaxf(lse_s, lse_o);
+                    const float es = lse_s == -INFINITY ? 0.f : fast_exp2(lse_s - Mc);
+                    const float eo = lse_o == -INFINITY ? 0.f : fast_exp2(lse_o - Mc);
+                    a_self = es / (es + eo);
+                    a_part = eo / (es + eo);                     // (NaN when the other gave up)
+                }
+                if (ok) {
+                    tc_fence_after();
+                    const float inv = ltot > 0.f ? 1.0f / ltot : 0.f;
+                    const float fs = w_self * inv * a_self, fo = w_other * inv * a_self;
+                    // 16 columns at a time (the partial columns are all in
+                    // registers already)
 #pragma unroll
-                for (int qt = 0; qt < 4; ++qt) {
-                    if (32 * qt >= c_n) break;
-                    const int cq = c_lo + 32 * qt;       // (the columns of O this thread writes)
-                    uint32_t os[32], oo[32];
-                    if (has_self) {
-                        tmem_ld16(ocol + (uint32_t)cq, *reinterpret_cast<uint32_t(*)[16]>(&os[0]));
-                        tmem_ld16(ocol + (uint32_t)(cq + 16), *reinterpret_cast<uint32_t(*)[16]>(&os[16]));
-                    }
-                    if (has_other) {
-                        tmem_ld16(o_other + (uint32_t)cq, *reinterpret_cast<uint32_t(*)[16]>(&oo[0]));
-                        tmem_ld16(o_other + (uint32_t)(cq + 16), *reinterpret_cast<uint32_t(*)[16]>(&oo[16]));
-                    }
-                    if (psrc && 32 * (qt + 1) < c_n) {
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) pr[(qt + 1) & 1][q] = __ldcg(psrc + 4 * (qt + 1) + q);
-                    }
-                    tmem_wait_ld();
-                    if (dst) {
-#pragma unroll
-                        for (int g16 = 0; g16 < 2; ++g16) {
+                    for (int qt = 0; qt < CN / 16; ++qt) {
+                        const int cq = c_lo + 16 * qt;       // (the columns of O this thread writes)
+                        uint32_t os[16], oo[16];
+                        if (has_self) tmem_ld16(ocol + (uint32_t)cq, os);
+                        if (TT == 1 && has_other) tmem_ld16(o_other + (uint32_t)cq, oo);
+                        tmem_wait_ld();
+                        if (dst) {
                             uint32_t pv[8];
 #pragma unroll
                             for (int u = 0; u < 8; ++u) {
-                                const int e = 16 * g16 + 2 * u;     // column pair within the quarter
+                                const int e = 2 * u;     // column pair within the 16
                                 float v0 = 0.f, v1 = 0.f;
                                 if (has_self) {
                                     v0 = __uint_as_float(os[e]) * fs;
                                     v1 = __uint_as_float(os[e + 1]) * fs;
                                 }
-                                if (has_other) {
+                                if (TT == 1 && has_other) {
                                     v0 = fmaf(__uint_as_float(oo[e]), fo, v0);
                                     v1 = fmaf(__uint_as_float(oo[e + 1]), fo, v1);
                                 }
                                 if (combine) {
-                                    const uint4 q4 = pr[qt & 1][e >> 3];
+                                    const uint4 q4 = pr[(2 * qt + (e >> 3)) & 7];
                                     const int wd = (e >> 1) & 3;
                                     const uint32_t pw = wd == 0 ? q4.x : wd == 1 ? q4.y : wd == 2 ? q4.z : q4.w;
                                     const float2 f = unpack_bf16(pw);
@@ -929,16 +929,24 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
                                 }
                                 pv[u] = pack_bf16(v0, v1);
                             }
-                            st_global_v8(dst + cq + 16 * g16, pv);
+                            st_global_v8(dst + cq, pv);
+                        }
+                        if (psrc && qt + 4 < CN / 16) {
+                            pr[(2 * qt) & 7] = __ldcg(psrc + 2 * (qt + 4));
+                            pr[(2 * qt + 1) & 7] = __ldcg(psrc + 2 * (qt + 4) + 1);
                         }
                     }
+                } else if (dst) {
+                    // Gave up: NaN rows (whole piece, or combined) or an invalid partial.
+                    const uint32_t fill = (pc.direct || combine) ? pack_bf16(NAN, NAN) : 0u;
+                    const uint32_t pv[8] = {fill, fill, fill, fill, fill, fill, fill, fill};
+                    for (int e = 0; e < CN; e += 16) st_global_v8(dst + c_lo + e, pv);
                 }
-            } else if (dst) {
-                // Gave up: NaN rows (whole piece, or combined) or an invalid partial.
-                const uint32_t fill = (pc.direct || combine) ? pack_bf16(NAN, NAN) : 0u;
-                const uint32_t pv[8] = {fill, fill, fill, fill, fill, fill, fill, fill};
-                for (int e = 0; e < c_n; e += 16) st_global_v8(dst + c_lo + e, pv);
-            }
+            };
+            if (T == 2)
+                rows_out(AlTiles<2>{});
+            else
+                rows_out(AlTiles<1>{});
             if (!pc.direct && !combine && rv && (T == 2 || s == 0))
                 a.part_lse[((size_t)pc.slot * T + tile) * 128 + row] =
                     ok ? (ltot > 0.f ? M + log2f(ltot) : -INFINITY) : NAN;
