@@ -7,7 +7,9 @@ Mixtral-attention workload (32 layers, prefix 16384, temperature 1).
 
 The float64 oracle cannot redo all 32 layers in seconds, so it checks samples
 that it can compute one by one: the first, a middle and the last layer's
-attention output and tree keys/values; the LM-head argmax of a sample of rows
+attention output and tree keys/values over every head, every layer's over one
+KV-head group (group l mod Hkv, so a wrong layer or head offset anywhere in
+the multi-layer call shows); the LM-head argmax of a sample of rows
 (every row's argmax is also checked against the planted closed form); the
 acceptance of the GPU's choices (bit-exact for greedy, a valid trail under the
 oracle's probabilities for sampling); the compacted rows of the sampled
@@ -62,6 +64,23 @@ def _check_tree_attention_compaction(cfg, inp, step, layers, keep, P):
         assert rel_err(out, ro) <= TOL_ATTN[kind], l
         assert rel_err(f64(step.treeK[l]), rK) <= TOL_ROT[kind], l
         np.testing.assert_array_equal(f64(step.treeV[l]), rV)
+    # Every layer, one KV-head group each (the query heads g G .. g G + G - 1
+    # that share KV head g).  The prefix rows read here are the cache's rows
+    # below P, which the compaction never writes.
+    Hkv = cfg["Hkv"]
+    G = cfg["Hq"] // Hkv
+    for l in range(cfg["L"]):
+        g = l % Hkv
+        hs = slice(g * G, (g + 1) * G)
+        gs = slice(g, g + 1)
+        ro, rK, rV = oracle.tree_attention(f64(inp.q[l][:, :, hs]), f64(inp.k_new[l][:, :, gs]),
+                                           f64(inp.v_new[l][:, :, gs]), f64(inp.cacheK[l][:, gs]),
+                                           f64(inp.cacheV[l][:, gs]), P, pos, anc, cfg["rope_base"])
+        out = f64(step.attn_out[l][:, :, hs])
+        assert np.isfinite(out).all(), (l, g)
+        assert rel_err(out, ro) <= TOL_ATTN[kind], (l, g)
+        assert rel_err(f64(step.treeK[l][:, gs]), rK) <= TOL_ROT[kind], (l, g)
+        np.testing.assert_array_equal(f64(step.treeV[l][:, gs]), rV)
     # Compaction of the sampled layers: accepted rows come from the tree
     # scratch, every other row keeps its bytes.
     path = step.path.cpu().numpy()
