@@ -80,7 +80,7 @@ static_assert(128 * AL_REG_LOW + 256 * AL_REG_HIGH <= 384 * 168, "register split
 constexpr uint32_t AL_OCOL = 256;          // O of tile t at columns 256 + 128 t
 constexpr uint32_t AL_TMEM_COLS = 512;
 constexpr int AL_MAXB = 64;                // sequences per call
-constexpr int AL_DSTART = 2;               // positions without a block before each unit's blocks (see Walk)
+constexpr int AL_DSTART = 3;               // positions without a block before each unit's blocks (see Walk)
 constexpr int AL_DEND = 0;                 // ... and after them
 
 // Shared memory: Q tiles | K ring | V ring | barriers | misc | the two
