@@ -50,7 +50,7 @@ TRAFFIC = {
         "bytes": 18778672,
         "sources": ["paper_2502_11018_gb300/csrc/attention_layers_sm103.cu",
                     "paper_2502_11018_gb300/csrc/attn_common.cuh", "paper_2502_11018_gb300/csrc/sm103.cuh"],
-        "sha256": "5b02f19d5ac37c3ca85f3267773cf28bb4887cb5e28b854948269372a1805ce9"},
+        "sha256": "9f530270965a268f699ed610bc391db4cac47cfd852901e7c9f828a0de29b2f3"},
     ("lmhead_select", "llama3_8b"): {
         "bytes": 1058401280,
         "sources": ["paper_2502_11018_gb300/csrc/lmhead_sm103.cu", "paper_2502_11018_gb300/csrc/sm103.cuh"],

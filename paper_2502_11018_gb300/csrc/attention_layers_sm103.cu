@@ -896,8 +896,8 @@ attn_layers_kernel(const __grid_constant__ CUtensorMap map_ck, const __grid_cons
                     tc_fence_after();
                     const float inv = ltot > 0.f ? 1.0f / ltot : 0.f;
                     const float fs = w_self * inv * a_self, fo = w_other * inv * a_self;
-                    // 16 columns at a time (the partial columns are all in
-                    // registers already)
+                    // 16 columns at a time; after each step the two ring
+                    // chunks it used are reloaded with those 64 columns on
 #pragma unroll
                     for (int qt = 0; qt < CN / 16; ++qt) {
                         const int cq = c_lo + 16 * qt;       // (the columns of O this thread writes)
