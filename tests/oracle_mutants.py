@@ -66,6 +66,42 @@ MUTANTS = [
  ("compact.py", "                    cacheV[layer, b, h, P + t, :] = treeV[layer, b, h, src, :]", "                    cacheV[layer, b, h, P + t, :] = treeV[layer, b, h, t, :]", "compaction copies tree rows in node order (V)"),
  ("compact.py", "        if P + n > S_max:", "        if P + n >= S_max:", "capacity check off by one"),
  ("compact.py", "        new_len[b] = P + n", "        new_len[b] = P + n - 1", "new length one short"),
+ # temperature sampling acceptance
+ ("accept.py", "    return np.maximum(p - q, 0.0)", "    return np.abs(p - q)", "residual |p - q| instead of max(p - q, 0)"),
+ ("accept.py", "                ratio = p[x] / qx\n                min_margin", "                ratio = qx / max(p[x], 1e-300)\n                min_margin", "acceptance ratio inverted"),
+ ("accept.py", "                if s > 0.0:\n                    p = r / s\n            if nxt is None:", "                if s > 0.0:\n                    p = r\n            if nxt is None:", "residual not renormalised"),
+ ("accept.py", "            for c in _children(parents[b], u):\n                x = int(tokens[b, c])\n                qx = 1.0 if q is None else q[x]\n                if qx == 0.0:", "            for c in reversed(_children(parents[b], u)):\n                x = int(tokens[b, c])\n                qx = 1.0 if q is None else q[x]\n                if qx == 0.0:", "children tried in decreasing index order"),
+ ("accept.py", "    z = np.asarray(x, dtype=np.float64) / T", "    z = np.asarray(x, dtype=np.float64)", "temperature ignored"),
+ ("accept.py", "                v, m = _inverse_cdf(p, float(u_res[b, u]))", "                v, m = _inverse_cdf(_softmax(target_logits[b, u], temperature), float(u_res[b, u]))", "bonus drawn from the target, not the residual"),
+ # training objective
+ ("tat.py", "        out[r] = 1 if ahead < k else 0", "        out[r] = 1 if ahead <= k else 0", "predictable mask top-(k+1)"),
+ ("tat.py", "((logits[r] == lx) & (ids < x))", "((logits[r] == lx) & (ids > x))", "predictable mask tie rule reversed"),
+ ("tat.py", "        out[r] = lse - logits[r, int(tokens[r])]", "        out[r] = lse - logits[r].max()", "token loss against the argmax"),
+ ("tat.py", "        lse = m + np.log(np.exp(logits[r] - m).sum())", "        lse = np.log(np.exp(logits[r] - m).sum())", "token loss log-sum-exp without the max"),
+ ("tat.py", "    return np.abs(fd - ft).sum(axis=1)", "    return ((fd - ft) ** 2).sum(axis=1)", "feature loss squared, not L1"),
+ ("tat.py", "                v *= int(mbar_prev[j - 1][b][t - n + j])", "                v *= int(mbar_prev[j - 1][b][t - n + j + 1])", "alignment chain shifted by one position"),
+ ("tat.py", "            if t - n + 1 < 0:", "            if t - n < 0:", "alignment start bound off by one"),
+ ("tat.py", "    ell = (lam_tok * token_loss(rows_logits, rows_tok)\n           + lam_feat * feature_loss(", "    ell = (lam_feat * token_loss(rows_logits, rows_tok)\n           + lam_tok * feature_loss(", "loss weights swapped"),
+ ("tat.py", "        seq_loss[b] = num / den if den > 0 else 0.0", "        seq_loss[b] = num / T if den > 0 else 0.0", "pass loss divided by the length, not the mask sum"),
+ # decoder layer
+ ("layer.py", "    ms = (x * x).mean(axis=1, keepdims=True)", "    ms = (x * x).sum(axis=1, keepdims=True)", "RMSNorm over the sum, not the mean"),
+ ("layer.py", "    return z / (1.0 + np.exp(-z))", "    return 1.0 / (1.0 + np.exp(-z))", "sigmoid instead of silu"),
+ ("layer.py", "    return silu(linear(x, Wg)) * linear(x, Wu)", "    return linear(x, Wg) * silu(linear(x, Wu))", "silu on the up projection"),
+ ("layer.py", "    h = h + linear(o.reshape(B * N, Hq * d), w[\"Wo\"])", "    h = linear(o.reshape(B * N, Hq * d), w[\"Wo\"])", "attention residual dropped"),
+ ("layer.py", "    x = rmsnorm(h, w[\"mlp_norm\"], eps)", "    x = rmsnorm(h, w[\"attn_norm\"], eps)", "MLP norm with the attention norm's gain"),
+ ("layer.py", "    k = linear(x, w[\"Wk\"]).reshape(B, N, Hkv, d)", "    k = linear(x, w[\"Wv\"]).reshape(B, N, Hkv, d)", "keys projected with Wv"),
+ # Token-Guided Fusion
+ ("tgf.py", "    var = ((x - mu) ** 2).mean(axis=1, keepdims=True)", "    var = ((x - mu) ** 2).sum(axis=1, keepdims=True) / (x.shape[1] - 1)", "layer norm with the sample variance"),
+ ("tgf.py", "    h = linear(np.concatenate([F, x], axis=1), w[\"Wm\"]) + w[\"bm\"]", "    h = linear(np.concatenate([x, F], axis=1), w[\"Wm\"]) + w[\"bm\"]", "Eq. 6 concatenation order swapped"),
+ ("tgf.py", "    o = linear(silu(z), w[\"Wd\"]) + w[\"bd\"] + h", "    o = linear(silu(z), w[\"Wd\"]) + w[\"bd\"]", "Eq. 8 residual dropped"),
+ ("tgf.py", "layernorm(h, w[\"g_h\"], w[\"b_h\"], eps)", "layernorm(h, w[\"g_x\"], w[\"b_x\"], eps)", "Eq. 7 norm of h with the token norm's gain"),
+ ("tgf.py", "    z = linear(zin, w[\"Wu\"]) + w[\"bu\"]", "    z = linear(zin, w[\"Wu\"])", "Eq. 7 bias dropped"),
+ # draft tree
+ ("draft_tree.py", "            pool[\"score\"].append(pool[\"score\"][pid] + lp[t])", "            pool[\"score\"].append(pool[\"score\"][pid] + np.exp(lp[t]))", "scores add probabilities, not log-probabilities"),
+ ("draft_tree.py", "            pool[\"score\"].append(pool[\"score\"][pid] + lp[t])", "            pool[\"score\"].append(lp[t])", "scores not cumulative"),
+ ("draft_tree.py", "    order = np.lexsort((np.arange(x.size), -x))", "    order = np.lexsort((-np.arange(x.size), -x))", "expansion top-k ties toward the higher id"),
+ ("draft_tree.py", "    order = np.lexsort((np.array(ids), -sc))", "    order = np.lexsort((-np.array(ids), -sc))", "selection ties toward the later pool node"),
+ ("draft_tree.py", "    kept, gap = best(pool, range(1, len(pool[\"token\"])), N - 1)", "    kept, gap = best(pool, range(1, len(pool[\"token\"])), N - 2)", "rerank keeps one node too few"),
 ]
 
 
@@ -83,8 +119,11 @@ def run(idx, base):
         return idx, "ANCHOR MISSING", []
     open(path, "w").write(text.replace(old, new))
     pins = sorted(glob.glob(os.path.join(d, "tests", "test_oracle_*.py")))
+    # One thread per run: parallel runs with a full BLAS / OpenMP pool each
+    # oversubscribe the cores badly enough to time out fast tests.
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
     r = subprocess.run([sys.executable, "-m", "pytest", *pins, "-q", "-m", "not gpu", "-p", "no:cacheprovider",
-                        "--tb=no", "--timeout=60"], cwd=d, capture_output=True, text=True)
+                        "--tb=no", "--timeout=120"], cwd=d, capture_output=True, text=True, env=env)
     failed = [ln.split()[1] for ln in r.stdout.splitlines() if ln.startswith("FAILED")]
     shutil.rmtree(d)
     return idx, ("caught" if failed else "SURVIVED"), failed

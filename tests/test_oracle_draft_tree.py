@@ -117,3 +117,27 @@ def test_flat_tail_keeps_the_first_level():
     out = draft_tree(0, steps, k, D, N=k + 1)
     assert out["parents"].tolist() == [-1] * 1 + [0] * k
     assert out["tokens"].tolist() == [0, 3, 9, 1, 30, 22]
+
+
+def test_uniform_logits_tie_rules_by_hand():
+    # Every logit equal (V = 4, k = 2, D = 3, N = 6): every candidate of a
+    # step scores the same, so the tie rules alone decide the tree.
+    # Step 0 expands the root: tokens 0, 1 (lower ids first) -> pool 1, 2,
+    # both -log 4.  Selection of the two nodes expanded next, ties toward the
+    # earlier pool node: slot 0 = pool 1, slot 1 = pool 2.  Step 1: slot 0's
+    # children are pool 3, 4 (tokens 0, 1), slot 1's pool 5, 6, all -2 log 4;
+    # the next expansion takes pool 3, 4 (both children of pool 1).  Step 2
+    # adds pool 7 .. 10 (children of 3 and 4), -3 log 4 each.  Rerank of the
+    # N - 1 = 5 best: pool 1, 2 and the three earliest of 3 .. 6, i.e. 3, 4, 5.
+    V, k, D, N = 4, 2, 3, 6
+    steps = [np.zeros((1, V)), np.zeros((k, V)), np.zeros((k, V))]
+    out = draft_tree(9, steps, k=k, D=D, N=N)
+    l4 = math.log(4)
+    assert out["expanded"] == [[0], [1, 2], [3, 4]]
+    assert out["pool"]["parent"] == [-1, 0, 0, 1, 1, 2, 2, 3, 3, 4, 4]
+    assert out["pool"]["token"] == [9, 0, 1, 0, 1, 0, 1, 0, 1, 0, 1]
+    np.testing.assert_allclose(out["pool"]["score"], [0] + [-l4] * 2 + [-2 * l4] * 4 + [-3 * l4] * 4,
+                               rtol=1e-13)
+    assert out["keep"] == [0, 1, 2, 3, 4, 5]
+    assert out["parents"].tolist() == [-1, 0, 0, 1, 1, 2]
+    assert out["tokens"].tolist() == [9, 0, 1, 0, 1, 0]

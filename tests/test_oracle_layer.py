@@ -1,10 +1,13 @@
 """Pins of the target-layer oracle (RMSNorm, linear, SwiGLU, one decoder
-layer around the tree attention) against closed forms, brute force and
-special cases that reduce the layer to a known expression."""
+layer around the tree attention) against closed forms, brute force,
+special cases that reduce the layer to a known expression, and an ordinary
+causal LLaMA layer written with torch's library attention."""
 
 import math
 
 import numpy as np
+import torch
+import torch.nn.functional as F
 
 from oracle.layer import decoder_layer, linear, rmsnorm, silu, swiglu
 from oracle.tree import tree_build
@@ -89,3 +92,64 @@ def test_single_token_layer_closed_form():
     gate = w["Wg"] @ x2
     ref = h1 + w["Wd"] @ (gate / (1.0 + np.exp(-gate)) * (w["Wu"] @ x2))
     np.testing.assert_allclose(got[0], ref, rtol=1e-10)
+
+
+def _rope_complex_torch(x, base):
+    """RoPE of x [S][heads][d] at positions 0 .. S-1 as the complex product
+    (x[j] + i x[j + d/2]) exp(i pos base^(-2j/d))."""
+    S, _, d = x.shape
+    half = d // 2
+    theta = torch.tensor([base ** (-2.0 * j / d) for j in range(half)], dtype=torch.float64)
+    ang = torch.arange(S, dtype=torch.float64)[:, None] * theta[None, :]
+    z = torch.complex(x[..., :half], x[..., half:]) * torch.polar(torch.ones_like(ang), ang)[:, None, :]
+    return torch.cat([z.real, z.imag], dim=-1)
+
+
+def _torch_llama_layer(hs, w, base, Hq, Hkv, d, eps=1e-5):
+    """A LLaMA decoder layer over a whole sequence in torch float64, causal
+    attention by scaled_dot_product_attention; returns the outputs and every
+    position's rotated key and value."""
+    t = {k: torch.from_numpy(np.asarray(v, dtype=np.float64)) for k, v in w.items()}
+    h = torch.from_numpy(hs)
+    S = h.shape[0]
+
+    def norm(v, g):
+        return v * torch.rsqrt(v.pow(2).mean(dim=-1, keepdim=True) + eps) * g
+
+    x = norm(h, t["attn_norm"])
+    q = _rope_complex_torch((x @ t["Wq"].T).view(S, Hq, d), base)
+    k = _rope_complex_torch((x @ t["Wk"].T).view(S, Hkv, d), base)
+    v = (x @ t["Wv"].T).view(S, Hkv, d)
+    G = Hq // Hkv
+    o = F.scaled_dot_product_attention(q.transpose(0, 1)[None], k.repeat_interleave(G, dim=1).transpose(0, 1)[None],
+                                       v.repeat_interleave(G, dim=1).transpose(0, 1)[None], is_causal=True)
+    h1 = h + o[0].transpose(0, 1).reshape(S, Hq * d) @ t["Wo"].T
+    x2 = norm(h1, t["mlp_norm"])
+    h2 = h1 + (F.silu(x2 @ t["Wg"].T) * (x2 @ t["Wu"].T)) @ t["Wd"].T
+    return h2.numpy(), k.numpy(), v.numpy()
+
+
+def test_chain_layer_equals_a_causal_llama_layer():
+    # A two-node chain after a three-token prefix is the last two positions of
+    # a five-token causal sequence: the tree layer, fed the prefix's rotated
+    # keys and values as its cache, must give what an ordinary LLaMA layer
+    # (torch, causal SDPA, RoPE as a complex product, GQA by repeated KV heads)
+    # gives there.  Unlike the one-token case, the keys decide the weights.
+    rng = np.random.default_rng(11)
+    Hq, Hkv, d, Fw, base = 4, 2, 8, 48, 1e4
+    H = Hq * d
+    w = _layer_weights(rng, H, Hq, Hkv, d, Fw, scale=0.3)
+    hs = rng.normal(size=(5, H))
+    ref, rk, rv = _torch_llama_layer(hs, w, base, Hq, Hkv, d)
+    P = np.array([3])
+    parents = np.array([[-1, 0]])
+    depth, pos, anc, st = tree_build(parents, P)
+    S = 8
+    cK = np.zeros((1, Hkv, S, d))
+    cV = np.zeros((1, Hkv, S, d))
+    cK[0, :, :3] = rk[:3].transpose(1, 0, 2)
+    cV[0, :, :3] = rv[:3].transpose(1, 0, 2)
+    got, tK, tV = decoder_layer(hs[3:], w, cK, cV, P, pos, anc, base, 1, 2, Hq, Hkv, d)
+    np.testing.assert_allclose(got, ref[3:], rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(tK[0], rk[3:].transpose(1, 0, 2), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(tV[0], rv[3:].transpose(1, 0, 2), rtol=1e-10, atol=1e-12)

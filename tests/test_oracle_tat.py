@@ -124,3 +124,25 @@ def test_sequence_without_aligned_tokens_has_zero_loss():
     out = tat_pass(lg, tok, fd, ft, k=3, n=2, mbar_prev=prev)
     assert (out["mask"] == 0).all()
     np.testing.assert_array_equal(out["seq_loss"], [0.0, 0.0])
+
+
+def test_pass_loss_is_the_mean_over_aligned_steps_hand_example():
+    # Eq. 5 by hand.  One sequence of T = 5 steps, V = 4 uniform logits (each
+    # step's cross-entropy is exactly log 4) and features differing by a
+    # constant c_t in each of H = 2 components (L1 distance 2 |c_t|), so with
+    # lam_feat = 0.1 the per-step losses are log 4 + (1.0, 0.2, 0.4, 1.4, 0.6).
+    # Pass n = 2 with the first pass's predictable mask (1, 1, 0, 1, 0): the
+    # alignment mask is (0, 1, 1, 0, 1) (step t looks at step t - 1; step 0
+    # has no chain), and the pass loss is the mean over those three steps,
+    # log 4 + (0.2 + 0.4 + 0.6) / 3 = log 4 + 0.4.
+    T, V, H = 5, 4, 2
+    logits = np.zeros((1, T, V))
+    tokens = np.array([[0, 1, 2, 3, 0]])
+    c = np.array([5.0, 1.0, 2.0, 7.0, 3.0])
+    ft = np.zeros((1, T, H))
+    fd = np.repeat(c[None, :, None], H, axis=2)
+    prev = [np.array([[1, 1, 0, 1, 0]], dtype=np.uint8)]
+    out = tat_pass(logits, tokens, fd, ft, k=2, n=2, mbar_prev=prev)
+    np.testing.assert_array_equal(out["mask"], [[0, 1, 1, 0, 1]])
+    np.testing.assert_allclose(out["ell"][0], math.log(4) + np.array([1.0, 0.2, 0.4, 1.4, 0.6]), rtol=1e-13)
+    assert abs(out["seq_loss"][0] - (math.log(4) + 0.4)) < 1e-13
