@@ -11,8 +11,8 @@ loop forever fails that way).  The script prints one line per mutant with the
 pins that caught it and exits non-zero if any mutant survives.
 
 Not collected by pytest (the file name does not start with ``test_``): it
-runs the whole pin suite once per mutant, about a quarter of an hour on 8
-cores (the chi-square losslessness pins take most of it).
+runs the whole pin suite once per mutant, about twenty minutes on 8 cores
+(the chi-square losslessness pins take most of it).
 """
 
 import concurrent.futures as cf
@@ -102,6 +102,16 @@ MUTANTS = [
  ("draft_tree.py", "    order = np.lexsort((np.arange(x.size), -x))", "    order = np.lexsort((-np.arange(x.size), -x))", "expansion top-k ties toward the higher id"),
  ("draft_tree.py", "    order = np.lexsort((np.array(ids), -sc))", "    order = np.lexsort((-np.array(ids), -sc))", "selection ties toward the later pool node"),
  ("draft_tree.py", "    kept, gap = best(pool, range(1, len(pool[\"token\"])), N - 1)", "    kept, gap = best(pool, range(1, len(pool[\"token\"])), N - 2)", "rerank keeps one node too few"),
+ # indexing across layers and sequences
+ ("attention.py", "            Kp = np.asarray(cacheK[b, g, :P, :], dtype=np.float64)", "            Kp = np.asarray(cacheK[0, g, :P, :], dtype=np.float64)", "every sequence reads sequence 0's prefix keys"),
+ ("compact.py", "        for layer in range(L):", "        for layer in range(1):", "only the first layer committed"),
+ ("tree.py", "                anc[b, i] = np.uint64(1) << np.uint64(i)", "                anc[b, i] = np.uint64(1)", "an invalid tree's nodes all see the root"),
+ # the step composition
+ ("step.py", "                                   as_f64(inp.v_new[layer]), as_f64(inp.cacheK[layer]),", "                                   as_f64(inp.v_new[layer]), as_f64(inp.cacheK[0]),", "every layer reads layer 0's key cache"),
+ ("step.py", "        o, tk, tv = tree_attention(as_f64(inp.q[layer]),", "        o, tk, tv = tree_attention(as_f64(inp.q[L - 1 - layer]),", "layers' queries in reverse order"),
+ ("step.py", "                                   as_f64(inp.cacheV[layer]), prefix_len, pos, anc,", "                                   as_f64(inp.cacheV[layer]), prefix_len, depth, anc,", "RoPE at depths, not positions"),
+ ("step.py", "                                          path, alen, prefix_len, st)", "                                          path, alen, prefix_len + 1, st)", "commit one row late"),
+ ("step.py", "        ck, cv, new_len, st2 = kv_compact(np.stack(treeK), np.stack(treeV),", "        ck, cv, new_len, st2 = kv_compact(np.stack(treeK[::-1]), np.stack(treeV),", "keys committed into the wrong layers"),
 ]
 
 
